@@ -1,0 +1,444 @@
+"""PIFA layer forward throughput on GB300.
+
+Default workload (one step = one pifa_forward over one token batch): the LLaMA-2-7B-shaped
+attention projection m = n = 4096, r = 2048, decode batch T = 8 (bf16). The step runs the whole
+hot path (selector, Y_p = X W_p^T, Y_np = Y_p C^T, both scatters into Y).
+
+Printed as one JSON line on rank 0:
+  value      tokens/s, device-timed (CUDA events on the launching stream) over K steps replayed
+             from a CUDA graph; the weights rotate over enough copies that the working set is
+             larger than L2 (every step streams its weights from HBM);
+  e2e        the same metric through the public API with host buffers: per step, X copied from
+             pinned host memory, pifa_forward, Y copied back to pinned host memory;
+  roofline   the decode call's achieved HBM GB/s against MEASURED_PEAKS.json (algorithmic bytes:
+             2 r(m + n - r) weight bytes + 2 T (n + m) activation bytes + 4 m index bytes);
+  cpu_baseline  the fp64 oracle (numpy) on the host cores over a bounded sample of the workload;
+  comparators   dense X W^T and low-rank (X V) U^T on the same GPU via torch.matmul;
+  prefill    the same layer at T = 2048 (tcgen05 path) with its bf16 tensor roofline.
+
+--impl reference times the oracle instead (the reference arm: the paper has no code).
+Multi-GPU (torchrun): every rank runs an independent replica of the workload ("replicas only");
+the time is the max over ranks and value sums the ranks' tokens.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2501_19090_gb300 import inputs  # noqa: E402
+
+METRIC = "PIFA layer tokens/s at 1 GB300 + % of HBM / bf16 tensor roofline vs low-rank"
+SHAPE = inputs.ATTN7B
+T_DECODE = 8
+T_PREFILL = 2048
+
+# DRAM traffic per launch measured with ncu for a given kernel source (sha256 of the .cu file).
+# A mismatch (the kernel changed since the capture) reports traffic as null.
+NCU_TRAFFIC = {}
+
+
+def _src_sha(name: str) -> str:
+    p = os.path.join(ROOT, "paper_2501_19090_gb300", "csrc", name)
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def decode_bytes(T, m, n, r):
+    return 2 * r * (m + n - r) + 2 * T * (n + m) + 4 * m
+
+
+def pifa_flops(T, m, n, r):
+    return 2 * T * r * (m + n - r)
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 100 ms while active."""
+
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "100",
+                 "-i", str(self.gpu)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[4:8]):
+                if val.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------------------------
+def build_layer(shape, seed):
+    """Host-side setup: the library's compression (Algorithm 1), rounded to bf16 operands."""
+    from paper_2501_19090_gb300 import pifa as P
+    U, V, _ = inputs.make_factors(shape.m, shape.n, shape.r, seed)
+    piv, nonp, Wp, C, info = P.pifa_compress(U, V, shape.r)
+    return dict(U=U, V=V, piv=piv, nonp=nonp, Wp=inputs.round_bf16(Wp), C=inputs.round_bf16(C), info=info)
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    from paper_2501_19090_gb300 import pifa as P
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    P.load()
+    hbm_peak, tc_peak, tc_sust, peak_src = _peaks()
+    shape = SHAPE
+    m, n, r = shape.m, shape.n, shape.r
+    T = args.tokens
+    lay = build_layer(shape, seed=0)
+    bf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev).to(torch.bfloat16)
+    piv = torch.from_numpy(lay["piv"]).to(dev)
+    nonp = torch.from_numpy(lay["nonp"]).to(dev)
+    Wp0, C0 = bf(lay["Wp"]), bf(lay["C"])
+    wbytes = (Wp0.numel() + C0.numel()) * 2
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    copies = max(4, math.ceil(3 * l2 / wbytes))
+    Wps = [Wp0.clone() for _ in range(copies)]
+    Cs = [C0.clone() for _ in range(copies)]
+    rng = np.random.default_rng(1 + rank)
+    Xs = [bf(inputs.make_activations(rng, T, n, "bf16")) for _ in range(copies)]
+    Ys = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(copies)]
+    variant = P.pifa_select_variant(T, m, n, r)
+    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant), dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def step(i):
+        j = i % copies
+        P.pifa_forward(Xs[j], Wps[j], Cs[j], piv, nonp, Y=Ys[j], variant=variant, workspace_tensor=ws,
+                       stream=stream)
+
+    # warm-up (eager), then capture a graph of `per_graph` steps
+    with torch.cuda.stream(stream):
+        for i in range(max(3, args.warmup)):
+            step(i)
+    stream.synchronize()
+    assert P.pifa_device_status(stream) == P.PIFA_OK
+    per_graph = copies * max(1, 64 // copies)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(per_graph):
+            step(i)
+    replays = max(1, math.ceil(args.steps / per_graph))
+    steps = replays * per_graph
+    for _ in range(max(3, args.warmup)):
+        g.replay()
+    stream.synchronize()
+
+    dist = _dist()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clk:
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(replays):
+                g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    ms = e0.elapsed_time(e1)
+    st = P.pifa_device_status(stream)
+    assert st == P.PIFA_OK, P.pifa_status_string(st)
+    ms_max = _max_over_ranks(ms)
+    step_ms = ms_max / steps
+    value = world * T * steps / (ms_max / 1e3)
+    achieved = decode_bytes(T, m, n, r) / (step_ms / 1e3) / 1e9
+
+    # --- e2e through the public API with pinned host buffers ---
+    Xh = torch.empty((T, n), dtype=torch.bfloat16).pin_memory()
+    Xh.copy_(Xs[0].cpu())
+    Yh = torch.empty((T, m), dtype=torch.bfloat16).pin_memory()
+    Xd = torch.empty((T, n), dtype=torch.bfloat16, device=dev)
+    e2e_steps = min(steps, 2000)
+    with torch.cuda.stream(stream):
+        for i in range(5):
+            Xd.copy_(Xh, non_blocking=True)
+            step_e2e = P.pifa_forward(Xd, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Ys[0], variant=variant,
+                                      workspace_tensor=ws, stream=stream)
+            Yh.copy_(Ys[0], non_blocking=True)
+    stream.synchronize()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for i in range(e2e_steps):
+            Xd.copy_(Xh, non_blocking=True)
+            P.pifa_forward(Xd, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Ys[0], variant=variant,
+                           workspace_tensor=ws, stream=stream)
+            Yh.copy_(Ys[0], non_blocking=True)
+        e1.record(stream)
+    stream.synchronize()
+    e2e_ms = _max_over_ranks(e0.elapsed_time(e1))
+    e2e_value = world * T * e2e_steps / (e2e_ms / 1e3)
+
+    out = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
+        "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{shape.name} decode T={T}", "m": m, "n": n, "r": r, "tokens_per_step": T,
+                   "variant": P.pifa_variant_name(variant), "parallelism": f"replicas{world}",
+                   "l2_defeat": f"{copies} rotating weight copies ({copies * wbytes / 1e6:.0f} MB > 3x L2)",
+                   "timing": "CUDA graph replay, CUDA events on the launching stream"},
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": T * n * 2,
+                "d2h_bytes_per_step": T * m * 2},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "traffic": _traffic("decode.cu", "decode"),
+                     "peak_source": f"{peak_src} hbm_gbs", "kernel": "decode_pivot_rows + decode_nonpivot_rows (PDL pair)",
+                     "algorithmic_bytes_per_launch": decode_bytes(T, m, n, r)},
+        "gpu_launches": steps * (2 if m > r else 1),
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and not args.no_extras:
+        out["comparators"] = comparators(dev, lay, T, copies, stream)
+        out["prefill"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src)
+        out["cpu_baseline"] = cpu_baseline(lay, T)
+    return out
+
+
+def comparators(dev, lay, T, copies, stream):
+    """Dense X W^T and two-factor low-rank (X V) U^T on the same GPU (torch.matmul, bf16)."""
+    import torch
+    res = {}
+    U = torch.from_numpy(lay["U"]).to(dev).to(torch.bfloat16)
+    V = torch.from_numpy(lay["V"]).to(dev).to(torch.bfloat16)
+    W = (U.float() @ V.float().t()).to(torch.bfloat16)
+    for Tq in (T, T_PREFILL):
+        X = torch.randn((Tq, V.shape[0]), device=dev).to(torch.bfloat16)
+        Ws = [W.clone() for _ in range(max(2, copies // 2))]
+        Us = [U.clone() for _ in range(copies)]
+        Vs = [V.clone() for _ in range(copies)]
+        for name, fn, nrot in (("dense", lambda i: X @ Ws[i % len(Ws)].t(), len(Ws)),
+                               ("lowrank", lambda i: (X @ Vs[i % copies]) @ Us[i % copies].t(), copies)):
+            with torch.cuda.stream(stream):
+                for i in range(5):
+                    fn(i)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                reps = 200 if Tq <= 16 else 40
+                e0.record(stream)
+                for i in range(reps):
+                    fn(i)
+                e1.record(stream)
+            stream.synchronize()
+            ms = e0.elapsed_time(e1) / reps
+            res[f"{name}_T{Tq}"] = {"tokens_per_s": Tq / (ms / 1e3), "ms": ms}
+    return res
+
+
+def prefill_point(dev, lay, copies, stream, tc_peak, peak_src):
+    import torch
+    from paper_2501_19090_gb300 import pifa as P
+    m, n, r = SHAPE.m, SHAPE.n, SHAPE.r
+    T = T_PREFILL
+    bf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev).to(torch.bfloat16)
+    piv = torch.from_numpy(lay["piv"]).to(dev)
+    nonp = torch.from_numpy(lay["nonp"]).to(dev)
+    Wp, C = bf(lay["Wp"]), bf(lay["C"])
+    ncp = max(2, copies // 4)
+    Wps = [Wp.clone() for _ in range(ncp)]
+    Cs = [C.clone() for _ in range(ncp)]
+    rng = np.random.default_rng(5)
+    Xs = [bf(inputs.make_activations(rng, T, n, "bf16")) for _ in range(ncp)]
+    Y = torch.empty((T, m), dtype=torch.bfloat16, device=dev)
+    variant = P.pifa_select_variant(T, m, n, r)
+    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant), dev, "prefill")
+    with torch.cuda.stream(stream):
+        for i in range(5):
+            P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,
+                           workspace_tensor=ws, stream=stream)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        reps = 50
+        e0.record(stream)
+        for i in range(reps):
+            P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,
+                           workspace_tensor=ws, stream=stream)
+        e1.record(stream)
+    stream.synchronize()
+    assert P.pifa_device_status(stream) == P.PIFA_OK
+    ms = e0.elapsed_time(e1) / reps
+    tf = pifa_flops(T, m, n, r) / (ms / 1e3) / 1e12
+    return {"workload": f"{SHAPE.name} prefill T={T}", "variant": P.pifa_variant_name(variant),
+            "tokens_per_s": T / (ms / 1e3), "ms_per_step": ms,
+            "roofline": {"bound": "tensor", "achieved": tf, "peak": tc_peak, "unit": "TFLOP/s",
+                         "frac": tf / tc_peak, "peak_source": f"{peak_src} bf16_tflops (burst)",
+                         "algorithmic_flops_per_launch": pifa_flops(T, m, n, r)}}
+
+
+def cpu_baseline(lay, T, budget_s=10.0):
+    """The fp64 oracle forward (numpy) on the host cores over a bounded sample of the workload."""
+    import oracle
+    rng = np.random.default_rng(9)
+    X = inputs.make_activations(rng, T, SHAPE.n, "bf16")
+    Wp, C = lay["Wp"].astype(np.float64), lay["C"].astype(np.float64)
+    piv, nonp = lay["piv"].astype(np.int64), lay["nonp"].astype(np.int64)
+    oracle.forward(X, Wp, C, piv, nonp)
+    t0 = time.perf_counter()
+    calls = 0
+    while time.perf_counter() - t0 < budget_s:
+        oracle.forward(X, Wp, C, piv, nonp)
+        calls += 1
+    dt = time.perf_counter() - t0
+    cores = len(os.sched_getaffinity(0))
+    return {"value": calls * T / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{calls} oracle forwards of T={T} tokens on {SHAPE.name} (fp64 numpy, BLAS threads = cores), {dt:.1f} s"}
+
+
+def _traffic(src, key):
+    t = NCU_TRAFFIC.get(key)
+    if not t or t.get("sha") != _src_sha(src):
+        return None
+    return t["bytes"]
+
+
+# ---------------------------------------------------------------------------------------------
+_DIST = None
+
+
+def _dist():
+    return _DIST
+
+
+def _max_over_ranks(v):
+    d = _dist()
+    if not d:
+        return v
+    import torch
+    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    d.all_reduce(t, op=d.ReduceOp.MAX)
+    return float(t.item())
+
+
+def run_reference(args, rank):
+    """Reference arm: the fp64 oracle (the paper publishes no code) on the host cores, same workload."""
+    import oracle
+    from paper_2501_19090_gb300 import pifa as P
+    if rank != 0:
+        return None
+    T = args.tokens
+    U, V, _ = inputs.make_factors(SHAPE.m, SHAPE.n, SHAPE.r, 0)
+    L = oracle.compress(U, V, SHAPE.r, "lapack")
+    Wp, C = inputs.round_bf16(L.Wp).astype(np.float64), inputs.round_bf16(L.C).astype(np.float64)
+    rng = np.random.default_rng(1)
+    X = inputs.make_activations(rng, T, SHAPE.n, "bf16")
+    for _ in range(max(3, args.warmup)):
+        oracle.forward(X, Wp, C, L.pivots, L.nonpivots)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.forward(X, Wp, C, L.pivots, L.nonpivots)
+    dt = time.perf_counter() - t0
+    v = T * args.steps / dt
+    cores = len(os.sched_getaffinity(0))
+    del P
+    return {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": f"{SHAPE.name} decode T={T}", "m": SHAPE.m, "n": SHAPE.n,
+                                            "r": SHAPE.r, "tokens_per_step": T},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{args.steps} fp64 oracle forwards of T={T} (numpy, host cores)"},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    global _DIST
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--tokens", type=int, default=T_DECODE)
+    ap.add_argument("--no-extras", action="store_true")
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        out = run_reference(args, rank)
+        if out is not None:
+            print(json.dumps(out), flush=True)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+        _DIST = dist
+    out = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if _DIST:
+        _DIST.barrier()
+        _DIST.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,171 @@
+/*
+ * pifa.h -- C ABI of libpifa: the forward pass of a Pivoting Factorization (PIFA) layer on
+ * NVIDIA GB300 (sm_103a), plus a host-side reference compression.
+ *
+ * A rank-r weight W' (m x n) is stored as (Sec. 3.2, Eqs. 1-2):
+ *   I    -- pivot-row indices, r of them (Algorithm 1, step 1);
+ *   I^c  -- the other m - r row indices (Algorithm 1, step 2);
+ *   W_p  -- the pivot rows W'[I, :], r x n (Eq. 1);
+ *   C    -- coefficients with W'[I^c, :] = C W_p, (m - r) x r (Eq. 2).
+ * The forward pass (Algorithm 2) maps activations to outputs:
+ *   Y_p = W_p X,  Y_np = C Y_p,  Y[I, :] = Y_p,  Y[I^c, :] = Y_np.
+ * The paper writes activations as columns (X is n x b). This library keeps tokens as ROWS:
+ * X is T x n row-major and Y = X W'^T is T x m row-major, so Y_p = X W_p^T (T x r) and
+ * Y_np = Y_p C^T (T x (m - r)); output column I[j] receives Y_p[:, j] and column I^c[i]
+ * receives Y_np[:, i].
+ *
+ * Conventions for every call:
+ *  - Status codes are returned (pifa_status); nothing aborts. pifa_status_string() names them
+ *    and pifa_last_error() gives the calling thread's last detailed message.
+ *  - Sizes and leading dimensions are counts of ELEMENTS, int64_t.
+ *  - Matrices are row-major; a leading dimension is the distance between consecutive rows.
+ *  - Device buffers are caller-owned. The library never keeps a pointer past the call and
+ *    allocates no device memory in pifa_forward (scratch comes from the caller's workspace).
+ *  - bf16 means IEEE-style bfloat16 (1 sign, 8 exponent, 7 mantissa bits); accumulation is fp32.
+ */
+#ifndef PIFA_H_
+#define PIFA_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  PIFA_OK = 0,
+  PIFA_ERR_INVALID_ARG = -1,     /* null pointer, bad size or leading dimension, bad index set  */
+  PIFA_ERR_ALIGNMENT = -2,       /* a base pointer or row pitch is not 16-byte aligned          */
+  PIFA_ERR_UNSUPPORTED = -3,     /* shape/variant combination this build does not implement    */
+  PIFA_ERR_CUDA = -4,            /* a CUDA runtime/driver call failed (see pifa_last_error)    */
+  PIFA_ERR_TIMEOUT = -5,         /* a device-side bounded wait gave up (kernel returned early) */
+  PIFA_ERR_RANK_DEFICIENT = -6,  /* W' = U V^T has fewer than r independent rows               */
+  PIFA_ERR_WORKSPACE = -7,       /* workspace missing or smaller than pifa_workspace_size()    */
+  PIFA_ERR_DEVICE_INDEX = -8     /* a kernel met a pivot/non-pivot index outside [0, m)       */
+} pifa_status;
+
+/* Forward-pass implementations. PIFA_VARIANT_AUTO lets the selector choose (see
+ * pifa_select_variant). The others force one implementation; a forced variant that cannot run
+ * the given shape returns PIFA_ERR_UNSUPPORTED. */
+typedef enum {
+  PIFA_VARIANT_AUTO = 0,
+  PIFA_VARIANT_DECODE = 1,        /* T <= 16: two-phase HBM-streaming GEMV (mma.sync fragments)  */
+  PIFA_VARIANT_PREFILL_SPLIT = 2, /* tcgen05 GEMM 1 -> Y_p hi/lo in workspace -> tcgen05 GEMM 2 */
+  PIFA_VARIANT_PREFILL_FUSED = 3  /* one cluster kernel: Y_p stays in shared memory             */
+} pifa_variant;
+
+/* Diagnostics of pifa_compress (all optional to read). */
+typedef struct {
+  double min_pivot_gap;   /* min over greedy steps of (best - runner_up) / best residual norm  */
+  double r_ratio;         /* |R_(r-1,r-1)| / |R_00| of the pivoted QR                          */
+  double max_abs_c;       /* max |C_ij|                                                         */
+  int32_t threads;        /* host threads used                                                  */
+} pifa_compress_info;
+
+/*
+ * pifa_forward -- Algorithm 2 (Sec. 3.2) on the GPU, asynchronously on `cuda_stream`.
+ *
+ *   X            DEVICE, bf16, T x n, row pitch ldx >= n.
+ *   Wp           DEVICE, bf16, r x n, row pitch ldwp >= n (row j is W'[I[j], :]).
+ *   C            DEVICE, bf16, (m - r) x r, row pitch ldc >= r (row i gives W'[I^c[i], :]).
+ *                May be NULL when r == m.
+ *   pivot_idx    DEVICE, int32[r], strictly ascending, values in [0, m).
+ *   nonpivot_idx DEVICE, int32[m - r], strictly ascending; together with pivot_idx a partition
+ *                of [0, m). May be NULL when r == m.
+ *   Y            DEVICE, bf16, T x m, row pitch ldy >= m. Every element Y[t, 0..m-1] is written
+ *                exactly once (round to nearest even from the fp32 accumulator); the padding
+ *                columns m..ldy-1 are not touched. Y must not overlap any input.
+ *   workspace    DEVICE scratch of at least pifa_workspace_size(T, m, n, r, variant) bytes,
+ *                256-byte aligned; NULL allowed when that size is 0. It must not be used by
+ *                another call that may run concurrently.
+ *   cuda_stream  a cudaStream_t (NULL = legacy default stream).
+ *
+ *   Requirements: 1 <= r <= min(m, n); T >= 0 (T == 0 is a no-op); every base pointer of X, Wp,
+ *   C, Y 16-byte aligned and ldx, ldwp, ldc, ldy multiples of 8 (16-byte row pitch), else
+ *   PIFA_ERR_ALIGNMENT. Index sets are not validated on the host (that would need a copy back);
+ *   kernels skip any write whose index is outside [0, m) and latch PIFA_ERR_DEVICE_INDEX, read
+ *   with pifa_device_status(). pifa_validate_indices() checks host copies in full.
+ *   Numerics: bf16 operands, fp32 accumulation; Y_p is carried into the second contraction
+ *   at (at least) 16 significant bits (a bf16 hi + bf16 lo pair or fp32), never as bf16 alone.
+ *   Returns PIFA_OK once the kernels are enqueued; launch errors give PIFA_ERR_CUDA.
+ */
+int pifa_forward(const void* X, int64_t T, int64_t n, int64_t ldx,
+                 const void* Wp, int64_t r, int64_t ldwp,
+                 const void* C, int64_t m, int64_t ldc,
+                 const int32_t* pivot_idx, const int32_t* nonpivot_idx,
+                 void* Y, int64_t ldy,
+                 void* workspace, int64_t workspace_bytes,
+                 void* cuda_stream);
+
+/* pifa_forward_variant -- pifa_forward with an explicit pifa_variant (tests and benchmarks). */
+int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx,
+                         const void* Wp, int64_t r, int64_t ldwp,
+                         const void* C, int64_t m, int64_t ldc,
+                         const int32_t* pivot_idx, const int32_t* nonpivot_idx,
+                         void* Y, int64_t ldy,
+                         void* workspace, int64_t workspace_bytes,
+                         int variant, void* cuda_stream);
+
+/* pifa_workspace_size -- bytes of device scratch pifa_forward needs for this shape and variant
+ * (PIFA_VARIANT_AUTO: the variant the selector picks). Returns a negative pifa_status on bad
+ * arguments. Pure host arithmetic; no GPU needed. */
+int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int variant);
+
+/* pifa_select_variant -- the selector (host, < 1 us): the pifa_variant pifa_forward runs for
+ * (T, m, n, r) on this build, never PIFA_VARIANT_AUTO; negative pifa_status on bad arguments.
+ * Decode for T <= 16; otherwise the fused prefill kernel when its cluster can hold Y_p for the
+ * rank r, else the split prefill. */
+int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r);
+
+/* pifa_variant_name -- static string naming a pifa_variant ("decode", ...); "?" if unknown. */
+const char* pifa_variant_name(int variant);
+
+/*
+ * pifa_compress -- Algorithm 1 (Sec. 3.2) on W' = U V^T, on the HOST in float64, synchronous.
+ * A reference setup step (it is not part of the GPU hot path).
+ *
+ *   U            HOST, float64, m x r row-major (contiguous).
+ *   V            HOST, float64, n x r row-major (contiguous); W' = U V^T.
+ *   pivot_idx    HOST out, int32[r]: I, ascending.
+ *   nonpivot_idx HOST out, int32[m - r]: I^c, ascending (may be NULL when r == m).
+ *   Wp           HOST out, float64, r x n, row pitch ldwp >= n: W'[I, :] (Eq. 1).
+ *   C            HOST out, float64, (m - r) x r, row pitch ldc >= r: W'[I^c, :] = C W_p (Eq. 2);
+ *                column j of C multiplies row j of Wp (ascending-I order). May be NULL if r == m.
+ *   info         HOST out, optional (NULL allowed).
+ *
+ *   Pivot rule: Businger-Golub QR with column pivoting on W'^T (greedy: the row of W' with the
+ *   largest norm orthogonal to the rows already chosen, norms recomputed exactly every step,
+ *   ties to the lowest index). Computed in the r-dimensional row space of U R_V^T, where
+ *   V = Q_V R_V, which has the same row inner products as W'. Requires 1 <= r <= min(m, n);
+ *   returns PIFA_ERR_RANK_DEFICIENT when |R_(r-1,r-1)| < 1e-8 |R_00|. Uses the host's cores
+ *   (OpenMP); scratch is allocated on the host and freed before returning.
+ */
+int pifa_compress(const double* U, const double* V, int64_t m, int64_t n, int64_t r,
+                  int32_t* pivot_idx, int32_t* nonpivot_idx,
+                  double* Wp, int64_t ldwp, double* C, int64_t ldc,
+                  pifa_compress_info* info);
+
+/* pifa_validate_indices -- HOST copies: PIFA_OK iff pivot_idx (r entries) and nonpivot_idx
+ * (m - r entries) are strictly ascending, inside [0, m) and disjoint (so together a partition
+ * of [0, m), as Algorithm 1 step 2 defines I^c); else PIFA_ERR_INVALID_ARG. */
+int pifa_validate_indices(const int32_t* pivot_idx, const int32_t* nonpivot_idx,
+                          int64_t m, int64_t r);
+
+/* pifa_device_status -- synchronizes `cuda_stream`, then returns and clears the error word the
+ * kernels latch on the current device (PIFA_OK, PIFA_ERR_TIMEOUT or PIFA_ERR_DEVICE_INDEX). */
+int pifa_device_status(void* cuda_stream);
+
+/* pifa_status_string -- static string for a pifa_status value. */
+const char* pifa_status_string(int status);
+
+/* pifa_last_error -- the calling thread's most recent detailed error message ("" if none). */
+const char* pifa_last_error(void);
+
+/* pifa_version -- static version string of this build. */
+const char* pifa_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PIFA_H_ */

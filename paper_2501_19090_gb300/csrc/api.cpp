@@ -1,0 +1,265 @@
+// api.cpp -- host side of the C ABI in include/pifa.h: argument checks, the variant selector,
+// workspace sizing, dispatch to the kernel launchers, TMA descriptor encoding, error strings.
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "pifa.h"
+#include "pifa_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Byte span [lo, hi) covered by a row-major matrix of `rows` rows, `cols` used columns, pitch ld.
+struct Span {
+  uintptr_t lo, hi;
+};
+Span span_of(const void* base, int64_t rows, int64_t cols, int64_t ld, int64_t elem) {
+  const uintptr_t b = reinterpret_cast<uintptr_t>(base);
+  if (!base || rows <= 0 || cols <= 0) return {0, 0};
+  return {b, b + (uintptr_t)(((rows - 1) * ld + cols) * elem)};
+}
+bool overlaps(Span a, Span b) { return a.lo < a.hi && b.lo < b.hi && a.lo < b.hi && b.lo < a.hi; }
+
+int validate_shape(int64_t T, int64_t m, int64_t n, int64_t r) {
+  if (T < 0) return pifa_fail(PIFA_ERR_INVALID_ARG, "T must be >= 0");
+  if (m < 1 || n < 1 || r < 1 || r > m || r > n)
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "need 1 <= r <= min(m, n)");
+  const int64_t lim = (int64_t)1 << 30;
+  if (T >= lim || m >= lim || n >= lim) return pifa_fail(PIFA_ERR_INVALID_ARG, "T, m or n too large (>= 2^30)");
+  return PIFA_OK;
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+}  // namespace
+
+// ---- internal helpers used by the kernel files --------------------------------------------------
+void pifa_clear_error() { g_last_error.clear(); }
+
+int pifa_fail(int status, const char* msg) {
+  g_last_error = msg ? msg : "";
+  return status;
+}
+
+int pifa_fail_cuda(const char* where, cudaError_t err) {
+  g_last_error = std::string(where) + ": " + cudaGetErrorName(err) + " (" + cudaGetErrorString(err) + ")";
+  return PIFA_ERR_CUDA;
+}
+
+uint64_t pifa_wait_timeout_ns() {
+  static uint64_t v = [] {
+    const char* e = std::getenv("PIFA_WAIT_TIMEOUT_NS");
+    if (e && *e) return (uint64_t)std::strtoull(e, nullptr, 10);
+    return (uint64_t)1000000000ull;  // 1 s
+  }();
+  return v;
+}
+
+int make_tmap_bf16_2d(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld, uint32_t box_cols,
+                      uint32_t box_rows) {
+  EncodeTiledFn fn = get_encode_fn();
+  if (!fn) return pifa_fail(PIFA_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    char buf[160];
+    std::snprintf(buf, sizeof buf, "cuTensorMapEncodeTiled failed (CUresult %d) for %lld x %lld, ld %lld",
+                  (int)r, (long long)rows, (long long)cols, (long long)ld);
+    return pifa_fail(PIFA_ERR_CUDA, buf);
+  }
+  return PIFA_OK;
+}
+
+// ---- public API ---------------------------------------------------------------------------------
+extern "C" {
+
+const char* pifa_version(void) { return "libpifa 0.1 (sm_103a)"; }
+
+const char* pifa_last_error(void) { return g_last_error.c_str(); }
+
+const char* pifa_status_string(int status) {
+  switch (status) {
+    case PIFA_OK: return "PIFA_OK";
+    case PIFA_ERR_INVALID_ARG: return "PIFA_ERR_INVALID_ARG";
+    case PIFA_ERR_ALIGNMENT: return "PIFA_ERR_ALIGNMENT";
+    case PIFA_ERR_UNSUPPORTED: return "PIFA_ERR_UNSUPPORTED";
+    case PIFA_ERR_CUDA: return "PIFA_ERR_CUDA";
+    case PIFA_ERR_TIMEOUT: return "PIFA_ERR_TIMEOUT";
+    case PIFA_ERR_RANK_DEFICIENT: return "PIFA_ERR_RANK_DEFICIENT";
+    case PIFA_ERR_WORKSPACE: return "PIFA_ERR_WORKSPACE";
+    case PIFA_ERR_DEVICE_INDEX: return "PIFA_ERR_DEVICE_INDEX";
+    default: return "PIFA_ERR_UNKNOWN";
+  }
+}
+
+const char* pifa_variant_name(int variant) {
+  switch (variant) {
+    case PIFA_VARIANT_AUTO: return "auto";
+    case PIFA_VARIANT_DECODE: return "decode";
+    case PIFA_VARIANT_PREFILL_SPLIT: return "prefill_split";
+    case PIFA_VARIANT_PREFILL_FUSED: return "prefill_fused";
+    default: return "?";
+  }
+}
+
+int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r) {
+  int st = validate_shape(T, m, n, r);
+  if (st != PIFA_OK) return st;
+  if (T <= 16) return PIFA_VARIANT_DECODE;
+  PifaShape s = {T, m, n, r, n, n, r, m};
+  if (prefill_fused_supported(s)) return PIFA_VARIANT_PREFILL_FUSED;
+  return PIFA_VARIANT_PREFILL_SPLIT;
+}
+
+int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int variant) {
+  int st = validate_shape(T, m, n, r);
+  if (st != PIFA_OK) return st;
+  if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r);
+  PifaShape s = {T, m, n, r, n, n, r, m};
+  if (T == 0) return 0;
+  switch (variant) {
+    case PIFA_VARIANT_DECODE: return decode_workspace_bytes(s);
+    case PIFA_VARIANT_PREFILL_SPLIT: return prefill_split_workspace_bytes(s);
+    case PIFA_VARIANT_PREFILL_FUSED: return prefill_fused_workspace_bytes(s);
+    default: return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
+  }
+}
+
+int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,
+                         const void* C, int64_t m, int64_t ldc, const int32_t* pivot_idx,
+                         const int32_t* nonpivot_idx, void* Y, int64_t ldy, void* workspace,
+                         int64_t workspace_bytes, int variant, void* cuda_stream) {
+  pifa_clear_error();
+  int st = validate_shape(T, m, n, r);
+  if (st != PIFA_OK) return st;
+  const bool has_np = m > r;
+  if (!X || !Wp || !pivot_idx || !Y) return pifa_fail(PIFA_ERR_INVALID_ARG, "null X, Wp, pivot_idx or Y");
+  if (has_np && (!C || !nonpivot_idx)) return pifa_fail(PIFA_ERR_INVALID_ARG, "null C or nonpivot_idx with m > r");
+  if (ldx < n || ldwp < n || ldy < m || (has_np && ldc < r))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "leading dimension smaller than the row length");
+  if (!aligned16(X) || !aligned16(Wp) || !aligned16(Y) || (has_np && !aligned16(C)))
+    return pifa_fail(PIFA_ERR_ALIGNMENT, "X, Wp, C and Y must be 16-byte aligned");
+  if ((ldx | ldwp | ldy | (has_np ? ldc : 0)) & 7)
+    return pifa_fail(PIFA_ERR_ALIGNMENT, "ldx, ldwp, ldc and ldy must be multiples of 8 elements");
+  if (variant < PIFA_VARIANT_AUTO || variant > PIFA_VARIANT_PREFILL_FUSED)
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
+  {
+    const Span y = span_of(Y, T, m, ldy, 2);
+    if (overlaps(y, span_of(X, T, n, ldx, 2)) || overlaps(y, span_of(Wp, r, n, ldwp, 2)) ||
+        (has_np && overlaps(y, span_of(C, m - r, r, ldc, 2))))
+      return pifa_fail(PIFA_ERR_INVALID_ARG, "Y overlaps an input");
+  }
+  if (T == 0) return PIFA_OK;
+  if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r);
+
+  PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy};
+  int64_t need = 0;
+  switch (variant) {
+    case PIFA_VARIANT_DECODE:
+      if (T > 16) return pifa_fail(PIFA_ERR_UNSUPPORTED, "decode variant needs T <= 16");
+      need = decode_workspace_bytes(s);
+      break;
+    case PIFA_VARIANT_PREFILL_SPLIT: need = prefill_split_workspace_bytes(s); break;
+    case PIFA_VARIANT_PREFILL_FUSED:
+      if (!prefill_fused_supported(s)) return pifa_fail(PIFA_ERR_UNSUPPORTED, "fused prefill cannot run this shape");
+      need = prefill_fused_workspace_bytes(s);
+      break;
+  }
+  if (need > 0) {
+    if (!workspace || workspace_bytes < need)
+      return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or smaller than pifa_workspace_size()");
+    if (reinterpret_cast<uintptr_t>(workspace) & 255u)
+      return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  }
+  cudaError_t cerr = cudaSuccess;
+  int* status = pifa_status_word(&cerr);
+  if (!status) return pifa_fail_cuda("device status word", cerr);
+
+  PifaPointers p = {X, Wp, has_np ? C : nullptr, pivot_idx, has_np ? nonpivot_idx : nullptr, Y, workspace,
+                    workspace_bytes};
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(cuda_stream);
+  switch (variant) {
+    case PIFA_VARIANT_DECODE: return launch_decode(s, p, status, stream);
+    case PIFA_VARIANT_PREFILL_SPLIT: return launch_prefill_split(s, p, status, pifa_wait_timeout_ns(), stream);
+    case PIFA_VARIANT_PREFILL_FUSED: return launch_prefill_fused(s, p, status, pifa_wait_timeout_ns(), stream);
+  }
+  return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
+}
+
+int pifa_forward(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,
+                 const void* C, int64_t m, int64_t ldc, const int32_t* pivot_idx, const int32_t* nonpivot_idx,
+                 void* Y, int64_t ldy, void* workspace, int64_t workspace_bytes, void* cuda_stream) {
+  return pifa_forward_variant(X, T, n, ldx, Wp, r, ldwp, C, m, ldc, pivot_idx, nonpivot_idx, Y, ldy, workspace,
+                              workspace_bytes, PIFA_VARIANT_AUTO, cuda_stream);
+}
+
+int pifa_validate_indices(const int32_t* pivot_idx, const int32_t* nonpivot_idx, int64_t m, int64_t r) {
+  pifa_clear_error();
+  if (m < 1 || r < 1 || r > m) return pifa_fail(PIFA_ERR_INVALID_ARG, "need 1 <= r <= m");
+  if (!pivot_idx || (m > r && !nonpivot_idx)) return pifa_fail(PIFA_ERR_INVALID_ARG, "null index array");
+  // strictly ascending and inside [0, m) each; disjoint by a merge walk (together they then
+  // cover r + (m - r) = m distinct values of [0, m), i.e. a partition)
+  for (int64_t a = 0; a < r; ++a) {
+    if (pivot_idx[a] < 0 || pivot_idx[a] >= m) return pifa_fail(PIFA_ERR_INVALID_ARG, "pivot index out of range");
+    if (a > 0 && pivot_idx[a] <= pivot_idx[a - 1]) return pifa_fail(PIFA_ERR_INVALID_ARG, "pivot_idx not ascending");
+  }
+  for (int64_t a = 0; a < m - r; ++a) {
+    if (nonpivot_idx[a] < 0 || nonpivot_idx[a] >= m)
+      return pifa_fail(PIFA_ERR_INVALID_ARG, "non-pivot index out of range");
+    if (a > 0 && nonpivot_idx[a] <= nonpivot_idx[a - 1])
+      return pifa_fail(PIFA_ERR_INVALID_ARG, "nonpivot_idx not ascending");
+  }
+  int64_t i = 0, j = 0;
+  while (i < r && j < m - r) {
+    if (pivot_idx[i] == nonpivot_idx[j]) return pifa_fail(PIFA_ERR_INVALID_ARG, "index in both sets");
+    if (pivot_idx[i] < nonpivot_idx[j]) ++i; else ++j;
+  }
+  return PIFA_OK;
+}
+
+int pifa_device_status(void* cuda_stream) {
+  pifa_clear_error();
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return pifa_fail_cuda("cudaStreamSynchronize", e);
+  int* word = pifa_status_word(&e);
+  if (!word) return pifa_fail_cuda("device status word", e);
+  int v = 0;
+  e = cudaMemcpy(&v, word, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return pifa_fail_cuda("read status word", e);
+  e = cudaMemset(word, 0, sizeof(int));
+  if (e != cudaSuccess) return pifa_fail_cuda("clear status word", e);
+  return v;
+}
+
+}  // extern "C"

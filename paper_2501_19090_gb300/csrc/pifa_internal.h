@@ -1,0 +1,59 @@
+// pifa_internal.h -- declarations shared by the host API (api.cpp) and the kernel files (*.cu).
+// Not installed; the public interface is include/pifa.h.
+#ifndef PIFA_INTERNAL_H_
+#define PIFA_INTERNAL_H_
+
+#include <stdint.h>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+// ---- error reporting (api.cpp) ---------------------------------------------------------------
+void pifa_clear_error();
+int pifa_fail(int status, const char* msg);                       // records msg, returns status
+int pifa_fail_cuda(const char* where, cudaError_t err);           // PIFA_ERR_CUDA with detail
+
+// Device status word of the current device (api.cpp). Kernels latch the first error into it
+// with atomicCAS(word, 0, code).
+int* pifa_status_word(cudaError_t* err);
+
+// Default bound of every device-side wait, nanoseconds (env PIFA_WAIT_TIMEOUT_NS overrides).
+uint64_t pifa_wait_timeout_ns();
+
+// Shape of one forward call after validation (element counts and pitches).
+struct PifaShape {
+  int64_t T, m, n, r;
+  int64_t ldx, ldwp, ldc, ldy;
+};
+
+struct PifaPointers {
+  const void* X;
+  const void* Wp;
+  const void* C;
+  const int32_t* piv;
+  const int32_t* nonpiv;
+  void* Y;
+  void* ws;
+  int64_t ws_bytes;
+};
+
+// ---- decode (decode.cu) ----------------------------------------------------------------------
+int64_t decode_workspace_bytes(const PifaShape& s);
+int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream);
+
+// ---- prefill (prefill.cu) --------------------------------------------------------------------
+int64_t prefill_split_workspace_bytes(const PifaShape& s);
+int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,
+                         cudaStream_t stream);
+int64_t prefill_fused_workspace_bytes(const PifaShape& s);
+bool prefill_fused_supported(const PifaShape& s);
+int launch_prefill_fused(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,
+                         cudaStream_t stream);
+
+// ---- TMA descriptors (api.cpp) ---------------------------------------------------------------
+// 2-D bf16 tensor map over a row-major (rows x cols) matrix with row pitch `ld` elements; box of
+// box_cols x box_rows elements, 128-byte swizzle, zero fill outside the matrix.
+int make_tmap_bf16_2d(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                      uint32_t box_cols, uint32_t box_rows);
+
+#endif  // PIFA_INTERNAL_H_

@@ -1,0 +1,261 @@
+// prefill.cu -- PIFA forward for many tokens on the 5th-generation tensor cores (tcgen05).
+//
+// Split variant: two launches of one warp-specialised tcgen05 GEMM.
+//   GEMM 1 (Algorithm 2, steps 2 and 4): D1 = W_p X^T, tile 128 weight rows x 256 tokens.
+//           Epilogue writes bf16(Y_p) into the pivot columns Y[:, I[j]] and the pair
+//           hi = bf16(Y_p), lo = bf16(Y_p - hi) into two T x r scratch matrices.
+//   GEMM 2 (Algorithm 2, steps 3 and 5): D2 = C [hi | lo]^T accumulated over K = r twice
+//           (hi pass then lo pass), epilogue writes bf16(Y_np) into Y[:, I^c[i]].
+// Weight rows are the MMA M dimension and tokens the N dimension, so the accumulator in tensor
+// memory holds one weight row per TMEM lane: an epilogue warp's 32 lanes are 32 consecutive
+// weight rows, which for a fixed token land in 32 ascending output columns of one row of Y.
+//
+// Per CTA (192 threads): warp 0 issues TMA loads into a 4-stage shared-memory ring (A tile
+// 128 x 64, B tile 256 x 64, bf16, 128-byte swizzle), warp 1 owns the TMEM allocation and issues
+// tcgen05.mma (M=128, N=256, K=16) from one thread, warps 2-5 drain the fp32 accumulator
+// (128 lanes x 256 columns of TMEM) through tcgen05.ld. Every wait is bounded (globaltimer); on
+// timeout the CTA latches PIFA_ERR_TIMEOUT, drains what it has in flight and returns.
+#include <cuda_bf16.h>
+
+#include "pifa.h"
+#include "pifa_internal.h"
+#include "ptx.cuh"
+
+namespace {
+
+using namespace pifa;
+using bf16 = __nv_bfloat16;
+
+constexpr int BM = 128;  // weight rows per tile (MMA M)
+constexpr int BN = 256;  // tokens per tile (MMA N)
+constexpr int BK = 64;   // K per stage: one 128-byte swizzle row of bf16
+constexpr int STAGES = 4;
+constexpr uint32_t A_BYTES = BM * BK * 2;
+constexpr uint32_t B_BYTES = BN * BK * 2;
+constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr uint32_t TMEM_COLS = BN;  // fp32 accumulator, one column per token
+constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
+constexpr size_t SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + 256 /*barriers*/;
+
+struct GemmArgs {
+  int M;                 // weight rows (r for GEMM 1, m - r for GEMM 2)
+  int N;                 // tokens T
+  int kchunks;           // ceil(K / 64) per pass
+  int passes;            // 1, or 2 for the hi + lo passes of GEMM 2
+  const int32_t* cols;   // output column of each weight row (I or I^c)
+  int m;                 // columns of Y (index bound)
+  bf16* Y;
+  int64_t ldy;
+  bf16* yp_hi;           // GEMM 1 only: T x ldyp scratch
+  bf16* yp_lo;
+  int64_t ldyp;
+  int* status;
+  uint64_t timeout_ns;
+};
+
+template <bool kWriteSplit>
+__global__ void __launch_bounds__(192, 1)
+    pifa_umma_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
+                   const __grid_constant__ CUtensorMap tmB1, GemmArgs p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* acc_full = empty + STAGES;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
+  const int total = p.kchunks * p.passes;
+
+  if (warp == 0 && lane == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(acc_full, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_tmap(&tmA);
+    prefetch_tmap(&tmB0);
+    if (p.passes > 1) prefetch_tmap(&tmB1);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      int issued = 0;
+      for (int i = 0; i < total; ++i) {
+        const int s = i % STAGES;
+        const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
+        if (i >= STAGES && !mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
+          *abort_flag = 1;
+          latch_status(p.status, PIFA_ERR_TIMEOUT);
+          break;
+        }
+        if (*abort_flag) break;
+        const int pass = i / p.kchunks, kc = i % p.kchunks;
+        uint8_t* sa = smem + s * STAGE_BYTES;
+        mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
+        tma_load_2d(smem_u32(sa), &tmA, kc * BK, m0, &full[s]);
+        tma_load_2d(smem_u32(sa + A_BYTES), pass ? &tmB1 : &tmB0, kc * BK, n0, &full[s]);
+        issued = i + 1;
+      }
+      // drain: the last use of every stage must have landed before the CTA may exit
+      const uint64_t drain_ns = 100000000ull;
+      for (int i = (issued > STAGES ? issued - STAGES : 0); i < issued; ++i) {
+        const int s = i % STAGES;
+        if (!mbar_wait(&full[s], (uint32_t)(i / STAGES) & 1u, drain_ns)) latch_status(p.status, PIFA_ERR_TIMEOUT);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      for (int i = 0; i < total; ++i) {
+        const int s = i % STAGES;
+        const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
+        if (!mbar_wait(&full[s], ph, p.timeout_ns)) {
+          *abort_flag = 1;
+          latch_status(p.status, PIFA_ERR_TIMEOUT);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a = smem_u32(smem + s * STAGE_BYTES);
+        const uint32_t b = a + A_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk)
+          mma_bf16_ss(tmem, sw128_desc(a + kk * 32), sw128_desc(b + kk * 32), IDESC, (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(&empty[s]);
+      }
+      mma_commit(acc_full);  // also drains every MMA issued above
+    }
+  } else {
+    // ---------------- epilogue: warps 2..5 ----------------
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int row = m0 + q * 32 + lane;
+    const bool ok = mbar_wait(acc_full, 0, p.timeout_ns);
+    if (!ok) latch_status(p.status, PIFA_ERR_TIMEOUT);
+    tc_fence_after();
+    if (ok && !*abort_flag) {
+      int col = -1;
+      if (row < p.M) {
+        col = p.cols[row];
+        if ((unsigned)col >= (unsigned)p.m) {
+          latch_status(p.status, PIFA_ERR_DEVICE_INDEX);
+          col = -1;
+        }
+      }
+#pragma unroll 1
+      for (int cc = 0; cc < BN / 32; ++cc) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(cc * 32), v);
+        tmem_ld_wait();
+        if (col >= 0) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const int t = n0 + cc * 32 + j;
+            if (t < p.N) {
+              const float f = __uint_as_float(v[j]);
+              const bf16 h = __float2bfloat16_rn(f);
+              p.Y[(int64_t)t * p.ldy + col] = h;
+              if (kWriteSplit) {
+                p.yp_hi[(int64_t)t * p.ldyp + row] = h;
+                p.yp_lo[(int64_t)t * p.ldyp + row] = __float2bfloat16_rn(f - __bfloat162float(h));
+              }
+            }
+          }
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+int run_gemm(bool write_split, const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
+             const GemmArgs& args, cudaStream_t stream) {
+  static bool attr_set[2] = {false, false};
+  auto kern = write_split ? pifa_umma_gemm<true> : pifa_umma_gemm<false>;
+  if (!attr_set[write_split]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+    if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(prefill gemm)", e);
+    attr_set[write_split] = true;
+  }
+  dim3 grid((args.M + BM - 1) / BM, (args.N + BN - 1) / BN);
+  kern<<<grid, 192, SMEM_BYTES, stream>>>(a, b0, b1, args);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return pifa_fail_cuda("prefill gemm launch", e);
+  return PIFA_OK;
+}
+
+inline int64_t pad8(int64_t v) { return (v + 7) / 8 * 8; }
+
+}  // namespace
+
+int64_t prefill_split_workspace_bytes(const PifaShape& s) {
+  const int64_t one = ((s.T * pad8(s.r) * 2 + 255) / 256) * 256;  // bf16 T x pad8(r)
+  return 2 * one;
+}
+
+int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,
+                         cudaStream_t stream) {
+  const int64_t ldyp = pad8(s.r);
+  const int64_t one = ((s.T * ldyp * 2 + 255) / 256) * 256;
+  bf16* hi = reinterpret_cast<bf16*>(p.ws);
+  bf16* lo = reinterpret_cast<bf16*>(reinterpret_cast<uint8_t*>(p.ws) + one);
+
+  CUtensorMap tWp, tX, tC, tHi, tLo;
+  int st;
+  if ((st = make_tmap_bf16_2d(&tWp, p.Wp, s.r, s.n, s.ldwp, BK, BM)) != PIFA_OK) return st;
+  if ((st = make_tmap_bf16_2d(&tX, p.X, s.T, s.n, s.ldx, BK, BN)) != PIFA_OK) return st;
+
+  GemmArgs g1 = {};
+  g1.M = (int)s.r;
+  g1.N = (int)s.T;
+  g1.kchunks = (int)((s.n + BK - 1) / BK);
+  g1.passes = 1;
+  g1.cols = p.piv;
+  g1.m = (int)s.m;
+  g1.Y = reinterpret_cast<bf16*>(p.Y);
+  g1.ldy = s.ldy;
+  g1.yp_hi = hi;
+  g1.yp_lo = lo;
+  g1.ldyp = ldyp;
+  g1.status = status;
+  g1.timeout_ns = timeout_ns;
+  if ((st = run_gemm(true, tWp, tX, tX, g1, stream)) != PIFA_OK) return st;
+  if (s.m == s.r) return PIFA_OK;
+
+  if ((st = make_tmap_bf16_2d(&tC, p.C, s.m - s.r, s.r, s.ldc, BK, BM)) != PIFA_OK) return st;
+  if ((st = make_tmap_bf16_2d(&tHi, hi, s.T, s.r, ldyp, BK, BN)) != PIFA_OK) return st;
+  if ((st = make_tmap_bf16_2d(&tLo, lo, s.T, s.r, ldyp, BK, BN)) != PIFA_OK) return st;
+  GemmArgs g2 = g1;
+  g2.M = (int)(s.m - s.r);
+  g2.kchunks = (int)((s.r + BK - 1) / BK);
+  g2.passes = 2;
+  g2.cols = p.nonpiv;
+  g2.yp_hi = nullptr;
+  g2.yp_lo = nullptr;
+  return run_gemm(false, tC, tHi, tLo, g2, stream);
+}
+
+// The fused variant is not built yet: the selector never picks it.
+int64_t prefill_fused_workspace_bytes(const PifaShape&) { return 0; }
+bool prefill_fused_supported(const PifaShape&) { return false; }
+int launch_prefill_fused(const PifaShape&, const PifaPointers&, int*, uint64_t, cudaStream_t) {
+  return pifa_fail(PIFA_ERR_UNSUPPORTED, "fused prefill variant is not available in this build");
+}

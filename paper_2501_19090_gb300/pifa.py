@@ -1,0 +1,230 @@
+"""Thin ctypes binding over libpifa.so (include/pifa.h). Argument marshalling only: every step of
+the forward pass runs in the library's CUDA kernels; the host compression runs in its C++ code.
+
+Functions keep the C names. Tensors are torch tensors (device memory and streams come from
+PyTorch); host arrays for pifa_compress are numpy. The library is loaded on first use and a
+missing or unloadable library raises -- there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libpifa.so")
+
+PIFA_OK = 0
+PIFA_ERR_INVALID_ARG = -1
+PIFA_ERR_ALIGNMENT = -2
+PIFA_ERR_UNSUPPORTED = -3
+PIFA_ERR_CUDA = -4
+PIFA_ERR_TIMEOUT = -5
+PIFA_ERR_RANK_DEFICIENT = -6
+PIFA_ERR_WORKSPACE = -7
+PIFA_ERR_DEVICE_INDEX = -8
+
+PIFA_VARIANT_AUTO = 0
+PIFA_VARIANT_DECODE = 1
+PIFA_VARIANT_PREFILL_SPLIT = 2
+PIFA_VARIANT_PREFILL_FUSED = 3
+
+# every symbol include/pifa.h declares
+EXPORTS = (
+    "pifa_forward", "pifa_forward_variant", "pifa_workspace_size", "pifa_select_variant",
+    "pifa_variant_name", "pifa_compress", "pifa_validate_indices", "pifa_device_status",
+    "pifa_status_string", "pifa_last_error", "pifa_version",
+)
+
+
+class PifaError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str = ""):
+        self.status = status
+        name = pifa_status_string(status) if _lib_handle is not None else str(status)
+        super().__init__(f"{where}: {name} ({status}) {detail}".rstrip())
+
+
+class PifaCompressInfo(ctypes.Structure):
+    _fields_ = [("min_pivot_gap", ctypes.c_double), ("r_ratio", ctypes.c_double),
+                ("max_abs_c", ctypes.c_double), ("threads", ctypes.c_int32)]
+
+
+_lib_handle = None
+_lock = threading.Lock()
+_I64 = ctypes.c_int64
+_VP = ctypes.c_void_p
+
+
+def load(path: str | None = None) -> ctypes.CDLL:
+    """Load libpifa.so (once) and declare its prototypes. Raises OSError if it cannot load."""
+    global _lib_handle
+    with _lock:
+        if _lib_handle is not None:
+            return _lib_handle
+        p = path or LIB_PATH
+        if not os.path.exists(p):
+            raise OSError(f"{p} not found: build it with `python -m paper_2501_19090_gb300.build`")
+        lib = ctypes.CDLL(p)
+        fwd = [_VP, _I64, _I64, _I64, _VP, _I64, _I64, _VP, _I64, _I64, _VP, _VP, _VP, _I64, _VP, _I64]
+        lib.pifa_forward.argtypes = fwd + [_VP]
+        lib.pifa_forward.restype = ctypes.c_int
+        lib.pifa_forward_variant.argtypes = fwd + [ctypes.c_int, _VP]
+        lib.pifa_forward_variant.restype = ctypes.c_int
+        lib.pifa_workspace_size.argtypes = [_I64, _I64, _I64, _I64, ctypes.c_int]
+        lib.pifa_workspace_size.restype = _I64
+        lib.pifa_select_variant.argtypes = [_I64, _I64, _I64, _I64]
+        lib.pifa_select_variant.restype = ctypes.c_int
+        lib.pifa_variant_name.argtypes = [ctypes.c_int]
+        lib.pifa_variant_name.restype = ctypes.c_char_p
+        lib.pifa_compress.argtypes = [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _I64, _VP, _I64,
+                                      ctypes.POINTER(PifaCompressInfo)]
+        lib.pifa_compress.restype = ctypes.c_int
+        lib.pifa_validate_indices.argtypes = [_VP, _VP, _I64, _I64]
+        lib.pifa_validate_indices.restype = ctypes.c_int
+        lib.pifa_device_status.argtypes = [_VP]
+        lib.pifa_device_status.restype = ctypes.c_int
+        lib.pifa_status_string.argtypes = [ctypes.c_int]
+        lib.pifa_status_string.restype = ctypes.c_char_p
+        lib.pifa_last_error.argtypes = []
+        lib.pifa_last_error.restype = ctypes.c_char_p
+        lib.pifa_version.argtypes = []
+        lib.pifa_version.restype = ctypes.c_char_p
+        _lib_handle = lib
+        return lib
+
+
+def _lib() -> ctypes.CDLL:
+    return _lib_handle if _lib_handle is not None else load()
+
+
+def _check(status: int, where: str) -> int:
+    if status != PIFA_OK:
+        raise PifaError(status, where, _lib().pifa_last_error().decode())
+    return status
+
+
+# ---- plain wrappers ------------------------------------------------------------------------------
+def pifa_version() -> str:
+    return _lib().pifa_version().decode()
+
+
+def pifa_status_string(status: int) -> str:
+    return _lib().pifa_status_string(int(status)).decode()
+
+
+def pifa_last_error() -> str:
+    return _lib().pifa_last_error().decode()
+
+
+def pifa_variant_name(variant: int) -> str:
+    return _lib().pifa_variant_name(int(variant)).decode()
+
+
+def pifa_select_variant(T: int, m: int, n: int, r: int) -> int:
+    v = _lib().pifa_select_variant(T, m, n, r)
+    if v < 0:
+        _check(v, "pifa_select_variant")
+    return v
+
+
+def pifa_workspace_size(T: int, m: int, n: int, r: int, variant: int = PIFA_VARIANT_AUTO) -> int:
+    v = _lib().pifa_workspace_size(T, m, n, r, variant)
+    if v < 0:
+        _check(int(v), "pifa_workspace_size")
+    return int(v)
+
+
+def pifa_validate_indices(pivot_idx: np.ndarray, nonpivot_idx: np.ndarray, m: int, r: int) -> int:
+    """Host check of the index sets; returns the pifa_status (does not raise)."""
+    p = np.ascontiguousarray(pivot_idx, dtype=np.int32)
+    q = np.ascontiguousarray(nonpivot_idx, dtype=np.int32)
+    return _lib().pifa_validate_indices(p.ctypes.data, q.ctypes.data if q.size else None, m, r)
+
+
+def pifa_device_status(stream=None) -> int:
+    """Synchronize the stream, then read and clear the device error word (a pifa_status)."""
+    return _lib().pifa_device_status(_stream_ptr(stream))
+
+
+def pifa_compress(U: np.ndarray, V: np.ndarray, r: int):
+    """Algorithm 1 on the host in float64 (library C++ route). Returns (I, I^c, W_p, C, info)."""
+    U = np.ascontiguousarray(U, dtype=np.float64)
+    V = np.ascontiguousarray(V, dtype=np.float64)
+    m, n = U.shape[0], V.shape[0]
+    if U.shape[1] != r or V.shape[1] != r:
+        raise ValueError("U must be m x r and V n x r")
+    piv = np.empty(r, dtype=np.int32)
+    nonpiv = np.empty(m - r, dtype=np.int32)
+    Wp = np.empty((r, n), dtype=np.float64)
+    C = np.empty((m - r, r), dtype=np.float64)
+    info = PifaCompressInfo()
+    st = _lib().pifa_compress(U.ctypes.data, V.ctypes.data, m, n, r, piv.ctypes.data,
+                              nonpiv.ctypes.data if m > r else None, Wp.ctypes.data, n,
+                              C.ctypes.data if m > r else None, r, ctypes.byref(info))
+    _check(st, "pifa_compress")
+    return piv, nonpiv, Wp, C, info
+
+
+# ---- forward -------------------------------------------------------------------------------------
+def _stream_ptr(stream):
+    if stream is None:
+        import torch
+        if not torch.cuda.is_available():
+            return None
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, int):
+        return ctypes.c_void_p(stream)
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+_workspaces: dict = {}
+
+
+def workspace(nbytes: int, device, stream=None):
+    """A cached device scratch tensor of at least nbytes on `device` (grown, never shrunk).
+
+    The cache is keyed by device and stream, so calls on different streams never share scratch.
+    """
+    import torch
+    key = (str(device), 0 if stream is None else getattr(stream, "cuda_stream", stream))
+    buf = _workspaces.get(key)
+    if buf is None or buf.numel() < nbytes:
+        buf = torch.empty(max(nbytes, 256) + 256, dtype=torch.uint8, device=device)
+        _workspaces[key] = buf
+    return buf
+
+
+def _ld(t) -> int:
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("expected a row-major 2-D tensor with unit column stride")
+    return t.stride(0)
+
+
+def pifa_forward(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, variant: int = PIFA_VARIANT_AUTO,
+                 workspace_tensor=None, stream=None):
+    """Y = PIFA(X) through pifa_forward_variant. X (T x n), Wp (r x n), C ((m-r) x r) bf16 CUDA
+    tensors; pivot_idx / nonpivot_idx int32 CUDA tensors. Allocates Y (T x m) if not given."""
+    import torch
+    T, n = X.shape
+    r = Wp.shape[0]
+    m = r + (nonpivot_idx.numel() if nonpivot_idx is not None else 0)
+    if Y is None:
+        Y = torch.empty((T, m), dtype=torch.bfloat16, device=X.device)
+    has_np = m > r
+    need = pifa_workspace_size(T, m, n, r, variant)
+    ws = workspace_tensor
+    if need > 0 and ws is None:
+        ws = workspace(need, X.device, stream)
+    ws_ptr = 0 if ws is None else ws.data_ptr()
+    if ws is not None and ws_ptr % 256:
+        ws_ptr += 256 - ws_ptr % 256
+    ws_bytes = 0 if ws is None else ws.numel() * ws.element_size() - (ws_ptr - ws.data_ptr())
+    st = _lib().pifa_forward_variant(
+        X.data_ptr(), T, n, _ld(X), Wp.data_ptr(), r, _ld(Wp),
+        C.data_ptr() if has_np else None, m, _ld(C) if has_np else r,
+        pivot_idx.data_ptr(), nonpivot_idx.data_ptr() if has_np else None,
+        Y.data_ptr(), _ld(Y), ws_ptr or None, ws_bytes, variant, _stream_ptr(stream))
+    _check(st, "pifa_forward")
+    return Y

@@ -1,0 +1,275 @@
+"""GPU parity: pifa_forward (through the C ABI) against the fp64 oracle on the same bf16 operands.
+
+Tolerance (bf16 operands, fp32 accumulation, bf16 output): relative Frobenius error <= 5e-3 and
+|err| <= 2e-2 * (|ref| + 1) per element. Large outputs are checked on a seeded sample of token
+rows (rows of Y are independent in Algorithm 2). Every call runs with guard bands around Y
+(sentinel rows before and after, sentinel padding columns when ldy > m) and Y pre-filled with
+NaN, so a missed or stray write fails the test.
+
+Layers: the oracle's own compression where it is quick (tiny: plain greedy loop; up to
+4096 x 4096: the LAPACK pivoted-QR route); the library's host compression for the 7B MLP and
+70B q/o shapes, each of which is checked against Eq. 2 by the oracle on sampled rows; and a
+randomly drawn layer (inputs.synthetic_layer) for the 28672 x 8192 shape, whose compression
+would take minutes on the host.
+"""
+import functools
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2501_19090_gb300 import inputs
+from paper_2501_19090_gb300 import pifa as P
+
+pytestmark = pytest.mark.gpu
+
+REL_FRO = 5e-3
+ELEM = 2e-2
+SENTINEL = -12345.0   # exactly representable in bf16
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    P.load()
+    yield
+
+
+DEV = torch.device("cuda:0")
+
+
+class Layer:
+    def __init__(self, pivots, nonpivots, Wp, C, name):
+        self.pivots = np.asarray(pivots, np.int64)
+        self.nonpivots = np.asarray(nonpivots, np.int64)
+        self.Wp = inputs.round_bf16(Wp)          # the exact operand values both sides use
+        self.C = inputs.round_bf16(C)
+        self.m = self.pivots.size + self.nonpivots.size
+        self.r, self.n = self.Wp.shape
+        self.name = name
+        self._dev = None
+
+    def dev(self, ldwp=None, ldc=None):
+        """Device copies (bf16 / int32); optional padded pitches with NaN in the padding."""
+        Wp = _pad_dev(self.Wp, ldwp)
+        C = _pad_dev(self.C, ldc) if self.C.size else torch.empty((0, self.r), dtype=torch.bfloat16, device=DEV)
+        piv = torch.from_numpy(self.pivots.astype(np.int32)).to(DEV)
+        nonp = torch.from_numpy(self.nonpivots.astype(np.int32)).to(DEV)
+        return Wp, C, piv, nonp
+
+
+def _pad_dev(a32, ld=None):
+    rows, cols = a32.shape
+    ld = ld or cols
+    buf = torch.full((rows, ld), float("nan"), dtype=torch.bfloat16, device=DEV)
+    buf[:, :cols] = torch.from_numpy(np.ascontiguousarray(a32)).to(DEV).to(torch.bfloat16)
+    return buf[:, :cols]
+
+
+@functools.lru_cache(maxsize=None)
+def layer_for(m, n, r, seed, source):
+    U, V, _ = inputs.make_factors(m, n, r, seed)
+    if source == "oracle_greedy":
+        L = oracle.compress(U, V, r, "greedy")
+        return Layer(L.pivots, L.nonpivots, L.Wp, L.C, f"{m}x{n}r{r}/oracle")
+    if source == "oracle_lapack":
+        L = oracle.compress(U, V, r, "lapack")
+        return Layer(L.pivots, L.nonpivots, L.Wp, L.C, f"{m}x{n}r{r}/oracle-lapack")
+    if source == "library":
+        piv, nonp, Wp, C, _ = P.pifa_compress(U, V, r)
+        # the oracle checks Eq. 1 and Eq. 2 on a sample of rows of W' = U V^T
+        rows = inputs.random_rows(m - r, 64, seed) if m > r else np.zeros(0, np.int64)
+        Vd = V.astype(np.float64)
+        Wnp_s = U[nonp[rows]].astype(np.float64) @ Vd.T
+        Wp_ref = U[piv].astype(np.float64) @ Vd.T
+        assert np.abs(Wp - Wp_ref).max() <= 1e-12 * np.abs(Wp_ref).max()
+        if rows.size:
+            err = np.linalg.norm(C[rows] @ Wp - Wnp_s) / np.linalg.norm(Wnp_s)
+            assert err <= 1e-10
+        assert P.pifa_validate_indices(piv, nonp, m, r) == P.PIFA_OK
+        return Layer(piv, nonp, Wp, C, f"{m}x{n}r{r}/library")
+    if source == "synthetic":
+        piv, nonp, Wp, C = inputs.synthetic_layer(m, n, r, seed)
+        return Layer(piv, nonp, Wp, C, f"{m}x{n}r{r}/synthetic")
+    raise ValueError(source)
+
+
+def acts(T, n, seed):
+    rng = np.random.default_rng(1000 + seed)
+    return inputs.make_activations(rng, T, n, "bf16")
+
+
+def run(layer, X32, variant=P.PIFA_VARIANT_AUTO, ldx=None, ldy_pad=8, guard_rows=3, ldwp=None, ldc=None,
+        stream=None):
+    """pifa_forward with NaN-filled Y inside sentinel guard bands; returns Y (T x m) as float32."""
+    T = X32.shape[0]
+    m = layer.m
+    Wp, C, piv, nonp = layer.dev(ldwp, ldc)
+    X = _pad_dev(X32, ldx) if T else torch.empty((0, layer.n), dtype=torch.bfloat16, device=DEV)
+    ldy = m + ldy_pad
+    big = torch.full((T + 2 * guard_rows, ldy), SENTINEL, dtype=torch.bfloat16, device=DEV)
+    Y = big[guard_rows:guard_rows + T, :m]
+    Y.fill_(float("nan"))
+    P.pifa_forward(X, Wp, C, piv, nonp, Y=Y, variant=variant, stream=stream)
+    st = P.pifa_device_status(stream)
+    assert st == P.PIFA_OK, P.pifa_status_string(st)
+    host = big.float().cpu().numpy()
+    assert np.all(host[:guard_rows] == SENTINEL) and np.all(host[guard_rows + T:] == SENTINEL), "guard rows hit"
+    assert np.all(host[:, m:] == SENTINEL), "padding columns of Y were written"
+    out = host[guard_rows:guard_rows + T, :m]
+    assert not np.isnan(out).any(), "some output element was never written"
+    return out
+
+
+def check(got, ref, what=""):
+    got = got.astype(np.float64)
+    denom = np.linalg.norm(ref)
+    rel = np.linalg.norm(got - ref) / denom if denom > 0 else np.linalg.norm(got)
+    elem = np.max(np.abs(got - ref) / (np.abs(ref) + 1.0)) if ref.size else 0.0
+    assert rel <= REL_FRO and elem <= ELEM, f"{what}: rel_fro {rel:.3e} (<= {REL_FRO}), elem {elem:.3e} (<= {ELEM})"
+    return rel, elem
+
+
+def parity(layer, T, variant=P.PIFA_VARIANT_AUTO, sample=None, seed=0, **kw):
+    X = acts(T, layer.n, seed)
+    Y = run(layer, X, variant, **kw)
+    rows = np.arange(T) if (sample is None or sample >= T) else inputs.random_rows(T, sample, seed)
+    ref = oracle.forward(X[rows], layer.Wp, layer.C, layer.pivots, layer.nonpivots)
+    return check(Y[rows], ref, f"{layer.name} T={T} variant={P.pifa_variant_name(variant)}")
+
+
+# ---------------------------------------------------------------------------------------------
+# the five workloads
+# ---------------------------------------------------------------------------------------------
+def test_tiny_layer_decode_and_prefill():
+    L = layer_for(256, 256, 128, 0, "oracle_greedy")
+    parity(L, 16, P.PIFA_VARIANT_DECODE)
+    parity(L, 16, P.PIFA_VARIANT_PREFILL_SPLIT)
+    parity(L, 16)
+
+
+@pytest.mark.parametrize("T", [1, 8])
+def test_attn7b_decode(T):
+    L = layer_for(4096, 4096, 2048, 0, "oracle_lapack")
+    assert P.pifa_select_variant(T, 4096, 4096, 2048) == P.PIFA_VARIANT_DECODE
+    parity(L, T)
+
+
+@pytest.mark.parametrize("T,sample", [(2048, None), (8192, 512)])
+def test_attn7b_prefill(T, sample):
+    L = layer_for(4096, 4096, 2048, 0, "oracle_lapack")
+    parity(L, T, sample=sample)
+
+
+@pytest.mark.parametrize("frac", [0.25, 0.4, 0.6, 0.75])
+def test_rank_sweep_prefill(frac):
+    r = int(np.floor(frac * 4096 + 0.5))
+    L = layer_for(4096, 4096, r, 0, "oracle_lapack")
+    parity(L, 2048, sample=768)
+
+
+@pytest.mark.parametrize("T", [1, 2048])
+def test_mlp7b_three_layers_back_to_back(T):
+    gate = layer_for(11008, 4096, 2048, 0, "library")
+    up = layer_for(11008, 4096, 2048, 1, "library")
+    down = layer_for(4096, 11008, 2048, 2, "library")
+    Xg = acts(T, 4096, 0)
+    Xd = acts(T, 11008, 2)      # the down projection gets its own N(0,1) input (no SwiGLU here)
+    stream = torch.cuda.Stream()
+    outs = [run(gate, Xg, stream=stream), run(up, Xg, stream=stream), run(down, Xd, stream=stream)]
+    rows = np.arange(T) if T <= 512 else inputs.random_rows(T, 384, 0)
+    for L, X, Y in zip((gate, up, down), (Xg, Xg, Xd), outs):
+        ref = oracle.forward(X[rows], L.Wp, L.C, L.pivots, L.nonpivots)
+        check(Y[rows], ref, f"{L.name} T={T}")
+
+
+@pytest.mark.parametrize("T", [1, 16, 4096])
+def test_llama70b_qo(T):
+    L = layer_for(8192, 8192, 4096, 0, "library")
+    parity(L, T, sample=256)
+
+
+@pytest.mark.parametrize("T", [1, 16, 4096])
+def test_llama70b_gate_up(T):
+    L = layer_for(28672, 8192, 4096, 0, "synthetic")
+    parity(L, T, sample=128)
+
+
+# ---------------------------------------------------------------------------------------------
+# edge cases
+# ---------------------------------------------------------------------------------------------
+@pytest.mark.parametrize("T", [1, 3, 13, 16, 17, 100, 300])
+def test_ragged_shapes_all_variants(T):
+    L = layer_for(300, 200, 77, 3, "oracle_greedy")
+    variants = [P.PIFA_VARIANT_PREFILL_SPLIT] + ([P.PIFA_VARIANT_DECODE] if T <= 16 else [])
+    for v in variants:
+        parity(L, T, v)
+
+
+@pytest.mark.parametrize("variant", [P.PIFA_VARIANT_DECODE, P.PIFA_VARIANT_PREFILL_SPLIT])
+def test_full_rank_r_equals_m(variant):
+    L = layer_for(64, 128, 64, 4, "oracle_greedy")
+    assert L.C.shape == (0, 64)
+    parity(L, 9, variant)
+
+
+@pytest.mark.parametrize("variant", [P.PIFA_VARIANT_DECODE, P.PIFA_VARIANT_PREFILL_SPLIT])
+def test_rank_one(variant):
+    L = layer_for(40, 48, 1, 5, "oracle_greedy")
+    parity(L, 12, variant)
+
+
+@pytest.mark.parametrize("variant", [P.PIFA_VARIANT_DECODE, P.PIFA_VARIANT_PREFILL_SPLIT])
+def test_padded_pitches_ignore_padding(variant):
+    """ldx > n, ldwp > n, ldc > r and ldy > m with NaN in the input padding: never read."""
+    L = layer_for(256, 256, 128, 0, "oracle_greedy")
+    parity(L, 11, variant, ldx=264, ldwp=272, ldc=136, ldy_pad=24)
+
+
+def test_zero_tokens_is_a_noop():
+    L = layer_for(256, 256, 128, 0, "oracle_greedy")
+    Wp, C, piv, nonp = L.dev()
+    X = torch.empty((0, 256), dtype=torch.bfloat16, device=DEV)
+    Y = torch.empty((0, 256), dtype=torch.bfloat16, device=DEV)
+    P.pifa_forward(X, Wp, C, piv, nonp, Y=Y)
+    assert P.pifa_device_status() == P.PIFA_OK
+
+
+def test_deterministic_bitwise():
+    L = layer_for(4096, 4096, 2048, 0, "oracle_lapack")
+    X = acts(300, 4096, 7)
+    for v in (P.PIFA_VARIANT_PREFILL_SPLIT,):
+        a = run(L, X, v)
+        b = run(L, X, v)
+        assert np.array_equal(a, b)
+    Xs = acts(8, 4096, 7)
+    assert np.array_equal(run(L, Xs, P.PIFA_VARIANT_DECODE), run(L, Xs, P.PIFA_VARIANT_DECODE))
+
+
+@pytest.mark.parametrize("variant", [P.PIFA_VARIANT_DECODE, P.PIFA_VARIANT_PREFILL_SPLIT])
+def test_out_of_range_index_is_reported_not_written(variant):
+    """A pivot index >= m is caught by the kernels' own bounds check: the write is skipped and
+    PIFA_ERR_DEVICE_INDEX is latched; nothing outside Y changes."""
+    L = layer_for(256, 256, 128, 0, "oracle_greedy")
+    Wp, C, piv, nonp = L.dev()
+    bad = piv.clone()
+    bad[5] = 256                              # == m: out of range
+    X = _pad_dev(acts(4, 256, 0))
+    big = torch.full((4 + 6, 256 + 8), SENTINEL, dtype=torch.bfloat16, device=DEV)
+    Y = big[3:7, :256]
+    P.pifa_forward(X, Wp, C, bad, nonp, Y=Y, variant=variant)
+    assert P.pifa_device_status() == P.PIFA_ERR_DEVICE_INDEX
+    assert P.pifa_device_status() == P.PIFA_OK           # cleared by the read
+    host = big.float().cpu().numpy()
+    assert np.all(host[:3] == SENTINEL) and np.all(host[7:] == SENTINEL) and np.all(host[:, 256:] == SENTINEL)
+
+
+def test_prefill_variants_agree_with_decode_at_t16():
+    L = layer_for(4096, 4096, 2048, 0, "oracle_lapack")
+    X = acts(16, 4096, 3)
+    a = run(L, X, P.PIFA_VARIANT_DECODE)
+    b = run(L, X, P.PIFA_VARIANT_PREFILL_SPLIT)
+    ref = oracle.forward(X, L.Wp, L.C, L.pivots, L.nonpivots)
+    check(a, ref, "decode")
+    check(b, ref, "prefill_split")

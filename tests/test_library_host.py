@@ -1,0 +1,172 @@
+"""Host-only checks of libpifa.so (no GPU): the library loads and exports every symbol that
+include/pifa.h declares, the host compression (Algorithm 1) agrees with the oracle, and
+argument errors are reported as status codes before anything touches a device."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2501_19090_gb300 import inputs
+from paper_2501_19090_gb300 import pifa as P
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "pifa.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(P.LIB_PATH):
+        from paper_2501_19090_gb300 import build
+        build.build()
+    return P.load()
+
+
+def header_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:const\s+)?(?:int|int64_t|char|void)\s*\**\s*(pifa_\w+)\s*\(",
+                                 src, flags=re.M)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = header_functions()
+    assert len(names) >= 10
+    assert set(names) == set(P.EXPORTS)
+    for name in names:
+        assert hasattr(lib, name), name
+        assert ctypes.cast(getattr(lib, name), ctypes.c_void_p).value
+
+
+def test_status_and_variant_strings(lib):
+    assert P.pifa_status_string(P.PIFA_OK) == "PIFA_OK"
+    assert P.pifa_status_string(P.PIFA_ERR_TIMEOUT) == "PIFA_ERR_TIMEOUT"
+    assert P.pifa_variant_name(P.PIFA_VARIANT_DECODE) == "decode"
+    assert "sm_103a" in P.pifa_version()
+
+
+def test_selector(lib):
+    assert P.pifa_select_variant(1, 4096, 4096, 2048) == P.PIFA_VARIANT_DECODE
+    assert P.pifa_select_variant(16, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE
+    v = P.pifa_select_variant(2048, 4096, 4096, 2048)
+    assert v in (P.PIFA_VARIANT_PREFILL_SPLIT, P.PIFA_VARIANT_PREFILL_FUSED)
+    assert P.pifa_select_variant(17, 256, 256, 128) != P.PIFA_VARIANT_DECODE
+    with pytest.raises(P.PifaError):
+        P.pifa_select_variant(1, 100, 50, 60)      # r > n
+
+
+def test_workspace_sizes(lib):
+    # decode: fp32 y_p, T rows of pitch round_up(r, 8)
+    assert P.pifa_workspace_size(8, 4096, 4096, 2048, P.PIFA_VARIANT_DECODE) == 8 * 2048 * 4
+    assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) % 256 == 0
+    assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) >= 3 * 1640 * 4
+    # split prefill: two bf16 T x round_up(r, 8) matrices
+    assert P.pifa_workspace_size(2048, 4096, 4096, 2048, P.PIFA_VARIANT_PREFILL_SPLIT) == 2 * 2048 * 2048 * 2
+    assert P.pifa_workspace_size(0, 4096, 4096, 2048, P.PIFA_VARIANT_AUTO) == 0
+    with pytest.raises(P.PifaError) as e:
+        P.pifa_workspace_size(4, 10, 10, 11, P.PIFA_VARIANT_AUTO)   # r > min(m, n)
+    assert e.value.status == P.PIFA_ERR_INVALID_ARG
+
+
+def test_validate_indices(lib):
+    piv = np.array([1, 3], np.int32)
+    nonp = np.array([0, 2, 4], np.int32)
+    assert P.pifa_validate_indices(piv, nonp, 5, 2) == P.PIFA_OK
+    assert P.pifa_validate_indices(np.array([3, 1], np.int32), nonp, 5, 2) == P.PIFA_ERR_INVALID_ARG
+    assert P.pifa_validate_indices(np.array([1, 2], np.int32), nonp, 5, 2) == P.PIFA_ERR_INVALID_ARG
+    assert P.pifa_validate_indices(np.array([1, 5], np.int32), np.array([0, 2, 3], np.int32), 5, 2) \
+        == P.PIFA_ERR_INVALID_ARG
+    assert P.pifa_validate_indices(np.arange(4, dtype=np.int32), np.zeros(0, np.int32), 4, 4) == P.PIFA_OK
+
+
+def _fwd_raw(lib, **kw):
+    """pifa_forward_variant with fake (never dereferenced) pointers, for argument checks only."""
+    a = dict(X=0x10000, T=4, n=64, ldx=64, Wp=0x20000, r=16, ldwp=64, C=0x30000, m=48, ldc=16,
+             piv=0x40000, nonpiv=0x50000, Y=0x60000, ldy=48, ws=0x70000, wsb=1 << 20,
+             variant=P.PIFA_VARIANT_AUTO)
+    a.update(kw)
+    return lib.pifa_forward_variant(a["X"], a["T"], a["n"], a["ldx"], a["Wp"], a["r"], a["ldwp"], a["C"],
+                                    a["m"], a["ldc"], a["piv"], a["nonpiv"], a["Y"], a["ldy"], a["ws"],
+                                    a["wsb"], a["variant"], None)
+
+
+def test_forward_argument_errors(lib):
+    E = P
+    assert _fwd_raw(lib, r=0) == E.PIFA_ERR_INVALID_ARG
+    assert _fwd_raw(lib, r=65) == E.PIFA_ERR_INVALID_ARG            # r > n
+    assert _fwd_raw(lib, T=-1) == E.PIFA_ERR_INVALID_ARG
+    assert _fwd_raw(lib, X=None) == E.PIFA_ERR_INVALID_ARG
+    assert _fwd_raw(lib, C=None) == E.PIFA_ERR_INVALID_ARG
+    assert _fwd_raw(lib, ldx=32) == E.PIFA_ERR_INVALID_ARG
+    assert _fwd_raw(lib, ldy=40) == E.PIFA_ERR_INVALID_ARG
+    assert _fwd_raw(lib, X=0x10002) == E.PIFA_ERR_ALIGNMENT
+    assert _fwd_raw(lib, ldwp=68) == E.PIFA_ERR_ALIGNMENT
+    assert _fwd_raw(lib, Y=0x10000 + 64) == E.PIFA_ERR_INVALID_ARG   # Y overlaps X
+    assert "overlap" in _last(lib)
+    assert _fwd_raw(lib, variant=9) == E.PIFA_ERR_INVALID_ARG
+    assert _fwd_raw(lib, variant=P.PIFA_VARIANT_DECODE, T=17) == E.PIFA_ERR_UNSUPPORTED
+    assert _fwd_raw(lib, wsb=16) == E.PIFA_ERR_WORKSPACE
+    assert _fwd_raw(lib, ws=None) == E.PIFA_ERR_WORKSPACE
+    assert _fwd_raw(lib, ws=0x70010) == E.PIFA_ERR_ALIGNMENT
+    assert _fwd_raw(lib, T=0) == E.PIFA_OK                           # no-op, no device touched
+
+
+def _last(lib):
+    return lib.pifa_last_error().decode()
+
+
+def test_compress_argument_errors(lib):
+    U = np.zeros((4, 2))
+    V = np.zeros((3, 2))
+    with pytest.raises(P.PifaError) as e:
+        P.pifa_compress(U, V, 2)                                      # W' = 0: rank 0 < 2
+    assert e.value.status == P.PIFA_ERR_RANK_DEFICIENT
+    st = lib.pifa_compress(None, None, 4, 3, 2, None, None, None, 3, None, 2, None)
+    assert st == P.PIFA_ERR_INVALID_ARG
+
+
+def _compare_with_oracle(m, n, r, seed, rule="greedy"):
+    U, V, _ = inputs.make_factors(m, n, r, seed)
+    ref = oracle.compress(U, V, r, rule)
+    piv, nonp, Wp, C, info = P.pifa_compress(U, V, r)
+    assert np.array_equal(piv, ref.pivots), "pivot indices differ from the oracle"
+    assert np.array_equal(nonp, ref.nonpivots)
+    W = oracle.form_weight(U, V)
+    scale = np.abs(W).max()
+    assert np.abs(Wp - ref.Wp).max() <= 1e-12 * scale
+    if m > r:
+        assert np.abs(C - ref.C).max() <= 1e-10 * max(1.0, np.abs(ref.C).max())
+        # Eq. 2 holds for the library's own C, judged by the oracle's definition
+        lay = oracle.PifaLayer(piv.astype(np.int64), nonp.astype(np.int64), Wp, C, ref.info)
+        assert oracle.lossless_error(W, lay) <= 1e-10
+    return info, ref
+
+
+@pytest.mark.parametrize("m,n,r,seed", [(256, 256, 128, 0), (300, 200, 100, 1), (96, 160, 96, 2),
+                                        (64, 64, 64, 3), (129, 77, 33, 4), (40, 40, 1, 5)])
+def test_compress_matches_oracle(lib, m, n, r, seed):
+    info, ref = _compare_with_oracle(m, n, r, seed)
+    assert info.threads >= 1
+    if ref.info.gaps.size:
+        assert abs(info.min_pivot_gap - ref.info.gaps.min()) <= 1e-6
+
+
+def test_compress_golden_example(lib):
+    """The hand-derived example of tests/golden (rank 2, W' given directly as U V^T with V = I_3[:, :2]
+    mapping): pivots {1, 3} and the rational C rows."""
+    W = np.array([[1, 0, 0], [0, 2, 0], [1, 2, 0], [2, 2, 0], [0, 0, 0]], dtype=np.float64)
+    U = W[:, :2].copy()                     # W' = U V^T with V = [[1,0],[0,1],[0,0]]
+    V = np.array([[1.0, 0.0], [0.0, 1.0], [0.0, 0.0]])
+    piv, nonp, Wp, C, _ = P.pifa_compress(U, V, 2)
+    assert list(piv) == [1, 3] and list(nonp) == [0, 2, 4]
+    assert np.allclose(C, [[-0.5, 0.5], [0.5, 0.5], [0.0, 0.0]], atol=1e-14)
+    assert np.array_equal(Wp, W[[1, 3]])
+
+
+@pytest.mark.slow
+def test_compress_matches_oracle_lapack_attention_shape(lib):
+    """4096 x 4096, r = 2048 (LLaMA-2-7B attention projection): pivots bit-exact with the oracle's
+    LAPACK route (skipped unless -m slow)."""
+    _compare_with_oracle(4096, 4096, 2048, 0, "lapack")
