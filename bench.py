@@ -220,7 +220,7 @@ def run_ours(args, rank, world, local_rank):
     with torch.cuda.stream(stream):
         for i in range(5):
             Xd.copy_(Xh, non_blocking=True)
-            step_e2e = P.pifa_forward(Xd, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Ys[0], variant=variant,
+            P.pifa_forward(Xd, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Ys[0], variant=variant,
                                       workspace_tensor=ws, stream=stream)
             Yh.copy_(Ys[0], non_blocking=True)
     stream.synchronize()
@@ -412,7 +412,7 @@ def main():
     global _DIST
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--steps", type=int, default=200000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--tokens", type=int, default=T_DECODE)

@@ -80,7 +80,8 @@ typedef struct {
  *                another call that may run concurrently.
  *   cuda_stream  a cudaStream_t (NULL = legacy default stream).
  *
- *   Requirements: 1 <= r <= min(m, n); T >= 0 (T == 0 is a no-op); every base pointer of X, Wp,
+ *   Requirements: 1 <= r <= min(m, n); T >= 0 (T == 0 is a no-op: nothing is read or written and
+ *   X and Y may be NULL); every base pointer of X, Wp,
  *   C, Y 16-byte aligned and ldx, ldwp, ldc, ldy multiples of 8 (16-byte row pitch), else
  *   PIFA_ERR_ALIGNMENT. Index sets are not validated on the host (that would need a copy back);
  *   kernels skip any write whose index is outside [0, m) and latch PIFA_ERR_DEVICE_INDEX, read

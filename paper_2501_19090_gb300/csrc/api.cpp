@@ -163,6 +163,7 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const
   int st = validate_shape(T, m, n, r);
   if (st != PIFA_OK) return st;
   const bool has_np = m > r;
+  if (T == 0) return PIFA_OK;  // no-op: nothing is read or written (X and Y may be null)
   if (!X || !Wp || !pivot_idx || !Y) return pifa_fail(PIFA_ERR_INVALID_ARG, "null X, Wp, pivot_idx or Y");
   if (has_np && (!C || !nonpivot_idx)) return pifa_fail(PIFA_ERR_INVALID_ARG, "null C or nonpivot_idx with m > r");
   if (ldx < n || ldwp < n || ldy < m || (has_np && ldc < r))
@@ -179,7 +180,6 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const
         (has_np && overlaps(y, span_of(C, m - r, r, ldc, 2))))
       return pifa_fail(PIFA_ERR_INVALID_ARG, "Y overlaps an input");
   }
-  if (T == 0) return PIFA_OK;
   if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r);
 
   PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy};

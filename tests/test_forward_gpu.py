@@ -26,7 +26,7 @@ pytestmark = pytest.mark.gpu
 
 REL_FRO = 5e-3
 ELEM = 2e-2
-SENTINEL = -12345.0   # exactly representable in bf16
+SENTINEL = -16384.0   # exactly representable in bf16 (a power of two)
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -59,9 +59,14 @@ class Layer:
         return Wp, C, piv, nonp
 
 
+def _round8(v):
+    return (v + 7) // 8 * 8
+
+
 def _pad_dev(a32, ld=None):
+    """Device bf16 copy with row pitch ld (default: cols rounded up to 8, the 16-byte rule)."""
     rows, cols = a32.shape
-    ld = ld or cols
+    ld = ld or _round8(cols)
     buf = torch.full((rows, ld), float("nan"), dtype=torch.bfloat16, device=DEV)
     buf[:, :cols] = torch.from_numpy(np.ascontiguousarray(a32)).to(DEV).to(torch.bfloat16)
     return buf[:, :cols]
@@ -107,7 +112,7 @@ def run(layer, X32, variant=P.PIFA_VARIANT_AUTO, ldx=None, ldy_pad=8, guard_rows
     m = layer.m
     Wp, C, piv, nonp = layer.dev(ldwp, ldc)
     X = _pad_dev(X32, ldx) if T else torch.empty((0, layer.n), dtype=torch.bfloat16, device=DEV)
-    ldy = m + ldy_pad
+    ldy = _round8(m + ldy_pad)
     big = torch.full((T + 2 * guard_rows, ldy), SENTINEL, dtype=torch.bfloat16, device=DEV)
     Y = big[guard_rows:guard_rows + T, :m]
     Y.fill_(float("nan"))
