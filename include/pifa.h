@@ -107,6 +107,29 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx,
                          void* workspace, int64_t workspace_bytes,
                          int variant, void* cuda_stream);
 
+/*
+ * pifa_forward_decode_noalloc -- the decode variant of pifa_forward (T <= 16) for callers that
+ * cannot allocate device memory, e.g. a runtime that plans all device memory up front and forbids
+ * a library's cudaMalloc, or a decode loop where an allocation's implicit synchronization is not
+ * acceptable. The paper has no counterpart; it is an interface convenience of this library.
+ *
+ *   Arguments, layouts and errors as pifa_forward, without the workspace: the call allocates
+ *   nothing (no cudaMalloc, cudaFree or allocating library routine). Its scratch, y_p in fp32
+ *   (T rows of pitch round_up(r, 8)), lives in a 1 MiB array in this library's static device
+ *   data, which every GPU that loads the library holds until the process exits. Shapes with
+ *   T * round_up(r, 8) * 4 > 1 MiB are rejected with PIFA_ERR_WORKSPACE; T > 16 with
+ *   PIFA_ERR_UNSUPPORTED.
+ *   The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
+ *   that device current; make that first call before any stream capture. Every call on a device
+ *   shares the one array and it keeps the last call's contents (nothing in it needs to start at
+ *   zero): calls that may overlap on the GPU, e.g. on different streams, race on it.
+ */
+int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, int64_t ldx,
+                                const void* Wp, int64_t r, int64_t ldwp,
+                                const void* C, int64_t m, int64_t ldc,
+                                const int32_t* pivot_idx, const int32_t* nonpivot_idx,
+                                void* Y, int64_t ldy, void* cuda_stream);
+
 /* pifa_workspace_size -- bytes of device scratch pifa_forward needs for this shape and variant
  * (PIFA_VARIANT_AUTO: the variant the selector picks). Returns a negative pifa_status on bad
  * arguments. Pure host arithmetic; no GPU needed. */

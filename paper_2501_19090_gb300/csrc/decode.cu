@@ -20,6 +20,8 @@
 // completed. y_p enters the second contraction as a bf16 hi + bf16 lo pair (16 significant bits):
 // C has large entries and Y_np = C Y_p cancels, so rounding y_p to bf16 alone would amplify its
 // rounding error several-fold.
+#include <mutex>
+
 #include <cuda_bf16.h>
 
 #include "pifa.h"
@@ -262,4 +264,74 @@ int64_t decode_workspace_bytes(const PifaShape& s) {
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
   if (s.T <= 8) return launch_decode_t<1, 16, 8>(s, p, status, stream);
   return launch_decode_t<2, 8, 8>(s, p, status, stream);
+}
+
+// ---- allocation-free decode entry point -------------------------------------------------------
+// For callers that cannot allocate device memory at all: for example an inference runtime that
+// plans every device byte ahead of time and forbids libraries from calling cudaMalloc, or code
+// running where an allocation would synchronize the device in the middle of a latency-critical
+// decode loop. Such callers cannot provide the workspace pifa_forward asks for, so this entry
+// point keeps the decode scratch (y_p, fp32, T rows of pitch round_up(r, 8)) in a fixed array in
+// the library's static device data instead. The array exists once per GPU that loads the
+// library and stays allocated until the process exits.
+namespace {
+
+constexpr int64_t kNoAllocScratchBytes = int64_t(1) << 20;  // 1 MiB: T * round_up(r, 8) * 4 bytes
+__device__ __align__(256) unsigned char g_decode_scratch[kNoAllocScratchBytes];
+
+constexpr int kNoAllocMaxDevices = 64;
+void* g_decode_scratch_addr[kNoAllocMaxDevices] = {};
+std::mutex g_decode_scratch_mu;
+
+bool noalloc_aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+extern "C" int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp,
+                                           int64_t r, int64_t ldwp, const void* C, int64_t m, int64_t ldc,
+                                           const int32_t* pivot_idx, const int32_t* nonpivot_idx, void* Y,
+                                           int64_t ldy, void* cuda_stream) {
+  pifa_clear_error();
+  if (T < 0 || m < 1 || n < 1 || r < 1 || r > m || r > n || m >= (int64_t(1) << 30) || n >= (int64_t(1) << 30))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "need T >= 0 and 1 <= r <= min(m, n) < 2^30");
+  if (T == 0) return PIFA_OK;
+  if (T > 16) return pifa_fail(PIFA_ERR_UNSUPPORTED, "pifa_forward_decode_noalloc needs T <= 16");
+  const bool has_np = m > r;
+  if (!X || !Wp || !pivot_idx || !Y || (has_np && (!C || !nonpivot_idx)))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "null X, Wp, C, pivot_idx, nonpivot_idx or Y");
+  if (ldx < n || ldwp < n || ldy < m || (has_np && ldc < r))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "leading dimension smaller than the row length");
+  if (!noalloc_aligned16(X) || !noalloc_aligned16(Wp) || !noalloc_aligned16(Y) || (has_np && !noalloc_aligned16(C)))
+    return pifa_fail(PIFA_ERR_ALIGNMENT, "X, Wp, C and Y must be 16-byte aligned");
+  if ((ldx | ldwp | ldy | (has_np ? ldc : 0)) & 7)
+    return pifa_fail(PIFA_ERR_ALIGNMENT, "ldx, ldwp, ldc and ldy must be multiples of 8 elements");
+  const PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy};
+  const int64_t need = decode_workspace_bytes(s);
+  if (need > kNoAllocScratchBytes)
+    return pifa_fail(PIFA_ERR_WORKSPACE,
+                     "T * round_up(r, 8) * 4 bytes exceeds the 1 MiB static scratch of pifa_forward_decode_noalloc");
+
+  // Set-up, once per device, with that device current: the device address of the static array.
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return pifa_fail_cuda("cudaGetDevice", e);
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return pifa_fail(PIFA_ERR_UNSUPPORTED, "device ordinal >= 64");
+  void* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_decode_scratch_mu);
+    if (!g_decode_scratch_addr[dev]) {
+      void* ptr = nullptr;
+      e = cudaGetSymbolAddress(&ptr, g_decode_scratch);
+      if (e != cudaSuccess) return pifa_fail_cuda("cudaGetSymbolAddress(decode scratch)", e);
+      g_decode_scratch_addr[dev] = ptr;
+    }
+    scratch = g_decode_scratch_addr[dev];
+  }
+  int* status = pifa_status_word(&e);
+  if (!status) return pifa_fail_cuda("device status word", e);
+  // y_p is written in full by the first phase before the second reads it, so nothing in the
+  // shared array has to start at zero.
+  const PifaPointers p = {X, Wp, has_np ? C : nullptr, pivot_idx, has_np ? nonpivot_idx : nullptr, Y, scratch,
+                          kNoAllocScratchBytes};
+  return launch_decode(s, p, status, reinterpret_cast<cudaStream_t>(cuda_stream));
 }

@@ -35,7 +35,7 @@ PIFA_VARIANT_PREFILL_FUSED = 3
 EXPORTS = (
     "pifa_forward", "pifa_forward_variant", "pifa_workspace_size", "pifa_select_variant",
     "pifa_variant_name", "pifa_compress", "pifa_validate_indices", "pifa_device_status",
-    "pifa_status_string", "pifa_last_error", "pifa_version",
+    "pifa_status_string", "pifa_last_error", "pifa_version", "pifa_forward_decode_noalloc",
 )
 
 
@@ -72,6 +72,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.pifa_forward.restype = ctypes.c_int
         lib.pifa_forward_variant.argtypes = fwd + [ctypes.c_int, _VP]
         lib.pifa_forward_variant.restype = ctypes.c_int
+        lib.pifa_forward_decode_noalloc.argtypes = fwd[:14] + [_VP]
+        lib.pifa_forward_decode_noalloc.restype = ctypes.c_int
         lib.pifa_workspace_size.argtypes = [_I64, _I64, _I64, _I64, ctypes.c_int]
         lib.pifa_workspace_size.restype = _I64
         lib.pifa_select_variant.argtypes = [_I64, _I64, _I64, _I64]
@@ -227,4 +229,23 @@ def pifa_forward(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, variant: int = PIFA_
         pivot_idx.data_ptr(), nonpivot_idx.data_ptr() if has_np else None,
         Y.data_ptr(), _ld(Y), ws_ptr or None, ws_bytes, variant, _stream_ptr(stream))
     _check(st, "pifa_forward")
+    return Y
+
+
+def pifa_forward_decode_noalloc(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, stream=None):
+    """Decode forward (T <= 16) without a workspace: the library's static 1 MiB device scratch
+    is used instead (see include/pifa.h). Allocates Y here only if the caller passes none."""
+    import torch
+    T, n = X.shape
+    r = Wp.shape[0]
+    m = r + (nonpivot_idx.numel() if nonpivot_idx is not None else 0)
+    if Y is None:
+        Y = torch.empty((T, m), dtype=torch.bfloat16, device=X.device)
+    has_np = m > r
+    st = _lib().pifa_forward_decode_noalloc(
+        X.data_ptr(), T, n, _ld(X), Wp.data_ptr(), r, _ld(Wp),
+        C.data_ptr() if has_np else None, m, _ld(C) if has_np else r,
+        pivot_idx.data_ptr(), nonpivot_idx.data_ptr() if has_np else None,
+        Y.data_ptr(), _ld(Y), _stream_ptr(stream))
+    _check(st, "pifa_forward_decode_noalloc")
     return Y
