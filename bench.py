@@ -130,12 +130,24 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------------------------
-def build_layer(shape, seed):
-    """Host-side setup: the library's compression (Algorithm 1), rounded to bf16 operands."""
+def build_layer(shape, seed, c_dtype="bf16"):
+    """Host-side setup: the library's compression (Algorithm 1); W_p rounded to bf16 and C to the
+    chosen storage type (bf16 by default, or fp16)."""
     from paper_2501_19090_gb300 import pifa as P
     U, V, _ = inputs.make_factors(shape.m, shape.n, shape.r, seed)
     piv, nonp, Wp, C, info = P.pifa_compress(U, V, shape.r)
-    return dict(U=U, V=V, piv=piv, nonp=nonp, Wp=inputs.round_bf16(Wp), C=inputs.round_bf16(C), info=info)
+    Cq = inputs.round_fp16(C) if c_dtype == "fp16" else inputs.round_bf16(C)
+    return dict(U=U, V=V, piv=piv, nonp=nonp, Wp=inputs.round_bf16(Wp), C=Cq, info=info, c_dtype=c_dtype)
+
+
+def _torch_c_dtype(lay):
+    import torch
+    return torch.float16 if lay["c_dtype"] == "fp16" else torch.bfloat16
+
+
+def _pifa_c_dtype(lay):
+    from paper_2501_19090_gb300 import pifa as P
+    return P.PIFA_DTYPE_FP16 if lay["c_dtype"] == "fp16" else P.PIFA_DTYPE_BF16
 
 
 def run_ours(args, rank, world, local_rank):
@@ -149,11 +161,13 @@ def run_ours(args, rank, world, local_rank):
     shape = SHAPE
     m, n, r = shape.m, shape.n, shape.r
     T = args.tokens
-    lay = build_layer(shape, seed=0)
+    lay = build_layer(shape, seed=0, c_dtype=args.c_dtype)
     bf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev).to(torch.bfloat16)
     piv = torch.from_numpy(lay["piv"]).to(dev)
     nonp = torch.from_numpy(lay["nonp"]).to(dev)
-    Wp0, C0 = bf(lay["Wp"]), bf(lay["C"])
+    Wp0 = bf(lay["Wp"])
+    C0 = torch.from_numpy(np.ascontiguousarray(lay["C"])).to(dev).to(_torch_c_dtype(lay))
+    cdt = _pifa_c_dtype(lay)
     wbytes = (Wp0.numel() + C0.numel()) * 2
     l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     copies = max(4, math.ceil(3 * l2 / wbytes))
@@ -162,8 +176,8 @@ def run_ours(args, rank, world, local_rank):
     rng = np.random.default_rng(1 + rank)
     Xs = [bf(inputs.make_activations(rng, T, n, "bf16")) for _ in range(copies)]
     Ys = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(copies)]
-    variant = P.pifa_select_variant(T, m, n, r)
-    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant), dev)
+    variant = P.pifa_select_variant(T, m, n, r, cdt)
+    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant, cdt), dev)
     stream = torch.cuda.Stream(device=dev)
 
     def step(i):
@@ -243,7 +257,8 @@ def run_ours(args, rank, world, local_rank):
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
         "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": f"{shape.name} decode T={T}", "m": m, "n": n, "r": r, "tokens_per_step": T,
+        "config": {"workload": f"{shape.name} {'decode' if T <= 16 else 'prefill'} T={T}", "m": m, "n": n, "r": r,
+                   "tokens_per_step": T, "c_dtype": lay["c_dtype"],
                    "variant": P.pifa_variant_name(variant), "parallelism": f"replicas{world}",
                    "l2_defeat": f"{copies} rotating weight copies ({copies * wbytes / 1e6:.0f} MB > 3x L2)",
                    "timing": "CUDA graph replay, CUDA events on the launching stream"},
@@ -259,6 +274,8 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0 and not args.no_extras:
         out["comparators"] = comparators(dev, lay, T, copies, stream)
         out["prefill"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src)
+        out["prefill_split"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src,
+                                             variant=P.PIFA_VARIANT_PREFILL_SPLIT)
         out["cpu_baseline"] = cpu_baseline(lay, T)
     return out
 
@@ -293,7 +310,7 @@ def comparators(dev, lay, T, copies, stream):
     return res
 
 
-def prefill_point(dev, lay, copies, stream, tc_peak, peak_src):
+def prefill_point(dev, lay, copies, stream, tc_peak, peak_src, variant=None):
     import torch
     from paper_2501_19090_gb300 import pifa as P
     m, n, r = SHAPE.m, SHAPE.n, SHAPE.r
@@ -301,15 +318,18 @@ def prefill_point(dev, lay, copies, stream, tc_peak, peak_src):
     bf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev).to(torch.bfloat16)
     piv = torch.from_numpy(lay["piv"]).to(dev)
     nonp = torch.from_numpy(lay["nonp"]).to(dev)
-    Wp, C = bf(lay["Wp"]), bf(lay["C"])
+    Wp = bf(lay["Wp"])
+    C = torch.from_numpy(np.ascontiguousarray(lay["C"])).to(dev).to(_torch_c_dtype(lay))
+    cdt = _pifa_c_dtype(lay)
     ncp = max(2, copies // 4)
     Wps = [Wp.clone() for _ in range(ncp)]
     Cs = [C.clone() for _ in range(ncp)]
     rng = np.random.default_rng(5)
     Xs = [bf(inputs.make_activations(rng, T, n, "bf16")) for _ in range(ncp)]
     Y = torch.empty((T, m), dtype=torch.bfloat16, device=dev)
-    variant = P.pifa_select_variant(T, m, n, r)
-    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant), dev, "prefill")
+    if variant is None:
+        variant = P.pifa_select_variant(T, m, n, r, cdt)
+    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant, cdt), dev, "prefill")
     with torch.cuda.stream(stream):
         for i in range(5):
             P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,
@@ -386,7 +406,8 @@ def run_reference(args, rank):
     T = args.tokens
     U, V, _ = inputs.make_factors(SHAPE.m, SHAPE.n, SHAPE.r, 0)
     L = oracle.compress(U, V, SHAPE.r, "lapack")
-    Wp, C = inputs.round_bf16(L.Wp).astype(np.float64), inputs.round_bf16(L.C).astype(np.float64)
+    Cq = inputs.round_fp16(L.C) if args.c_dtype == "fp16" else inputs.round_bf16(L.C)
+    Wp, C = inputs.round_bf16(L.Wp).astype(np.float64), Cq.astype(np.float64)
     rng = np.random.default_rng(1)
     X = inputs.make_activations(rng, T, SHAPE.n, "bf16")
     for _ in range(max(3, args.warmup)):
@@ -417,6 +438,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--tokens", type=int, default=T_DECODE)
     ap.add_argument("--no-extras", action="store_true")
+    ap.add_argument("--c-dtype", default="bf16", choices=["bf16", "fp16"])
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

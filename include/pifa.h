@@ -41,8 +41,15 @@ typedef enum {
   PIFA_ERR_TIMEOUT = -5,         /* a device-side bounded wait gave up (kernel returned early) */
   PIFA_ERR_RANK_DEFICIENT = -6,  /* W' = U V^T has fewer than r independent rows               */
   PIFA_ERR_WORKSPACE = -7,       /* workspace missing or smaller than pifa_workspace_size()    */
-  PIFA_ERR_DEVICE_INDEX = -8     /* a kernel met a pivot/non-pivot index outside [0, m)       */
+  PIFA_ERR_DEVICE_INDEX = -8,    /* a kernel met a pivot/non-pivot index outside [0, m)       */
+  PIFA_ERR_RANGE = -9            /* a Y_p value exceeded the fp16 range (C stored as fp16)      */
 } pifa_status;
+
+/* Storage type of C. W_p, X and Y are always bf16. C may be bf16 or fp16 (both 2 bytes per
+ * element). Y_p enters the second contraction as a hi + lo pair of C's type (bf16: 16
+ * significant bits, fp16: 22). Y_p values beyond +-65504 cannot be represented in fp16: with
+ * fp16 C they saturate and PIFA_ERR_RANGE is latched. */
+typedef enum { PIFA_DTYPE_BF16 = 0, PIFA_DTYPE_FP16 = 1 } pifa_dtype;
 
 /* Forward-pass implementations. PIFA_VARIANT_AUTO lets the selector choose (see
  * pifa_select_variant). The others force one implementation; a forced variant that cannot run
@@ -50,8 +57,9 @@ typedef enum {
 typedef enum {
   PIFA_VARIANT_AUTO = 0,
   PIFA_VARIANT_DECODE = 1,        /* T <= 16: two-phase HBM-streaming GEMV (mma.sync fragments)  */
-  PIFA_VARIANT_PREFILL_SPLIT = 2, /* tcgen05 GEMM 1 -> Y_p hi/lo in workspace -> tcgen05 GEMM 2 */
-  PIFA_VARIANT_PREFILL_FUSED = 3  /* one cluster kernel: Y_p stays in shared memory             */
+  PIFA_VARIANT_PREFILL_SPLIT = 2, /* tcgen05 GEMM 1 -> Y_p in workspace -> tcgen05 GEMM 2        */
+  PIFA_VARIANT_PREFILL_FUSED = 3  /* one persistent cluster kernel per token tile: GEMM 1, Y_p kept
+                                     on chip (L2 + shared memory), GEMM 2                        */
 } pifa_variant;
 
 /* Diagnostics of pifa_compress (all optional to read). */
@@ -67,17 +75,21 @@ typedef struct {
  *
  *   X            DEVICE, bf16, T x n, row pitch ldx >= n.
  *   Wp           DEVICE, bf16, r x n, row pitch ldwp >= n (row j is W'[I[j], :]).
- *   C            DEVICE, bf16, (m - r) x r, row pitch ldc >= r (row i gives W'[I^c[i], :]).
- *                May be NULL when r == m.
+ *   C            DEVICE, (m - r) x r, row pitch ldc >= r (row i gives W'[I^c[i], :]), stored as
+ *                c_dtype (a pifa_dtype: bf16 or fp16). May be NULL when r == m.
  *   pivot_idx    DEVICE, int32[r], strictly ascending, values in [0, m).
  *   nonpivot_idx DEVICE, int32[m - r], strictly ascending; together with pivot_idx a partition
  *                of [0, m). May be NULL when r == m.
  *   Y            DEVICE, bf16, T x m, row pitch ldy >= m. Every element Y[t, 0..m-1] is written
  *                exactly once (round to nearest even from the fp32 accumulator); the padding
  *                columns m..ldy-1 are not touched. Y must not overlap any input.
- *   workspace    DEVICE scratch of at least pifa_workspace_size(T, m, n, r, variant) bytes,
- *                256-byte aligned; NULL allowed when that size is 0. It must not be used by
- *                another call that may run concurrently.
+ *   workspace    DEVICE scratch of at least pifa_workspace_size(T, m, n, r, c_dtype, variant) bytes,
+ *                256-byte aligned. Its first 256 bytes are library state (the decode kernel's
+ *                grid-barrier words): zero-fill the workspace once before its first use (e.g. a
+ *                cudaMemset at allocation); every completed call leaves those bytes zero again,
+ *                for any shape and variant. After a call that returned or latched
+ *                PIFA_ERR_TIMEOUT, zero them again. A workspace must not be used by another call
+ *                that may run concurrently.
  *   cuda_stream  a cudaStream_t (NULL = legacy default stream).
  *
  *   Requirements: 1 <= r <= min(m, n); T >= 0 (T == 0 is a no-op: nothing is read or written and
@@ -86,13 +98,13 @@ typedef struct {
  *   PIFA_ERR_ALIGNMENT. Index sets are not validated on the host (that would need a copy back);
  *   kernels skip any write whose index is outside [0, m) and latch PIFA_ERR_DEVICE_INDEX, read
  *   with pifa_device_status(). pifa_validate_indices() checks host copies in full.
- *   Numerics: bf16 operands, fp32 accumulation; Y_p is carried into the second contraction
- *   at (at least) 16 significant bits (a bf16 hi + bf16 lo pair or fp32), never as bf16 alone.
+ *   Numerics: bf16 X and W_p, fp32 accumulation; Y_p enters the second contraction as a hi + lo
+ *   pair of C's storage type, never as one bf16 or fp16 value.
  *   Returns PIFA_OK once the kernels are enqueued; launch errors give PIFA_ERR_CUDA.
  */
 int pifa_forward(const void* X, int64_t T, int64_t n, int64_t ldx,
                  const void* Wp, int64_t r, int64_t ldwp,
-                 const void* C, int64_t m, int64_t ldc,
+                 const void* C, int64_t m, int64_t ldc, int c_dtype,
                  const int32_t* pivot_idx, const int32_t* nonpivot_idx,
                  void* Y, int64_t ldy,
                  void* workspace, int64_t workspace_bytes,
@@ -101,7 +113,7 @@ int pifa_forward(const void* X, int64_t T, int64_t n, int64_t ldx,
 /* pifa_forward_variant -- pifa_forward with an explicit pifa_variant (tests and benchmarks). */
 int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx,
                          const void* Wp, int64_t r, int64_t ldwp,
-                         const void* C, int64_t m, int64_t ldc,
+                         const void* C, int64_t m, int64_t ldc, int c_dtype,
                          const int32_t* pivot_idx, const int32_t* nonpivot_idx,
                          void* Y, int64_t ldy,
                          void* workspace, int64_t workspace_bytes,
@@ -113,16 +125,19 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx,
  * a library's cudaMalloc, or a decode loop where an allocation's implicit synchronization is not
  * acceptable. The paper has no counterpart; it is an interface convenience of this library.
  *
- *   Arguments, layouts and errors as pifa_forward, without the workspace: the call allocates
- *   nothing (no cudaMalloc, cudaFree or allocating library routine). Its scratch, y_p in fp32
- *   (T rows of pitch round_up(r, 8)), lives in a 1 MiB array in this library's static device
- *   data, which every GPU that loads the library holds until the process exits. Shapes with
- *   T * round_up(r, 8) * 4 > 1 MiB are rejected with PIFA_ERR_WORKSPACE; T > 16 with
- *   PIFA_ERR_UNSUPPORTED.
+ *   Arguments, layouts and errors as pifa_forward with C in bf16, without the workspace: the
+ *   call allocates
+ *   nothing (no cudaMalloc, cudaFree or allocating library routine). Its scratch -- 256 bytes of
+ *   grid-barrier words, then y_p in fp32 (T rows of pitch round_up(r, 8)) -- lives in a 1 MiB
+ *   array in this library's static device data, which every GPU that loads the library holds
+ *   until the process exits. Shapes with 256 + T * round_up(r, 8) * 4 > 1 MiB are rejected
+ *   with PIFA_ERR_WORKSPACE; T > 16 with PIFA_ERR_UNSUPPORTED.
  *   The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
  *   that device current; make that first call before any stream capture. Every call on a device
- *   shares the one array and it keeps the last call's contents (nothing in it needs to start at
- *   zero): calls that may overlap on the GPU, e.g. on different streams, race on it.
+ *   shares the one array and it keeps the last call's contents: the barrier words start at zero
+ *   (static data is zero-initialised) and every completed call leaves them zero; y_p is fully
+ *   written before it is read. Calls that may overlap on the GPU, e.g. on different streams,
+ *   race on the array.
  */
 int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, int64_t ldx,
                                 const void* Wp, int64_t r, int64_t ldwp,
@@ -130,16 +145,16 @@ int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, int64_t ldx
                                 const int32_t* pivot_idx, const int32_t* nonpivot_idx,
                                 void* Y, int64_t ldy, void* cuda_stream);
 
-/* pifa_workspace_size -- bytes of device scratch pifa_forward needs for this shape and variant
- * (PIFA_VARIANT_AUTO: the variant the selector picks). Returns a negative pifa_status on bad
- * arguments. Pure host arithmetic; no GPU needed. */
-int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int variant);
+/* pifa_workspace_size -- bytes of device scratch pifa_forward needs for this shape, C dtype and
+ * variant (PIFA_VARIANT_AUTO: the variant the selector picks). Returns a negative pifa_status on
+ * bad arguments. Pure host arithmetic; no GPU needed. */
+int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype, int variant);
 
 /* pifa_select_variant -- the selector (host, < 1 us): the pifa_variant pifa_forward runs for
- * (T, m, n, r) on this build, never PIFA_VARIANT_AUTO; negative pifa_status on bad arguments.
- * Decode for T <= 16; otherwise the fused prefill kernel when its cluster can hold Y_p for the
- * rank r, else the split prefill. */
-int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r);
+ * (T, m, n, r, c_dtype) on this build, never PIFA_VARIANT_AUTO; negative pifa_status on bad
+ * arguments. Decode for T <= 16; otherwise the fused prefill kernel when the device can run
+ * its thread-block cluster, else the split prefill. */
+int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype);
 
 /* pifa_variant_name -- static string naming a pifa_variant ("decode", ...); "?" if unknown. */
 const char* pifa_variant_name(int variant);
@@ -178,6 +193,19 @@ int pifa_validate_indices(const int32_t* pivot_idx, const int32_t* nonpivot_idx,
 /* pifa_device_status -- synchronizes `cuda_stream`, then returns and clears the error word the
  * kernels latch on the current device (PIFA_OK, PIFA_ERR_TIMEOUT or PIFA_ERR_DEVICE_INDEX). */
 int pifa_device_status(void* cuda_stream);
+
+/* pifa_set_wait_timeout -- bound, in nanoseconds, of every device-side wait of kernels launched
+ * after this call (default 1 s, or the environment variable PIFA_WAIT_TIMEOUT_NS at load time;
+ * ns == 0 restores that default). A wait that runs out makes its CTA latch PIFA_ERR_TIMEOUT, wait
+ * (with a fixed bound) for its own copies in flight, and return; the outputs of that call are then
+ * undefined. Process-wide; PIFA_ERR_INVALID_ARG for ns < 0. */
+int pifa_set_wait_timeout(int64_t ns);
+
+/* pifa_selftest_wait_timeout -- enqueues on `cuda_stream` a one-CTA kernel that waits, with the
+ * current bound (pifa_set_wait_timeout), on an mbarrier that nothing arrives on, so the wait runs
+ * out and PIFA_ERR_TIMEOUT is latched for pifa_device_status(). Checks the failure-detection path
+ * of the bounded device waits without faulting or hanging the GPU. Not part of the paper. */
+int pifa_selftest_wait_timeout(void* cuda_stream);
 
 /* pifa_status_string -- static string for a pifa_status value. */
 const char* pifa_status_string(int status);

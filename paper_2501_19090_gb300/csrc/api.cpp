@@ -3,6 +3,7 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 #include <string>
 
@@ -71,24 +72,28 @@ int pifa_fail_cuda(const char* where, cudaError_t err) {
   return PIFA_ERR_CUDA;
 }
 
-uint64_t pifa_wait_timeout_ns() {
-  static uint64_t v = [] {
-    const char* e = std::getenv("PIFA_WAIT_TIMEOUT_NS");
-    if (e && *e) return (uint64_t)std::strtoull(e, nullptr, 10);
-    return (uint64_t)1000000000ull;  // 1 s
-  }();
-  return v;
+namespace {
+uint64_t default_wait_timeout_ns() {
+  const char* e = std::getenv("PIFA_WAIT_TIMEOUT_NS");
+  if (e && *e) return (uint64_t)std::strtoull(e, nullptr, 10);
+  return (uint64_t)1000000000ull;  // 1 s
 }
+std::atomic<uint64_t> g_wait_timeout_ns{default_wait_timeout_ns()};
+}  // namespace
 
-int make_tmap_bf16_2d(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld, uint32_t box_cols,
-                      uint32_t box_rows) {
+uint64_t pifa_wait_timeout_ns() { return g_wait_timeout_ns.load(std::memory_order_relaxed); }
+
+int make_tmap_2d(CUtensorMap* map, int dtype, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                 uint32_t box_cols, uint32_t box_rows) {
   EncodeTiledFn fn = get_encode_fn();
   if (!fn) return pifa_fail(PIFA_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
   cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
   cuuint64_t strides[1] = {(cuuint64_t)(ld * 2)};
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+  const CUtensorMapDataType dt =
+      dtype == PIFA_DTYPE_FP16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+  CUresult r = fn(map, dt, 2, const_cast<void*>(base), dims, strides, box, estr,
                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
@@ -105,6 +110,12 @@ extern "C" {
 
 const char* pifa_version(void) { return "libpifa 0.1 (sm_103a)"; }
 
+int pifa_set_wait_timeout(int64_t ns) {
+  if (ns < 0) return pifa_fail(PIFA_ERR_INVALID_ARG, "timeout must be >= 0");
+  g_wait_timeout_ns.store(ns == 0 ? default_wait_timeout_ns() : (uint64_t)ns, std::memory_order_relaxed);
+  return PIFA_OK;
+}
+
 const char* pifa_last_error(void) { return g_last_error.c_str(); }
 
 const char* pifa_status_string(int status) {
@@ -118,6 +129,7 @@ const char* pifa_status_string(int status) {
     case PIFA_ERR_RANK_DEFICIENT: return "PIFA_ERR_RANK_DEFICIENT";
     case PIFA_ERR_WORKSPACE: return "PIFA_ERR_WORKSPACE";
     case PIFA_ERR_DEVICE_INDEX: return "PIFA_ERR_DEVICE_INDEX";
+    case PIFA_ERR_RANGE: return "PIFA_ERR_RANGE";
     default: return "PIFA_ERR_UNKNOWN";
   }
 }
@@ -132,37 +144,40 @@ const char* pifa_variant_name(int variant) {
   }
 }
 
-int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r) {
+int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype) {
   int st = validate_shape(T, m, n, r);
   if (st != PIFA_OK) return st;
+  if (c_dtype != PIFA_DTYPE_BF16 && c_dtype != PIFA_DTYPE_FP16) return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown c_dtype");
   if (T <= 16) return PIFA_VARIANT_DECODE;
-  PifaShape s = {T, m, n, r, n, n, r, m};
+  PifaShape s = {T, m, n, r, n, n, r, m, c_dtype};
   if (prefill_fused_supported(s)) return PIFA_VARIANT_PREFILL_FUSED;
   return PIFA_VARIANT_PREFILL_SPLIT;
 }
 
-int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int variant) {
+int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype, int variant) {
   int st = validate_shape(T, m, n, r);
   if (st != PIFA_OK) return st;
-  if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r);
-  PifaShape s = {T, m, n, r, n, n, r, m};
+  if (c_dtype != PIFA_DTYPE_BF16 && c_dtype != PIFA_DTYPE_FP16) return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown c_dtype");
+  if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r, c_dtype);
+  PifaShape s = {T, m, n, r, n, n, r, m, c_dtype};
   if (T == 0) return 0;
   switch (variant) {
-    case PIFA_VARIANT_DECODE: return decode_workspace_bytes(s);
-    case PIFA_VARIANT_PREFILL_SPLIT: return prefill_split_workspace_bytes(s);
-    case PIFA_VARIANT_PREFILL_FUSED: return prefill_fused_workspace_bytes(s);
+    case PIFA_VARIANT_DECODE: return kWorkspaceReserve + decode_workspace_bytes(s);
+    case PIFA_VARIANT_PREFILL_SPLIT: return kWorkspaceReserve + prefill_split_workspace_bytes(s);
+    case PIFA_VARIANT_PREFILL_FUSED: return kWorkspaceReserve + prefill_fused_workspace_bytes(s);
     default: return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
   }
 }
 
 int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,
-                         const void* C, int64_t m, int64_t ldc, const int32_t* pivot_idx,
+                         const void* C, int64_t m, int64_t ldc, int c_dtype, const int32_t* pivot_idx,
                          const int32_t* nonpivot_idx, void* Y, int64_t ldy, void* workspace,
                          int64_t workspace_bytes, int variant, void* cuda_stream) {
   pifa_clear_error();
   int st = validate_shape(T, m, n, r);
   if (st != PIFA_OK) return st;
   const bool has_np = m > r;
+  if (c_dtype != PIFA_DTYPE_BF16 && c_dtype != PIFA_DTYPE_FP16) return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown c_dtype");
   if (T == 0) return PIFA_OK;  // no-op: nothing is read or written (X and Y may be null)
   if (!X || !Wp || !pivot_idx || !Y) return pifa_fail(PIFA_ERR_INVALID_ARG, "null X, Wp, pivot_idx or Y");
   if (has_np && (!C || !nonpivot_idx)) return pifa_fail(PIFA_ERR_INVALID_ARG, "null C or nonpivot_idx with m > r");
@@ -180,9 +195,9 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const
         (has_np && overlaps(y, span_of(C, m - r, r, ldc, 2))))
       return pifa_fail(PIFA_ERR_INVALID_ARG, "Y overlaps an input");
   }
-  if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r);
+  if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r, c_dtype);
 
-  PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy};
+  PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy, c_dtype};
   int64_t need = 0;
   switch (variant) {
     case PIFA_VARIANT_DECODE:
@@ -195,18 +210,18 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const
       need = prefill_fused_workspace_bytes(s);
       break;
   }
-  if (need > 0) {
-    if (!workspace || workspace_bytes < need)
-      return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or smaller than pifa_workspace_size()");
-    if (reinterpret_cast<uintptr_t>(workspace) & 255u)
-      return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
-  }
+  need += kWorkspaceReserve;
+  if (!workspace || workspace_bytes < need)
+    return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or smaller than pifa_workspace_size()");
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u)
+    return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
   cudaError_t cerr = cudaSuccess;
   int* status = pifa_status_word(&cerr);
   if (!status) return pifa_fail_cuda("device status word", cerr);
 
-  PifaPointers p = {X, Wp, has_np ? C : nullptr, pivot_idx, has_np ? nonpivot_idx : nullptr, Y, workspace,
-                    workspace_bytes};
+  PifaPointers p = {X, Wp, has_np ? C : nullptr, pivot_idx, has_np ? nonpivot_idx : nullptr, Y,
+                    static_cast<uint8_t*>(workspace) + kWorkspaceReserve, workspace_bytes - kWorkspaceReserve,
+                    static_cast<unsigned*>(workspace)};
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(cuda_stream);
   switch (variant) {
     case PIFA_VARIANT_DECODE: return launch_decode(s, p, status, stream);
@@ -217,9 +232,10 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const
 }
 
 int pifa_forward(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,
-                 const void* C, int64_t m, int64_t ldc, const int32_t* pivot_idx, const int32_t* nonpivot_idx,
-                 void* Y, int64_t ldy, void* workspace, int64_t workspace_bytes, void* cuda_stream) {
-  return pifa_forward_variant(X, T, n, ldx, Wp, r, ldwp, C, m, ldc, pivot_idx, nonpivot_idx, Y, ldy, workspace,
+                 const void* C, int64_t m, int64_t ldc, int c_dtype, const int32_t* pivot_idx,
+                 const int32_t* nonpivot_idx, void* Y, int64_t ldy, void* workspace, int64_t workspace_bytes,
+                 void* cuda_stream) {
+  return pifa_forward_variant(X, T, n, ldx, Wp, r, ldwp, C, m, ldc, c_dtype, pivot_idx, nonpivot_idx, Y, ldy, workspace,
                               workspace_bytes, PIFA_VARIANT_AUTO, cuda_stream);
 }
 

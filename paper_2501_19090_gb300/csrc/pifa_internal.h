@@ -24,7 +24,13 @@ uint64_t pifa_wait_timeout_ns();
 struct PifaShape {
   int64_t T, m, n, r;
   int64_t ldx, ldwp, ldc, ldy;
+  int c_dtype;  // PIFA_DTYPE_BF16 or PIFA_DTYPE_FP16 (storage type of C)
 };
+
+// The first kWorkspaceReserve bytes of every workspace hold library state that must be zero before
+// the first call and that every call leaves zero (the decode kernel's grid-barrier count and
+// generation); per-call scratch starts after them.
+constexpr int64_t kWorkspaceReserve = 256;
 
 struct PifaPointers {
   const void* X;
@@ -33,8 +39,9 @@ struct PifaPointers {
   const int32_t* piv;
   const int32_t* nonpiv;
   void* Y;
-  void* ws;
-  int64_t ws_bytes;
+  void* ws;           // per-call scratch (workspace + kWorkspaceReserve)
+  int64_t ws_bytes;   // bytes available at ws
+  unsigned* sync;     // the reserved words at the start of the workspace
 };
 
 // ---- decode (decode.cu) ----------------------------------------------------------------------
@@ -51,9 +58,10 @@ int launch_prefill_fused(const PifaShape& s, const PifaPointers& p, int* status,
                          cudaStream_t stream);
 
 // ---- TMA descriptors (api.cpp) ---------------------------------------------------------------
-// 2-D bf16 tensor map over a row-major (rows x cols) matrix with row pitch `ld` elements; box of
-// box_cols x box_rows elements, 128-byte swizzle, zero fill outside the matrix.
-int make_tmap_bf16_2d(CUtensorMap* map, const void* base, int64_t rows, int64_t cols, int64_t ld,
-                      uint32_t box_cols, uint32_t box_rows);
+// 2-D tensor map over a row-major (rows x cols) matrix of 2-byte elements (bf16 or fp16, a
+// PIFA_DTYPE_*) with row pitch `ld` elements; box of box_cols x box_rows elements, 128-byte
+// swizzle, zero fill outside the matrix.
+int make_tmap_2d(CUtensorMap* map, int dtype, const void* base, int64_t rows, int64_t cols, int64_t ld,
+                 uint32_t box_cols, uint32_t box_rows);
 
 #endif  // PIFA_INTERNAL_H_

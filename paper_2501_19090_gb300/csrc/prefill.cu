@@ -3,9 +3,10 @@
 // Split variant: two launches of one warp-specialised tcgen05 GEMM.
 //   GEMM 1 (Algorithm 2, steps 2 and 4): D1 = W_p X^T, tile 128 weight rows x 256 tokens.
 //           Epilogue writes bf16(Y_p) into the pivot columns Y[:, I[j]] and the pair
-//           hi = bf16(Y_p), lo = bf16(Y_p - hi) into two T x r scratch matrices.
-//   GEMM 2 (Algorithm 2, steps 3 and 5): D2 = C [hi | lo]^T accumulated over K = r twice
-//           (hi pass then lo pass), epilogue writes bf16(Y_np) into Y[:, I^c[i]].
+//           hi = rnd(Y_p), lo = rnd(Y_p - hi) into two T x r scratch matrices, rnd rounding to
+//           C's storage type (bf16 or fp16).
+//   GEMM 2 (Algorithm 2, steps 3 and 5): D2 = C [hi | lo]^T accumulated over K = r twice (hi pass
+//           then lo pass), epilogue writes bf16(Y_np) into Y[:, I^c[i]].
 // Weight rows are the MMA M dimension and tokens the N dimension, so the accumulator in tensor
 // memory holds one weight row per TMEM lane: an epilogue warp's 32 lanes are 32 consecutive
 // weight rows, which for a fixed token land in 32 ascending output columns of one row of Y.
@@ -16,6 +17,7 @@
 // (128 lanes x 256 columns of TMEM) through tcgen05.ld. Every wait is bounded (globaltimer); on
 // timeout the CTA latches PIFA_ERR_TIMEOUT, drains what it has in flight and returns.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include "pifa.h"
 #include "pifa_internal.h"
@@ -34,10 +36,13 @@ constexpr uint32_t A_BYTES = BM * BK * 2;
 constexpr uint32_t B_BYTES = BN * BK * 2;
 constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr uint32_t TMEM_COLS = BN;  // fp32 accumulator, one column per token
-constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 constexpr size_t SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + 256 /*barriers*/;
 
+// Epilogue modes: what GEMM 1 also writes besides Y (GEMM 2 writes Y only).
+enum { EPI_Y_ONLY = 0, EPI_SPLIT_BF16 = 1, EPI_SPLIT_F16 = 2 };
+
 struct GemmArgs {
+  uint32_t idesc;        // tcgen05 instruction descriptor (bf16 or fp16 operands)
   int M;                 // weight rows (r for GEMM 1, m - r for GEMM 2)
   int N;                 // tokens T
   int kchunks;           // ceil(K / 64) per pass
@@ -46,14 +51,14 @@ struct GemmArgs {
   int m;                 // columns of Y (index bound)
   bf16* Y;
   int64_t ldy;
-  bf16* yp_hi;           // GEMM 1 only: T x ldyp scratch
-  bf16* yp_lo;
+  void* yp_hi;           // GEMM 1 only: T x ldyp scratch, hi part (bf16 or fp16)
+  void* yp_lo;           // lo part
   int64_t ldyp;
   int* status;
   uint64_t timeout_ns;
 };
 
-template <bool kWriteSplit>
+template <int kEpi>
 __global__ void __launch_bounds__(192, 1)
     pifa_umma_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, GemmArgs p) {
@@ -133,10 +138,12 @@ __global__ void __launch_bounds__(192, 1)
         const uint32_t b = a + A_BYTES;
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk)
-          mma_bf16_ss(tmem, sw128_desc(a + kk * 32), sw128_desc(b + kk * 32), IDESC, (i > 0 || kk > 0) ? 1u : 0u);
+          mma_bf16_ss(tmem, sw128_desc(a + kk * 32), sw128_desc(b + kk * 32), p.idesc, (i > 0 || kk > 0) ? 1u : 0u);
         mma_commit(&empty[s]);
       }
-      mma_commit(acc_full);  // also drains every MMA issued above
+      mma_commit(acc_full);  // arrives once every MMA issued above has completed
+      // the CTA frees TMEM only after its MMAs are done, even if the epilogue gave up waiting
+      if (!mbar_wait(acc_full, 0, 100000000ull)) latch_status(p.status, PIFA_ERR_TIMEOUT);
     }
   } else {
     // ---------------- epilogue: warps 2..5 ----------------
@@ -160,6 +167,7 @@ __global__ void __launch_bounds__(192, 1)
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(cc * 32), v);
         tmem_ld_wait();
         if (col >= 0) {
+          bool range_err = false;
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
             const int t = n0 + cc * 32 + j;
@@ -167,12 +175,23 @@ __global__ void __launch_bounds__(192, 1)
               const float f = __uint_as_float(v[j]);
               const bf16 h = __float2bfloat16_rn(f);
               p.Y[(int64_t)t * p.ldy + col] = h;
-              if (kWriteSplit) {
-                p.yp_hi[(int64_t)t * p.ldyp + row] = h;
-                p.yp_lo[(int64_t)t * p.ldyp + row] = __float2bfloat16_rn(f - __bfloat162float(h));
+              if (kEpi == EPI_SPLIT_BF16) {
+                reinterpret_cast<bf16*>(p.yp_hi)[(int64_t)t * p.ldyp + row] = h;
+                reinterpret_cast<bf16*>(p.yp_lo)[(int64_t)t * p.ldyp + row] =
+                    __float2bfloat16_rn(f - __bfloat162float(h));
+              } else if (kEpi == EPI_SPLIT_F16) {
+                float fs = f;
+                if (fabsf(fs) > 65504.0f) {
+                  range_err = true;
+                  fs = copysignf(65504.0f, fs);
+                }
+                const __half hh = __float2half_rn(fs);
+                reinterpret_cast<__half*>(p.yp_hi)[(int64_t)t * p.ldyp + row] = hh;
+                reinterpret_cast<__half*>(p.yp_lo)[(int64_t)t * p.ldyp + row] = __float2half_rn(fs - __half2float(hh));
               }
             }
           }
+          if (range_err) latch_status(p.status, PIFA_ERR_RANGE);
         }
       }
     }
@@ -186,18 +205,16 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
-int run_gemm(bool write_split, const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
-             const GemmArgs& args, cudaStream_t stream) {
-  static bool attr_set[2] = {false, false};
-  auto kern = write_split ? pifa_umma_gemm<true> : pifa_umma_gemm<false>;
-  if (!attr_set[write_split]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
-    if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(prefill gemm)", e);
-    attr_set[write_split] = true;
-  }
+int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1, const GemmArgs& args,
+             cudaStream_t stream) {
+  auto kern = epi == EPI_SPLIT_BF16 ? pifa_umma_gemm<EPI_SPLIT_BF16>
+              : epi == EPI_SPLIT_F16 ? pifa_umma_gemm<EPI_SPLIT_F16>
+                                    : pifa_umma_gemm<EPI_Y_ONLY>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
+  if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(prefill gemm)", e);
   dim3 grid((args.M + BM - 1) / BM, (args.N + BN - 1) / BN);
   kern<<<grid, 192, SMEM_BYTES, stream>>>(a, b0, b1, args);
-  cudaError_t e = cudaGetLastError();
+  e = cudaGetLastError();
   if (e != cudaSuccess) return pifa_fail_cuda("prefill gemm launch", e);
   return PIFA_OK;
 }
@@ -207,23 +224,25 @@ inline int64_t pad8(int64_t v) { return (v + 7) / 8 * 8; }
 }  // namespace
 
 int64_t prefill_split_workspace_bytes(const PifaShape& s) {
-  const int64_t one = ((s.T * pad8(s.r) * 2 + 255) / 256) * 256;  // bf16 T x pad8(r)
-  return 2 * one;
+  const int64_t one = ((s.T * pad8(s.r) * 2 + 255) / 256) * 256;  // 2-byte T x pad8(r)
+  return 2 * one;  // hi and lo
 }
 
 int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,
                          cudaStream_t stream) {
+  const bool f16 = s.c_dtype == PIFA_DTYPE_FP16;
   const int64_t ldyp = pad8(s.r);
   const int64_t one = ((s.T * ldyp * 2 + 255) / 256) * 256;
-  bf16* hi = reinterpret_cast<bf16*>(p.ws);
-  bf16* lo = reinterpret_cast<bf16*>(reinterpret_cast<uint8_t*>(p.ws) + one);
+  void* hi = p.ws;
+  void* lo = reinterpret_cast<uint8_t*>(p.ws) + one;
 
   CUtensorMap tWp, tX, tC, tHi, tLo;
   int st;
-  if ((st = make_tmap_bf16_2d(&tWp, p.Wp, s.r, s.n, s.ldwp, BK, BM)) != PIFA_OK) return st;
-  if ((st = make_tmap_bf16_2d(&tX, p.X, s.T, s.n, s.ldx, BK, BN)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tWp, PIFA_DTYPE_BF16, p.Wp, s.r, s.n, s.ldwp, BK, BM)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tX, PIFA_DTYPE_BF16, p.X, s.T, s.n, s.ldx, BK, BN)) != PIFA_OK) return st;
 
   GemmArgs g1 = {};
+  g1.idesc = idesc_bf16_f32(BM, BN);
   g1.M = (int)s.r;
   g1.N = (int)s.T;
   g1.kchunks = (int)((s.n + BK - 1) / BK);
@@ -237,25 +256,20 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
   g1.ldyp = ldyp;
   g1.status = status;
   g1.timeout_ns = timeout_ns;
-  if ((st = run_gemm(true, tWp, tX, tX, g1, stream)) != PIFA_OK) return st;
+  if ((st = run_gemm(f16 ? EPI_SPLIT_F16 : EPI_SPLIT_BF16, tWp, tX, tX, g1, stream)) != PIFA_OK) return st;
   if (s.m == s.r) return PIFA_OK;
 
-  if ((st = make_tmap_bf16_2d(&tC, p.C, s.m - s.r, s.r, s.ldc, BK, BM)) != PIFA_OK) return st;
-  if ((st = make_tmap_bf16_2d(&tHi, hi, s.T, s.r, ldyp, BK, BN)) != PIFA_OK) return st;
-  if ((st = make_tmap_bf16_2d(&tLo, lo, s.T, s.r, ldyp, BK, BN)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tC, s.c_dtype, p.C, s.m - s.r, s.r, s.ldc, BK, BM)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tHi, s.c_dtype, hi, s.T, s.r, ldyp, BK, BN)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tLo, s.c_dtype, lo, s.T, s.r, ldyp, BK, BN)) != PIFA_OK) return st;
   GemmArgs g2 = g1;
+  g2.idesc = f16 ? idesc_f16_f32(BM, BN) : idesc_bf16_f32(BM, BN);
   g2.M = (int)(s.m - s.r);
   g2.kchunks = (int)((s.r + BK - 1) / BK);
   g2.passes = 2;
   g2.cols = p.nonpiv;
   g2.yp_hi = nullptr;
   g2.yp_lo = nullptr;
-  return run_gemm(false, tC, tHi, tLo, g2, stream);
+  return run_gemm(EPI_Y_ONLY, tC, tHi, tLo, g2, stream);
 }
 
-// The fused variant is not built yet: the selector never picks it.
-int64_t prefill_fused_workspace_bytes(const PifaShape&) { return 0; }
-bool prefill_fused_supported(const PifaShape&) { return false; }
-int launch_prefill_fused(const PifaShape&, const PifaPointers&, int*, uint64_t, cudaStream_t) {
-  return pifa_fail(PIFA_ERR_UNSUPPORTED, "fused prefill variant is not available in this build");
-}

@@ -4,7 +4,9 @@
 
 #include <cuda_runtime.h>
 
+#include "pifa.h"
 #include "pifa_internal.h"
+#include "ptx.cuh"
 
 namespace {
 __device__ int g_pifa_status_word = 0;
@@ -32,4 +34,30 @@ int* pifa_status_word(cudaError_t* err) {
     g_word_addr[dev] = static_cast<int*>(p);
   }
   return g_word_addr[dev];
+}
+
+namespace {
+// Waits, with the library's bound, on an mbarrier that nothing ever arrives on, then latches
+// PIFA_ERR_TIMEOUT: the failure-detection path of every bounded wait, exercised on its own.
+__global__ void wait_timeout_selftest(int* status, uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    pifa::mbar_init(&bar, 1);
+    pifa::fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !pifa::mbar_wait(&bar, 0, limit_ns)) pifa::latch_status(status, PIFA_ERR_TIMEOUT);
+  __syncthreads();
+}
+}  // namespace
+
+extern "C" int pifa_selftest_wait_timeout(void* cuda_stream) {
+  pifa_clear_error();
+  cudaError_t e = cudaSuccess;
+  int* status = pifa_status_word(&e);
+  if (!status) return pifa_fail_cuda("device status word", e);
+  wait_timeout_selftest<<<1, 32, 0, reinterpret_cast<cudaStream_t>(cuda_stream)>>>(status, pifa_wait_timeout_ns());
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return pifa_fail_cuda("wait-timeout self-test launch", e);
+  return PIFA_OK;
 }

@@ -68,6 +68,13 @@ def round_bf16(a) -> np.ndarray:
     return rounded.view(np.float64).astype(np.float32)
 
 
+def round_fp16(a) -> np.ndarray:
+    """Round float64 values to IEEE fp16 (round to nearest even, numpy's cast); return float32.
+
+    Values beyond +-65504 become inf: callers keep C (|C| of order 1) well inside the range."""
+    return np.asarray(a, dtype=np.float64).astype(np.float16).astype(np.float32)
+
+
 def bf16_bits(a32: np.ndarray) -> np.ndarray:
     """The 16-bit bf16 encodings of float32 values that are already exactly bf16 (see round_bf16)."""
     a32 = np.ascontiguousarray(np.asarray(a32, dtype=np.float32))

@@ -25,6 +25,10 @@ PIFA_ERR_TIMEOUT = -5
 PIFA_ERR_RANK_DEFICIENT = -6
 PIFA_ERR_WORKSPACE = -7
 PIFA_ERR_DEVICE_INDEX = -8
+PIFA_ERR_RANGE = -9
+
+PIFA_DTYPE_BF16 = 0
+PIFA_DTYPE_FP16 = 1
 
 PIFA_VARIANT_AUTO = 0
 PIFA_VARIANT_DECODE = 1
@@ -36,6 +40,7 @@ EXPORTS = (
     "pifa_forward", "pifa_forward_variant", "pifa_workspace_size", "pifa_select_variant",
     "pifa_variant_name", "pifa_compress", "pifa_validate_indices", "pifa_device_status",
     "pifa_status_string", "pifa_last_error", "pifa_version", "pifa_forward_decode_noalloc",
+    "pifa_set_wait_timeout", "pifa_selftest_wait_timeout",
 )
 
 
@@ -67,16 +72,17 @@ def load(path: str | None = None) -> ctypes.CDLL:
         if not os.path.exists(p):
             raise OSError(f"{p} not found: build it with `python -m paper_2501_19090_gb300.build`")
         lib = ctypes.CDLL(p)
-        fwd = [_VP, _I64, _I64, _I64, _VP, _I64, _I64, _VP, _I64, _I64, _VP, _VP, _VP, _I64, _VP, _I64]
-        lib.pifa_forward.argtypes = fwd + [_VP]
+        fwd = [_VP, _I64, _I64, _I64, _VP, _I64, _I64, _VP, _I64, _I64]
+        tail = [_VP, _VP, _VP, _I64, _VP, _I64]
+        lib.pifa_forward.argtypes = fwd + [ctypes.c_int] + tail + [_VP]
         lib.pifa_forward.restype = ctypes.c_int
-        lib.pifa_forward_variant.argtypes = fwd + [ctypes.c_int, _VP]
+        lib.pifa_forward_variant.argtypes = fwd + [ctypes.c_int] + tail + [ctypes.c_int, _VP]
         lib.pifa_forward_variant.restype = ctypes.c_int
-        lib.pifa_forward_decode_noalloc.argtypes = fwd[:14] + [_VP]
+        lib.pifa_forward_decode_noalloc.argtypes = fwd + tail[:4] + [_VP]
         lib.pifa_forward_decode_noalloc.restype = ctypes.c_int
-        lib.pifa_workspace_size.argtypes = [_I64, _I64, _I64, _I64, ctypes.c_int]
+        lib.pifa_workspace_size.argtypes = [_I64, _I64, _I64, _I64, ctypes.c_int, ctypes.c_int]
         lib.pifa_workspace_size.restype = _I64
-        lib.pifa_select_variant.argtypes = [_I64, _I64, _I64, _I64]
+        lib.pifa_select_variant.argtypes = [_I64, _I64, _I64, _I64, ctypes.c_int]
         lib.pifa_select_variant.restype = ctypes.c_int
         lib.pifa_variant_name.argtypes = [ctypes.c_int]
         lib.pifa_variant_name.restype = ctypes.c_char_p
@@ -91,6 +97,10 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.pifa_status_string.restype = ctypes.c_char_p
         lib.pifa_last_error.argtypes = []
         lib.pifa_last_error.restype = ctypes.c_char_p
+        lib.pifa_set_wait_timeout.argtypes = [_I64]
+        lib.pifa_set_wait_timeout.restype = ctypes.c_int
+        lib.pifa_selftest_wait_timeout.argtypes = [_VP]
+        lib.pifa_selftest_wait_timeout.restype = ctypes.c_int
         lib.pifa_version.argtypes = []
         lib.pifa_version.restype = ctypes.c_char_p
         _lib_handle = lib
@@ -116,6 +126,16 @@ def pifa_status_string(status: int) -> str:
     return _lib().pifa_status_string(int(status)).decode()
 
 
+def pifa_set_wait_timeout(ns: int) -> None:
+    """Bound of every device-side wait of later launches, in ns (0 restores the default 1 s)."""
+    _check(_lib().pifa_set_wait_timeout(int(ns)), "pifa_set_wait_timeout")
+
+
+def pifa_selftest_wait_timeout(stream=None) -> None:
+    """Enqueue the bounded-wait self-test kernel (latches PIFA_ERR_TIMEOUT; see include/pifa.h)."""
+    _check(_lib().pifa_selftest_wait_timeout(_stream_ptr(stream)), "pifa_selftest_wait_timeout")
+
+
 def pifa_last_error() -> str:
     return _lib().pifa_last_error().decode()
 
@@ -124,15 +144,16 @@ def pifa_variant_name(variant: int) -> str:
     return _lib().pifa_variant_name(int(variant)).decode()
 
 
-def pifa_select_variant(T: int, m: int, n: int, r: int) -> int:
-    v = _lib().pifa_select_variant(T, m, n, r)
+def pifa_select_variant(T: int, m: int, n: int, r: int, c_dtype: int = PIFA_DTYPE_BF16) -> int:
+    v = _lib().pifa_select_variant(T, m, n, r, c_dtype)
     if v < 0:
         _check(v, "pifa_select_variant")
     return v
 
 
-def pifa_workspace_size(T: int, m: int, n: int, r: int, variant: int = PIFA_VARIANT_AUTO) -> int:
-    v = _lib().pifa_workspace_size(T, m, n, r, variant)
+def pifa_workspace_size(T: int, m: int, n: int, r: int, variant: int = PIFA_VARIANT_AUTO,
+                        c_dtype: int = PIFA_DTYPE_BF16) -> int:
+    v = _lib().pifa_workspace_size(T, m, n, r, c_dtype, variant)
     if v < 0:
         _check(int(v), "pifa_workspace_size")
     return int(v)
@@ -193,7 +214,8 @@ def workspace(nbytes: int, device, stream=None):
     key = (str(device), 0 if stream is None else getattr(stream, "cuda_stream", stream))
     buf = _workspaces.get(key)
     if buf is None or buf.numel() < nbytes:
-        buf = torch.empty(max(nbytes, 256) + 256, dtype=torch.uint8, device=device)
+        # zero-filled: its first 256 bytes are library state that must start at zero
+        buf = torch.zeros(max(nbytes, 256) + 256, dtype=torch.uint8, device=device)
         _workspaces[key] = buf
     return buf
 
@@ -204,10 +226,21 @@ def _ld(t) -> int:
     return t.stride(0)
 
 
+def c_dtype_of(C) -> int:
+    """The pifa_dtype of a torch tensor C (bfloat16 or float16)."""
+    import torch
+    if C is None or C.dtype == torch.bfloat16:
+        return PIFA_DTYPE_BF16
+    if C.dtype == torch.float16:
+        return PIFA_DTYPE_FP16
+    raise TypeError(f"C must be bfloat16 or float16, got {C.dtype}")
+
+
 def pifa_forward(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, variant: int = PIFA_VARIANT_AUTO,
                  workspace_tensor=None, stream=None):
-    """Y = PIFA(X) through pifa_forward_variant. X (T x n), Wp (r x n), C ((m-r) x r) bf16 CUDA
-    tensors; pivot_idx / nonpivot_idx int32 CUDA tensors. Allocates Y (T x m) if not given."""
+    """Y = PIFA(X) through pifa_forward_variant. X (T x n), Wp (r x n) bf16 CUDA tensors; C
+    ((m-r) x r) bf16 or fp16; pivot_idx / nonpivot_idx int32 CUDA tensors. Allocates Y (T x m)
+    if not given."""
     import torch
     T, n = X.shape
     r = Wp.shape[0]
@@ -215,7 +248,8 @@ def pifa_forward(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, variant: int = PIFA_
     if Y is None:
         Y = torch.empty((T, m), dtype=torch.bfloat16, device=X.device)
     has_np = m > r
-    need = pifa_workspace_size(T, m, n, r, variant)
+    cdt = c_dtype_of(C if has_np else None)
+    need = pifa_workspace_size(T, m, n, r, variant, cdt)
     ws = workspace_tensor
     if need > 0 and ws is None:
         ws = workspace(need, X.device, stream)
@@ -225,7 +259,7 @@ def pifa_forward(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, variant: int = PIFA_
     ws_bytes = 0 if ws is None else ws.numel() * ws.element_size() - (ws_ptr - ws.data_ptr())
     st = _lib().pifa_forward_variant(
         X.data_ptr(), T, n, _ld(X), Wp.data_ptr(), r, _ld(Wp),
-        C.data_ptr() if has_np else None, m, _ld(C) if has_np else r,
+        C.data_ptr() if has_np else None, m, _ld(C) if has_np else r, cdt,
         pivot_idx.data_ptr(), nonpivot_idx.data_ptr() if has_np else None,
         Y.data_ptr(), _ld(Y), ws_ptr or None, ws_bytes, variant, _stream_ptr(stream))
     _check(st, "pifa_forward")

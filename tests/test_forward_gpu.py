@@ -40,11 +40,12 @@ DEV = torch.device("cuda:0")
 
 
 class Layer:
-    def __init__(self, pivots, nonpivots, Wp, C, name):
+    def __init__(self, pivots, nonpivots, Wp, C, name, c_dtype="bf16"):
         self.pivots = np.asarray(pivots, np.int64)
         self.nonpivots = np.asarray(nonpivots, np.int64)
         self.Wp = inputs.round_bf16(Wp)          # the exact operand values both sides use
-        self.C = inputs.round_bf16(C)
+        self.c_dtype = c_dtype
+        self.C = inputs.round_bf16(C) if c_dtype == "bf16" else inputs.round_fp16(C)
         self.m = self.pivots.size + self.nonpivots.size
         self.r, self.n = self.Wp.shape
         self.name = name
@@ -53,7 +54,8 @@ class Layer:
     def dev(self, ldwp=None, ldc=None):
         """Device copies (bf16 / int32); optional padded pitches with NaN in the padding."""
         Wp = _pad_dev(self.Wp, ldwp)
-        C = _pad_dev(self.C, ldc) if self.C.size else torch.empty((0, self.r), dtype=torch.bfloat16, device=DEV)
+        cdt = torch.bfloat16 if self.c_dtype == "bf16" else torch.float16
+        C = _pad_dev(self.C, ldc, cdt) if self.C.size else torch.empty((0, self.r), dtype=cdt, device=DEV)
         piv = torch.from_numpy(self.pivots.astype(np.int32)).to(DEV)
         nonp = torch.from_numpy(self.nonpivots.astype(np.int32)).to(DEV)
         return Wp, C, piv, nonp
@@ -63,24 +65,25 @@ def _round8(v):
     return (v + 7) // 8 * 8
 
 
-def _pad_dev(a32, ld=None):
-    """Device bf16 copy with row pitch ld (default: cols rounded up to 8, the 16-byte rule)."""
+def _pad_dev(a32, ld=None, dtype=torch.bfloat16):
+    """Device copy (bf16 or fp16; values already exact in that type) with row pitch ld (default:
+    cols rounded up to 8, the 16-byte rule) and NaN in the padding."""
     rows, cols = a32.shape
     ld = ld or _round8(cols)
-    buf = torch.full((rows, ld), float("nan"), dtype=torch.bfloat16, device=DEV)
-    buf[:, :cols] = torch.from_numpy(np.ascontiguousarray(a32)).to(DEV).to(torch.bfloat16)
+    buf = torch.full((rows, ld), float("nan"), dtype=dtype, device=DEV)
+    buf[:, :cols] = torch.from_numpy(np.ascontiguousarray(a32)).to(DEV).to(dtype)
     return buf[:, :cols]
 
 
 @functools.lru_cache(maxsize=None)
-def layer_for(m, n, r, seed, source):
+def _compressed(m, n, r, seed, source):
     U, V, _ = inputs.make_factors(m, n, r, seed)
     if source == "oracle_greedy":
         L = oracle.compress(U, V, r, "greedy")
-        return Layer(L.pivots, L.nonpivots, L.Wp, L.C, f"{m}x{n}r{r}/oracle")
+        return L.pivots, L.nonpivots, L.Wp, L.C
     if source == "oracle_lapack":
         L = oracle.compress(U, V, r, "lapack")
-        return Layer(L.pivots, L.nonpivots, L.Wp, L.C, f"{m}x{n}r{r}/oracle-lapack")
+        return L.pivots, L.nonpivots, L.Wp, L.C
     if source == "library":
         piv, nonp, Wp, C, _ = P.pifa_compress(U, V, r)
         # the oracle checks Eq. 1 and Eq. 2 on a sample of rows of W' = U V^T
@@ -93,11 +96,16 @@ def layer_for(m, n, r, seed, source):
             err = np.linalg.norm(C[rows] @ Wp - Wnp_s) / np.linalg.norm(Wnp_s)
             assert err <= 1e-10
         assert P.pifa_validate_indices(piv, nonp, m, r) == P.PIFA_OK
-        return Layer(piv, nonp, Wp, C, f"{m}x{n}r{r}/library")
+        return piv, nonp, Wp, C
     if source == "synthetic":
-        piv, nonp, Wp, C = inputs.synthetic_layer(m, n, r, seed)
-        return Layer(piv, nonp, Wp, C, f"{m}x{n}r{r}/synthetic")
+        return inputs.synthetic_layer(m, n, r, seed)
     raise ValueError(source)
+
+
+@functools.lru_cache(maxsize=None)
+def layer_for(m, n, r, seed, source, c_dtype="bf16"):
+    piv, nonp, Wp, C = _compressed(m, n, r, seed, source)
+    return Layer(piv, nonp, Wp, C, f"{m}x{n}r{r}/{source}/C-{c_dtype}", c_dtype)
 
 
 def acts(T, n, seed):
@@ -278,3 +286,113 @@ def test_prefill_variants_agree_with_decode_at_t16():
     ref = oracle.forward(X, L.Wp, L.C, L.pivots, L.nonpivots)
     check(a, ref, "decode")
     check(b, ref, "prefill_split")
+
+
+# ---------------------------------------------------------------------------------------------
+# C stored as fp16: decode, split prefill (single fp16 pass) and the fused cluster kernel
+# ---------------------------------------------------------------------------------------------
+FUSED = P.PIFA_VARIANT_PREFILL_FUSED
+SPLIT = P.PIFA_VARIANT_PREFILL_SPLIT
+
+
+def test_fp16_c_tiny_all_variants():
+    L = layer_for(256, 256, 128, 0, "oracle_greedy", "fp16")
+    for v in (P.PIFA_VARIANT_DECODE, SPLIT, FUSED):
+        parity(L, 16, v)
+
+
+@pytest.mark.parametrize("T", [1, 8, 16])
+def test_fp16_c_attn7b_decode(T):
+    parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16"), T)
+
+
+def test_selector_picks_fused_prefill():
+    assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == FUSED, P.pifa_last_error()
+    assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == FUSED, P.pifa_last_error()
+    assert P.pifa_select_variant(16, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
+
+
+def test_bf16_c_fused_attn7b_and_ragged():
+    parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack"), 2048, FUSED)
+    L = layer_for(300, 200, 77, 3, "oracle_greedy")
+    for T in (1, 17, 300):
+        parity(L, T, FUSED)
+
+
+@pytest.mark.parametrize("T,sample", [(2048, None), (8192, 512), (300, None), (17, None)])
+def test_fp16_c_attn7b_fused(T, sample):
+    L = layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16")
+    parity(L, T, FUSED, sample=sample)
+
+
+@pytest.mark.parametrize("T", [2048])
+def test_fp16_c_attn7b_split(T):
+    parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16"), T, SPLIT)
+
+
+@pytest.mark.parametrize("frac", [0.25, 0.4, 0.6, 0.75])
+def test_fp16_c_rank_sweep_fused(frac):
+    r = int(np.floor(frac * 4096 + 0.5))
+    parity(layer_for(4096, 4096, r, 0, "oracle_lapack", "fp16"), 2048, FUSED, sample=512)
+
+
+@pytest.mark.parametrize("T", [1, 2048])
+def test_fp16_c_mlp7b(T):
+    for m, n, seed in ((11008, 4096, 0), (4096, 11008, 2)):
+        parity(layer_for(m, n, 2048, seed, "library", "fp16"), T, sample=384)
+
+
+@pytest.mark.parametrize("T", [16, 4096])
+def test_fp16_c_llama70b(T):
+    parity(layer_for(8192, 8192, 4096, 0, "library", "fp16"), T, sample=256)
+    parity(layer_for(28672, 8192, 4096, 0, "synthetic", "fp16"), T, sample=128)
+
+
+@pytest.mark.parametrize("T", [1, 17, 100, 300, 513])
+def test_fp16_c_ragged_fused_and_split(T):
+    L = layer_for(300, 200, 77, 3, "oracle_greedy", "fp16")
+    for v in ([SPLIT, FUSED] if T > 16 else [P.PIFA_VARIANT_DECODE, SPLIT, FUSED]):
+        parity(L, T, v)
+
+
+@pytest.mark.parametrize("variant", [P.PIFA_VARIANT_DECODE, SPLIT, FUSED])
+def test_fp16_c_full_rank_and_rank_one(variant):
+    parity(layer_for(64, 128, 64, 4, "oracle_greedy", "fp16"), 16 if variant == P.PIFA_VARIANT_DECODE else 40,
+           variant)
+    parity(layer_for(40, 48, 1, 5, "oracle_greedy", "fp16"), 12, variant)
+
+
+def test_fp16_c_fused_deterministic_and_padded():
+    L = layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16")
+    X = acts(600, 4096, 7)
+    a = run(L, X, FUSED)
+    b = run(L, X, FUSED, ldx=4104, ldwp=4112, ldc=2056, ldy_pad=24)
+    assert np.array_equal(a, b)
+
+
+# ---------------------------------------------------------------------------------------------
+# failure detection without a GPU fault
+# ---------------------------------------------------------------------------------------------
+def test_wait_timeout_is_reported_and_recoverable():
+    """Failure detection without a GPU fault: a kernel waits, with a 2 ms bound, on an mbarrier
+    that nothing arrives on. The wait runs out, PIFA_ERR_TIMEOUT is latched and read back, the
+    context stays usable, and a forward pass right after is correct."""
+    L = layer_for(256, 256, 128, 0, "oracle_greedy")
+    try:
+        P.pifa_set_wait_timeout(2_000_000)
+        P.pifa_selftest_wait_timeout()
+        assert P.pifa_device_status() == P.PIFA_ERR_TIMEOUT
+        assert P.pifa_device_status() == P.PIFA_OK       # read-and-clear
+    finally:
+        P.pifa_set_wait_timeout(0)
+    for v in (P.PIFA_VARIANT_DECODE, P.PIFA_VARIANT_PREFILL_SPLIT, P.PIFA_VARIANT_PREFILL_FUSED):
+        parity(L, 16, v)
+
+
+def test_workspace_shared_across_shapes_and_variants():
+    """One workspace (the binding's per-stream cache) serves decode at several T, then prefill,
+    then decode again: the reserved head stays valid across shapes and variants."""
+    L = layer_for(300, 200, 77, 3, "oracle_greedy")
+    for T, v in ((8, P.PIFA_VARIANT_DECODE), (1, P.PIFA_VARIANT_DECODE), (100, SPLIT), (16, P.PIFA_VARIANT_DECODE),
+                 (300, FUSED), (3, P.PIFA_VARIANT_DECODE)):
+        parity(L, T, v)

@@ -53,17 +53,25 @@ def test_selector(lib):
     v = P.pifa_select_variant(2048, 4096, 4096, 2048)
     assert v in (P.PIFA_VARIANT_PREFILL_SPLIT, P.PIFA_VARIANT_PREFILL_FUSED)
     assert P.pifa_select_variant(17, 256, 256, 128) != P.PIFA_VARIANT_DECODE
+    # without a GPU the cluster kernel cannot be planned: the selector falls back to the split one
+    assert P.pifa_select_variant(4096, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) in (
+        P.PIFA_VARIANT_PREFILL_SPLIT, P.PIFA_VARIANT_PREFILL_FUSED)
     with pytest.raises(P.PifaError):
         P.pifa_select_variant(1, 100, 50, 60)      # r > n
 
 
 def test_workspace_sizes(lib):
     # decode: fp32 y_p, T rows of pitch round_up(r, 8)
-    assert P.pifa_workspace_size(8, 4096, 4096, 2048, P.PIFA_VARIANT_DECODE) == 8 * 2048 * 4
+    # every size includes the 256 reserved bytes at the head of the workspace
+    assert P.pifa_workspace_size(8, 4096, 4096, 2048, P.PIFA_VARIANT_DECODE) == 256 + 8 * 2048 * 4
     assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) % 256 == 0
-    assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) >= 3 * 1640 * 4
-    # split prefill: two bf16 T x round_up(r, 8) matrices
-    assert P.pifa_workspace_size(2048, 4096, 4096, 2048, P.PIFA_VARIANT_PREFILL_SPLIT) == 2 * 2048 * 2048 * 2
+    assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) >= 256 + 3 * 1640 * 4
+    # split and fused prefill: Y_p hi and lo, two 2-byte T x round_up(r, 8) matrices
+    assert P.pifa_workspace_size(2048, 4096, 4096, 2048, P.PIFA_VARIANT_PREFILL_SPLIT) == 256 + 2 * 2048 * 2048 * 2
+    assert P.pifa_workspace_size(2048, 4096, 4096, 2048, P.PIFA_VARIANT_PREFILL_SPLIT,
+                                 P.PIFA_DTYPE_FP16) == 256 + 2 * 2048 * 2048 * 2
+    assert P.pifa_workspace_size(2048, 4096, 4096, 1638, P.PIFA_VARIANT_PREFILL_FUSED,
+                                 P.PIFA_DTYPE_FP16) == 256 + 2 * 2048 * 1640 * 2
     assert P.pifa_workspace_size(0, 4096, 4096, 2048, P.PIFA_VARIANT_AUTO) == 0
     with pytest.raises(P.PifaError) as e:
         P.pifa_workspace_size(4, 10, 10, 11, P.PIFA_VARIANT_AUTO)   # r > min(m, n)
@@ -84,12 +92,12 @@ def test_validate_indices(lib):
 def _fwd_raw(lib, **kw):
     """pifa_forward_variant with fake (never dereferenced) pointers, for argument checks only."""
     a = dict(X=0x10000, T=4, n=64, ldx=64, Wp=0x20000, r=16, ldwp=64, C=0x30000, m=48, ldc=16,
-             piv=0x40000, nonpiv=0x50000, Y=0x60000, ldy=48, ws=0x70000, wsb=1 << 20,
-             variant=P.PIFA_VARIANT_AUTO)
+             cdt=P.PIFA_DTYPE_BF16, piv=0x40000, nonpiv=0x50000, Y=0x60000, ldy=48, ws=0x70000,
+             wsb=1 << 20, variant=P.PIFA_VARIANT_AUTO)
     a.update(kw)
     return lib.pifa_forward_variant(a["X"], a["T"], a["n"], a["ldx"], a["Wp"], a["r"], a["ldwp"], a["C"],
-                                    a["m"], a["ldc"], a["piv"], a["nonpiv"], a["Y"], a["ldy"], a["ws"],
-                                    a["wsb"], a["variant"], None)
+                                    a["m"], a["ldc"], a["cdt"], a["piv"], a["nonpiv"], a["Y"], a["ldy"],
+                                    a["ws"], a["wsb"], a["variant"], None)
 
 
 def test_forward_argument_errors(lib):
@@ -106,11 +114,13 @@ def test_forward_argument_errors(lib):
     assert _fwd_raw(lib, Y=0x10000 + 64) == E.PIFA_ERR_INVALID_ARG   # Y overlaps X
     assert "overlap" in _last(lib)
     assert _fwd_raw(lib, variant=9) == E.PIFA_ERR_INVALID_ARG
+    assert _fwd_raw(lib, cdt=7) == E.PIFA_ERR_INVALID_ARG
     assert _fwd_raw(lib, variant=P.PIFA_VARIANT_DECODE, T=17) == E.PIFA_ERR_UNSUPPORTED
     assert _fwd_raw(lib, wsb=16) == E.PIFA_ERR_WORKSPACE
     assert _fwd_raw(lib, ws=None) == E.PIFA_ERR_WORKSPACE
     assert _fwd_raw(lib, ws=0x70010) == E.PIFA_ERR_ALIGNMENT
     assert _fwd_raw(lib, T=0) == E.PIFA_OK                           # no-op, no device touched
+    assert _fwd_raw(lib, wsb=256) == E.PIFA_ERR_WORKSPACE             # only the reserved head
 
 
 def _last(lib):

@@ -66,7 +66,7 @@ def test_noalloc_decode_matches_pifa_forward_twice():
 def test_noalloc_rejects_sizes_beyond_the_static_scratch():
     lib = P.load()
     fake = 0x100000                              # never dereferenced: rejected before any launch
-    # T * round_up(r, 8) * 4 bytes: 16 * 16384 * 4 = 1 MiB fits, r = 16392 does not
+    # 256 + T * round_up(r, 8) * 4 bytes must fit in 1 MiB: r = 16392 at T = 16 does not
     st = lib.pifa_forward_decode_noalloc(fake, 16, 20000, 20000, fake * 2, 16392, 20000, fake * 3,
                                          20000, 16392, fake * 4, fake * 5, fake * 6, 20000, None)
     assert st == P.PIFA_ERR_WORKSPACE
