@@ -84,14 +84,14 @@ typedef struct {
  *                exactly once (round to nearest even from the fp32 accumulator); the padding
  *                columns m..ldy-1 are not touched. Y must not overlap any input.
  *   workspace    DEVICE scratch of at least pifa_workspace_size(T, m, n, r, c_dtype, variant) bytes,
- *                256-byte aligned. Its first 256 bytes are library state (the decode kernel's
- *                grid-barrier words): zero-fill the workspace once before its first use (e.g. a
- *                cudaMemset at allocation); every completed call leaves those bytes zero again,
- *                for any shape and variant. After a call that returned or latched
- *                PIFA_ERR_TIMEOUT, zero them again. A workspace must not be used by another call
- *                that may run concurrently.
+ *                256-byte aligned; it needs no initialisation. Its first 256 bytes are reserved
+ *                for library state (no kernel of this version reads or writes them); the rest
+ *                holds Y_p between the two contractions. A workspace must not be used by another
+ *                call that may run concurrently.
  *   cuda_stream  a cudaStream_t (NULL = legacy default stream).
  *
+ *   Every matrix buffer spans rows x pitch elements: kernels may read a row's padding up to the
+ *   next multiple of 8 columns (never write it) and ignore what it holds.
  *   Requirements: 1 <= r <= min(m, n); T >= 0 (T == 0 is a no-op: nothing is read or written and
  *   X and Y may be NULL); every base pointer of X, Wp,
  *   C, Y 16-byte aligned and ldx, ldwp, ldc, ldy multiples of 8 (16-byte row pitch), else
@@ -126,18 +126,17 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx,
  * acceptable. The paper has no counterpart; it is an interface convenience of this library.
  *
  *   Arguments, layouts and errors as pifa_forward with C in bf16, without the workspace: the
- *   call allocates
- *   nothing (no cudaMalloc, cudaFree or allocating library routine). Its scratch -- 256 bytes of
- *   grid-barrier words, then y_p in fp32 (T rows of pitch round_up(r, 8)) -- lives in a 1 MiB
- *   array in this library's static device data, which every GPU that loads the library holds
- *   until the process exits. Shapes with 256 + T * round_up(r, 8) * 4 > 1 MiB are rejected
- *   with PIFA_ERR_WORKSPACE; T > 16 with PIFA_ERR_UNSUPPORTED.
+ *   call allocates nothing (no cudaMalloc, cudaFree or allocating library routine). Its scratch
+ *   -- 256 reserved bytes, then y_p as bf16 hi and lo planes (T rows of pitch round_up(r, 8)
+ *   each) -- lives in a 1 MiB array in this library's static device data, which every GPU that
+ *   loads the library holds until the process exits. Shapes with
+ *   256 + T * round_up(r, 8) * 4 > 1 MiB are rejected with PIFA_ERR_WORKSPACE; T > 16 with
+ *   PIFA_ERR_UNSUPPORTED.
  *   The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
  *   that device current; make that first call before any stream capture. Every call on a device
- *   shares the one array and it keeps the last call's contents: the barrier words start at zero
- *   (static data is zero-initialised) and every completed call leaves them zero; y_p is fully
- *   written before it is read. Calls that may overlap on the GPU, e.g. on different streams,
- *   race on the array.
+ *   shares the one array and it keeps the last call's contents, which no call depends on: y_p is
+ *   fully written before it is read. Calls that may overlap on the GPU, e.g. on different
+ *   streams, race on the array.
  */
 int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, int64_t ldx,
                                 const void* Wp, int64_t r, int64_t ldwp,

@@ -220,8 +220,7 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const
   if (!status) return pifa_fail_cuda("device status word", cerr);
 
   PifaPointers p = {X, Wp, has_np ? C : nullptr, pivot_idx, has_np ? nonpivot_idx : nullptr, Y,
-                    static_cast<uint8_t*>(workspace) + kWorkspaceReserve, workspace_bytes - kWorkspaceReserve,
-                    static_cast<unsigned*>(workspace)};
+                    static_cast<uint8_t*>(workspace) + kWorkspaceReserve, workspace_bytes - kWorkspaceReserve};
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(cuda_stream);
   switch (variant) {
     case PIFA_VARIANT_DECODE: return launch_decode(s, p, status, stream);

@@ -1,30 +1,33 @@
 // decode.cu -- PIFA forward for small token counts (T <= 16): Algorithm 2 as two HBM-streaming
-// GEMV phases.
+// phases, one kernel each.
 //
-//   phase 1: Y_p = X W_p^T   (r rows of W_p streamed once)   -> y_p fp32 in the workspace,
-//            Y[:, I[j]] = bf16(Y_p[:, j])                     (Algorithm 2, steps 2 and 4)
-//   phase 2: Y_np = Y_p C^T  (m - r rows of C streamed once)  -> Y[:, I^c[i]] = bf16(Y_np[:, i])
-//                                                              (Algorithm 2, steps 3 and 5)
+//   phase 1: Y_p = X W_p^T  (the r rows of W_p, each read once)  -> Y[:, I[j]] = bf16(Y_p[:, j]),
+//            and y_p to the workspace as a hi + lo pair of C's dtype  (Algorithm 2, steps 2 and 4)
+//   phase 2: Y_np = Y_p C^T (the m - r rows of C, each read once) -> Y[:, I^c[i]] = bf16(Y_np[:, i])
+//                                                                     (Algorithm 2, steps 3 and 5)
 //
-// The work is memory bound: every weight byte is read exactly once; x and y_p are tiny and stay in
-// L1/L2. One CTA (16 warps) owns 16 consecutive weight rows (one m16 MMA fragment); its warps split
-// the K dimension. For a 32-wide K step, lane (g = lane/4, c = lane%4) holds 8 consecutive elements
-// of rows g and g+8 at offset 8c and uses them directly as the A fragments of two m16n8k16 MMAs,
-// permuting K identically in both operands (a dot product does not depend on the order of its
-// terms): MMA step s takes elements 4s..4s+3. The lane loads the matching 8 activations of token g
-// as the B fragment. Warps then reduce their 16 x 8 partial tiles through shared memory.
+// Both phases have one shape. A CTA owns 16 consecutive weight rows (one m16 MMA fragment). At
+// launch -- before it waits on its predecessor (programmatic dependent launch, PDL) -- one thread
+// bulk-copies the CTA's rows into shared memory: all of K when it fits, else K-chunks through two
+// stages refilled as they are used. The weights do not depend on the previous kernel, so their
+// HBM traffic overlaps its compute: phase 2 stages its rows of C while phase 1 computes, and the
+// next call's phase 1 stages its W_p while this call's phase 2 computes. The stage budgets let a
+// phase-1 CTA and a phase-2 CTA share one SM.
 //
-// Both phases are launched with programmatic dependent launch (PDL) and start their weight traffic
-// before waiting on the previous kernel: phase 1 bulk-prefetches its W_p rows into L2 and then
-// streams them with 128-bit loads straight into registers; phase 2 -- launched while phase 1 still
-// runs -- bulk-copies its rows of C into shared memory (rows 64 bytes apart beyond their length, so
-// fragment loads hit eight different bank groups per quarter warp). Only after griddepcontrol.wait
-// do they read X or y_p or write outputs. The next call's phase 1 likewise starts pulling its W_p
-// while this call's phase 2 computes.
+// Once the predecessor has completed, each warp loads the B fragments of its K-steps (x for
+// phase 1; the y_p hi and lo planes for phase 2) from L2 into registers in one batch and runs
+// mma.sync.m16n8k16 over its steps with A from shared memory. For a 32-wide K step, lane
+// (g = lane/4, c = lane%4) takes 8 consecutive elements of rows g and g+8 at offset 8c as the A
+// fragments of two k16 MMAs and the matching 8 elements of token g as its B fragment: K is
+// permuted identically in both operands, which a dot product does not notice. The warps' 16 x 8
+// partial tiles are summed through shared memory in a fixed order (the result is deterministic).
+//
 // y_p enters the second contraction as a hi + lo pair of C's storage type (bf16 or fp16): C has
 // large entries and Y_np = C Y_p cancels, so rounding y_p to one bf16 alone would amplify its
-// rounding error several-fold.
+// rounding error several-fold. Phase 1 splits each value once; phase 2 runs one MMA per plane.
+#include <map>
 #include <mutex>
+#include <utility>
 
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
@@ -38,34 +41,33 @@ namespace {
 using namespace pifa;
 using bf16 = __nv_bfloat16;
 
-constexpr int kRows = 16;       // weight rows per CTA
-constexpr int kChunk = 32;      // K elements per warp step (two k16 MMAs)
-constexpr int kRowPad = 64;     // bytes between consecutive rows of a stage beyond their length
+constexpr int kRows = 16;    // weight rows per CTA
+constexpr int kChunk = 32;   // K elements per warp step (two k16 MMAs)
+constexpr int kRowPad = 64;  // bytes between consecutive staged rows beyond their length
+constexpr int kWarps = 8;    // warps per CTA, both phases
+// Shared-memory budgets of the weight stages of one CTA. 136 KB (phase 1) + 70 KB (phase 2) and
+// the small rest fit in one SM's 228 KB, so a phase-2 CTA can stage its rows of C beside a
+// computing phase-1 CTA (and a phase-1 CTA its rows of W_p beside a phase-2 CTA).
+constexpr uint32_t kStageBudget1 = 136u * 1024u;
+constexpr uint32_t kStageBudget2 = 70u * 1024u;
+// K steps whose B fragments a warp holds in registers at once: 64 registers for any NT and NB
+template <int NT, int NB>
+constexpr int kBatch = 16 / (NT * NB);
 
 __device__ __forceinline__ uint32_t pack2(uint16_t a, uint16_t b) { return (uint32_t)a | ((uint32_t)b << 16); }
 
-// 8 consecutive bf16 of `row` starting at column k; zero beyond column K or for an invalid row.
-// kStream: weights read exactly once, not allocated in L1.
-// kCoherent: data another kernel may have just written (L2 only, never a stale L1 line).
-template <bool kStream = false, bool kCoherent = false>
-__device__ __forceinline__ uint4 load8_bf16(const bf16* __restrict__ base, int64_t ld, int64_t row, bool row_ok,
-                                            int k, int K) {
-  uint4 v = make_uint4(0u, 0u, 0u, 0u);
-  if (!row_ok || k >= K) return v;
-  const bf16* p = base + row * ld + k;
-  if (k + 8 <= K) {
-    if (kStream) return ld_stream_16(p);
-    if (kCoherent) return __ldcg(reinterpret_cast<const uint4*>(p));
-    return __ldg(reinterpret_cast<const uint4*>(p));
-  }
+// 8 consecutive 16-bit elements of row `row` starting at column k; zero beyond column K or when
+// !ok. Read through L2 only (ld.global.cg): the data may have been written by the previous kernel
+// and a stale L1 line must never be used.
+__device__ __forceinline__ uint4 ldg8_cg(const uint16_t* __restrict__ base, int64_t ld, int row, bool ok, int k,
+                                         int K) {
+  if (!ok || k >= K) return make_uint4(0u, 0u, 0u, 0u);
+  const uint16_t* p = base + (int64_t)row * ld + k;
+  if (k + 8 <= K) return __ldcg(reinterpret_cast<const uint4*>(p));
   uint16_t e[8];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) e[i] = (k + i < K) ? __bfloat16_as_ushort(p[i]) : (uint16_t)0;
-  v.x = pack2(e[0], e[1]);
-  v.y = pack2(e[2], e[3]);
-  v.z = pack2(e[4], e[5]);
-  v.w = pack2(e[6], e[7]);
-  return v;
+  for (int i = 0; i < 8; ++i) e[i] = (k + i < K) ? __ldcg(p + i) : (uint16_t)0;
+  return make_uint4(pack2(e[0], e[1]), pack2(e[2], e[3]), pack2(e[4], e[5]), pack2(e[6], e[7]));
 }
 
 // 8 weights of one staged row at local column kl; elements at or beyond `len` are zeroed (the
@@ -78,8 +80,7 @@ __device__ __forceinline__ uint4 lds8_masked(const uint8_t* rowp, int kl, int le
     uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      const int e0 = 2 * i, e1 = 2 * i + 1;
-      const uint32_t m0 = e0 < keep ? 0x0000FFFFu : 0u, m1 = e1 < keep ? 0xFFFF0000u : 0u;
+      const uint32_t m0 = 2 * i < keep ? 0x0000FFFFu : 0u, m1 = 2 * i + 1 < keep ? 0xFFFF0000u : 0u;
       w[i] &= (m0 | m1);
     }
     v = make_uint4(w[0], w[1], w[2], w[3]);
@@ -106,204 +107,59 @@ __device__ __forceinline__ void split2(float f, uint16_t& h, uint16_t& l, bool& 
   }
 }
 
-// 8 consecutive fp32 y_p values of one token at column k (zero beyond K), split into hi and lo.
 template <bool kF16>
-__device__ __forceinline__ void load8_split(const float* __restrict__ yp, bool t_ok, int k, int K, uint4& hi,
-                                            uint4& lo, bool& range_err) {
-  float f[8];
-  if (t_ok && k + 8 <= K) {
-    const float4 a = __ldcg(reinterpret_cast<const float4*>(yp + k));
-    const float4 b = __ldcg(reinterpret_cast<const float4*>(yp + k + 4));
-    f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
-    f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) f[i] = (t_ok && k + i < K) ? __ldcg(yp + k + i) : 0.0f;
-  }
-  uint16_t h[8], l[8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i) split2<kF16>(f[i], h[i], l[i], range_err);
-  hi = make_uint4(pack2(h[0], h[1]), pack2(h[2], h[3]), pack2(h[4], h[5]), pack2(h[6], h[7]));
-  lo = make_uint4(pack2(l[0], l[1]), pack2(l[2], l[3]), pack2(l[4], l[5]), pack2(l[6], l[7]));
-}
-
-// 8 consecutive fp32 y_p values of one token at column k from its staged row in shared memory
-// (zero beyond K or for an absent token), split into hi and lo.
-template <bool kF16>
-__device__ __forceinline__ void lds8_split(const float* row, bool t_ok, int k, int K, uint4& hi, uint4& lo,
-                                           bool& range_err) {
-  float f[8];
-  if (t_ok && k + 8 <= K) {
-    const float4 a = *reinterpret_cast<const float4*>(row + k);
-    const float4 b = *reinterpret_cast<const float4*>(row + k + 4);
-    f[0] = a.x; f[1] = a.y; f[2] = a.z; f[3] = a.w;
-    f[4] = b.x; f[5] = b.y; f[6] = b.z; f[7] = b.w;
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) f[i] = (t_ok && k + i < K) ? row[k + i] : 0.0f;
-  }
-  uint16_t h[8], l[8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i) split2<kF16>(f[i], h[i], l[i], range_err);
-  hi = make_uint4(pack2(h[0], h[1]), pack2(h[2], h[3]), pack2(h[4], h[5]), pack2(h[6], h[7]));
-  lo = make_uint4(pack2(l[0], l[1]), pack2(l[2], l[3]), pack2(l[4], l[5]), pack2(l[6], l[7]));
+__device__ __forceinline__ void mma16816(float (&d)[4], const uint4& wa, const uint4& wb, uint32_t b0, uint32_t b1,
+                                         bool upper) {
+  const uint32_t a0 = upper ? wa.z : wa.x, a1 = upper ? wb.z : wb.x;
+  const uint32_t a2 = upper ? wa.w : wa.y, a3 = upper ? wb.w : wb.y;
+  if (kF16)
+    mma_m16n8k16_f16(d, a0, a1, a2, a3, b0, b1);
+  else
+    mma_m16n8k16_bf16(d, a0, a1, a2, a3, b0, b1);
 }
 
 struct DecodeArgs {
-  const uint16_t* A;     // weight rows (W_p for phase 1, C for phase 2), 2-byte elements
+  const uint16_t* A;    // weight rows: W_p (phase 1) or C (phase 2), 2-byte elements
   int64_t lda;
-  int R, K;              // rows and columns of A
-  const bf16* X;         // phase 1: activations T x K
-  int64_t ldx;
-  float* yp;             // y_p, T rows of pitch ldyp (phase 1 writes it, phase 2 reads it)
+  int R, K;             // rows and columns of A
+  const uint16_t* B0;   // B operand, T rows of K: X (phase 1) or the y_p hi plane (phase 2)
+  const uint16_t* B1;   // phase 2: the y_p lo plane
+  int64_t ldb;
+  uint16_t* yph;        // phase 1 with m > r: y_p as hi and lo planes, T rows of pitch ldyp each
+  uint16_t* ypl;
   int64_t ldyp;
-  const int32_t* cols;   // output column of each weight row (I or I^c)
+  const int32_t* cols;  // output column of each weight row (I or I^c)
   int m;
   bf16* Y;
   int64_t ldy;
   int T;
-  int kc;                // phase 2: K columns per shared-memory stage (multiple of 32)
-  int stages;            // phase 2: 1 (all of K resident) or 2
+  int kc;               // K columns per shared-memory stage (multiple of 32)
+  int stages;           // 1 (all of K resident) or 2
   int* status;
   uint64_t timeout_ns;
 };
 
-constexpr int kWarps = 16;                 // phase 1 warps per CTA
-// Phase 2 runs 8 warps so that one of its CTAs fits in the registers an SM has left beside a
-// phase-1 CTA: phase 2 can then launch (PDL) and pull its C rows while phase 1 still streams W_p.
-constexpr int kWarps2 = 8;
-template <int NT>
-constexpr int kUnroll2 = 2;  // phase 2: 32-column steps in flight per warp
-// phase 1: 32-column steps in flight per warp (fewer with two token tiles, to stay in 64 registers)
-template <int NT>
-constexpr int kUnroll1 = NT == 1 ? 4 : 2;
-
-// Cross-warp reduction of the per-warp 16 x (8*NT) partial tiles, then the outputs of this CTA's
-// 16 rows: y_p (phase 1 only) and the bf16 values in their output columns of Y.
-template <int NT, int PHASE, int WARPS>
-__device__ __forceinline__ void reduce_and_store(const DecodeArgs& a, float (*red)[kRows][8 * NT],
-                                                 const float (&acc)[NT][4], int64_t row0, int nrows,
-                                                 const int* s_cols) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, c = lane & 3;
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
-    red[warp][g][nt * 8 + 2 * c] = acc[nt][0];
-    red[warp][g][nt * 8 + 2 * c + 1] = acc[nt][1];
-    red[warp][g + 8][nt * 8 + 2 * c] = acc[nt][2];
-    red[warp][g + 8][nt * 8 + 2 * c + 1] = acc[nt][3];
-  }
-  __syncthreads();
-  for (int idx = threadIdx.x; idx < kRows * 8 * NT; idx += WARPS * 32) {
-    const int row = idx / (8 * NT), t = idx % (8 * NT);
-    if (t >= a.T || row >= nrows) continue;
-    float sum = 0.0f;
-#pragma unroll
-    for (int w = 0; w < WARPS; ++w) sum += red[w][row][t];
-    const int64_t i = row0 + row;
-    if (PHASE == 1) a.yp[(int64_t)t * a.ldyp + i] = sum;
-    const int col = s_cols[row];
-    if ((unsigned)col >= (unsigned)a.m) {
-      latch_status(a.status, PIFA_ERR_DEVICE_INDEX);
-      continue;
-    }
-    a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(sum);
-  }
-}
-
-// The output columns of this CTA's rows are layer constants: read them at launch, before waiting
-// on the previous kernel, so no dependent global load is left for the end of the kernel.
-__device__ __forceinline__ void load_cols(const DecodeArgs& a, int64_t row0, int nrows, int* s_cols) {
-  if (threadIdx.x < kRows) s_cols[threadIdx.x] = threadIdx.x < nrows ? a.cols[row0 + threadIdx.x] : 0;
-}
-
-// ---- phase 1: Y_p = X W_p^T, streamed with 128-bit loads straight into MMA fragments ----------
-template <int NT>
-__global__ void __launch_bounds__(kWarps * 32) decode_pivot_rows(DecodeArgs a) {
-  __shared__ float red[kWarps][kRows][8 * NT];
+// One CTA: weight rows row0 .. row0 + 15 against the T tokens. PHASE 1: bf16 MMAs against x, and
+// y_p split in C's dtype (kF16C). PHASE 2: MMAs in C's dtype against the y_p hi and lo planes.
+template <int PHASE, int NT, bool kF16C>
+__global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
+  constexpr int NB = PHASE == 1 ? 1 : 2;  // B planes
+  constexpr bool kF16Mma = PHASE == 2 && kF16C;
+  constexpr int NBATCH = kBatch<NT, NB>;
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ uint64_t full[2];
   __shared__ int s_cols[kRows];
-  pdl_launch_dependents();  // phase 2 may launch now and start pulling its rows of C
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, c = lane & 3;
-  const int64_t row0 = (int64_t)blockIdx.x * kRows;
-  const int nrows = (int)((int64_t)a.R - row0 < kRows ? (int64_t)a.R - row0 : kRows);
-  if (threadIdx.x < nrows)  // start this CTA's W_p rows towards L2 before waiting on anything
-    prefetch_l2_bulk(a.A + (row0 + threadIdx.x) * a.lda, ((uint32_t)a.K * 2u + 15u) & ~15u);
-  load_cols(a, row0, nrows, s_cols);
-  // One thread waits for the previous kernel (X valid, y_p and Y free) while the other warps park
-  // in the CTA barrier: warps waiting on the previous grid would otherwise compete for issue slots
-  // with the CTAs that are still working on this SM.
-  if (threadIdx.x == 0) pdl_wait_primary();
-  __syncthreads();
-  const bf16* W = reinterpret_cast<const bf16*>(a.A);
-  const bool ok0 = g < nrows, ok1 = g + 8 < nrows;
-  // one accumulator per unrolled step: independent MMA chains instead of one long dependent one
-  float accu[kUnroll1<NT>][NT][4];
-#pragma unroll
-  for (int u = 0; u < kUnroll1<NT>; ++u)
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt) accu[u][nt][0] = accu[u][nt][1] = accu[u][nt][2] = accu[u][nt][3] = 0.0f;
-  const int nchunks = (a.K + kChunk - 1) / kChunk;
-  for (int base = warp; base < nchunks; base += kWarps * kUnroll1<NT>) {
-    uint4 wa[kUnroll1<NT>], wb[kUnroll1<NT>], xv[kUnroll1<NT>][NT];
-#pragma unroll
-    for (int u = 0; u < kUnroll1<NT>; ++u) {
-      const int ch = base + u * kWarps;
-      const int k = ch * kChunk + 8 * c;
-      const bool in = ch < nchunks;
-      wa[u] = load8_bf16<true>(W, a.lda, row0 + g, in && ok0, k, a.K);
-      wb[u] = load8_bf16<true>(W, a.lda, row0 + g + 8, in && ok1, k, a.K);
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        const int t = nt * 8 + g;
-        xv[u][nt] = load8_bf16<false, true>(a.X, a.ldx, t, in && t < a.T, k, a.K);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll1<NT>; ++u) {
-#pragma unroll
-      for (int nt = 0; nt < NT; ++nt) {
-        mma_m16n8k16_bf16(accu[u][nt], wa[u].x, wb[u].x, wa[u].y, wb[u].y, xv[u][nt].x, xv[u][nt].y);
-        mma_m16n8k16_bf16(accu[u][nt], wa[u].z, wb[u].z, wa[u].w, wb[u].w, xv[u][nt].z, xv[u][nt].w);
-      }
-    }
-  }
-  float acc[NT][4];
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float v = 0.0f;
-#pragma unroll
-      for (int u = 0; u < kUnroll1<NT>; ++u) v += accu[u][nt][i];
-      acc[nt][i] = v;
-    }
-  reduce_and_store<NT, 1, kWarps>(a, red, acc, row0, nrows, s_cols);
-}
-
-// ---- phase 2: Y_np = Y_p C^T from C rows staged in shared memory -------------------------------
-// At launch (before waiting on phase 1) thread 0 bulk-copies the CTA's 16 rows of C into shared
-// memory -- all of K when it fits, else K-chunks through two stages refilled after each is used.
-template <int NT, bool kF16C, bool kYs>
-__global__ void __launch_bounds__(kWarps2 * 32) decode_nonpivot_rows(DecodeArgs a) {
-  extern __shared__ __align__(16) uint8_t smem[];
-  const uint32_t pitch = (uint32_t)(a.kc * 2 + kRowPad);
+  pdl_launch_dependents();  // the next kernel may launch now and start staging its weights
+  const uint32_t pitch = (uint32_t)a.kc * 2u + kRowPad;
   const uint32_t stage_bytes = (uint32_t)kRows * pitch;
-  // y_p staged in shared memory: T rows of ldyp floats, 16 bytes apart beyond their length so that
-  // the two float4 loads of a quarter warp fall into distinct bank groups
-  const uint32_t ypitch = (uint32_t)a.ldyp * 4u + 16u;
-  float* ys = reinterpret_cast<float*>(smem + a.stages * stage_bytes);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + a.stages * stage_bytes + (kYs ? (uint32_t)a.T * ypitch : 0u));
-  uint64_t* ybar = full + 2;
-  float(*red)[kRows][8 * NT] = reinterpret_cast<float(*)[kRows][8 * NT]>(full + 3);
-  __shared__ int s_cols[kRows];
-  pdl_launch_dependents();  // the next call's phase 1 may launch and prefetch its W_p
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, c = lane & 3;
   const int64_t row0 = (int64_t)blockIdx.x * kRows;
   const int nrows = (int)((int64_t)a.R - row0 < kRows ? (int64_t)a.R - row0 : kRows);
   const int nchunks = (a.K + a.kc - 1) / a.kc;
-  auto issue = [&](int j) {  // thread 0: chunk j into stage j % stages
+  auto issue = [&](int j) {  // thread 0: K-chunk j of the CTA's rows into stage j % stages
     const int s = j % a.stages;
     const int len = min(a.kc, a.K - j * a.kc);
-    const uint32_t bytes = (uint32_t)((len + 7) & ~7) * 2u;  // stays inside the 16-byte row pitch
+    const uint32_t bytes = (uint32_t)((len + 7) & ~7) * 2u;  // 16-byte multiple within the row pitch
     mbar_arrive_expect_tx(&full[s], bytes * (uint32_t)nrows);
     uint8_t* st = smem + s * stage_bytes;
     for (int rr = 0; rr < nrows; ++rr)
@@ -311,120 +167,174 @@ __global__ void __launch_bounds__(kWarps2 * 32) decode_nonpivot_rows(DecodeArgs 
   };
   if (threadIdx.x == 0) {
     for (int s = 0; s < a.stages; ++s) mbar_init(&full[s], 1);
-    mbar_init(ybar, 1);
     fence_mbar_init();
     for (int j = 0; j < a.stages && j < nchunks; ++j) issue(j);
   }
-  load_cols(a, row0, nrows, s_cols);
-  if (threadIdx.x == 0) pdl_wait_primary();  // phase 1 has completed: y_p is valid (see phase 1)
-  if (kYs && threadIdx.x == 0) {  // all of y_p into shared memory in T bulk copies
-    const uint32_t ybytes = (uint32_t)a.ldyp * 4u;
-    mbar_arrive_expect_tx(ybar, ybytes * (uint32_t)a.T);
-    for (int t = 0; t < a.T; ++t)
-      bulk_copy_g2s(smem_u32(reinterpret_cast<uint8_t*>(ys) + t * ypitch), a.yp + (int64_t)t * a.ldyp, ybytes, ybar);
-  }
-  __syncthreads();  // barriers initialised before anyone waits on them
-  const bool ok0 = g < nrows, ok1 = g + 8 < nrows;
-  bool range_err = false, dead = false;
-  // separate accumulators per unrolled step and per hi / lo pass: short independent MMA chains
-  float accu[kUnroll2<NT>][2][NT][4];
+  // the output columns of this CTA's rows are layer constants: read them before waiting
+  if (threadIdx.x < kRows) s_cols[threadIdx.x] = threadIdx.x < nrows ? a.cols[row0 + threadIdx.x] : 0;
+  // One thread waits for the previous kernel (its outputs visible, ours free to overwrite) while
+  // the other warps park in the CTA barrier instead of taking issue slots from co-resident CTAs.
+  if (threadIdx.x == 0) pdl_wait_primary();
+  __syncthreads();  // also: barriers initialised before anyone waits on them
+  // independent accumulator chains: the hi and lo planes in phase 2, even and odd steps in phase 1
+  constexpr int NU = NB == 1 ? 2 : 1;
+  float acc[NU][NB][NT][4];
 #pragma unroll
-  for (int u = 0; u < kUnroll2<NT>; ++u)
+  for (int u = 0; u < NU; ++u)
 #pragma unroll
-    for (int h = 0; h < 2; ++h)
+    for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) accu[u][h][nt][0] = accu[u][h][nt][1] = accu[u][h][nt][2] = accu[u][h][nt][3] = 0.0f;
-  if (kYs && !mbar_wait(ybar, 0, a.timeout_ns)) {
-    latch_status(a.status, PIFA_ERR_TIMEOUT);
-    dead = true;
-  }
+      for (int nt = 0; nt < NT; ++nt) acc[u][nb][nt][0] = acc[u][nb][nt][1] = acc[u][nb][nt][2] = acc[u][nb][nt][3] = 0.0f;
+  // This lane's B rows: token t = 8 nt + g, clamped to T - 1. The output columns of tokens >= T
+  // are computed from a duplicate row and never stored, and so are the output rows of weight
+  // rows >= nrows (their stage rows hold stale bytes): an MMA row or column only ever affects
+  // itself. Only the K tail beyond the last full step needs masking, and it gets its own step.
+  const uint16_t* brow[NB][NT];
+#pragma unroll
+  for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+      const int t = nt * 8 + g < a.T ? nt * 8 + g : a.T - 1;
+      brow[nb][nt] = (nb == 0 ? a.B0 : a.B1) + (int64_t)t * a.ldb + 8 * c;
+    }
+  bool dead = false;
   for (int j = 0; j < nchunks; ++j) {
     const int s = j % a.stages;
-    const int len = min(a.kc, a.K - j * a.kc);
-    const int steps = (len + kChunk - 1) / kChunk;
-    if (!mbar_wait(&full[s], (uint32_t)(j / a.stages) & 1u, a.timeout_ns)) {
+    const int kbase = j * a.kc;
+    const int len = min(a.kc, a.K - kbase);
+    if (!dead && !mbar_wait(&full[s], (uint32_t)(j / a.stages) & 1u, a.timeout_ns)) {
       latch_status(a.status, PIFA_ERR_TIMEOUT);
       dead = true;
     }
+    dead = __any_sync(0xffffffffu, dead);  // the MMAs below are warp-collective
     if (!dead) {
-      const uint8_t* st = smem + s * stage_bytes;
-      for (int base = warp; base < steps; base += kWarps2 * kUnroll2<NT>) {
-        uint4 hi[kUnroll2<NT>][NT], lo[kUnroll2<NT>][NT], wa[kUnroll2<NT>], wb[kUnroll2<NT>];
+      // The hot loop is kept short: this code runs once per launch, and its instruction fetch
+      // (not its arithmetic) would otherwise dominate the kernel.
+      const uint8_t* wlo = smem + s * stage_bytes + g * pitch + 16 * c;  // weight row g
+      const uint8_t* whi = wlo + 8 * pitch;                               // weight row g + 8
+      const int nfull = len / kChunk;
+      for (int s0 = warp; s0 < nfull; s0 += kWarps * NBATCH) {
+        const int nmine = min(NBATCH, (nfull - s0 + kWarps - 1) / kWarps);  // this batch's steps
+        uint4 bv[NBATCH][NB][NT];  // every load of the batch in flight together
 #pragma unroll
-        for (int u = 0; u < kUnroll2<NT>; ++u) {  // several steps' y_p loads in flight together
-          const int stp = base + u * kWarps2;
-          const int kl = stp * kChunk + 8 * c;
-          const bool in = stp < steps;
-          wa[u] = lds8_masked(st + g * pitch, kl, len, in && ok0);
-          wb[u] = lds8_masked(st + (g + 8) * pitch, kl, len, in && ok1);
+        for (int i = 0; i < NBATCH; ++i)
+          if (i < nmine)
+#pragma unroll
+            for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt)
+                bv[i][nb][nt] = __ldcg(reinterpret_cast<const uint4*>(brow[nb][nt] + kbase + (s0 + i * kWarps) * kChunk));
+#pragma unroll
+        for (int i = 0; i < NBATCH; ++i)
+          if (i < nmine) {
+            const int off = (s0 + i * kWarps) * kChunk * 2;
+            const uint4 wa = *reinterpret_cast<const uint4*>(wlo + off);
+            const uint4 wb = *reinterpret_cast<const uint4*>(whi + off);
+#pragma unroll
+            for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt) {
+                mma16816<kF16Mma>(acc[i % NU][nb][nt], wa, wb, bv[i][nb][nt].x, bv[i][nb][nt].y, false);
+                mma16816<kF16Mma>(acc[i % NU][nb][nt], wa, wb, bv[i][nb][nt].z, bv[i][nb][nt].w, true);
+              }
+          }
+      }
+      if (nfull * kChunk < len && warp == nfull % kWarps) {  // ragged K tail, masked
+        const int kl = nfull * kChunk + 8 * c;
+        const uint8_t* st = smem + s * stage_bytes;
+        const uint4 wa = lds8_masked(st + g * pitch, kl, len, true);
+        const uint4 wb = lds8_masked(st + (g + 8) * pitch, kl, len, true);
+#pragma unroll
+        for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            const int t = nt * 8 + g;
-            if (kYs)
-              lds8_split<kF16C>(reinterpret_cast<const float*>(reinterpret_cast<const uint8_t*>(ys) +
-                                                              (t < a.T ? t : 0) * ypitch),
-                                in && t < a.T, j * a.kc + kl, a.K, hi[u][nt], lo[u][nt], range_err);
-            else
-              load8_split<kF16C>(a.yp + (int64_t)(t < a.T ? t : 0) * a.ldyp, in && t < a.T, j * a.kc + kl, a.K,
-                                 hi[u][nt], lo[u][nt], range_err);
+            const int t = nt * 8 + g < a.T ? nt * 8 + g : a.T - 1;
+            const uint4 b = ldg8_cg(nb == 0 ? a.B0 : a.B1, a.ldb, t, true, kbase + kl, a.K);
+            mma16816<kF16Mma>(acc[0][nb][nt], wa, wb, b.x, b.y, false);
+            mma16816<kF16Mma>(acc[0][nb][nt], wa, wb, b.z, b.w, true);
           }
-        }
-#pragma unroll
-        for (int u = 0; u < kUnroll2<NT>; ++u) {
-#pragma unroll
-          for (int nt = 0; nt < NT; ++nt) {
-            if (kF16C) {
-              mma_m16n8k16_f16(accu[u][0][nt], wa[u].x, wb[u].x, wa[u].y, wb[u].y, hi[u][nt].x, hi[u][nt].y);
-              mma_m16n8k16_f16(accu[u][1][nt], wa[u].x, wb[u].x, wa[u].y, wb[u].y, lo[u][nt].x, lo[u][nt].y);
-              mma_m16n8k16_f16(accu[u][0][nt], wa[u].z, wb[u].z, wa[u].w, wb[u].w, hi[u][nt].z, hi[u][nt].w);
-              mma_m16n8k16_f16(accu[u][1][nt], wa[u].z, wb[u].z, wa[u].w, wb[u].w, lo[u][nt].z, lo[u][nt].w);
-            } else {
-              mma_m16n8k16_bf16(accu[u][0][nt], wa[u].x, wb[u].x, wa[u].y, wb[u].y, hi[u][nt].x, hi[u][nt].y);
-              mma_m16n8k16_bf16(accu[u][1][nt], wa[u].x, wb[u].x, wa[u].y, wb[u].y, lo[u][nt].x, lo[u][nt].y);
-              mma_m16n8k16_bf16(accu[u][0][nt], wa[u].z, wb[u].z, wa[u].w, wb[u].w, hi[u][nt].z, hi[u][nt].w);
-              mma_m16n8k16_bf16(accu[u][1][nt], wa[u].z, wb[u].z, wa[u].w, wb[u].w, lo[u][nt].z, lo[u][nt].w);
-            }
-          }
-        }
       }
     }
     if (j + a.stages < nchunks) {  // refill stage s once every warp is done with it
-      __syncthreads();
+      dead = __syncthreads_or(dead);
       if (threadIdx.x == 0 && !dead) issue(j + a.stages);
     }
   }
   if (threadIdx.x == 0) {
-    // nothing may still be landing in shared memory when the CTA exits
+    // nothing may still be landing in shared memory when it is reused or the CTA exits
     for (int j = nchunks > a.stages ? nchunks - a.stages : 0; j < nchunks; ++j)
       if (!mbar_wait(&full[j % a.stages], (uint32_t)(j / a.stages) & 1u, 100000000ull))
         latch_status(a.status, PIFA_ERR_TIMEOUT);
-    if (kYs && !mbar_wait(ybar, 0, 100000000ull)) latch_status(a.status, PIFA_ERR_TIMEOUT);
   }
-  if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
-  float acc[NT][4];
+  __syncthreads();  // every warp is done with the stages: they hold the cross-warp reduction now
+  float(*red)[kRows][8 * NT + 1] = reinterpret_cast<float(*)[kRows][8 * NT + 1]>(smem);
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt)
+  for (int nt = 0; nt < NT; ++nt) {
+    float v[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      float v = 0.0f;
+      v[i] = 0.0f;
 #pragma unroll
-      for (int u = 0; u < kUnroll2<NT>; ++u) v += accu[u][0][nt][i] + accu[u][1][nt][i];
-      acc[nt][i] = v;
+      for (int u = 0; u < NU; ++u)
+#pragma unroll
+        for (int nb = 0; nb < NB; ++nb) v[i] += acc[u][nb][nt][i];
     }
-  reduce_and_store<NT, 2, kWarps2>(a, red, acc, row0, nrows, s_cols);
+    red[warp][g][nt * 8 + 2 * c] = v[0];
+    red[warp][g][nt * 8 + 2 * c + 1] = v[1];
+    red[warp][g + 8][nt * 8 + 2 * c] = v[2];
+    red[warp][g + 8][nt * 8 + 2 * c + 1] = v[3];
+  }
+  __syncthreads();
+  bool range_err = false;
+  for (int idx = threadIdx.x; idx < kRows * 8 * NT; idx += kWarps * 32) {
+    const int row = idx % kRows, t = idx / kRows;  // neighbouring threads: neighbouring rows
+    if (t >= a.T || row >= nrows) continue;
+    float sum = 0.0f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) sum += red[w][row][t];
+    if (PHASE == 1 && a.yph != nullptr) {
+      uint16_t h, l;
+      split2<kF16C>(sum, h, l, range_err);
+      a.yph[(int64_t)t * a.ldyp + row0 + row] = h;
+      a.ypl[(int64_t)t * a.ldyp + row0 + row] = l;
+    }
+    const int col = s_cols[row];
+    if ((unsigned)col >= (unsigned)a.m) {
+      latch_status(a.status, PIFA_ERR_DEVICE_INDEX);
+      continue;
+    }
+    a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(sum);
+  }
+  if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
+}
+
+// Once per kernel, device and size: the dynamic shared-memory limit, and the largest shared-memory
+// carveout, so that a phase-1 CTA and a phase-2 CTA fit on one SM together.
+int prepare_kernel(const void* fn, size_t smem, const char* what) {
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, size_t> done;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return pifa_fail_cuda(what, e);
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = done.find({fn, dev});
+  if (it != done.end() && it->second >= smem) return PIFA_OK;
+  e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, (int)cudaSharedmemCarveoutMaxShared);
+  if (e != cudaSuccess) return pifa_fail_cuda(what, e);
+  done[{fn, dev}] = smem;
+  return PIFA_OK;
 }
 
 template <typename Kern>
-int launch_pdl(Kern kernel, unsigned grid, unsigned threads, size_t smem, cudaStream_t stream,
-               const DecodeArgs& args, const char* what) {
-  if (smem > 48 * 1024) {
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return pifa_fail_cuda(what, e);
-  }
-
+int launch_pdl(Kern kernel, unsigned grid, size_t smem, cudaStream_t stream, const DecodeArgs& args,
+               const char* what) {
+  const int st = prepare_kernel(reinterpret_cast<const void*>(kernel), smem, what);
+  if (st != PIFA_OK) return st;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(threads);
+  cfg.blockDim = dim3(kWarps * 32);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
@@ -437,17 +347,40 @@ int launch_pdl(Kern kernel, unsigned grid, unsigned threads, size_t smem, cudaSt
   return PIFA_OK;
 }
 
-template <int NT>
+// K columns per stage and stage count for rows of K elements within `budget` bytes of stages.
+void plan_stages(int K, uint32_t budget, DecodeArgs& a) {
+  const int k32 = (K + kChunk - 1) / kChunk * kChunk;
+  if ((uint64_t)kRows * (uint64_t)(k32 * 2 + kRowPad) <= budget) {
+    a.kc = k32;
+    a.stages = 1;
+    return;
+  }
+  a.stages = 2;
+  const int row_bytes = (int)(budget / 2u / kRows) - kRowPad;
+  a.kc = row_bytes / 2 / 256 * 256;
+}
+
+size_t smem_bytes(const DecodeArgs& a, int NT) {
+  const size_t stages = (size_t)a.stages * kRows * ((size_t)a.kc * 2 + kRowPad);
+  const size_t red = (size_t)kWarps * kRows * (8 * NT + 1) * 4;
+  return stages > red ? stages : red;
+}
+
+template <int NT, bool kF16C>
 int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
+  const int64_t ldyp = (s.r + 7) / 8 * 8;  // 16-byte rows keep the fragment loads aligned
+  uint16_t* yph = reinterpret_cast<uint16_t*>(p.ws);
+  uint16_t* ypl = yph + s.T * ldyp;
   DecodeArgs a = {};
   a.A = reinterpret_cast<const uint16_t*>(p.Wp);
   a.lda = s.ldwp;
   a.R = (int)s.r;
   a.K = (int)s.n;
-  a.X = reinterpret_cast<const bf16*>(p.X);
-  a.ldx = s.ldx;
-  a.yp = reinterpret_cast<float*>(p.ws);
-  a.ldyp = (s.r + 7) / 8 * 8;  // 32-byte row pitch keeps the 16-byte loads aligned
+  a.B0 = reinterpret_cast<const uint16_t*>(p.X);
+  a.ldb = s.ldx;
+  a.yph = s.m > s.r ? yph : nullptr;
+  a.ypl = s.m > s.r ? ypl : nullptr;
+  a.ldyp = ldyp;
   a.cols = p.piv;
   a.m = (int)s.m;
   a.Y = reinterpret_cast<bf16*>(p.Y);
@@ -455,55 +388,37 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   a.T = (int)s.T;
   a.status = status;
   a.timeout_ns = pifa_wait_timeout_ns();
-  int st = launch_pdl(decode_pivot_rows<NT>, (unsigned)((s.r + kRows - 1) / kRows), kWarps * 32, 0, stream, a,
-                      "decode phase 1 launch");
+  plan_stages(a.K, kStageBudget1, a);
+  int st = launch_pdl(decode_rows<1, NT, kF16C>, (unsigned)((s.r + kRows - 1) / kRows), smem_bytes(a, NT), stream,
+                      a, "decode phase 1 launch");
   if (st != PIFA_OK || s.m == s.r) return st;
   DecodeArgs b = a;
   b.A = reinterpret_cast<const uint16_t*>(p.C);
   b.lda = s.ldc;
   b.R = (int)(s.m - s.r);
   b.K = (int)s.r;
-  b.X = nullptr;
+  b.B0 = yph;
+  b.B1 = ypl;
+  b.ldb = ldyp;
+  b.yph = b.ypl = nullptr;
   b.cols = p.nonpiv;
-  // Shared memory: C all of K in one stage and y_p staged whole when both fit in ~190 KB; else C
-  // alone in one stage (y_p read from L2); else C in 2048-column chunks through 2 stages.
-  const size_t ys_bytes = (size_t)s.T * (size_t)(b.ldyp * 4 + 16);
-  const size_t tail = 32 + (size_t)kWarps2 * kRows * 8 * NT * 4;
-  const int kc_all = (b.K + kChunk - 1) / kChunk * kChunk;
-  const size_t c_all = (size_t)kRows * (kc_all * 2 + kRowPad);
-  bool ys = false;
-  if (c_all + ys_bytes + tail <= 190 * 1024) {
-    b.kc = kc_all;
-    b.stages = 1;
-    ys = true;
-  } else if (c_all + tail <= 190 * 1024) {
-    b.kc = kc_all;
-    b.stages = 1;
-  } else {
-    b.kc = 2048;
-    b.stages = 2;
-  }
-  const size_t smem = (size_t)b.stages * kRows * (b.kc * 2 + kRowPad) + (ys ? ys_bytes : 0) + tail;
-  const unsigned grid2 = (unsigned)((s.m - s.r + kRows - 1) / kRows);
-  const bool f16 = s.c_dtype == PIFA_DTYPE_FP16;
-  const unsigned th = kWarps2 * 32;
-  const char* what = "decode phase 2 launch";
-  if (f16 && ys) return launch_pdl(decode_nonpivot_rows<NT, true, true>, grid2, th, smem, stream, b, what);
-  if (f16) return launch_pdl(decode_nonpivot_rows<NT, true, false>, grid2, th, smem, stream, b, what);
-  if (ys) return launch_pdl(decode_nonpivot_rows<NT, false, true>, grid2, th, smem, stream, b, what);
-  return launch_pdl(decode_nonpivot_rows<NT, false, false>, grid2, th, smem, stream, b, what);
+  plan_stages(b.K, kStageBudget2, b);
+  return launch_pdl(decode_rows<2, NT, kF16C>, (unsigned)((s.m - s.r + kRows - 1) / kRows), smem_bytes(b, NT),
+                    stream, b, "decode phase 2 launch");
 }
 
 }  // namespace
 
 int64_t decode_workspace_bytes(const PifaShape& s) {
-  // y_p, fp32, T rows of pitch round_up(r, 8), rounded up to 256 bytes
+  // y_p as hi and lo planes of 2-byte elements, T rows of pitch round_up(r, 8) each, rounded up
+  // to 256 bytes
   return ((s.T * ((s.r + 7) / 8 * 8) * 4 + 255) / 256) * 256;
 }
 
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
-  if (s.T <= 8) return launch_decode_t<1>(s, p, status, stream);
-  return launch_decode_t<2>(s, p, status, stream);
+  const bool f16 = s.c_dtype == PIFA_DTYPE_FP16;
+  if (s.T <= 8) return f16 ? launch_decode_t<1, true>(s, p, status, stream) : launch_decode_t<1, false>(s, p, status, stream);
+  return f16 ? launch_decode_t<2, true>(s, p, status, stream) : launch_decode_t<2, false>(s, p, status, stream);
 }
 
 // ---- allocation-free decode entry point -------------------------------------------------------
@@ -511,7 +426,8 @@ int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaSt
 // plans every device byte ahead of time and forbids libraries from calling cudaMalloc, or code
 // running where an allocation would synchronize the device in the middle of a latency-critical
 // decode loop. Such callers cannot provide the workspace pifa_forward asks for, so this entry
-// point keeps the decode scratch (y_p, fp32, T rows of pitch round_up(r, 8)) in a fixed array in
+// point keeps the decode scratch (y_p as hi and lo planes of 2-byte elements, T rows of pitch
+// round_up(r, 8) each) in a fixed array in
 // the library's static device data instead. The array exists once per GPU that loads the
 // library and stays allocated until the process exits.
 namespace {
@@ -570,9 +486,8 @@ extern "C" int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, 
   }
   int* status = pifa_status_word(&e);
   if (!status) return pifa_fail_cuda("device status word", e);
-  // The array starts zeroed (static device data). Its first kWorkspaceReserve bytes hold the
-  // decode kernel's grid-barrier words, which every completed call leaves at zero; y_p after them
-  // is written in full before it is read.
+  // The first kWorkspaceReserve bytes of the array are reserved like those of a workspace; y_p
+  // after them is written in full before it is read.
   const PifaPointers p = {X,
                           Wp,
                           has_np ? C : nullptr,
@@ -580,7 +495,6 @@ extern "C" int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, 
                           has_np ? nonpivot_idx : nullptr,
                           Y,
                           static_cast<uint8_t*>(scratch) + kWorkspaceReserve,
-                          kNoAllocScratchBytes - kWorkspaceReserve,
-                          static_cast<unsigned*>(scratch)};
+                          kNoAllocScratchBytes - kWorkspaceReserve};
   return launch_decode(s, p, status, reinterpret_cast<cudaStream_t>(cuda_stream));
 }

@@ -27,9 +27,8 @@ struct PifaShape {
   int c_dtype;  // PIFA_DTYPE_BF16 or PIFA_DTYPE_FP16 (storage type of C)
 };
 
-// The first kWorkspaceReserve bytes of every workspace hold library state that must be zero before
-// the first call and that every call leaves zero (the decode kernel's grid-barrier count and
-// generation); per-call scratch starts after them.
+// The first kWorkspaceReserve bytes of every workspace are reserved for library state (no kernel
+// of this version uses them); per-call scratch starts after them.
 constexpr int64_t kWorkspaceReserve = 256;
 
 struct PifaPointers {
@@ -41,7 +40,6 @@ struct PifaPointers {
   void* Y;
   void* ws;           // per-call scratch (workspace + kWorkspaceReserve)
   int64_t ws_bytes;   // bytes available at ws
-  unsigned* sync;     // the reserved words at the start of the workspace
 };
 
 // ---- decode (decode.cu) ----------------------------------------------------------------------

@@ -214,8 +214,7 @@ def workspace(nbytes: int, device, stream=None):
     key = (str(device), 0 if stream is None else getattr(stream, "cuda_stream", stream))
     buf = _workspaces.get(key)
     if buf is None or buf.numel() < nbytes:
-        # zero-filled: its first 256 bytes are library state that must start at zero
-        buf = torch.zeros(max(nbytes, 256) + 256, dtype=torch.uint8, device=device)
+        buf = torch.empty(max(nbytes, 256) + 256, dtype=torch.uint8, device=device)
         _workspaces[key] = buf
     return buf
 
