@@ -6,21 +6,28 @@
 //   phase 2: Y_np = Y_p C^T (the m - r rows of C, each read once) -> Y[:, I^c[i]] = bf16(Y_np[:, i])
 //                                                                     (Algorithm 2, steps 3 and 5)
 //
-// Both phases have one shape. A CTA owns 16 consecutive weight rows (one m16 MMA fragment). At
-// launch -- before it waits on its predecessor (programmatic dependent launch, PDL) -- one thread
-// bulk-copies the CTA's rows into shared memory: all of K when it fits, else K-chunks through two
+// Both phases have one shape. A CTA owns a tile of 16 RG consecutive weight rows (RG m16 MMA row
+// groups; RG = 1 or 4 by token count) and a K range; a thread-block cluster of up to 8 CTAs
+// splits K when a tile's rows do not fit one stage, so each CTA reads only
+// its slice of the broadcast operand (x or y_p). Every CTA of the grid reads the whole broadcast
+// slice of its K range once, so taller tiles mean proportionally less of that L2 traffic, which
+// otherwise competes with the weight streams and delays the dependent step. At launch -- before
+// the CTA waits on its predecessor (programmatic dependent launch, PDL) -- warp 0 bulk-copies the
+// CTA's weight rows into shared memory: the whole K range when it fits, else K-chunks through two
 // stages refilled as they are used. The weights do not depend on the previous kernel, so their
 // HBM traffic overlaps its compute: phase 2 stages its rows of C while phase 1 computes, and the
 // next call's phase 1 stages its W_p while this call's phase 2 computes. The stage budgets let a
 // phase-1 CTA and a phase-2 CTA share one SM.
 //
-// Once the predecessor has completed, each warp loads the B fragments of its K-steps (x for
-// phase 1; the y_p hi and lo planes for phase 2) from L2 into registers in one batch and runs
-// mma.sync.m16n8k16 over its steps with A from shared memory. For a 32-wide K step, lane
-// (g = lane/4, c = lane%4) takes 8 consecutive elements of rows g and g+8 at offset 8c as the A
-// fragments of two k16 MMAs and the matching 8 elements of token g as its B fragment: K is
-// permuted identically in both operands, which a dot product does not notice. The warps' 16 x 8
-// partial tiles are summed through shared memory in a fixed order (the result is deterministic).
+// Once the predecessor has completed, each warp loads the B fragments of its K steps from L2
+// into registers and runs mma.sync.m16n8k16 over its steps and all RG row groups with A from
+// shared memory. For a 32-wide K step, lane (g = lane/4, c = lane%4) takes 8 consecutive elements
+// of rows g and g+8 of a row group at offset 8c as the A fragments of two k16 MMAs and the
+// matching 8 elements of token g as its B fragment: K is permuted identically in both operands,
+// which a dot product does not notice. The warps' partial tiles are summed through shared memory,
+// then the cluster's K slices through distributed shared memory, each CTA finishing 16 RG / ks
+// rows;
+// both sums run in a fixed order, so the result is deterministic.
 //
 // y_p enters the second contraction as a hi + lo pair of C's storage type (bf16 or fp16): C has
 // large entries and Y_np = C Y_p cancels, so rounding y_p to one bf16 alone would amplify its
@@ -41,18 +48,19 @@ namespace {
 using namespace pifa;
 using bf16 = __nv_bfloat16;
 
-constexpr int kRows = 16;    // weight rows per CTA
-constexpr int kChunk = 32;   // K elements per warp step (two k16 MMAs)
-constexpr int kRowPad = 64;  // bytes between consecutive staged rows beyond their length
-constexpr int kWarps = 8;    // warps per CTA, both phases
-// Shared-memory budgets of the weight stages of one CTA. 136 KB (phase 1) + 70 KB (phase 2) and
-// the small rest fit in one SM's 228 KB, so a phase-2 CTA can stage its rows of C beside a
-// computing phase-1 CTA (and a phase-1 CTA its rows of W_p beside a phase-2 CTA).
-constexpr uint32_t kStageBudget1 = 136u * 1024u;
-constexpr uint32_t kStageBudget2 = 70u * 1024u;
-// K steps whose B fragments a warp holds in registers at once: 64 registers for any NT and NB
-template <int NT, int NB>
-constexpr int kBatch = 16 / (NT * NB);
+// Weight rows per CTA: RG MMA row groups of 16. RG = 4 (64 rows, K split over a cluster) reads
+// 4x less of the broadcast operand per weight byte than RG = 1 (16 rows, whole K per CTA) and wins
+// from T of a few tokens up; RG = 1 needs no cross-CTA reduction and wins at T <= 4.
+template <int RG>
+constexpr int kRowsOf = 16 * RG;
+constexpr int kChunk = 32;          // K elements per warp step (two k16 MMAs)
+constexpr int kWarps = 8;           // warps per CTA, both phases
+constexpr int kMaxCluster = 8;      // CTAs per cluster splitting K (portable cluster size)
+// Shared-memory budgets of one CTA's weight stages. 144 KB (phase 1) + 76 KB (phase 2) and the
+// small rest fit in one SM's 228 KB, so a phase-2 CTA can stage its rows of C beside a computing
+// phase-1 CTA (and a phase-1 CTA its rows of W_p beside a phase-2 CTA).
+constexpr uint32_t kStageBudget1 = 144u * 1024u;
+constexpr uint32_t kStageBudget2 = 76u * 1024u;
 
 __device__ __forceinline__ uint32_t pack2(uint16_t a, uint16_t b) { return (uint32_t)a | ((uint32_t)b << 16); }
 
@@ -133,62 +141,84 @@ struct DecodeArgs {
   bf16* Y;
   int64_t ldy;
   int T;
-  int kc;               // K columns per shared-memory stage (multiple of 32)
-  int stages;           // 1 (all of K resident) or 2
+  int ks;               // CTAs of a cluster, splitting K (1, 2, 4 or 8)
+  int kcta;             // K columns per CTA (multiple of 32)
+  int kc;               // K columns per shared-memory stage (multiple of 32, at most kcta)
+  int stages;           // 1 (the CTA's whole K range resident) or 2
   int* status;
   uint64_t timeout_ns;
 };
 
-// One CTA: weight rows row0 .. row0 + 15 against the T tokens. PHASE 1: bf16 MMAs against x, and
-// y_p split in C's dtype (kF16C). PHASE 2: MMAs in C's dtype against the y_p hi and lo planes.
-template <int PHASE, int NT, bool kF16C>
+// Bytes between staged rows: the row's bytes, plus 64 when they are a multiple of 128, so that
+// rows g and g + 1 start 64 bytes apart and a quarter warp's 16-byte fragment loads (two rows,
+// four 16-byte columns each) cover all 32 banks.
+__host__ __device__ constexpr uint32_t row_pitch(int kc) {
+  return (uint32_t)kc * 2u + (((uint32_t)kc * 2u) % 128u == 0u ? 64u : 0u);
+}
+
+// One CTA: 16 RG weight rows x its K range [q kcta, (q + 1) kcta) against the T tokens, q = its
+// rank in the cluster. The cluster's CTAs sum their partial tiles through distributed shared
+// memory, each finishing kRows / ks of the rows. PHASE 1: bf16 MMAs against x, and y_p split in
+// C's dtype (kF16C). PHASE 2: MMAs in C's dtype against the y_p hi and lo planes.
+template <int PHASE, int NT, bool kF16C, int RG>
 __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
-  constexpr int NB = PHASE == 1 ? 1 : 2;  // B planes
+  constexpr int kRows = kRowsOf<RG>;
+  constexpr int NB = PHASE == 1 ? 1 : 2;  // B planes (both accumulate into one tile)
   constexpr bool kF16Mma = PHASE == 2 && kF16C;
-  constexpr int NBATCH = kBatch<NT, NB>;
+  // K steps whose B fragments a warp loads at once (about 64 registers of B and accumulators)
+  constexpr int NBATCH = 16 / (RG * NB * NT) > 0 ? 16 / (RG * NB * NT) : 1;
+  constexpr int NU = RG == 1 ? 2 : 1;     // accumulator sets (even / odd steps): shorter MMA chains
+  constexpr int RP = 8 * NT + 1;          // floats per row of the reduction tiles
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ uint64_t full[2];
   __shared__ int s_cols[kRows];
   pdl_launch_dependents();  // the next kernel may launch now and start staging its weights
-  const uint32_t pitch = (uint32_t)a.kc * 2u + kRowPad;
+  const uint32_t pitch = row_pitch(a.kc);
   const uint32_t stage_bytes = (uint32_t)kRows * pitch;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, c = lane & 3;
-  const int64_t row0 = (int64_t)blockIdx.x * kRows;
+  const int q = (int)cluster_ctarank();
+  const int64_t row0 = (int64_t)(blockIdx.x / a.ks) * kRows;
   const int nrows = (int)((int64_t)a.R - row0 < kRows ? (int64_t)a.R - row0 : kRows);
-  const int nchunks = (a.K + a.kc - 1) / a.kc;
-  auto issue = [&](int j) {  // thread 0: K-chunk j of the CTA's rows into stage j % stages
+  const int k0 = q * a.kcta;
+  const int klen = max(0, min(a.kcta, a.K - k0));
+  const int nchunks = (klen + a.kc - 1) / a.kc;
+  // Warp 0 stages K-chunk j: lane 0 arms the stage barrier, then each lane copies every 32nd row.
+  auto issue = [&](int j) {
     const int s = j % a.stages;
-    const int len = min(a.kc, a.K - j * a.kc);
+    const int len = min(a.kc, klen - j * a.kc);
     const uint32_t bytes = (uint32_t)((len + 7) & ~7) * 2u;  // 16-byte multiple within the row pitch
-    mbar_arrive_expect_tx(&full[s], bytes * (uint32_t)nrows);
+    if (lane == 0) mbar_arrive_expect_tx(&full[s], bytes * (uint32_t)nrows);
+    __syncwarp();
     uint8_t* st = smem + s * stage_bytes;
-    for (int rr = 0; rr < nrows; ++rr)
-      bulk_copy_g2s(smem_u32(st + rr * pitch), a.A + (row0 + rr) * a.lda + (int64_t)j * a.kc, bytes, &full[s]);
+    for (int rr = lane; rr < nrows; rr += 32)
+      bulk_copy_g2s(smem_u32(st + rr * pitch), a.A + (row0 + rr) * a.lda + k0 + (int64_t)j * a.kc, bytes, &full[s]);
   };
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < a.stages; ++s) mbar_init(&full[s], 1);
-    fence_mbar_init();
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int s = 0; s < a.stages; ++s) mbar_init(&full[s], 1);
+      fence_mbar_init();
+    }
+    __syncwarp();
     for (int j = 0; j < a.stages && j < nchunks; ++j) issue(j);
   }
   // the output columns of this CTA's rows are layer constants: read them before waiting
-  if (threadIdx.x < kRows) s_cols[threadIdx.x] = threadIdx.x < nrows ? a.cols[row0 + threadIdx.x] : 0;
+  for (int i = threadIdx.x; i < kRows; i += kWarps * 32) s_cols[i] = i < nrows ? a.cols[row0 + i] : 0;
   // One thread waits for the previous kernel (its outputs visible, ours free to overwrite) while
   // the other warps park in the CTA barrier instead of taking issue slots from co-resident CTAs.
   if (threadIdx.x == 0) pdl_wait_primary();
   __syncthreads();  // also: barriers initialised before anyone waits on them
-  // independent accumulator chains: the hi and lo planes in phase 2, even and odd steps in phase 1
-  constexpr int NU = NB == 1 ? 2 : 1;
-  float acc[NU][NB][NT][4];
+
+  float acc[NU][RG][NT][4];
 #pragma unroll
   for (int u = 0; u < NU; ++u)
 #pragma unroll
-    for (int nb = 0; nb < NB; ++nb)
+    for (int gq = 0; gq < RG; ++gq)
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) acc[u][nb][nt][0] = acc[u][nb][nt][1] = acc[u][nb][nt][2] = acc[u][nb][nt][3] = 0.0f;
+      for (int nt = 0; nt < NT; ++nt) acc[u][gq][nt][0] = acc[u][gq][nt][1] = acc[u][gq][nt][2] = acc[u][gq][nt][3] = 0.0f;
   // This lane's B rows: token t = 8 nt + g, clamped to T - 1. The output columns of tokens >= T
   // are computed from a duplicate row and never stored, and so are the output rows of weight
   // rows >= nrows (their stage rows hold stale bytes): an MMA row or column only ever affects
-  // itself. Only the K tail beyond the last full step needs masking, and it gets its own step.
+  // itself. Only a K tail beyond the last full step needs masking, and it gets its own step.
   const uint16_t* brow[NB][NT];
 #pragma unroll
   for (int nb = 0; nb < NB; ++nb)
@@ -200,22 +230,21 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
   bool dead = false;
   for (int j = 0; j < nchunks; ++j) {
     const int s = j % a.stages;
-    const int kbase = j * a.kc;
-    const int len = min(a.kc, a.K - kbase);
+    const int kb = k0 + j * a.kc;  // first K column of the chunk
+    const int len = min(a.kc, klen - j * a.kc);
     if (!dead && !mbar_wait(&full[s], (uint32_t)(j / a.stages) & 1u, a.timeout_ns)) {
       latch_status(a.status, PIFA_ERR_TIMEOUT);
       dead = true;
     }
     dead = __any_sync(0xffffffffu, dead);  // the MMAs below are warp-collective
     if (!dead) {
-      // The hot loop is kept short: this code runs once per launch, and its instruction fetch
-      // (not its arithmetic) would otherwise dominate the kernel.
-      const uint8_t* wlo = smem + s * stage_bytes + g * pitch + 16 * c;  // weight row g
-      const uint8_t* whi = wlo + 8 * pitch;                               // weight row g + 8
+      // The hot loop is kept short: it runs once per launch, and its instruction fetch (not its
+      // arithmetic) would otherwise dominate the kernel.
+      const uint32_t wbase = smem_u32(smem + s * stage_bytes) + g * pitch + 16 * c;
       const int nfull = len / kChunk;
       for (int s0 = warp; s0 < nfull; s0 += kWarps * NBATCH) {
         const int nmine = min(NBATCH, (nfull - s0 + kWarps - 1) / kWarps);  // this batch's steps
-        uint4 bv[NBATCH][NB][NT];  // every load of the batch in flight together
+        uint4 bv[NBATCH][NB][NT];  // the batch's B loads in flight together
 #pragma unroll
         for (int i = 0; i < NBATCH; ++i)
           if (i < nmine)
@@ -223,41 +252,53 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
             for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
               for (int nt = 0; nt < NT; ++nt)
-                bv[i][nb][nt] = __ldcg(reinterpret_cast<const uint4*>(brow[nb][nt] + kbase + (s0 + i * kWarps) * kChunk));
+                bv[i][nb][nt] = __ldcg(reinterpret_cast<const uint4*>(brow[nb][nt] + kb + (s0 + i * kWarps) * kChunk));
 #pragma unroll
         for (int i = 0; i < NBATCH; ++i)
           if (i < nmine) {
-            const int off = (s0 + i * kWarps) * kChunk * 2;
-            const uint4 wa = *reinterpret_cast<const uint4*>(wlo + off);
-            const uint4 wb = *reinterpret_cast<const uint4*>(whi + off);
+            const uint32_t at = wbase + (uint32_t)((s0 + i * kWarps) * kChunk * 2);
 #pragma unroll
-            for (int nb = 0; nb < NB; ++nb)
+            for (int gq = 0; gq < RG; ++gq) {
+              const uint4 wa = lds128(at + (uint32_t)(16 * gq) * pitch);      // row 16 gq + g
+              const uint4 wb = lds128(at + (uint32_t)(16 * gq + 8) * pitch);  // row 16 gq + g + 8
 #pragma unroll
-              for (int nt = 0; nt < NT; ++nt) {
-                mma16816<kF16Mma>(acc[i % NU][nb][nt], wa, wb, bv[i][nb][nt].x, bv[i][nb][nt].y, false);
-                mma16816<kF16Mma>(acc[i % NU][nb][nt], wa, wb, bv[i][nb][nt].z, bv[i][nb][nt].w, true);
-              }
+              for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                  mma16816<kF16Mma>(acc[i % NU][gq][nt], wa, wb, bv[i][nb][nt].x, bv[i][nb][nt].y, false);
+                  mma16816<kF16Mma>(acc[i % NU][gq][nt], wa, wb, bv[i][nb][nt].z, bv[i][nb][nt].w, true);
+                }
+            }
           }
       }
       if (nfull * kChunk < len && warp == nfull % kWarps) {  // ragged K tail, masked
         const int kl = nfull * kChunk + 8 * c;
         const uint8_t* st = smem + s * stage_bytes;
-        const uint4 wa = lds8_masked(st + g * pitch, kl, len, true);
-        const uint4 wb = lds8_masked(st + (g + 8) * pitch, kl, len, true);
+        uint4 bt[NB][NT];
 #pragma unroll
         for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
             const int t = nt * 8 + g < a.T ? nt * 8 + g : a.T - 1;
-            const uint4 b = ldg8_cg(nb == 0 ? a.B0 : a.B1, a.ldb, t, true, kbase + kl, a.K);
-            mma16816<kF16Mma>(acc[0][nb][nt], wa, wb, b.x, b.y, false);
-            mma16816<kF16Mma>(acc[0][nb][nt], wa, wb, b.z, b.w, true);
+            bt[nb][nt] = ldg8_cg(nb == 0 ? a.B0 : a.B1, a.ldb, t, true, kb + kl, a.K);
           }
+#pragma unroll
+        for (int gq = 0; gq < RG; ++gq) {
+          const uint4 wa = lds8_masked(st + (16 * gq + g) * pitch, kl, len, true);
+          const uint4 wb = lds8_masked(st + (16 * gq + g + 8) * pitch, kl, len, true);
+#pragma unroll
+          for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+              mma16816<kF16Mma>(acc[0][gq][nt], wa, wb, bt[nb][nt].x, bt[nb][nt].y, false);
+              mma16816<kF16Mma>(acc[0][gq][nt], wa, wb, bt[nb][nt].z, bt[nb][nt].w, true);
+            }
+        }
       }
     }
     if (j + a.stages < nchunks) {  // refill stage s once every warp is done with it
       dead = __syncthreads_or(dead);
-      if (threadIdx.x == 0 && !dead) issue(j + a.stages);
+      if (warp == 0 && !dead) issue(j + a.stages);
     }
   }
   if (threadIdx.x == 0) {
@@ -266,32 +307,50 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
       if (!mbar_wait(&full[j % a.stages], (uint32_t)(j / a.stages) & 1u, 100000000ull))
         latch_status(a.status, PIFA_ERR_TIMEOUT);
   }
-  __syncthreads();  // every warp is done with the stages: they hold the cross-warp reduction now
-  float(*red)[kRows][8 * NT + 1] = reinterpret_cast<float(*)[kRows][8 * NT + 1]>(smem);
+  __syncthreads();  // every warp is done with the stages: they hold the reduction tiles now
+
+  // 1. the warps' partial tiles, red[warp][row][t]; 2. their sum, in place in warp 0's tile
+  float* red = reinterpret_cast<float*>(smem);
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
-    float v[4];
+  for (int gq = 0; gq < RG; ++gq)
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      v[i] = 0.0f;
+    for (int nt = 0; nt < NT; ++nt) {
+      float v[4];
 #pragma unroll
-      for (int u = 0; u < NU; ++u)
+      for (int e = 0; e < 4; ++e) {
+        v[e] = acc[0][gq][nt][e];
 #pragma unroll
-        for (int nb = 0; nb < NB; ++nb) v[i] += acc[u][nb][nt][i];
+        for (int u = 1; u < NU; ++u) v[e] += acc[u][gq][nt][e];
+      }
+      float* r0p = red + (warp * kRows + 16 * gq + g) * RP + nt * 8 + 2 * c;
+      r0p[0] = v[0];
+      r0p[1] = v[1];
+      r0p[8 * RP] = v[2];
+      r0p[8 * RP + 1] = v[3];
     }
-    red[warp][g][nt * 8 + 2 * c] = v[0];
-    red[warp][g][nt * 8 + 2 * c + 1] = v[1];
-    red[warp][g + 8][nt * 8 + 2 * c] = v[2];
-    red[warp][g + 8][nt * 8 + 2 * c + 1] = v[3];
-  }
   __syncthreads();
-  bool range_err = false;
   for (int idx = threadIdx.x; idx < kRows * 8 * NT; idx += kWarps * 32) {
-    const int row = idx % kRows, t = idx / kRows;  // neighbouring threads: neighbouring rows
-    if (t >= a.T || row >= nrows) continue;
+    const int row = idx % kRows, t = idx / kRows;  // each (row, t) belongs to one thread
     float sum = 0.0f;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) sum += red[w][row][t];
+    for (int w = 0; w < kWarps; ++w) sum += red[(w * kRows + row) * RP + t];
+    red[row * RP + t] = sum;
+  }
+  // 3. the cluster's K-slices: CTA q sums rows [q rpr, (q + 1) rpr) over all ranks, in rank order
+  if (a.ks > 1) cluster_sync_all();
+  else __syncthreads();
+  const int rpr = kRows / a.ks;
+  bool range_err = false;
+  for (int idx = threadIdx.x; idx < rpr * 8 * NT; idx += kWarps * 32) {
+    const int row = q * rpr + idx % rpr, t = idx / rpr;
+    if (t >= a.T || row >= nrows) continue;
+    float sum = 0.0f;
+    if (a.ks == 1) {
+      sum = red[row * RP + t];
+    } else {
+      const uint32_t la = smem_u32(red + row * RP + t);
+      for (int rk = 0; rk < a.ks; ++rk) sum += ld_dsmem_f32(mapa_shared(la, (uint32_t)rk));
+    }
     if (PHASE == 1 && a.yph != nullptr) {
       uint16_t h, l;
       split2<kF16C>(sum, h, l, range_err);
@@ -306,6 +365,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
     a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(sum);
   }
   if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
+  if (a.ks > 1) cluster_sync_relaxed();  // peers may still be reading this CTA's partial tile
 }
 
 // Once per kernel, device and size: the dynamic shared-memory limit, and the largest shared-memory
@@ -327,47 +387,60 @@ int prepare_kernel(const void* fn, size_t smem, const char* what) {
   return PIFA_OK;
 }
 
+// Launch with programmatic dependent launch and a (ks, 1, 1) cluster.
 template <typename Kern>
-int launch_pdl(Kern kernel, unsigned grid, size_t smem, cudaStream_t stream, const DecodeArgs& args,
-               const char* what) {
+int launch_phase(Kern kernel, int rows, const DecodeArgs& args, size_t smem, cudaStream_t stream, const char* what) {
   const int st = prepare_kernel(reinterpret_cast<const void*>(kernel), smem, what);
   if (st != PIFA_OK) return st;
+  const unsigned tiles = (unsigned)((args.R + rows - 1) / rows);
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = dim3(tiles * (unsigned)args.ks);
   cfg.blockDim = dim3(kWarps * 32);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)args.ks;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, args);
   if (e != cudaSuccess) return pifa_fail_cuda(what, e);
   return PIFA_OK;
 }
 
-// K columns per stage and stage count for rows of K elements within `budget` bytes of stages.
-void plan_stages(int K, uint32_t budget, DecodeArgs& a) {
-  const int k32 = (K + kChunk - 1) / kChunk * kChunk;
-  if ((uint64_t)kRows * (uint64_t)(k32 * 2 + kRowPad) <= budget) {
-    a.kc = k32;
-    a.stages = 1;
-    return;
+// The K split and the stages of one phase: the fewest CTAs per cluster (1, 2, 4, 8) whose K range
+// fits one stage within `budget`; else 8 CTAs, each streaming its range through two stages.
+void plan_phase(int kRows, uint32_t budget, DecodeArgs& a) {
+  for (int ks = 1; ks <= kMaxCluster; ks *= 2) {
+    const int kcta = ((a.K + ks - 1) / ks + kChunk - 1) / kChunk * kChunk;
+    if ((uint64_t)kRows * row_pitch(kcta) <= budget) {
+      a.ks = ks;
+      a.kcta = a.kc = kcta;
+      a.stages = 1;
+      return;
+    }
   }
+  a.ks = kMaxCluster;
+  a.kcta = ((a.K + kMaxCluster - 1) / kMaxCluster + kChunk - 1) / kChunk * kChunk;
   a.stages = 2;
-  const int row_bytes = (int)(budget / 2u / kRows) - kRowPad;
-  a.kc = row_bytes / 2 / 256 * 256;
+  int kc = kChunk;
+  while (kc + kChunk <= a.kcta && 2ull * kRows * row_pitch(kc + kChunk) <= budget) kc += kChunk;
+  a.kc = kc;
 }
 
-size_t smem_bytes(const DecodeArgs& a, int NT) {
-  const size_t stages = (size_t)a.stages * kRows * ((size_t)a.kc * 2 + kRowPad);
+size_t smem_bytes(int kRows, const DecodeArgs& a, int NT) {
+  const size_t stages = (size_t)a.stages * kRows * row_pitch(a.kc);
   const size_t red = (size_t)kWarps * kRows * (8 * NT + 1) * 4;
   return stages > red ? stages : red;
 }
 
-template <int NT, bool kF16C>
+template <int NT, bool kF16C, int RG>
 int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
+  constexpr int kRows = kRowsOf<RG>;
   const int64_t ldyp = (s.r + 7) / 8 * 8;  // 16-byte rows keep the fragment loads aligned
   uint16_t* yph = reinterpret_cast<uint16_t*>(p.ws);
   uint16_t* ypl = yph + s.T * ldyp;
@@ -388,9 +461,9 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   a.T = (int)s.T;
   a.status = status;
   a.timeout_ns = pifa_wait_timeout_ns();
-  plan_stages(a.K, kStageBudget1, a);
-  int st = launch_pdl(decode_rows<1, NT, kF16C>, (unsigned)((s.r + kRows - 1) / kRows), smem_bytes(a, NT), stream,
-                      a, "decode phase 1 launch");
+  plan_phase(kRows, kStageBudget1, a);
+  int st = launch_phase(decode_rows<1, NT, kF16C, RG>, kRows, a, smem_bytes(kRows, a, NT), stream,
+                        "decode phase 1 launch");
   if (st != PIFA_OK || s.m == s.r) return st;
   DecodeArgs b = a;
   b.A = reinterpret_cast<const uint16_t*>(p.C);
@@ -402,9 +475,9 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   b.ldb = ldyp;
   b.yph = b.ypl = nullptr;
   b.cols = p.nonpiv;
-  plan_stages(b.K, kStageBudget2, b);
-  return launch_pdl(decode_rows<2, NT, kF16C>, (unsigned)((s.m - s.r + kRows - 1) / kRows), smem_bytes(b, NT),
-                    stream, b, "decode phase 2 launch");
+  plan_phase(kRows, kStageBudget2, b);
+  return launch_phase(decode_rows<2, NT, kF16C, RG>, kRows, b, smem_bytes(kRows, b, NT), stream,
+                      "decode phase 2 launch");
 }
 
 }  // namespace
@@ -417,8 +490,9 @@ int64_t decode_workspace_bytes(const PifaShape& s) {
 
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
   const bool f16 = s.c_dtype == PIFA_DTYPE_FP16;
-  if (s.T <= 8) return f16 ? launch_decode_t<1, true>(s, p, status, stream) : launch_decode_t<1, false>(s, p, status, stream);
-  return f16 ? launch_decode_t<2, true>(s, p, status, stream) : launch_decode_t<2, false>(s, p, status, stream);
+  if (s.T <= 4) return f16 ? launch_decode_t<1, true, 1>(s, p, status, stream) : launch_decode_t<1, false, 1>(s, p, status, stream);
+  if (s.T <= 8) return f16 ? launch_decode_t<1, true, 4>(s, p, status, stream) : launch_decode_t<1, false, 4>(s, p, status, stream);
+  return f16 ? launch_decode_t<2, true, 4>(s, p, status, stream) : launch_decode_t<2, false, 4>(s, p, status, stream);
 }
 
 // ---- allocation-free decode entry point -------------------------------------------------------
