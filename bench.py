@@ -47,7 +47,11 @@ T_PREFILL = 2048
 
 # DRAM traffic per launch measured with ncu for a given kernel source (sha256 of the .cu file).
 # A mismatch (the kernel changed since the capture) reports traffic as null.
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {
+    # decode_rows phase 1 + phase 2 of one call, attn 4096x4096 r=2048 T=8:
+    # dram__bytes_read.sum 16.88 MB + 8.50 MB, dram__bytes_write.sum 0 (profiles/decode_attn7b_T8_ncu_full.md)
+    "decode": {"sha": "a50d3f72ac5c1c35", "bytes": 16884736 + 8497152},
+}
 
 
 def _src_sha(name: str) -> str:
@@ -265,8 +269,8 @@ def run_ours(args, rank, world, local_rank):
         "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": T * n * 2,
                 "d2h_bytes_per_step": T * m * 2},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": achieved / hbm_peak, "traffic": _traffic("decode.cu", "decode"),
-                     "peak_source": f"{peak_src} hbm_gbs", "kernel": "decode_pivot_rows + decode_nonpivot_rows (PDL pair)",
+                     "frac": achieved / hbm_peak, "traffic": _traffic("decode.cu", "decode") if (T, m, n, r) == (8, 4096, 4096, 2048) else None,
+                     "peak_source": f"{peak_src} hbm_gbs", "kernel": "decode_rows phase 1 + phase 2 (one PDL-chained pair per call)",
                      "algorithmic_bytes_per_launch": decode_bytes(T, m, n, r)},
         "gpu_launches": steps * (2 if m > r else 1),
         "clocks": clk.summary(),
@@ -274,8 +278,8 @@ def run_ours(args, rank, world, local_rank):
     if rank == 0 and not args.no_extras:
         out["comparators"] = comparators(dev, lay, T, copies, stream)
         out["prefill"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src)
-        out["prefill_split"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src,
-                                             variant=P.PIFA_VARIANT_PREFILL_SPLIT)
+        out["prefill_fused"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src,
+                                             variant=P.PIFA_VARIANT_PREFILL_FUSED)
         out["cpu_baseline"] = cpu_baseline(lay, T)
     return out
 
@@ -412,20 +416,24 @@ def run_reference(args, rank):
     X = inputs.make_activations(rng, T, SHAPE.n, "bf16")
     for _ in range(max(3, args.warmup)):
         oracle.forward(X, Wp, C, L.pivots, L.nonpivots)
+    # bounded sample: at most ~60 s of oracle forwards, however many steps were asked for
     t0 = time.perf_counter()
-    for _ in range(args.steps):
+    done = 0
+    while done < args.steps and (done == 0 or time.perf_counter() - t0 < 60.0):
         oracle.forward(X, Wp, C, L.pivots, L.nonpivots)
+        done += 1
     dt = time.perf_counter() - t0
-    v = T * args.steps / dt
+    v = T * done / dt
     cores = len(os.sched_getaffinity(0))
     del P
     return {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
+            "steps": done, "requested_steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / done,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic", "config": {"workload": f"{SHAPE.name} decode T={T}", "m": SHAPE.m, "n": SHAPE.n,
                                             "r": SHAPE.r, "tokens_per_step": T},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                             "sample": f"{args.steps} fp64 oracle forwards of T={T} (numpy, host cores)"},
+                             "sample": f"{done} of {args.steps} requested fp64 oracle forwards of T={T} "
+                                       f"(numpy, host cores; capped at ~60 s)"},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 

@@ -151,8 +151,8 @@ int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dt
 
 /* pifa_select_variant -- the selector (host, < 1 us): the pifa_variant pifa_forward runs for
  * (T, m, n, r, c_dtype) on this build, never PIFA_VARIANT_AUTO; negative pifa_status on bad
- * arguments. Decode for T <= 16; otherwise the fused prefill kernel when the device can run
- * its thread-block cluster, else the split prefill. */
+ * arguments. Decode for T <= 16, else the split prefill (the fused prefill kernel is measured
+ * slower on GB300 and runs only when requested). */
 int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype);
 
 /* pifa_variant_name -- static string naming a pifa_variant ("decode", ...); "?" if unknown. */

@@ -149,8 +149,8 @@ int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype)
   if (st != PIFA_OK) return st;
   if (c_dtype != PIFA_DTYPE_BF16 && c_dtype != PIFA_DTYPE_FP16) return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown c_dtype");
   if (T <= 16) return PIFA_VARIANT_DECODE;
-  PifaShape s = {T, m, n, r, n, n, r, m, c_dtype};
-  if (prefill_fused_supported(s)) return PIFA_VARIANT_PREFILL_FUSED;
+  // The fused cluster kernel is correct but measured slower than the split GEMMs on GB300 (attn
+  // 4096 x 4096, r = 2048, T = 2048: 171 us against 70 us); it runs only when asked for.
   return PIFA_VARIANT_PREFILL_SPLIT;
 }
 

@@ -306,10 +306,12 @@ def test_fp16_c_attn7b_decode(T):
     parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16"), T)
 
 
-def test_selector_picks_fused_prefill():
-    assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == FUSED, P.pifa_last_error()
-    assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == FUSED, P.pifa_last_error()
+def test_selector_picks_split_prefill_and_fused_still_plans():
+    assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == SPLIT, P.pifa_last_error()
+    assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(16, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
+    # the fused kernel is still runnable on request for this shape
+    assert P.pifa_workspace_size(2048, 4096, 4096, 2048, FUSED) > 0
 
 
 def test_bf16_c_fused_attn7b_and_ragged():

@@ -50,12 +50,9 @@ def test_status_and_variant_strings(lib):
 def test_selector(lib):
     assert P.pifa_select_variant(1, 4096, 4096, 2048) == P.PIFA_VARIANT_DECODE
     assert P.pifa_select_variant(16, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE
-    v = P.pifa_select_variant(2048, 4096, 4096, 2048)
-    assert v in (P.PIFA_VARIANT_PREFILL_SPLIT, P.PIFA_VARIANT_PREFILL_FUSED)
-    assert P.pifa_select_variant(17, 256, 256, 128) != P.PIFA_VARIANT_DECODE
-    # without a GPU the cluster kernel cannot be planned: the selector falls back to the split one
-    assert P.pifa_select_variant(4096, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) in (
-        P.PIFA_VARIANT_PREFILL_SPLIT, P.PIFA_VARIANT_PREFILL_FUSED)
+    assert P.pifa_select_variant(2048, 4096, 4096, 2048) == P.PIFA_VARIANT_PREFILL_SPLIT
+    assert P.pifa_select_variant(17, 256, 256, 128) == P.PIFA_VARIANT_PREFILL_SPLIT
+    assert P.pifa_select_variant(4096, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == P.PIFA_VARIANT_PREFILL_SPLIT
     with pytest.raises(P.PifaError):
         P.pifa_select_variant(1, 100, 50, 60)      # r > n
 
