@@ -226,7 +226,7 @@ def run_ours(args, rank, world, local_rank):
     assert st == P.PIFA_OK, P.pifa_status_string(st)
     ms_max = _max_over_ranks(ms)
     step_ms = ms_max / steps
-    value = world * T * steps / (ms_max / 1e3)
+    value = _job_value(world, T, steps, ms_max)
     achieved = decode_bytes(T, m, n, r) / (step_ms / 1e3) / 1e9
 
     # --- e2e through the public API with pinned host buffers ---
@@ -255,7 +255,7 @@ def run_ours(args, rank, world, local_rank):
         e1.record(stream)
     stream.synchronize()
     e2e_ms = _max_over_ranks(e0.elapsed_time(e1))
-    e2e_value = world * T * e2e_steps / (e2e_ms / 1e3)
+    e2e_value = _job_value(world, T, e2e_steps, e2e_ms)
 
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
@@ -392,13 +392,21 @@ def _dist():
 
 
 def _max_over_ranks(v):
+    """The slowest rank's value (every rank gets it); a no-op on one process."""
     d = _dist()
     if not d:
         return v
     import torch
-    t = torch.tensor([v], dtype=torch.float64, device="cuda")
+    dev = "cuda" if d.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
     d.all_reduce(t, op=d.ReduceOp.MAX)
     return float(t.item())
+
+
+def _job_value(world, tokens_per_step, steps, ms_max):
+    """Whole-job tokens/s: each of `world` replicas ran `steps` steps of `tokens_per_step` tokens,
+    and the job took as long as its slowest rank (`ms_max`)."""
+    return world * tokens_per_step * steps / (ms_max / 1e3)
 
 
 def run_reference(args, rank):
