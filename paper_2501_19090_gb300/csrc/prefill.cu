@@ -11,11 +11,15 @@
 // memory holds one weight row per TMEM lane: an epilogue warp's 32 lanes are 32 consecutive
 // weight rows, which for a fixed token land in 32 ascending output columns of one row of Y.
 //
-// Per CTA (192 threads): warp 0 issues TMA loads into a 4-stage shared-memory ring (A tile
+// Per CTA (576 threads): warp 0 issues TMA loads into a 4-stage shared-memory ring (A tile
 // 128 x 64, B tile 256 x 64, bf16, 128-byte swizzle), warp 1 owns the TMEM allocation and issues
-// tcgen05.mma (M=128, N=256, K=16) from one thread, warps 2-5 drain the fp32 accumulator
-// (128 lanes x 256 columns of TMEM) through tcgen05.ld. Every wait is bounded (globaltimer); on
-// timeout the CTA latches PIFA_ERR_TIMEOUT, drains what it has in flight and returns.
+// tcgen05.mma (M=128, N=256, K=16) from one thread, warps 2-17 drain the fp32 accumulator
+// (128 lanes x 256 columns of TMEM) through tcgen05.ld. The epilogue, not the tensor cores, was
+// the largest cost of this kernel (16 of 66 us at 4096 x 4096, r = 2048, T = 2048): its output is
+// a column scatter into Y of 2-byte stores. Sixteen warps issue them, and Y_p's hi/lo planes go
+// out as 16-byte stores after a transpose through shared memory. Every wait is bounded
+// (globaltimer); on timeout the CTA latches PIFA_ERR_TIMEOUT, drains what it has in flight and
+// returns.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -32,6 +36,8 @@ constexpr int BM = 128;  // weight rows per tile (MMA M)
 constexpr int BN = 256;  // tokens per tile (MMA N)
 constexpr int BK = 64;   // K per stage: one 128-byte swizzle row of bf16
 constexpr int STAGES = 4;
+constexpr int EPI_WARPS = 16;                 // epilogue warps: four per TMEM lane quarter
+constexpr int THREADS = 64 + 32 * EPI_WARPS;  // + the TMA producer and the MMA warp
 constexpr uint32_t A_BYTES = BM * BK * 2;
 constexpr uint32_t B_BYTES = BN * BK * 2;
 constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
@@ -59,7 +65,7 @@ struct GemmArgs {
 };
 
 template <int kEpi>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(THREADS, 1)
     pifa_umma_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, GemmArgs p) {
   extern __shared__ uint8_t smem_raw[];
@@ -146,9 +152,19 @@ __global__ void __launch_bounds__(192, 1)
       if (!mbar_wait(acc_full, 0, 100000000ull)) latch_status(p.status, PIFA_ERR_TIMEOUT);
     }
   } else {
-    // ---------------- epilogue: warps 2..5 ----------------
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    // ---------------- epilogue: warps 2 .. 2 + EPI_WARPS - 1 ----------------
+    // Warp w may access TMEM lanes 32 (w % 4) .. + 31, one quarter of the tile's weight rows; the
+    // EPI_WARPS / 4 warps of a quarter split the tile's tokens. Many warps keep the store issue
+    // rate up: the scattered 2-byte stores into Y's columns are instruction-bound.
+    constexpr int kSlices = EPI_WARPS / 4;
+    constexpr int kChunks = BN / 32 / kSlices;  // 32-token chunks per warp
+    const int q = warp & 3;
+    const int slice = (warp - 2) >> 2;
     const int row = m0 + q * 32 + lane;
+    // Y_p's hi and lo planes are written transposed through this warp's 4 KB of the stage memory
+    // (free once every MMA has completed) as 16-byte stores of 8 consecutive weight rows.
+    uint16_t* st_hi = reinterpret_cast<uint16_t*>(smem) + (warp - 2) * 2048;
+    uint16_t* st_lo = st_hi + 1024;
     const bool ok = mbar_wait(acc_full, 0, p.timeout_ns);
     if (!ok) latch_status(p.status, PIFA_ERR_TIMEOUT);
     tc_fence_after();
@@ -161,39 +177,51 @@ __global__ void __launch_bounds__(192, 1)
           col = -1;
         }
       }
+      bool range_err = false;
 #pragma unroll 1
-      for (int cc = 0; cc < BN / 32; ++cc) {
+      for (int ci = 0; ci < kChunks; ++ci) {
+        const int tb = n0 + (slice * kChunks + ci) * 32;  // first token of the chunk
         uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(cc * 32), v);
+        tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(tb - n0), v);
         tmem_ld_wait();
-        if (col >= 0) {
-          bool range_err = false;
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int t = n0 + cc * 32 + j;
-            if (t < p.N) {
-              const float f = __uint_as_float(v[j]);
-              const bf16 h = __float2bfloat16_rn(f);
-              p.Y[(int64_t)t * p.ldy + col] = h;
-              if (kEpi == EPI_SPLIT_BF16) {
-                reinterpret_cast<bf16*>(p.yp_hi)[(int64_t)t * p.ldyp + row] = h;
-                reinterpret_cast<bf16*>(p.yp_lo)[(int64_t)t * p.ldyp + row] =
-                    __float2bfloat16_rn(f - __bfloat162float(h));
-              } else if (kEpi == EPI_SPLIT_F16) {
-                float fs = f;
-                if (fabsf(fs) > 65504.0f) {
-                  range_err = true;
-                  fs = copysignf(65504.0f, fs);
-                }
-                const __half hh = __float2half_rn(fs);
-                reinterpret_cast<__half*>(p.yp_hi)[(int64_t)t * p.ldyp + row] = hh;
-                reinterpret_cast<__half*>(p.yp_lo)[(int64_t)t * p.ldyp + row] = __float2half_rn(fs - __half2float(hh));
-              }
+        for (int j = 0; j < 32; ++j) {
+          const float f = __uint_as_float(v[j]);
+          if (col >= 0 && tb + j < p.N) p.Y[(int64_t)(tb + j) * p.ldy + col] = __float2bfloat16_rn(f);
+          if (kEpi == EPI_SPLIT_BF16) {
+            const bf16 h = __float2bfloat16_rn(f);
+            st_hi[j * 32 + lane] = __bfloat16_as_ushort(h);
+            st_lo[j * 32 + lane] = __bfloat16_as_ushort(__float2bfloat16_rn(f - __bfloat162float(h)));
+          } else if (kEpi == EPI_SPLIT_F16) {
+            float fs = f;
+            if (fabsf(fs) > 65504.0f) {
+              range_err = true;
+              fs = copysignf(65504.0f, fs);
+            }
+            const __half hh = __float2half_rn(fs);
+            st_hi[j * 32 + lane] = __half_as_ushort(hh);
+            st_lo[j * 32 + lane] = __half_as_ushort(__float2half_rn(fs - __half2float(hh)));
+          }
+        }
+        if (kEpi != EPI_Y_ONLY) {
+          __syncwarp();
+          // 128 chunks of 16 bytes per plane: token j = c / 4, weight rows 8 (c % 4) .. + 7
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const int c = lane + 32 * k;
+            const int t = tb + (c >> 2);
+            const int rr = m0 + q * 32 + (c & 3) * 8;  // rows beyond M hold zeros (padding columns)
+            if (t < p.N && rr < p.ldyp) {
+              *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(p.yp_hi) + (int64_t)t * p.ldyp + rr) =
+                  *reinterpret_cast<const uint4*>(st_hi + c * 8);
+              *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(p.yp_lo) + (int64_t)t * p.ldyp + rr) =
+                  *reinterpret_cast<const uint4*>(st_lo + c * 8);
             }
           }
-          if (range_err) latch_status(p.status, PIFA_ERR_RANGE);
+          __syncwarp();  // the next chunk reuses the staging
         }
       }
+      if (range_err) latch_status(p.status, PIFA_ERR_RANGE);
     }
   }
 
@@ -213,7 +241,7 @@ int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtenso
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(prefill gemm)", e);
   dim3 grid((args.M + BM - 1) / BM, (args.N + BN - 1) / BN);
-  kern<<<grid, 192, SMEM_BYTES, stream>>>(a, b0, b1, args);
+  kern<<<grid, THREADS, SMEM_BYTES, stream>>>(a, b0, b1, args);
   e = cudaGetLastError();
   if (e != cudaSuccess) return pifa_fail_cuda("prefill gemm launch", e);
   return PIFA_OK;
