@@ -48,9 +48,10 @@ namespace {
 using namespace pifa;
 using bf16 = __nv_bfloat16;
 
-// Weight rows per CTA: RG MMA row groups of 16. RG = 4 (64 rows, K split over a cluster) reads
-// 4x less of the broadcast operand per weight byte than RG = 1 (16 rows, whole K per CTA) and wins
-// from T of a few tokens up; RG = 1 needs no cross-CTA reduction and wins at T <= 4.
+// Weight rows per CTA: RG MMA row groups of 16. Taller tiles read less of the broadcast operand
+// per weight byte (RG = 4 reads 4x less than RG = 1) but split K over larger clusters whose
+// partial tiles must be summed; RG = 1 (no cluster) wins at T <= 2, RG = 4 up to T = 8, RG = 2
+// with two token tiles.
 template <int RG>
 constexpr int kRowsOf = 16 * RG;
 constexpr int kChunk = 32;          // K elements per warp step (two k16 MMAs)
@@ -490,9 +491,11 @@ int64_t decode_workspace_bytes(const PifaShape& s) {
 
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
   const bool f16 = s.c_dtype == PIFA_DTYPE_FP16;
-  if (s.T <= 4) return f16 ? launch_decode_t<1, true, 1>(s, p, status, stream) : launch_decode_t<1, false, 1>(s, p, status, stream);
+  // Tile height by token count (measured on the 4096 x 4096, r = 2048 layer): 16 rows for T <= 2,
+  // 64 rows for T <= 8, 32 rows for T <= 16 (two token tiles).
+  if (s.T <= 2) return f16 ? launch_decode_t<1, true, 1>(s, p, status, stream) : launch_decode_t<1, false, 1>(s, p, status, stream);
   if (s.T <= 8) return f16 ? launch_decode_t<1, true, 4>(s, p, status, stream) : launch_decode_t<1, false, 4>(s, p, status, stream);
-  return f16 ? launch_decode_t<2, true, 4>(s, p, status, stream) : launch_decode_t<2, false, 4>(s, p, status, stream);
+  return f16 ? launch_decode_t<2, true, 2>(s, p, status, stream) : launch_decode_t<2, false, 2>(s, p, status, stream);
 }
 
 // ---- allocation-free decode entry point -------------------------------------------------------
