@@ -25,9 +25,9 @@
 // of rows g and g+8 of a row group at offset 8c as the A fragments of two k16 MMAs and the
 // matching 8 elements of token g as its B fragment: K is permuted identically in both operands,
 // which a dot product does not notice. The warps' partial tiles are summed through shared memory,
-// then the cluster's K slices through distributed shared memory, each CTA finishing 16 RG / ks
-// rows;
-// both sums run in a fixed order, so the result is deterministic.
+// then the cluster's K slices: each CTA stores its sums of a peer's rows into that peer's shared
+// memory and finishes 16 RG / ks rows itself. Both sums run in a fixed order, so the result is
+// deterministic.
 //
 // y_p enters the second contraction as a hi + lo pair of C's storage type (bf16 or fp16): C has
 // large entries and Y_np = C Y_p cancels, so rounding y_p to one bf16 alone would amplify its
@@ -146,6 +146,7 @@ struct DecodeArgs {
   int kcta;             // K columns per CTA (multiple of 32)
   int kc;               // K columns per shared-memory stage (multiple of 32, at most kcta)
   int stages;           // 1 (the CTA's whole K range resident) or 2
+  uint32_t recv_off;    // ks > 1: byte offset in dynamic shared memory of the receive buffer
   int* status;
   uint64_t timeout_ns;
 };
@@ -312,6 +313,9 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
 
   // 1. the warps' partial tiles, red[warp][row][t]; 2. their sum, in place in warp 0's tile
   float* red = reinterpret_cast<float*>(smem);
+  // ks > 1: the cluster's partial sums of the rows this CTA finishes, [source rank][token][row],
+  // beyond the stages and partial tiles (peers write it while this CTA may still be computing)
+  float* recv = reinterpret_cast<float*>(smem + a.recv_off);
 #pragma unroll
   for (int gq = 0; gq < RG; ++gq)
 #pragma unroll
@@ -330,28 +334,32 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
       r0p[8 * RP + 1] = v[3];
     }
   __syncthreads();
+  // CTA q of the cluster finishes rows [q rpr, (q + 1) rpr): every CTA stores its sums of those
+  // rows straight into q's receive buffer (remote stores before the cluster barrier, so no CTA
+  // reads another's shared memory after it and none has to wait for its peers before exiting)
+  const int rpr = kRows / a.ks;
   for (int idx = threadIdx.x; idx < kRows * 8 * NT; idx += kWarps * 32) {
     const int row = idx % kRows, t = idx / kRows;  // each (row, t) belongs to one thread
     float sum = 0.0f;
 #pragma unroll
     for (int w = 0; w < kWarps; ++w) sum += red[(w * kRows + row) * RP + t];
-    red[row * RP + t] = sum;
+    if (a.ks == 1)
+      red[row * RP + t] = sum;
+    else if (t < a.T)  // consecutive threads store consecutive words of the owner's buffer
+      st_dsmem_f32(mapa_shared(smem_u32(recv + (q * 8 * NT + t) * rpr + row % rpr), (uint32_t)(row / rpr)), sum);
   }
-  // 3. the cluster's K-slices: CTA q sums rows [q rpr, (q + 1) rpr) over all ranks, in rank order
+  // 3. the cluster's K-slices, summed in rank order
   if (a.ks > 1) cluster_sync_all();
   else __syncthreads();
-  const int rpr = kRows / a.ks;
   bool range_err = false;
   for (int idx = threadIdx.x; idx < rpr * 8 * NT; idx += kWarps * 32) {
     const int row = q * rpr + idx % rpr, t = idx / rpr;
     if (t >= a.T || row >= nrows) continue;
     float sum = 0.0f;
-    if (a.ks == 1) {
+    if (a.ks == 1)
       sum = red[row * RP + t];
-    } else {
-      const uint32_t la = smem_u32(red + row * RP + t);
-      for (int rk = 0; rk < a.ks; ++rk) sum += ld_dsmem_f32(mapa_shared(la, (uint32_t)rk));
-    }
+    else
+      for (int rk = 0; rk < a.ks; ++rk) sum += recv[(rk * 8 * NT + t) * rpr + idx % rpr];
     if (PHASE == 1 && a.yph != nullptr) {
       uint16_t h, l;
       split2<kF16C>(sum, h, l, range_err);
@@ -366,7 +374,6 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
     a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(sum);
   }
   if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
-  if (a.ks > 1) cluster_sync_relaxed();  // peers may still be reading this CTA's partial tile
 }
 
 // Once per kernel, device and size: the dynamic shared-memory limit, and the largest shared-memory
@@ -433,10 +440,14 @@ void plan_phase(int kRows, uint32_t budget, DecodeArgs& a) {
   a.kc = kc;
 }
 
-size_t smem_bytes(int kRows, const DecodeArgs& a, int NT) {
+// Dynamic shared memory of one CTA: the stages, overlaid by the warps' partial tiles, then (ks > 1)
+// the receive buffer at a.recv_off, which this sets.
+size_t smem_bytes(int kRows, DecodeArgs& a, int NT) {
   const size_t stages = (size_t)a.stages * kRows * row_pitch(a.kc);
   const size_t red = (size_t)kWarps * kRows * (8 * NT + 1) * 4;
-  return stages > red ? stages : red;
+  const size_t body = ((stages > red ? stages : red) + 15) / 16 * 16;
+  a.recv_off = (uint32_t)body;
+  return a.ks > 1 ? body + (size_t)kRows * 8 * NT * 4 : body;
 }
 
 template <int NT, bool kF16C, int RG>
@@ -463,8 +474,8 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   a.status = status;
   a.timeout_ns = pifa_wait_timeout_ns();
   plan_phase(kRows, kStageBudget1, a);
-  int st = launch_phase(decode_rows<1, NT, kF16C, RG>, kRows, a, smem_bytes(kRows, a, NT), stream,
-                        "decode phase 1 launch");
+  const size_t smem1 = smem_bytes(kRows, a, NT);  // sets a.recv_off, so before a is passed on
+  int st = launch_phase(decode_rows<1, NT, kF16C, RG>, kRows, a, smem1, stream, "decode phase 1 launch");
   if (st != PIFA_OK || s.m == s.r) return st;
   DecodeArgs b = a;
   b.A = reinterpret_cast<const uint16_t*>(p.C);
@@ -477,8 +488,8 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   b.yph = b.ypl = nullptr;
   b.cols = p.nonpiv;
   plan_phase(kRows, kStageBudget2, b);
-  return launch_phase(decode_rows<2, NT, kF16C, RG>, kRows, b, smem_bytes(kRows, b, NT), stream,
-                      "decode phase 2 launch");
+  const size_t smem2 = smem_bytes(kRows, b, NT);
+  return launch_phase(decode_rows<2, NT, kF16C, RG>, kRows, b, smem2, stream, "decode phase 2 launch");
 }
 
 }  // namespace

@@ -139,6 +139,10 @@ __device__ __forceinline__ float ld_dsmem_f32(uint32_t cluster_saddr) {
   asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(cluster_saddr) : "memory");
   return v;
 }
+// 32-bit store into the shared memory of a CTA of this cluster (shared::cluster address).
+__device__ __forceinline__ void st_dsmem_f32(uint32_t cluster_saddr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(cluster_saddr), "f"(v) : "memory");
+}
 // 128-bit load from this CTA's shared memory at a 32-bit shared-window address.
 __device__ __forceinline__ uint4 lds128(uint32_t saddr) {
   uint4 v;
