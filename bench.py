@@ -280,6 +280,7 @@ def run_ours(args, rank, world, local_rank):
         out["prefill"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src)
         out["prefill_fused"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src,
                                              variant=P.PIFA_VARIANT_PREFILL_FUSED)
+        out["decode_sweep"] = decode_sweep(dev, stream, hbm_peak, peak_src)
         out["cpu_baseline"] = cpu_baseline(lay, T)
     return out
 
@@ -312,6 +313,90 @@ def comparators(dev, lay, T, copies, stream):
             ms = e0.elapsed_time(e1) / reps
             res[f"{name}_T{Tq}"] = {"tokens_per_s": Tq / (ms / 1e3), "ms": ms}
     return res
+
+
+DECODE_SWEEP = [(inputs.ATTN7B, (1, 8, 16)), (inputs.MLP7B_GATE, (1,)), (inputs.MLP7B_DOWN, (1,)),
+                (inputs.ATTN70B, (1, 16)), (inputs.MLP70B_GATE, (1, 16))]
+
+
+def decode_sweep(dev, stream, hbm_peak, peak_src):
+    """The decode variant on every decode-sized layer shape (HBM-bound), beside the two-factor
+    low-rank layer of the same shape. Timing inputs only: W_p and C are seeded N(0, 1) bf16 and the
+    pivot set a seeded random r-subset (kernel time does not depend on the values); weight copies
+    rotate so that every call streams its weights from HBM."""
+    import torch
+    from paper_2501_19090_gb300 import pifa as P
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    out = []
+    for shape, Ts in DECODE_SWEEP:
+        m, n, r = shape.m, shape.n, shape.r
+        rng = np.random.default_rng(11)
+        perm = rng.permutation(m)
+        piv = torch.from_numpy(np.sort(perm[:r]).astype(np.int32)).to(dev)
+        nonp = torch.from_numpy(np.sort(perm[r:]).astype(np.int32)).to(dev)
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(12)
+        wbytes = 2 * r * (m + n - r)
+        copies = max(2, math.ceil(3 * l2 / wbytes))
+        Wps = [torch.randn((r, n), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
+        Cs = [torch.randn((m - r, r), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
+        lr_copies = max(2, math.ceil(3 * l2 / (2 * r * (m + n))))
+        Us = [torch.randn((m, r), device=dev, generator=gen).to(torch.bfloat16) for _ in range(lr_copies)]
+        Vs = [torch.randn((n, r), device=dev, generator=gen).to(torch.bfloat16) for _ in range(lr_copies)]
+        for T in Ts:
+            X = torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16)
+            Y = torch.empty((T, m), dtype=torch.bfloat16, device=dev)
+            variant = P.pifa_select_variant(T, m, n, r, P.PIFA_DTYPE_BF16)
+            ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant), dev, "sweep")
+
+            def step(i):
+                P.pifa_forward(X, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Y, variant=variant,
+                               workspace_tensor=ws, stream=stream)
+
+            with torch.cuda.stream(stream):
+                for i in range(4):
+                    step(i)
+            per_graph = copies * max(1, 32 // copies)
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for i in range(per_graph):
+                    step(i)
+            ms = _graph_ms(g, stream, replays=max(2, 256 // per_graph)) / per_graph
+            assert P.pifa_device_status(stream) == P.PIFA_OK
+            lr = lambda i: (X @ Vs[i % lr_copies]) @ Us[i % lr_copies].t()
+            with torch.cuda.stream(stream):
+                for i in range(4):
+                    lr(i)
+            g2 = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g2, stream=stream):
+                for i in range(per_graph):
+                    lr(i)
+            lr_ms = _graph_ms(g2, stream, replays=max(2, 256 // per_graph)) / per_graph
+            gbs = decode_bytes(T, m, n, r) / (ms / 1e3) / 1e9
+            out.append({"workload": f"{shape.name} decode T={T}", "us_per_call": ms * 1e3,
+                        "tokens_per_s": T / (ms / 1e3), "hbm_gbs": gbs, "frac": gbs / hbm_peak,
+                        "lowrank_us_per_call": lr_ms * 1e3, "speedup_vs_lowrank": lr_ms / ms,
+                        "weight_copies": copies, "peak_source": f"{peak_src} hbm_gbs"})
+            del g, g2
+        del Wps, Cs, Us, Vs
+        torch.cuda.empty_cache()
+    return out
+
+
+def _graph_ms(g, stream, replays):
+    import torch
+    for _ in range(2):
+        g.replay()
+    stream.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(replays):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    return e0.elapsed_time(e1) / replays
 
 
 def prefill_point(dev, lay, copies, stream, tc_peak, peak_src, variant=None):

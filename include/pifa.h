@@ -200,6 +200,18 @@ int pifa_device_status(void* cuda_stream);
  * undefined. Process-wide; PIFA_ERR_INVALID_ARG for ns < 0. */
 int pifa_set_wait_timeout(int64_t ns);
 
+/* pifa_set_decode_grid -- how the decode variant (T <= 16) lays out each of its two phases for
+ * calls made after this one (process-wide): PIFA_DECODE_GRID_AUTO (0, the default) runs a phase
+ * as waves of one-tile clusters, every CTA staging its weight rows at launch, while it takes at
+ * most two waves, and otherwise as a persistent grid of co-resident clusters that stream their
+ * tiles through a ring of TMA-filled stages; PIFA_DECODE_GRID_WAVES (1) and
+ * PIFA_DECODE_GRID_PERSISTENT (2) force one layout (a tuning and test knob: both compute the same
+ * result up to the summation order of fp32 partial sums). PIFA_ERR_INVALID_ARG for other values. */
+#define PIFA_DECODE_GRID_AUTO 0
+#define PIFA_DECODE_GRID_WAVES 1
+#define PIFA_DECODE_GRID_PERSISTENT 2
+int pifa_set_decode_grid(int mode);
+
 /* pifa_selftest_wait_timeout -- enqueues on `cuda_stream` a one-CTA kernel that waits, with the
  * current bound (pifa_set_wait_timeout), on an mbarrier that nothing arrives on, so the wait runs
  * out and PIFA_ERR_TIMEOUT is latched for pifa_device_status(). Checks the failure-detection path

@@ -29,11 +29,20 @@
 // memory and finishes 16 RG / ks rows itself. Both sums run in a fixed order, so the result is
 // deterministic.
 //
+// Layers with more row tiles than one wave of clusters holds run a second kernel, decode_stream:
+// a persistent grid (as many clusters as are co-resident) in which every cluster streams the
+// K-chunks of its tiles through a ring of shared-memory stages filled by 2-D TMA boxes (few large
+// copies: per-row bulk copies of 1-2 KB stream well below the HBM rate), with the CTA's K range
+// of the broadcast operand resident in shared memory for all its tiles (per-chunk L2 loads of it
+// wait behind the weight stream).
+//
 // y_p enters the second contraction as a hi + lo pair of C's storage type (bf16 or fp16): C has
 // large entries and Y_np = C Y_p cancels, so rounding y_p to one bf16 alone would amplify its
 // rounding error several-fold. Phase 1 splits each value once; phase 2 runs one MMA per plane.
+#include <atomic>
 #include <map>
 #include <mutex>
+#include <tuple>
 #include <utility>
 
 #include <cuda_bf16.h>
@@ -62,6 +71,9 @@ constexpr int kMaxCluster = 8;      // CTAs per cluster splitting K (portable cl
 // phase-1 CTA (and a phase-1 CTA its rows of W_p beside a phase-2 CTA).
 constexpr uint32_t kStageBudget1 = 144u * 1024u;
 constexpr uint32_t kStageBudget2 = 76u * 1024u;
+// decode_stream: shared memory of one CTA (two fit an SM), and its largest ring
+constexpr uint32_t kStreamBudget = 108u * 1024u;
+constexpr int kMaxStages = 8;
 
 __device__ __forceinline__ uint32_t pack2(uint16_t a, uint16_t b) { return (uint32_t)a | ((uint32_t)b << 16); }
 
@@ -146,7 +158,12 @@ struct DecodeArgs {
   int kcta;             // K columns per CTA (multiple of 32)
   int kc;               // K columns per shared-memory stage (multiple of 32, at most kcta)
   int stages;           // 1 (the CTA's whole K range resident) or 2
-  uint32_t recv_off;    // ks > 1: byte offset in dynamic shared memory of the receive buffer
+  uint32_t recv_off;    // ks > 1: byte offset in dynamic shared memory of the receive buffer(s)
+  // decode_stream only
+  int ntiles;           // row tiles of kRows rows
+  int ncl;              // clusters in the grid: cluster c owns tiles c, c + ncl, c + 2 ncl, ...
+  uint32_t bres_off;    // byte offset of the resident B rows (NB planes x T, pitch row_pitch(kcta))
+  uint32_t red_off;     // byte offset of the warps' partial tiles
   int* status;
   uint64_t timeout_ns;
 };
@@ -376,6 +393,236 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
   if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
 }
 
+// MMA row g of a 16-row group reads shared-memory row rho(g) = (g >> 1) | ((g & 1) << 2) of that
+// group in decode_stream's TMA blocks. A quarter warp's fragment loads (MMA rows 2i and 2i + 1,
+// four 16-byte columns each) then hit rows i and i + 4 of a 128-byte-swizzled block, whose chunks
+// the swizzle places in opposite halves of the 128-byte bank window: no bank conflicts.
+__device__ __forceinline__ int rho8(int g) { return (g >> 1) | ((g & 1) << 2); }
+
+// Persistent form of decode_rows. Cluster cid (of ncl) owns the row tiles cid, cid + ncl, ...;
+// CTA q of the cluster covers the K range [q kcta, (q + 1) kcta) of each. Its K range of the B
+// operand (NB planes x T rows) is copied into shared memory once, after the dependency wait, and
+// zero-padded to whole 32-column steps. The weights stream through `stages` stages of kc / 64 TMA
+// boxes each (64 columns x kRows rows, 128-byte swizzle, zero-filled beyond the layer), the
+// first stages issued before the wait. Per tile, the warps' partial tiles are summed as in
+// decode_rows, through a region of their own (the ring stays in flight), and the cluster's
+// partials through two alternating receive buffers.
+template <int PHASE, int NT, bool kF16C, int RG>
+__global__ void __launch_bounds__(kWarps * 32, 2)
+    decode_stream(const __grid_constant__ CUtensorMap tmA, DecodeArgs a) {
+  constexpr int kRows = kRowsOf<RG>;
+  constexpr int NB = PHASE == 1 ? 1 : 2;
+  constexpr bool kF16Mma = PHASE == 2 && kF16C;
+  constexpr int NU = RG == 1 ? 2 : 1;     // accumulator sets (alternate steps): shorter MMA chains
+  constexpr int RP = 8 * NT + 1;
+  constexpr uint32_t kBlk = kRows * 128;  // one TMA box: 64 columns x kRows rows
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  __shared__ uint64_t full[kMaxStages];
+  __shared__ uint64_t bbar;
+  __shared__ int s_cols[kRows];
+  pdl_launch_dependents();  // the next kernel may launch now and start staging its weights
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t stage_bytes = (uint32_t)(a.kc / 64) * kBlk;
+  const uint32_t bpitch = row_pitch(a.kcta);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, c = lane & 3;
+  const int q = (int)cluster_ctarank();
+  const int cid = (int)blockIdx.x / a.ks;
+  const int ntile = cid < a.ntiles ? (a.ntiles - 1 - cid) / a.ncl + 1 : 0;
+  const int k0 = q * a.kcta;
+  const int klen = max(0, min(a.kcta, a.K - k0));
+  const int nchunks = (klen + a.kc - 1) / a.kc;
+  const int nitems = ntile * nchunks;
+  auto tile_row0 = [&](int t) { return (int64_t)(cid + t * a.ncl) * kRows; };
+  auto tile_rows = [&](int64_t r0) { return (int)((int64_t)a.R - r0 < kRows ? (int64_t)a.R - r0 : kRows); };
+  // one thread stages item `it` (tile it / nchunks, K-chunk it % nchunks) into stage it % stages
+  auto issue = [&](int it) {
+    const int s = it % a.stages, j = it % nchunks;
+    const int len = min(a.kc, klen - j * a.kc);
+    const int nblk = (len + 63) / 64;
+    uint8_t* st = smem + s * stage_bytes;
+    mbar_arrive_expect_tx(&full[s], (uint32_t)nblk * kBlk);  // zero-filled parts count too
+    for (int b = 0; b < nblk; ++b)
+      tma_load_2d(smem_u32(st + b * kBlk), &tmA, k0 + j * a.kc + 64 * b, (int)tile_row0(it / nchunks), &full[s]);
+  };
+  if (threadIdx.x == 0) {
+    prefetch_tmap(&tmA);
+    for (int s = 0; s < a.stages; ++s) mbar_init(&full[s], 1);
+    mbar_init(&bbar, 1);
+    fence_mbar_init();
+    for (int it = 0; it < a.stages && it < nitems; ++it) issue(it);
+  }
+  if (ntile > 0)
+    for (int i = threadIdx.x; i < kRows; i += kWarps * 32) s_cols[i] = i < tile_rows(tile_row0(0)) ? a.cols[tile_row0(0) + i] : 0;
+  if (threadIdx.x == 0) pdl_wait_primary();
+  __syncthreads();
+
+  // B rows, resident: [0, klen rounded down to 8) by bulk copies, the rest up to whole steps by
+  // plain loads and zeros (the steps read up to kpad; the TMA boxes are zero beyond K as well)
+  uint8_t* bres = smem + a.bres_off;
+  const int kbulk = klen & ~7, kpad = (klen + kChunk - 1) / kChunk * kChunk;
+  if (warp == 0) {
+    const uint32_t bytes = (uint32_t)kbulk * 2u;
+    if (lane == 0) mbar_arrive_expect_tx(&bbar, bytes * (uint32_t)(NB * a.T));
+    __syncwarp();
+    if (bytes)
+      for (int i = lane; i < NB * a.T; i += 32)
+        bulk_copy_g2s(smem_u32(bres + i * bpitch), (i < a.T ? a.B0 : a.B1) + (int64_t)(i % a.T) * a.ldb + k0, bytes, &bbar);
+  }
+  const int wtail = kpad - kbulk;
+  if (wtail > 0)
+    for (int idx = threadIdx.x; idx < NB * a.T * wtail; idx += kWarps * 32) {
+      const int i = idx / wtail, col = kbulk + idx % wtail;
+      const uint16_t v = col < klen ? __ldcg((i < a.T ? a.B0 : a.B1) + (int64_t)(i % a.T) * a.ldb + k0 + col) : (uint16_t)0;
+      reinterpret_cast<uint16_t*>(bres + i * bpitch)[col] = v;
+    }
+  bool dead = false;
+  if (threadIdx.x == 0 && !mbar_wait(&bbar, 0, a.timeout_ns)) {
+    latch_status(a.status, PIFA_ERR_TIMEOUT);
+    dead = true;
+  }
+  dead = __syncthreads_or(dead);
+
+  const int arow = rho8(g);
+  const uint32_t lane_off = (uint32_t)arow * 128u + (uint32_t)((c ^ arow) << 4);
+  uint32_t boff[NB][NT];  // this lane's B row (token 8 nt + g, clamped to T - 1) and column 8 c
+#pragma unroll
+  for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+      boff[nb][nt] = smem_u32(bres) + (uint32_t)(nb * a.T + (nt * 8 + g < a.T ? nt * 8 + g : a.T - 1)) * bpitch + 16u * c;
+  float* red = reinterpret_cast<float*>(smem + a.red_off);
+  bool range_err = false;
+  const int rpr = kRows / a.ks;
+  for (int tt = 0; tt < ntile; ++tt) {
+    const int64_t row0 = tile_row0(tt);
+    const int nrows = tile_rows(row0);
+    if (tt > 0)  // the columns of this tile's rows, in flight while it computes
+      for (int i = threadIdx.x; i < kRows; i += kWarps * 32)
+        if (i < nrows) cp_async4(smem_u32(&s_cols[i]), a.cols + row0 + i);
+    float acc[NU][RG][NT][4];
+#pragma unroll
+    for (int u = 0; u < NU; ++u)
+#pragma unroll
+      for (int gq = 0; gq < RG; ++gq)
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) acc[u][gq][nt][0] = acc[u][gq][nt][1] = acc[u][gq][nt][2] = acc[u][gq][nt][3] = 0.0f;
+    for (int j = 0; j < nchunks; ++j) {
+      const int it = tt * nchunks + j;
+      const int s = it % a.stages;
+      const int nst = (min(a.kc, klen - j * a.kc) + kChunk - 1) / kChunk;
+      if (warp < nst) {
+        if (!dead && !mbar_wait(&full[s], (uint32_t)(it / a.stages) & 1u, a.timeout_ns)) {
+          latch_status(a.status, PIFA_ERR_TIMEOUT);
+          dead = true;
+        }
+        dead = __any_sync(0xffffffffu, dead);
+      }
+      if (!dead) {
+        const uint32_t sb = smem_u32(smem + s * stage_bytes) + lane_off;
+        const uint32_t bj = (uint32_t)(j * a.kc) * 2u;
+        // one 32-column step: the stage base is 1024-byte aligned and kBlk a multiple of 1024,
+        // so the odd step's chunk flip (bit 6) acts on lane_off alone
+        auto step = [&](int st, float (&ac)[RG][NT][4]) {
+          const uint32_t at = (sb + (uint32_t)(st >> 1) * kBlk) ^ ((uint32_t)(st & 1) << 6);
+          uint4 bv[NB][NT];
+#pragma unroll
+          for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) bv[nb][nt] = lds128(boff[nb][nt] + bj + (uint32_t)st * 64u);
+#pragma unroll
+          for (int gq = 0; gq < RG; ++gq) {
+            const uint4 wa = lds128(at + (uint32_t)(16 * gq) * 128u);      // MMA row g
+            const uint4 wb = lds128(at + (uint32_t)(16 * gq + 8) * 128u);  // MMA row g + 8
+#pragma unroll
+            for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+              for (int nt = 0; nt < NT; ++nt) {
+                mma16816<kF16Mma>(ac[gq][nt], wa, wb, bv[nb][nt].x, bv[nb][nt].y, false);
+                mma16816<kF16Mma>(ac[gq][nt], wa, wb, bv[nb][nt].z, bv[nb][nt].w, true);
+              }
+          }
+        };
+#pragma unroll 1
+        for (int st = warp; st < nst; st += kWarps * NU) {
+          step(st, acc[0]);
+          if (NU > 1 && st + kWarps < nst) step(st + kWarps, acc[NU - 1]);
+        }
+      }
+      if (it + a.stages < nitems) {  // refill stage s once every warp is done with it
+        dead = __syncthreads_or(dead);
+        if (threadIdx.x == 0 && !dead) issue(it + a.stages);
+      }
+    }
+    if (tt + 1 == ntile && threadIdx.x == 0) {
+      // nothing may still be landing in shared memory when the CTA exits
+      for (int it = nitems > a.stages ? nitems - a.stages : 0; it < nitems; ++it)
+        if (!mbar_wait(&full[it % a.stages], (uint32_t)(it / a.stages) & 1u, 100000000ull))
+          latch_status(a.status, PIFA_ERR_TIMEOUT);
+    }
+    __syncthreads();  // every warp is done with the previous tile's partials and columns
+
+    // the warps' partial tiles, red[warp][row][t] in weight-row order, and their sum
+#pragma unroll
+    for (int gq = 0; gq < RG; ++gq)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        float v[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          v[e] = acc[0][gq][nt][e];
+#pragma unroll
+          for (int u = 1; u < NU; ++u) v[e] += acc[u][gq][nt][e];
+        }
+        float* r0p = red + (warp * kRows + 16 * gq + arow) * RP + nt * 8 + 2 * c;
+        r0p[0] = v[0];
+        r0p[1] = v[1];
+        r0p[8 * RP] = v[2];
+        r0p[8 * RP + 1] = v[3];
+      }
+    __syncthreads();
+    // the cluster's partial sums, pushed into the owner's receive buffer (alternating by tile: a
+    // peer's next-tile stores cannot overtake the owner's reads, which precede its arrival at the
+    // next tile's barrier)
+    float* recv = reinterpret_cast<float*>(smem + a.recv_off) + (tt & 1) * (kRows * 8 * NT);
+    for (int idx = threadIdx.x; idx < kRows * 8 * NT; idx += kWarps * 32) {
+      const int row = idx % kRows, t = idx / kRows;
+      float sum = 0.0f;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) sum += red[(w * kRows + row) * RP + t];
+      if (a.ks == 1)
+        red[row * RP + t] = sum;
+      else if (t < a.T)
+        st_dsmem_f32(mapa_shared(smem_u32(recv + (q * 8 * NT + t) * rpr + row % rpr), (uint32_t)(row / rpr)), sum);
+    }
+    cp_async_wait_all();  // this thread's column loads (if any) have landed
+    if (a.ks > 1) cluster_sync_all();
+    else __syncthreads();
+    for (int idx = threadIdx.x; idx < rpr * 8 * NT; idx += kWarps * 32) {
+      const int row = q * rpr + idx % rpr, t = idx / rpr;
+      if (t >= a.T || row >= nrows) continue;
+      float sum = 0.0f;
+      if (a.ks == 1)
+        sum = red[row * RP + t];
+      else
+        for (int rk = 0; rk < a.ks; ++rk) sum += recv[(rk * 8 * NT + t) * rpr + idx % rpr];
+      if (PHASE == 1 && a.yph != nullptr) {
+        uint16_t h, l;
+        split2<kF16C>(sum, h, l, range_err);
+        a.yph[(int64_t)t * a.ldyp + row0 + row] = h;
+        a.ypl[(int64_t)t * a.ldyp + row0 + row] = l;
+      }
+      const int col = s_cols[row];
+      if ((unsigned)col >= (unsigned)a.m) {
+        latch_status(a.status, PIFA_ERR_DEVICE_INDEX);
+        continue;
+      }
+      a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(sum);
+    }
+    if (tt + 1 < ntile) __syncthreads();  // the partials and the columns are rewritten next tile
+  }
+  if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
+}
+
 // Once per kernel, device and size: the dynamic shared-memory limit, and the largest shared-memory
 // carveout, so that a phase-1 CTA and a phase-2 CTA fit on one SM together.
 int prepare_kernel(const void* fn, size_t smem, const char* what) {
@@ -450,9 +697,154 @@ size_t smem_bytes(int kRows, DecodeArgs& a, int NT) {
   return a.ks > 1 ? body + (size_t)kRows * 8 * NT * 4 : body;
 }
 
-template <int NT, bool kF16C, int RG>
-int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
+// Co-resident clusters of ks CTAs of `fn` with `smem` bytes of dynamic shared memory each, on the
+// current device (cached per kernel, device, cluster size and size). 0 if unknown.
+int max_clusters(const void* fn, int ks, size_t smem) {
+  static std::mutex mu;
+  static std::map<std::tuple<const void*, int, int, size_t>, int> cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  const auto key = std::make_tuple(fn, dev, ks, smem);
+  auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  int n = 0;
+  if (ks == 1) {
+    int per_sm = 0, sms = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kWarps * 32, smem) == cudaSuccess &&
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+      n = per_sm * sms;
+  } else {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)ks);
+    cfg.blockDim = dim3(kWarps * 32);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = (unsigned)ks;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    if (cudaOccupancyMaxActiveClusters(&n, fn, &cfg) != cudaSuccess) n = 0;
+  }
+  cudaGetLastError();  // a failed query leaves no sticky error behind
+  cache[key] = n;
+  return n;
+}
+
+std::atomic<int> g_decode_grid{PIFA_DECODE_GRID_AUTO};  // pifa_set_decode_grid
+
+int kcta_of(int K, int ks) { return ((K + ks - 1) / ks + kChunk - 1) / kChunk * kChunk; }
+
+int sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      n = 1;
+  }
+  return n;
+}
+
+// decode_stream's split of one phase into (ks, kcta, kc, stages, ntiles, ncl) and its shared memory
+// (returned, with 1 KB of alignment slack): the fewest CTAs per cluster giving at least two
+// (tile, K-range) units per SM, with resident B rows of at most a third of the budget; then
+// chunks of whole 64-column blocks, four stages where they fit.
+size_t plan_stream(const void* fn, int kRows, int NT, int NB, DecodeArgs& a, const char* what, int* st) {
+  auto round16 = [](size_t b) { return (b + 15) / 16 * 16; };
+  a.ntiles = (a.R + kRows - 1) / kRows;
+  const size_t red = round16((size_t)kWarps * kRows * (8 * NT + 1) * 4);
+  const size_t recv1 = (size_t)kRows * 8 * NT * 4;
+  int ks = 1;
+  while (ks < kMaxCluster && ((int64_t)a.ntiles * ks < 2 * sm_count() ||
+                              (size_t)NB * a.T * row_pitch(kcta_of(a.K, ks)) > kStreamBudget / 3))
+    ks *= 2;
+  a.ks = ks;
+  a.kcta = kcta_of(a.K, ks);
+  const size_t bres = round16((size_t)NB * a.T * row_pitch(a.kcta));
+  const size_t side = bres + red + (ks > 1 ? 2 * recv1 : 0);
+  const size_t blk = (size_t)kRows * 128;
+  const size_t ring = kStreamBudget > side + 2 * blk ? kStreamBudget - side : 2 * blk;
+  const int kblocks = (a.kcta + 63) / 64;
+  int nblk = (int)(ring / (4 * blk));
+  if (nblk < 1) nblk = 1;
+  if (nblk > kblocks) nblk = kblocks;
+  a.kc = 64 * nblk;
+  const size_t stage = (size_t)nblk * blk;
+  a.stages = (int)(ring / stage);
+  if (a.stages > kMaxStages) a.stages = kMaxStages;
+  if (a.stages < 2) a.stages = 2;
+  a.bres_off = (uint32_t)(a.stages * stage);
+  a.red_off = a.bres_off + (uint32_t)bres;
+  a.recv_off = a.red_off + (uint32_t)red;
+  const size_t smem = 1024 + a.recv_off + (ks > 1 ? 2 * recv1 : 0);
+  *st = prepare_kernel(fn, smem, what);
+  if (*st != PIFA_OK) return 0;
+  // as many clusters as are co-resident, but the tiles dealt evenly: rounds = ceil(ntiles / cap)
+  // tiles for every cluster (a last round on a few clusters would run at their share of HBM alone)
+  const int cap = max_clusters(fn, ks, smem) > 0 ? max_clusters(fn, ks, smem) : 1;
+  const int rounds = (a.ntiles + cap - 1) / cap;
+  a.ncl = (a.ntiles + rounds - 1) / rounds;
+  return smem;
+}
+
+template <typename Kern>
+int launch_stream(Kern kernel, const CUtensorMap& tm, const DecodeArgs& args, size_t smem, cudaStream_t stream,
+                  const char* what) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(args.ncl * args.ks));
+  cfg.blockDim = dim3(kWarps * 32);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)args.ks;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, tm, args);
+  if (e != cudaSuccess) return pifa_fail_cuda(what, e);
+  return PIFA_OK;
+}
+
+// One phase: decode_rows (16 RG-row tiles) or decode_stream (16 RGS-row tiles, over a TMA map of
+// the weights in their storage type `dtype`). The stream reads its B operand once per CTA, so its
+// tiles can be taller than decode_rows': 32 rows make 4 KB TMA boxes (2 KB boxes of 16 rows
+// issue too many copies per byte).
+template <int PHASE, int NT, bool kF16C, int RG, int RGS>
+int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, cudaStream_t stream) {
   constexpr int kRows = kRowsOf<RG>;
+  const char* what = PHASE == 1 ? "decode phase 1 launch" : "decode phase 2 launch";
+  const auto kr = decode_rows<PHASE, NT, kF16C, RG>;
+  plan_phase(kRows, budget, a);
+  const size_t smem = smem_bytes(kRows, a, NT);
+  int st = prepare_kernel(reinterpret_cast<const void*>(kr), smem, what);
+  if (st != PIFA_OK) return st;
+  // decode_rows in waves while a phase takes at most two of them (its weights staged at launch,
+  // before the dependency wait, outweigh the persistent grid's streaming), and always for two
+  // token tiles (T > 8: measured slower persistent, the per-tile reductions of 16 tokens being
+  // twice as long); else decode_stream
+  const int tiles = (a.R + kRows - 1) / kRows;
+  const int mode = g_decode_grid.load(std::memory_order_relaxed);
+  if (mode == PIFA_DECODE_GRID_WAVES ||
+      (mode == PIFA_DECODE_GRID_AUTO &&
+       (NT > 1 || tiles <= 2 * max_clusters(reinterpret_cast<const void*>(kr), a.ks, smem))))
+    return launch_phase(kr, kRows, a, smem, stream, what);
+  const auto ks = decode_stream<PHASE, NT, kF16C, RGS>;
+  const size_t smem_s =
+      plan_stream(reinterpret_cast<const void*>(ks), kRowsOf<RGS>, NT, PHASE == 1 ? 1 : 2, a, what, &st);
+  if (st != PIFA_OK) return st;
+  CUtensorMap tm;
+  if ((st = make_tmap_2d(&tm, dtype, a.A, a.R, a.K, a.lda, 64, kRowsOf<RGS>)) != PIFA_OK) return st;
+  return launch_stream(ks, tm, a, smem_s, stream, what);
+}
+
+template <int NT, bool kF16C, int RG, int RGS>
+int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
   const int64_t ldyp = (s.r + 7) / 8 * 8;  // 16-byte rows keep the fragment loads aligned
   uint16_t* yph = reinterpret_cast<uint16_t*>(p.ws);
   uint16_t* ypl = yph + s.T * ldyp;
@@ -473,9 +865,7 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   a.T = (int)s.T;
   a.status = status;
   a.timeout_ns = pifa_wait_timeout_ns();
-  plan_phase(kRows, kStageBudget1, a);
-  const size_t smem1 = smem_bytes(kRows, a, NT);  // sets a.recv_off, so before a is passed on
-  int st = launch_phase(decode_rows<1, NT, kF16C, RG>, kRows, a, smem1, stream, "decode phase 1 launch");
+  int st = launch_one_phase<1, NT, kF16C, RG, RGS>(a, kStageBudget1, PIFA_DTYPE_BF16, stream);
   if (st != PIFA_OK || s.m == s.r) return st;
   DecodeArgs b = a;
   b.A = reinterpret_cast<const uint16_t*>(p.C);
@@ -487,12 +877,17 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   b.ldb = ldyp;
   b.yph = b.ypl = nullptr;
   b.cols = p.nonpiv;
-  plan_phase(kRows, kStageBudget2, b);
-  const size_t smem2 = smem_bytes(kRows, b, NT);
-  return launch_phase(decode_rows<2, NT, kF16C, RG>, kRows, b, smem2, stream, "decode phase 2 launch");
+  return launch_one_phase<2, NT, kF16C, RG, RGS>(b, kStageBudget2, (int)s.c_dtype, stream);
 }
 
 }  // namespace
+
+extern "C" int pifa_set_decode_grid(int mode) {
+  if (mode != PIFA_DECODE_GRID_AUTO && mode != PIFA_DECODE_GRID_WAVES && mode != PIFA_DECODE_GRID_PERSISTENT)
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "decode grid mode must be 0 (auto), 1 (waves) or 2 (persistent)");
+  g_decode_grid.store(mode, std::memory_order_relaxed);
+  return PIFA_OK;
+}
 
 int64_t decode_workspace_bytes(const PifaShape& s) {
   // y_p as hi and lo planes of 2-byte elements, T rows of pitch round_up(r, 8) each, rounded up
@@ -504,9 +899,12 @@ int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaSt
   const bool f16 = s.c_dtype == PIFA_DTYPE_FP16;
   // Tile height by token count (measured on the 4096 x 4096, r = 2048 layer): 16 rows for T <= 2,
   // 64 rows for T <= 8, 32 rows for T <= 16 (two token tiles).
-  if (s.T <= 2) return f16 ? launch_decode_t<1, true, 1>(s, p, status, stream) : launch_decode_t<1, false, 1>(s, p, status, stream);
-  if (s.T <= 8) return f16 ? launch_decode_t<1, true, 4>(s, p, status, stream) : launch_decode_t<1, false, 4>(s, p, status, stream);
-  return f16 ? launch_decode_t<2, true, 2>(s, p, status, stream) : launch_decode_t<2, false, 2>(s, p, status, stream);
+  // Persistent-grid tiles (layers beyond two waves): 32 rows (4 KB TMA boxes) at any T.
+  if (s.T <= 2)
+    return f16 ? launch_decode_t<1, true, 1, 2>(s, p, status, stream) : launch_decode_t<1, false, 1, 2>(s, p, status, stream);
+  if (s.T <= 8)
+    return f16 ? launch_decode_t<1, true, 4, 2>(s, p, status, stream) : launch_decode_t<1, false, 4, 2>(s, p, status, stream);
+  return f16 ? launch_decode_t<2, true, 2, 2>(s, p, status, stream) : launch_decode_t<2, false, 2, 2>(s, p, status, stream);
 }
 
 // ---- allocation-free decode entry point -------------------------------------------------------

@@ -35,12 +35,16 @@ PIFA_VARIANT_DECODE = 1
 PIFA_VARIANT_PREFILL_SPLIT = 2
 PIFA_VARIANT_PREFILL_FUSED = 3
 
+PIFA_DECODE_GRID_AUTO = 0
+PIFA_DECODE_GRID_WAVES = 1
+PIFA_DECODE_GRID_PERSISTENT = 2
+
 # every symbol include/pifa.h declares
 EXPORTS = (
     "pifa_forward", "pifa_forward_variant", "pifa_workspace_size", "pifa_select_variant",
     "pifa_variant_name", "pifa_compress", "pifa_validate_indices", "pifa_device_status",
     "pifa_status_string", "pifa_last_error", "pifa_version", "pifa_forward_decode_noalloc",
-    "pifa_set_wait_timeout", "pifa_selftest_wait_timeout",
+    "pifa_set_wait_timeout", "pifa_selftest_wait_timeout", "pifa_set_decode_grid",
 )
 
 
@@ -101,6 +105,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.pifa_set_wait_timeout.restype = ctypes.c_int
         lib.pifa_selftest_wait_timeout.argtypes = [_VP]
         lib.pifa_selftest_wait_timeout.restype = ctypes.c_int
+        lib.pifa_set_decode_grid.argtypes = [ctypes.c_int]
+        lib.pifa_set_decode_grid.restype = ctypes.c_int
         lib.pifa_version.argtypes = []
         lib.pifa_version.restype = ctypes.c_char_p
         _lib_handle = lib
@@ -129,6 +135,11 @@ def pifa_status_string(status: int) -> str:
 def pifa_set_wait_timeout(ns: int) -> None:
     """Bound of every device-side wait of later launches, in ns (0 restores the default 1 s)."""
     _check(_lib().pifa_set_wait_timeout(int(ns)), "pifa_set_wait_timeout")
+
+
+def pifa_set_decode_grid(mode: int) -> None:
+    """Layout of the decode phases for later calls: PIFA_DECODE_GRID_AUTO, _WAVES or _PERSISTENT."""
+    _check(_lib().pifa_set_decode_grid(int(mode)), "pifa_set_decode_grid")
 
 
 def pifa_selftest_wait_timeout(stream=None) -> None:

@@ -197,16 +197,43 @@ def test_mlp7b_three_layers_back_to_back(T):
         check(Y[rows], ref, f"{L.name} T={T}")
 
 
-@pytest.mark.parametrize("T", [1, 16, 4096])
+@pytest.mark.parametrize("T", [1, 8, 16, 4096])
 def test_llama70b_qo(T):
     L = layer_for(8192, 8192, 4096, 0, "library")
     parity(L, T, sample=256)
 
 
-@pytest.mark.parametrize("T", [1, 16, 4096])
+@pytest.mark.parametrize("T", [1, 8, 16, 4096])
 def test_llama70b_gate_up(T):
     L = layer_for(28672, 8192, 4096, 0, "synthetic")
     parity(L, T, sample=128)
+
+
+@pytest.mark.parametrize("T", [1, 3, 8, 16])
+@pytest.mark.parametrize("grid", [P.PIFA_DECODE_GRID_PERSISTENT, P.PIFA_DECODE_GRID_WAVES])
+def test_decode_grids_many_tiles_ragged(T, grid):
+    """Both decode layouts on a layer with more row tiles than co-resident clusters: the
+    persistent grid (every cluster streaming several tiles through its TMA-filled stage ring) and
+    waves of one-tile clusters; ragged K in both phases (520 and 264 columns), a partial last
+    tile."""
+    L = layer_for(40000, 520, 264, 3, "synthetic")
+    P.pifa_set_decode_grid(grid)
+    try:
+        parity(L, T, P.PIFA_VARIANT_DECODE)
+    finally:
+        P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
+
+
+@pytest.mark.parametrize("T", [2, 8, 16])
+def test_decode_persistent_grid_fp16_c_and_padding(T):
+    """The persistent decode grid with C stored in fp16 (its TMA map in C's type), on padded
+    pitches that hold NaN (the TMA boxes must not read past K)."""
+    L = layer_for(3000, 1000, 600, 4, "synthetic", "fp16")
+    P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_PERSISTENT)
+    try:
+        parity(L, T, P.PIFA_VARIANT_DECODE, ldx=1000 + 24, ldwp=1000 + 40, ldc=600 + 16)
+    finally:
+        P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
 # ---------------------------------------------------------------------------------------------

@@ -47,6 +47,16 @@ def test_status_and_variant_strings(lib):
     assert "sm_103a" in P.pifa_version()
 
 
+def test_decode_grid_setter(lib):
+    """The decode layout knob takes the three declared modes and rejects anything else (no GPU
+    work: the mode only steers later launches)."""
+    for mode in (P.PIFA_DECODE_GRID_WAVES, P.PIFA_DECODE_GRID_PERSISTENT, P.PIFA_DECODE_GRID_AUTO):
+        assert lib.pifa_set_decode_grid(mode) == P.PIFA_OK
+    for bad in (-1, 3, 99):
+        assert lib.pifa_set_decode_grid(bad) == P.PIFA_ERR_INVALID_ARG
+    assert lib.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO) == P.PIFA_OK
+
+
 def test_selector(lib):
     assert P.pifa_select_variant(1, 4096, 4096, 2048) == P.PIFA_VARIANT_DECODE
     assert P.pifa_select_variant(16, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE
