@@ -399,16 +399,20 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
 // the swizzle places in opposite halves of the 128-byte bank window: no bank conflicts.
 __device__ __forceinline__ int rho8(int g) { return (g >> 1) | ((g & 1) << 2); }
 
-// Persistent form of decode_rows. Cluster cid (of ncl) owns the row tiles cid, cid + ncl, ...;
-// CTA q of the cluster covers the K range [q kcta, (q + 1) kcta) of each. Its K range of the B
-// operand (NB planes x T rows) is copied into shared memory once, after the dependency wait, and
-// zero-padded to whole 32-column steps. The weights stream through `stages` stages of kc / 64 TMA
-// boxes each (64 columns x kRows rows, 128-byte swizzle, zero-filled beyond the layer), the
-// first stages issued before the wait. Per tile, the warps' partial tiles are summed as in
-// decode_rows, through a region of their own (the ring stays in flight), and the cluster's
-// partials through two alternating receive buffers.
+// Persistent form of decode_rows, warp-specialised. Cluster cid (of ncl) owns the row tiles cid,
+// cid + ncl, ...; CTA q of the cluster covers the K range [q kcta, (q + 1) kcta) of each. A producer
+// warp streams the weights through `stages` stages of kc / 64 TMA boxes each (64 columns x kRows
+// rows, 128-byte swizzle, zero-filled beyond the layer), the first stages before the dependency
+// wait, each later one as soon as all eight consumer warps have released the stage (an "empty"
+// mbarrier): issuing never stalls the MMAs. The consumers hold their K range of the B operand
+// (NB planes x T rows) in shared memory, copied once after the dependency wait and zero-padded to
+// whole 32-column steps. Per tile the warps' partial tiles are summed through a region of their
+// own, and the cluster's partials are pushed into the owners' receive buffers (two, alternating
+// by tile) with mbarrier hand-offs in both directions -- "ready" when a source's pushes are
+// visible, "released" when an owner has read them -- instead of cluster barriers, which the
+// producer, running ahead, could not join.
 template <int PHASE, int NT, bool kF16C, int RG>
-__global__ void __launch_bounds__(kWarps * 32, 2)
+__global__ void __launch_bounds__((kWarps + 1) * 32, 2)
     decode_stream(const __grid_constant__ CUtensorMap tmA, DecodeArgs a) {
   constexpr int kRows = kRowsOf<RG>;
   constexpr int NB = PHASE == 1 ? 1 : 2;
@@ -416,9 +420,10 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
   constexpr int NU = RG == 1 ? 2 : 1;     // accumulator sets (alternate steps): shorter MMA chains
   constexpr int RP = 8 * NT + 1;
   constexpr uint32_t kBlk = kRows * 128;  // one TMA box: 64 columns x kRows rows
+  constexpr uint32_t kCons = kWarps * 32; // consumer threads (named barrier 1)
   extern __shared__ __align__(128) uint8_t smem_raw[];
-  __shared__ uint64_t full[kMaxStages];
-  __shared__ uint64_t bbar;
+  __shared__ uint64_t full[kMaxStages], empty[kMaxStages];
+  __shared__ uint64_t bbar, rready[2], rfree[2];
   __shared__ int s_cols[kRows];
   pdl_launch_dependents();  // the next kernel may launch now and start staging its weights
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -434,27 +439,53 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
   const int nitems = ntile * nchunks;
   auto tile_row0 = [&](int t) { return (int64_t)(cid + t * a.ncl) * kRows; };
   auto tile_rows = [&](int64_t r0) { return (int)((int64_t)a.R - r0 < kRows ? (int64_t)a.R - r0 : kRows); };
-  // one thread stages item `it` (tile it / nchunks, K-chunk it % nchunks) into stage it % stages
-  auto issue = [&](int it) {
-    const int s = it % a.stages, j = it % nchunks;
-    const int len = min(a.kc, klen - j * a.kc);
-    const int nblk = (len + 63) / 64;
-    uint8_t* st = smem + s * stage_bytes;
-    mbar_arrive_expect_tx(&full[s], (uint32_t)nblk * kBlk);  // zero-filled parts count too
-    for (int b = 0; b < nblk; ++b)
-      tma_load_2d(smem_u32(st + b * kBlk), &tmA, k0 + j * a.kc + 64 * b, (int)tile_row0(it / nchunks), &full[s]);
-  };
   if (threadIdx.x == 0) {
-    prefetch_tmap(&tmA);
-    for (int s = 0; s < a.stages; ++s) mbar_init(&full[s], 1);
+    for (int s = 0; s < a.stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], kWarps);
+    }
     mbar_init(&bbar, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&rready[b], (uint32_t)a.ks);  // one arrival per source CTA
+      mbar_init(&rfree[b], (uint32_t)a.ks);   // one arrival per owner CTA
+    }
     fence_mbar_init();
-    for (int it = 0; it < a.stages && it < nitems; ++it) issue(it);
   }
+  // the peers' barriers are initialised before anyone arrives on them remotely
+  if (a.ks > 1) cluster_sync_all();
+  else __syncthreads();
+
+  if (warp == kWarps) {  // ---- producer ----
+    if (lane == 0) {
+      prefetch_tmap(&tmA);
+      int issued = 0;
+      for (int it = 0; it < nitems; ++it) {
+        const int s = it % a.stages, j = it % nchunks;
+        if (it >= a.stages && !mbar_wait(&empty[s], (uint32_t)((it / a.stages) - 1) & 1u, a.timeout_ns)) {
+          latch_status(a.status, PIFA_ERR_TIMEOUT);
+          break;
+        }
+        const int len = min(a.kc, klen - j * a.kc);
+        const int nblk = (len + 63) / 64;
+        uint8_t* st = smem + s * stage_bytes;
+        mbar_arrive_expect_tx(&full[s], (uint32_t)nblk * kBlk);  // zero-filled parts count too
+        for (int b = 0; b < nblk; ++b)
+          tma_load_2d(smem_u32(st + b * kBlk), &tmA, k0 + j * a.kc + 64 * b, (int)tile_row0(it / nchunks), &full[s]);
+        issued = it + 1;
+      }
+      // nothing may land in shared memory after the CTA retires: wait for the last copies
+      for (int it = issued > a.stages ? issued - a.stages : 0; it < issued; ++it)
+        if (!mbar_wait(&full[it % a.stages], (uint32_t)(it / a.stages) & 1u, 100000000ull))
+          latch_status(a.status, PIFA_ERR_TIMEOUT);
+    }
+    return;  // from here on the consumers synchronise on named barrier 1 only
+  }
+
+  // ---- consumers ----
   if (ntile > 0)
-    for (int i = threadIdx.x; i < kRows; i += kWarps * 32) s_cols[i] = i < tile_rows(tile_row0(0)) ? a.cols[tile_row0(0) + i] : 0;
+    for (int i = threadIdx.x; i < kRows; i += kCons) s_cols[i] = i < tile_rows(tile_row0(0)) ? a.cols[tile_row0(0) + i] : 0;
   if (threadIdx.x == 0) pdl_wait_primary();
-  __syncthreads();
+  named_barrier_sync(1, kCons);
 
   // B rows, resident: [0, klen rounded down to 8) by bulk copies, the rest up to whole steps by
   // plain loads and zeros (the steps read up to kpad; the TMA boxes are zero beyond K as well)
@@ -470,7 +501,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
   }
   const int wtail = kpad - kbulk;
   if (wtail > 0)
-    for (int idx = threadIdx.x; idx < NB * a.T * wtail; idx += kWarps * 32) {
+    for (int idx = threadIdx.x; idx < NB * a.T * wtail; idx += kCons) {
       const int i = idx / wtail, col = kbulk + idx % wtail;
       const uint16_t v = col < klen ? __ldcg((i < a.T ? a.B0 : a.B1) + (int64_t)(i % a.T) * a.ldb + k0 + col) : (uint16_t)0;
       reinterpret_cast<uint16_t*>(bres + i * bpitch)[col] = v;
@@ -480,7 +511,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
     latch_status(a.status, PIFA_ERR_TIMEOUT);
     dead = true;
   }
-  dead = __syncthreads_or(dead);
+  dead = named_barrier_or(1, kCons, dead);
 
   const int arow = rho8(g);
   const uint32_t lane_off = (uint32_t)arow * 128u + (uint32_t)((c ^ arow) << 4);
@@ -497,7 +528,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
     const int64_t row0 = tile_row0(tt);
     const int nrows = tile_rows(row0);
     if (tt > 0)  // the columns of this tile's rows, in flight while it computes
-      for (int i = threadIdx.x; i < kRows; i += kWarps * 32)
+      for (int i = threadIdx.x; i < kRows; i += kCons)
         if (i < nrows) cp_async4(smem_u32(&s_cols[i]), a.cols + row0 + i);
     float acc[NU][RG][NT][4];
 #pragma unroll
@@ -516,52 +547,44 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
           dead = true;
         }
         dead = __any_sync(0xffffffffu, dead);
-      }
-      if (!dead) {
-        const uint32_t sb = smem_u32(smem + s * stage_bytes) + lane_off;
-        const uint32_t bj = (uint32_t)(j * a.kc) * 2u;
-        // one 32-column step: the stage base is 1024-byte aligned and kBlk a multiple of 1024,
-        // so the odd step's chunk flip (bit 6) acts on lane_off alone
-        auto step = [&](int st, float (&ac)[RG][NT][4]) {
-          const uint32_t at = (sb + (uint32_t)(st >> 1) * kBlk) ^ ((uint32_t)(st & 1) << 6);
-          uint4 bv[NB][NT];
-#pragma unroll
-          for (int nb = 0; nb < NB; ++nb)
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) bv[nb][nt] = lds128(boff[nb][nt] + bj + (uint32_t)st * 64u);
-#pragma unroll
-          for (int gq = 0; gq < RG; ++gq) {
-            const uint4 wa = lds128(at + (uint32_t)(16 * gq) * 128u);      // MMA row g
-            const uint4 wb = lds128(at + (uint32_t)(16 * gq + 8) * 128u);  // MMA row g + 8
+        if (!dead) {
+          const uint32_t sb = smem_u32(smem + s * stage_bytes) + lane_off;
+          const uint32_t bj = (uint32_t)(j * a.kc) * 2u;
+          // one 32-column step: the stage base is 1024-byte aligned and kBlk a multiple of 1024,
+          // so the odd step's chunk flip (bit 6) acts on lane_off alone
+          auto step = [&](int st, float (&ac)[RG][NT][4]) {
+            const uint32_t at = (sb + (uint32_t)(st >> 1) * kBlk) ^ ((uint32_t)(st & 1) << 6);
+            uint4 bv[NB][NT];
 #pragma unroll
             for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-              for (int nt = 0; nt < NT; ++nt) {
-                mma16816<kF16Mma>(ac[gq][nt], wa, wb, bv[nb][nt].x, bv[nb][nt].y, false);
-                mma16816<kF16Mma>(ac[gq][nt], wa, wb, bv[nb][nt].z, bv[nb][nt].w, true);
-              }
-          }
-        };
+              for (int nt = 0; nt < NT; ++nt) bv[nb][nt] = lds128(boff[nb][nt] + bj + (uint32_t)st * 64u);
+#pragma unroll
+            for (int gq = 0; gq < RG; ++gq) {
+              const uint4 wa = lds128(at + (uint32_t)(16 * gq) * 128u);      // MMA row g
+              const uint4 wb = lds128(at + (uint32_t)(16 * gq + 8) * 128u);  // MMA row g + 8
+#pragma unroll
+              for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) {
+                  mma16816<kF16Mma>(ac[gq][nt], wa, wb, bv[nb][nt].x, bv[nb][nt].y, false);
+                  mma16816<kF16Mma>(ac[gq][nt], wa, wb, bv[nb][nt].z, bv[nb][nt].w, true);
+                }
+            }
+          };
 #pragma unroll 1
-        for (int st = warp; st < nst; st += kWarps * NU) {
-          step(st, acc[0]);
-          if (NU > 1 && st + kWarps < nst) step(st + kWarps, acc[NU - 1]);
+          for (int st = warp; st < nst; st += kWarps * NU) {
+            step(st, acc[0]);
+            if (NU > 1 && st + kWarps < nst) step(st + kWarps, acc[NU - 1]);
+          }
         }
       }
-      if (it + a.stages < nitems) {  // refill stage s once every warp is done with it
-        dead = __syncthreads_or(dead);
-        if (threadIdx.x == 0 && !dead) issue(it + a.stages);
-      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[s]);  // this warp is done with stage s
     }
-    if (tt + 1 == ntile && threadIdx.x == 0) {
-      // nothing may still be landing in shared memory when the CTA exits
-      for (int it = nitems > a.stages ? nitems - a.stages : 0; it < nitems; ++it)
-        if (!mbar_wait(&full[it % a.stages], (uint32_t)(it / a.stages) & 1u, 100000000ull))
-          latch_status(a.status, PIFA_ERR_TIMEOUT);
-    }
-    __syncthreads();  // every warp is done with the previous tile's partials and columns
+    named_barrier_sync(1, kCons);  // every warp is done with the previous tile's partials and columns
 
-    // the warps' partial tiles, red[warp][row][t] in weight-row order, and their sum
+    // the warps' partial tiles, red[warp][row][t] in weight-row order
 #pragma unroll
     for (int gq = 0; gq < RG; ++gq)
 #pragma unroll
@@ -579,12 +602,16 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
         r0p[8 * RP] = v[2];
         r0p[8 * RP + 1] = v[3];
       }
-    __syncthreads();
-    // the cluster's partial sums, pushed into the owner's receive buffer (alternating by tile: a
-    // peer's next-tile stores cannot overtake the owner's reads, which precede its arrival at the
-    // next tile's barrier)
-    float* recv = reinterpret_cast<float*>(smem + a.recv_off) + (tt & 1) * (kRows * 8 * NT);
-    for (int idx = threadIdx.x; idx < kRows * 8 * NT; idx += kWarps * 32) {
+    const int b = tt & 1;
+    float* recv = reinterpret_cast<float*>(smem + a.recv_off) + b * (kRows * 8 * NT);
+    if (a.ks > 1 && tt >= 2 && threadIdx.x == 0 &&
+        !mbar_wait_cluster(&rfree[b], (uint32_t)((tt - 2) >> 1) & 1u, a.timeout_ns)) {
+      latch_status(a.status, PIFA_ERR_TIMEOUT);  // every owner has read this buffer's last pushes
+      dead = true;
+    }
+    dead = named_barrier_or(1, kCons, dead);
+    // the sum over the warps; with a cluster, pushed into the owner's receive buffer
+    for (int idx = threadIdx.x; idx < kRows * 8 * NT; idx += kCons) {
       const int row = idx % kRows, t = idx / kRows;
       float sum = 0.0f;
 #pragma unroll
@@ -595,9 +622,21 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
         st_dsmem_f32(mapa_shared(smem_u32(recv + (q * 8 * NT + t) * rpr + row % rpr), (uint32_t)(row / rpr)), sum);
     }
     cp_async_wait_all();  // this thread's column loads (if any) have landed
-    if (a.ks > 1) cluster_sync_all();
-    else __syncthreads();
-    for (int idx = threadIdx.x; idx < rpr * 8 * NT; idx += kWarps * 32) {
+    named_barrier_sync(1, kCons);
+    if (a.ks > 1) {
+      if (threadIdx.x == 0) {
+        // this CTA's pushes (ordered before by the barrier) are released with one arrival at
+        // every owner; then wait until every source's pushes to this CTA are visible
+        asm volatile("fence.acq_rel.cluster;" ::: "memory");
+        for (int o = 0; o < a.ks; ++o) mbar_arrive_remote(mapa_shared(smem_u32(&rready[b]), (uint32_t)o));
+        if (!mbar_wait_cluster(&rready[b], (uint32_t)(tt >> 1) & 1u, a.timeout_ns)) {
+          latch_status(a.status, PIFA_ERR_TIMEOUT);
+          dead = true;
+        }
+      }
+      dead = named_barrier_or(1, kCons, dead);
+    }
+    for (int idx = threadIdx.x; idx < rpr * 8 * NT; idx += kCons) {
       const int row = q * rpr + idx % rpr, t = idx / rpr;
       if (t >= a.T || row >= nrows) continue;
       float sum = 0.0f;
@@ -618,7 +657,13 @@ __global__ void __launch_bounds__(kWarps * 32, 2)
       }
       a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(sum);
     }
-    if (tt + 1 < ntile) __syncthreads();  // the partials and the columns are rewritten next tile
+    if (tt + 1 < ntile) {
+      named_barrier_sync(1, kCons);  // the partials, the columns and buffer b have been read
+      // release buffer b to every source that will push into it again (tile tt + 2); a source
+      // with no such tile may have retired, and gets no arrival
+      if (a.ks > 1 && tt + 2 < ntile && threadIdx.x == 0)
+        for (int o = 0; o < a.ks; ++o) mbar_arrive_remote(mapa_shared(smem_u32(&rfree[b]), (uint32_t)o));
+    }
   }
   if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
 }
@@ -699,7 +744,7 @@ size_t smem_bytes(int kRows, DecodeArgs& a, int NT) {
 
 // Co-resident clusters of ks CTAs of `fn` with `smem` bytes of dynamic shared memory each, on the
 // current device (cached per kernel, device, cluster size and size). 0 if unknown.
-int max_clusters(const void* fn, int ks, size_t smem) {
+int max_clusters(const void* fn, int ks, size_t smem, int threads = kWarps * 32) {
   static std::mutex mu;
   static std::map<std::tuple<const void*, int, int, size_t>, int> cache;
   int dev = 0;
@@ -711,13 +756,13 @@ int max_clusters(const void* fn, int ks, size_t smem) {
   int n = 0;
   if (ks == 1) {
     int per_sm = 0, sms = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kWarps * 32, smem) == cudaSuccess &&
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, threads, smem) == cudaSuccess &&
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
       n = per_sm * sms;
   } else {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)ks);
-    cfg.blockDim = dim3(kWarps * 32);
+    cfg.blockDim = dim3((unsigned)threads);
     cfg.dynamicSmemBytes = smem;
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeClusterDimension;
@@ -783,7 +828,8 @@ size_t plan_stream(const void* fn, int kRows, int NT, int NB, DecodeArgs& a, con
   if (*st != PIFA_OK) return 0;
   // as many clusters as are co-resident, but the tiles dealt evenly: rounds = ceil(ntiles / cap)
   // tiles for every cluster (a last round on a few clusters would run at their share of HBM alone)
-  const int cap = max_clusters(fn, ks, smem) > 0 ? max_clusters(fn, ks, smem) : 1;
+  const int nclu = max_clusters(fn, ks, smem, (kWarps + 1) * 32);
+  const int cap = nclu > 0 ? nclu : 1;
   const int rounds = (a.ntiles + cap - 1) / cap;
   a.ncl = (a.ntiles + rounds - 1) / rounds;
   return smem;
@@ -794,7 +840,7 @@ int launch_stream(Kern kernel, const CUtensorMap& tm, const DecodeArgs& args, si
                   const char* what) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(args.ncl * args.ks));
-  cfg.blockDim = dim3(kWarps * 32);
+  cfg.blockDim = dim3((kWarps + 1) * 32);  // eight consumer warps and the producer warp
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
