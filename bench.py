@@ -315,8 +315,8 @@ def comparators(dev, lay, T, copies, stream):
     return res
 
 
-DECODE_SWEEP = [(inputs.ATTN7B, (1, 8, 16)), (inputs.MLP7B_GATE, (1,)), (inputs.MLP7B_DOWN, (1,)),
-                (inputs.ATTN70B, (1, 16)), (inputs.MLP70B_GATE, (1, 16))]
+DECODE_SWEEP = [(inputs.ATTN7B, (1, 8, 16)), (inputs.MLP7B_GATE, (1, 8)), (inputs.MLP7B_DOWN, (1, 8)),
+                (inputs.ATTN70B, (1, 8, 16)), (inputs.MLP70B_GATE, (1, 8, 16))]
 
 
 def decode_sweep(dev, stream, hbm_peak, peak_src):

@@ -423,7 +423,7 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
   constexpr uint32_t kCons = kWarps * 32; // consumer threads (named barrier 1)
   extern __shared__ __align__(128) uint8_t smem_raw[];
   __shared__ uint64_t full[kMaxStages], empty[kMaxStages];
-  __shared__ uint64_t bbar, rready[2], rfree[2];
+  __shared__ uint64_t bbar, rready[2], rfree[2], done;
   __shared__ int s_cols[kRows];
   pdl_launch_dependents();  // the next kernel may launch now and start staging its weights
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -445,6 +445,7 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
       mbar_init(&empty[s], kWarps);
     }
     mbar_init(&bbar, 1);
+    mbar_init(&done, (uint32_t)a.ks);  // one arrival per CTA of the cluster
     for (int b = 0; b < 2; ++b) {
       mbar_init(&rready[b], (uint32_t)a.ks);  // one arrival per source CTA
       mbar_init(&rfree[b], (uint32_t)a.ks);   // one arrival per owner CTA
@@ -541,12 +542,14 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
       const int it = tt * nchunks + j;
       const int s = it % a.stages;
       const int nst = (min(a.kc, klen - j * a.kc) + kChunk - 1) / kChunk;
+      // every warp waits for the stage, steps or not: a warp that released stages it had not
+      // waited for could run ahead and count its release of a later item toward this one's
+      if (!dead && !mbar_wait(&full[s], (uint32_t)(it / a.stages) & 1u, a.timeout_ns)) {
+        latch_status(a.status, PIFA_ERR_TIMEOUT);
+        dead = true;
+      }
+      dead = __any_sync(0xffffffffu, dead);
       if (warp < nst) {
-        if (!dead && !mbar_wait(&full[s], (uint32_t)(it / a.stages) & 1u, a.timeout_ns)) {
-          latch_status(a.status, PIFA_ERR_TIMEOUT);
-          dead = true;
-        }
-        dead = __any_sync(0xffffffffu, dead);
         if (!dead) {
           const uint32_t sb = smem_u32(smem + s * stage_bytes) + lane_off;
           const uint32_t bj = (uint32_t)(j * a.kc) * 2u;
@@ -604,7 +607,7 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
       }
     const int b = tt & 1;
     float* recv = reinterpret_cast<float*>(smem + a.recv_off) + b * (kRows * 8 * NT);
-    if (a.ks > 1 && tt >= 2 && threadIdx.x == 0 &&
+    if (a.ks > 1 && tt >= 2 && threadIdx.x == 0 && !dead &&
         !mbar_wait_cluster(&rfree[b], (uint32_t)((tt - 2) >> 1) & 1u, a.timeout_ns)) {
       latch_status(a.status, PIFA_ERR_TIMEOUT);  // every owner has read this buffer's last pushes
       dead = true;
@@ -629,7 +632,7 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
         // every owner; then wait until every source's pushes to this CTA are visible
         asm volatile("fence.acq_rel.cluster;" ::: "memory");
         for (int o = 0; o < a.ks; ++o) mbar_arrive_remote(mapa_shared(smem_u32(&rready[b]), (uint32_t)o));
-        if (!mbar_wait_cluster(&rready[b], (uint32_t)(tt >> 1) & 1u, a.timeout_ns)) {
+        if (!dead && !mbar_wait_cluster(&rready[b], (uint32_t)(tt >> 1) & 1u, a.timeout_ns)) {
           latch_status(a.status, PIFA_ERR_TIMEOUT);
           dead = true;
         }
@@ -666,6 +669,17 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
     }
   }
   if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
+  // No CTA retires before every CTA of its cluster has made its last remote access to it (pushes
+  // and arrivals precede each CTA's arrival here): after a timeout the waits above are skipped,
+  // and a CTA could otherwise leave while a peer still writes into its shared memory.
+  if (a.ks > 1) {
+    named_barrier_sync(1, kCons);
+    if (threadIdx.x == 0) {
+      for (int o = 0; o < a.ks; ++o) mbar_arrive_remote(mapa_shared(smem_u32(&done), (uint32_t)o));
+      if (!mbar_wait_cluster(&done, 0, a.timeout_ns)) latch_status(a.status, PIFA_ERR_TIMEOUT);
+    }
+    named_barrier_sync(1, kCons);
+  }
 }
 
 // Once per kernel, device and size: the dynamic shared-memory limit, and the largest shared-memory
@@ -793,16 +807,17 @@ int sm_count() {
 }
 
 // decode_stream's split of one phase into (ks, kcta, kc, stages, ntiles, ncl) and its shared memory
-// (returned, with 1 KB of alignment slack): the fewest CTAs per cluster giving at least two
-// (tile, K-range) units per SM, with resident B rows of at most a third of the budget; then
-// chunks of whole 64-column blocks, four stages where they fit.
+// (returned, with 1 KB of alignment slack): the fewest CTAs per cluster giving at least one
+// (tile, K-range) unit per SM (measured: two per SM, through larger clusters, cost more in per-tile
+// reductions than they gain), with resident B rows of at most a third of the budget; then chunks
+// of whole 64-column blocks, four stages where they fit.
 size_t plan_stream(const void* fn, int kRows, int NT, int NB, DecodeArgs& a, const char* what, int* st) {
   auto round16 = [](size_t b) { return (b + 15) / 16 * 16; };
   a.ntiles = (a.R + kRows - 1) / kRows;
   const size_t red = round16((size_t)kWarps * kRows * (8 * NT + 1) * 4);
   const size_t recv1 = (size_t)kRows * 8 * NT * 4;
   int ks = 1;
-  while (ks < kMaxCluster && ((int64_t)a.ntiles * ks < 2 * sm_count() ||
+  while (ks < kMaxCluster && ((int64_t)a.ntiles * ks < sm_count() ||
                               (size_t)NB * a.T * row_pitch(kcta_of(a.K, ks)) > kStreamBudget / 3))
     ks *= 2;
   a.ks = ks;

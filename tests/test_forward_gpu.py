@@ -203,6 +203,19 @@ def test_llama70b_qo(T):
     parity(L, T, sample=256)
 
 
+@pytest.mark.parametrize("T", [4, 16])
+def test_llama70b_qo_persistent_grid(T):
+    """The persistent decode grid forced on the 70B q/o layer: chunks on which some warps have no
+    step, several chunks per tile, three or more tiles per cluster of up to eight CTAs (both
+    receive buffers reused)."""
+    L = layer_for(8192, 8192, 4096, 0, "library")
+    P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_PERSISTENT)
+    try:
+        parity(L, T, P.PIFA_VARIANT_DECODE)
+    finally:
+        P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
+
+
 @pytest.mark.parametrize("T", [1, 8, 16, 4096])
 def test_llama70b_gate_up(T):
     L = layer_for(28672, 8192, 4096, 0, "synthetic")
