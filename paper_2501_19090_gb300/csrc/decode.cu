@@ -164,6 +164,8 @@ struct DecodeArgs {
   int ncl;              // clusters in the grid: cluster c owns tiles c, c + ncl, c + 2 ncl, ...
   uint32_t bres_off;    // byte offset of the resident B rows (NB planes x T, pitch row_pitch(kcta))
   uint32_t red_off;     // byte offset of the warps' partial tiles
+  int bstaged;          // 1: the chunk's B rows ride in each stage (TMA boxes of tb rows), else resident
+  int tb;               // B box rows: T rounded up to 8
   int* status;
   uint64_t timeout_ns;
 };
@@ -413,7 +415,8 @@ __device__ __forceinline__ int rho8(int g) { return (g >> 1) | ((g & 1) << 2); }
 // producer, running ahead, could not join.
 template <int PHASE, int NT, bool kF16C, int RG>
 __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
-    decode_stream(const __grid_constant__ CUtensorMap tmA, DecodeArgs a) {
+    decode_stream(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
+                  const __grid_constant__ CUtensorMap tmB1, DecodeArgs a) {
   constexpr int kRows = kRowsOf<RG>;
   constexpr int NB = PHASE == 1 ? 1 : 2;
   constexpr bool kF16Mma = PHASE == 2 && kF16C;
@@ -427,7 +430,10 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
   __shared__ int s_cols[kRows];
   pdl_launch_dependents();  // the next kernel may launch now and start staging its weights
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t stage_bytes = (uint32_t)(a.kc / 64) * kBlk;
+  const int nblkmax = a.kc / 64;  // 64-column blocks of a stage
+  const uint32_t bblk = (uint32_t)a.tb * 128u;  // one staged B box: 64 columns x tb token rows
+  const uint32_t bplane = a.bstaged ? (uint32_t)nblkmax * bblk : 0u;
+  const uint32_t stage_bytes = (uint32_t)nblkmax * kBlk + (uint32_t)NB * bplane;
   const uint32_t bpitch = row_pitch(a.kcta);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, c = lane & 3;
   const int q = (int)cluster_ctarank();
@@ -459,19 +465,45 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
   if (warp == kWarps) {  // ---- producer ----
     if (lane == 0) {
       prefetch_tmap(&tmA);
-      int issued = 0;
-      for (int it = 0; it < nitems; ++it) {
+      if (a.bstaged) {
+        prefetch_tmap(&tmB0);
+        if (NB > 1) prefetch_tmap(&tmB1);
+      }
+      // item `it` into stage it % stages: its weight boxes (wa) and/or B boxes (wb); the barrier's
+      // one arrival comes with the last part (zero-filled parts of a box count too)
+      auto issue = [&](int it, bool wa, bool wb) {
         const int s = it % a.stages, j = it % nchunks;
-        if (it >= a.stages && !mbar_wait(&empty[s], (uint32_t)((it / a.stages) - 1) & 1u, a.timeout_ns)) {
+        const int nblk = (min(a.kc, klen - j * a.kc) + 63) / 64;
+        const uint32_t tx = (wa ? (uint32_t)nblk * kBlk : 0u) + (wb ? (uint32_t)(NB * nblk) * bblk : 0u);
+        if (wb || !a.bstaged)
+          mbar_arrive_expect_tx(&full[s], tx);
+        else
+          mbar_expect_tx(&full[s], tx);
+        uint8_t* st = smem + s * stage_bytes;
+        const int x0 = k0 + j * a.kc;
+        if (wa)
+          for (int b = 0; b < nblk; ++b)
+            tma_load_2d(smem_u32(st + b * kBlk), &tmA, x0 + 64 * b, (int)tile_row0(it / nchunks), &full[s]);
+        if (wb)
+          for (int nb = 0; nb < NB; ++nb)
+            for (int b = 0; b < nblk; ++b)
+              tma_load_2d(smem_u32(st + nblkmax * kBlk + nb * bplane + b * bblk), nb ? &tmB1 : &tmB0, x0 + 64 * b, 0,
+                          &full[s]);
+      };
+      const int pre = min(a.stages, nitems);
+      for (int it = 0; it < pre; ++it) issue(it, true, false);  // weights: before the dependency wait
+      if (a.bstaged) {  // B depends on the previous kernel
+        pdl_wait_primary();
+        for (int it = 0; it < pre; ++it) issue(it, false, true);
+      }
+      int issued = pre;
+      for (int it = pre; it < nitems; ++it) {
+        const int s = it % a.stages;
+        if (!mbar_wait(&empty[s], (uint32_t)((it / a.stages) - 1) & 1u, a.timeout_ns)) {
           latch_status(a.status, PIFA_ERR_TIMEOUT);
           break;
         }
-        const int len = min(a.kc, klen - j * a.kc);
-        const int nblk = (len + 63) / 64;
-        uint8_t* st = smem + s * stage_bytes;
-        mbar_arrive_expect_tx(&full[s], (uint32_t)nblk * kBlk);  // zero-filled parts count too
-        for (int b = 0; b < nblk; ++b)
-          tma_load_2d(smem_u32(st + b * kBlk), &tmA, k0 + j * a.kc + 64 * b, (int)tile_row0(it / nchunks), &full[s]);
+        issue(it, true, a.bstaged != 0);
         issued = it + 1;
       }
       // nothing may land in shared memory after the CTA retires: wait for the last copies
@@ -491,8 +523,8 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
   // B rows, resident: [0, klen rounded down to 8) by bulk copies, the rest up to whole steps by
   // plain loads and zeros (the steps read up to kpad; the TMA boxes are zero beyond K as well)
   uint8_t* bres = smem + a.bres_off;
-  const int kbulk = klen & ~7, kpad = (klen + kChunk - 1) / kChunk * kChunk;
-  if (warp == 0) {
+  const int kbulk = a.bstaged ? 0 : klen & ~7, kpad = a.bstaged ? 0 : (klen + kChunk - 1) / kChunk * kChunk;
+  if (warp == 0 && !a.bstaged) {
     const uint32_t bytes = (uint32_t)kbulk * 2u;
     if (lane == 0) mbar_arrive_expect_tx(&bbar, bytes * (uint32_t)(NB * a.T));
     __syncwarp();
@@ -508,7 +540,7 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
       reinterpret_cast<uint16_t*>(bres + i * bpitch)[col] = v;
     }
   bool dead = false;
-  if (threadIdx.x == 0 && !mbar_wait(&bbar, 0, a.timeout_ns)) {
+  if (threadIdx.x == 0 && !a.bstaged && !mbar_wait(&bbar, 0, a.timeout_ns)) {
     latch_status(a.status, PIFA_ERR_TIMEOUT);
     dead = true;
   }
@@ -516,12 +548,19 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
 
   const int arow = rho8(g);
   const uint32_t lane_off = (uint32_t)arow * 128u + (uint32_t)((c ^ arow) << 4);
-  uint32_t boff[NB][NT];  // this lane's B row (token 8 nt + g, clamped to T - 1) and column 8 c
+  // this lane's B row (token t = 8 nt + g, clamped to T - 1) and column 8 c:
+  //   resident: bres + (nb T + t) bpitch + 16 c  (+ 2 column)
+  //   staged:   stage + nblkmax kBlk + nb bplane + (st / 2) bblk + t 128 + ((4 (st & 1) + c) ^ (t & 7)) 16
+  uint32_t boff[NB][NT];
 #pragma unroll
   for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-      boff[nb][nt] = smem_u32(bres) + (uint32_t)(nb * a.T + (nt * 8 + g < a.T ? nt * 8 + g : a.T - 1)) * bpitch + 16u * c;
+    for (int nt = 0; nt < NT; ++nt) {
+      const int t = nt * 8 + g < a.T ? nt * 8 + g : a.T - 1;
+      boff[nb][nt] = a.bstaged ? (uint32_t)nblkmax * kBlk + (uint32_t)nb * bplane + (uint32_t)t * 128u +
+                                     (uint32_t)((c ^ (t & 7)) << 4)
+                               : smem_u32(bres) + (uint32_t)(nb * a.T + t) * bpitch + 16u * c;
+    }
   float* red = reinterpret_cast<float*>(smem + a.red_off);
   bool range_err = false;
   const int rpr = kRows / a.ks;
@@ -551,7 +590,8 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
       dead = __any_sync(0xffffffffu, dead);
       if (warp < nst) {
         if (!dead) {
-          const uint32_t sb = smem_u32(smem + s * stage_bytes) + lane_off;
+          const uint32_t sbase = smem_u32(smem + s * stage_bytes);
+          const uint32_t sb = sbase + lane_off;
           const uint32_t bj = (uint32_t)(j * a.kc) * 2u;
           // one 32-column step: the stage base is 1024-byte aligned and kBlk a multiple of 1024,
           // so the odd step's chunk flip (bit 6) acts on lane_off alone
@@ -561,7 +601,9 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
 #pragma unroll
             for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-              for (int nt = 0; nt < NT; ++nt) bv[nb][nt] = lds128(boff[nb][nt] + bj + (uint32_t)st * 64u);
+              for (int nt = 0; nt < NT; ++nt)
+                bv[nb][nt] = lds128(a.bstaged ? sbase + (uint32_t)(st >> 1) * bblk + (boff[nb][nt] ^ ((uint32_t)(st & 1) << 6))
+                                              : boff[nb][nt] + bj + (uint32_t)st * 64u);
 #pragma unroll
             for (int gq = 0; gq < RG; ++gq) {
               const uint4 wa = lds128(at + (uint32_t)(16 * gq) * 128u);      // MMA row g
@@ -816,15 +858,19 @@ size_t plan_stream(const void* fn, int kRows, int NT, int NB, DecodeArgs& a, con
   a.ntiles = (a.R + kRows - 1) / kRows;
   const size_t red = round16((size_t)kWarps * kRows * (8 * NT + 1) * 4);
   const size_t recv1 = (size_t)kRows * 8 * NT * 4;
+  // B rows: resident for T <= 2 (a few KB per CTA, no per-chunk traffic), else staged with the
+  // weights in every stage, which frees the cluster split from the resident rows' size
+  a.bstaged = a.T > 2 ? 1 : 0;
+  a.tb = (a.T + 7) / 8 * 8;
   int ks = 1;
   while (ks < kMaxCluster && ((int64_t)a.ntiles * ks < sm_count() ||
-                              (size_t)NB * a.T * row_pitch(kcta_of(a.K, ks)) > kStreamBudget / 3))
+                              (!a.bstaged && (size_t)NB * a.T * row_pitch(kcta_of(a.K, ks)) > kStreamBudget / 3)))
     ks *= 2;
   a.ks = ks;
   a.kcta = kcta_of(a.K, ks);
-  const size_t bres = round16((size_t)NB * a.T * row_pitch(a.kcta));
+  const size_t bres = a.bstaged ? 0 : round16((size_t)NB * a.T * row_pitch(a.kcta));
   const size_t side = bres + red + (ks > 1 ? 2 * recv1 : 0);
-  const size_t blk = (size_t)kRows * 128;
+  const size_t blk = (size_t)kRows * 128 + (a.bstaged ? (size_t)NB * a.tb * 128 : 0);  // one 64-column block
   const size_t ring = kStreamBudget > side + 2 * blk ? kStreamBudget - side : 2 * blk;
   const int kblocks = (a.kcta + 63) / 64;
   int nblk = (int)(ring / (4 * blk));
@@ -851,8 +897,8 @@ size_t plan_stream(const void* fn, int kRows, int NT, int NB, DecodeArgs& a, con
 }
 
 template <typename Kern>
-int launch_stream(Kern kernel, const CUtensorMap& tm, const DecodeArgs& args, size_t smem, cudaStream_t stream,
-                  const char* what) {
+int launch_stream(Kern kernel, const CUtensorMap& tm, const CUtensorMap& tb0, const CUtensorMap& tb1,
+                  const DecodeArgs& args, size_t smem, cudaStream_t stream, const char* what) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)(args.ncl * args.ks));
   cfg.blockDim = dim3((kWarps + 1) * 32);  // eight consumer warps and the producer warp
@@ -867,7 +913,7 @@ int launch_stream(Kern kernel, const CUtensorMap& tm, const DecodeArgs& args, si
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, tm, args);
+  cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, tm, tb0, tb1, args);
   if (e != cudaSuccess) return pifa_fail_cuda(what, e);
   return PIFA_OK;
 }
@@ -886,22 +932,22 @@ int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, cudaStream_t str
   int st = prepare_kernel(reinterpret_cast<const void*>(kr), smem, what);
   if (st != PIFA_OK) return st;
   // decode_rows in waves while a phase takes at most two of them (its weights staged at launch,
-  // before the dependency wait, outweigh the persistent grid's streaming), and always for two
-  // token tiles (T > 8: measured slower persistent, the per-tile reductions of 16 tokens being
-  // twice as long); else decode_stream
+  // before the dependency wait, outweigh the persistent grid's streaming); else decode_stream
   const int tiles = (a.R + kRows - 1) / kRows;
   const int mode = g_decode_grid.load(std::memory_order_relaxed);
   if (mode == PIFA_DECODE_GRID_WAVES ||
-      (mode == PIFA_DECODE_GRID_AUTO &&
-       (NT > 1 || tiles <= 2 * max_clusters(reinterpret_cast<const void*>(kr), a.ks, smem))))
+      (mode == PIFA_DECODE_GRID_AUTO && tiles <= 2 * max_clusters(reinterpret_cast<const void*>(kr), a.ks, smem)))
     return launch_phase(kr, kRows, a, smem, stream, what);
   const auto ks = decode_stream<PHASE, NT, kF16C, RGS>;
   const size_t smem_s =
       plan_stream(reinterpret_cast<const void*>(ks), kRowsOf<RGS>, NT, PHASE == 1 ? 1 : 2, a, what, &st);
   if (st != PIFA_OK) return st;
-  CUtensorMap tm;
+  CUtensorMap tm, tb0 = {}, tb1 = {};  // B maps (x, or the y_p planes in C's type): staged B only
   if ((st = make_tmap_2d(&tm, dtype, a.A, a.R, a.K, a.lda, 64, kRowsOf<RGS>)) != PIFA_OK) return st;
-  return launch_stream(ks, tm, a, smem_s, stream, what);
+  if (a.bstaged && (st = make_tmap_2d(&tb0, dtype, a.B0, a.T, a.K, a.ldb, 64, a.tb)) != PIFA_OK) return st;
+  if (a.bstaged && PHASE == 2 && (st = make_tmap_2d(&tb1, dtype, a.B1, a.T, a.K, a.ldb, 64, a.tb)) != PIFA_OK)
+    return st;
+  return launch_stream(ks, tm, tb0, tb1, a, smem_s, stream, what);
 }
 
 template <int NT, bool kF16C, int RG, int RGS>
