@@ -144,6 +144,20 @@ def build_layer(shape, seed, c_dtype="bf16"):
     return dict(U=U, V=V, piv=piv, nonp=nonp, Wp=inputs.round_bf16(Wp), C=Cq, info=info, c_dtype=c_dtype)
 
 
+# --shape: the decode measurement on another decode-config layer shape (profiling; the default line
+# is the 7B attention layer). Other shapes use seeded random operands (inputs.synthetic_layer): the
+# kernels' time does not depend on the values, and Algorithm 1 on a 28672 x 8192 layer takes minutes
+# on the host.
+SHAPES = {s.name: s for s in (inputs.ATTN7B, inputs.MLP7B_GATE, inputs.MLP7B_DOWN, inputs.ATTN70B,
+                              inputs.MLP70B_GATE)}
+
+
+def synthetic_layer_dict(shape, c_dtype="bf16"):
+    piv, nonp, Wp, C = inputs.synthetic_layer(shape.m, shape.n, shape.r, 0)
+    Cq = inputs.round_fp16(C) if c_dtype == "fp16" else C
+    return dict(piv=piv.astype(np.int32), nonp=nonp.astype(np.int32), Wp=Wp, C=Cq, c_dtype=c_dtype)
+
+
 def _torch_c_dtype(lay):
     import torch
     return torch.float16 if lay["c_dtype"] == "fp16" else torch.bfloat16
@@ -162,10 +176,11 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.set_device(dev)
     P.load()
     hbm_peak, tc_peak, tc_sust, peak_src = _peaks()
-    shape = SHAPE
+    shape = SHAPES[args.shape]
     m, n, r = shape.m, shape.n, shape.r
     T = args.tokens
-    lay = build_layer(shape, seed=0, c_dtype=args.c_dtype)
+    lay = (build_layer(shape, seed=0, c_dtype=args.c_dtype) if shape is SHAPE
+           else synthetic_layer_dict(shape, args.c_dtype))
     bf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev).to(torch.bfloat16)
     piv = torch.from_numpy(lay["piv"]).to(dev)
     nonp = torch.from_numpy(lay["nonp"]).to(dev)
@@ -275,7 +290,7 @@ def run_ours(args, rank, world, local_rank):
         "gpu_launches": steps * (2 if m > r else 1),
         "clocks": clk.summary(),
     }
-    if rank == 0 and not args.no_extras:
+    if rank == 0 and not args.no_extras and shape is SHAPE:
         out["comparators"] = comparators(dev, lay, T, copies, stream)
         out["prefill"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src)
         out["prefill_fused"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src,
@@ -540,6 +555,8 @@ def main():
     ap.add_argument("--tokens", type=int, default=T_DECODE)
     ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--c-dtype", default="bf16", choices=["bf16", "fp16"])
+    ap.add_argument("--shape", default=SHAPE.name, choices=sorted(SHAPES),
+                    help="decode layer shape of the main line (other shapes: synthetic operands, no extras)")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
