@@ -76,6 +76,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_full + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
+  pdl_launch_dependents();  // the next kernel may launch now (its CTAs take SMs this grid leaves idle)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
   const int total = p.kchunks * p.passes;
@@ -104,11 +105,25 @@ __global__ void __launch_bounds__(THREADS, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer ----------------
-      int issued = 0;
-      for (int i = 0; i < total; ++i) {
+      // The weight tiles (A) do not depend on the previous kernel: those of the first stages go out
+      // before the dependency wait, raising the expected bytes without arriving; the activation
+      // tiles (B: X, or the y_p planes GEMM 1 wrote) follow the wait and bring the arrival.
+      const int pre = total < STAGES ? total : STAGES;
+      for (int i = 0; i < pre; ++i) {
+        mbar_expect_tx(&full[i], A_BYTES);
+        tma_load_2d(smem_u32(smem + i * STAGE_BYTES), &tmA, (i % p.kchunks) * BK, m0, &full[i]);
+      }
+      pdl_wait_primary();
+      for (int i = 0; i < pre; ++i) {
+        const int pass = i / p.kchunks, kc = i % p.kchunks;
+        mbar_arrive_expect_tx(&full[i], B_BYTES);
+        tma_load_2d(smem_u32(smem + i * STAGE_BYTES + A_BYTES), pass ? &tmB1 : &tmB0, kc * BK, n0, &full[i]);
+      }
+      int issued = pre;
+      for (int i = pre; i < total; ++i) {
         const int s = i % STAGES;
         const uint32_t ph = (uint32_t)(i / STAGES) & 1u;
-        if (i >= STAGES && !mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
+        if (!mbar_wait(&empty[s], ph ^ 1u, p.timeout_ns)) {
           *abort_flag = 1;
           latch_status(p.status, PIFA_ERR_TIMEOUT);
           break;
@@ -240,9 +255,19 @@ int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtenso
                                     : pifa_umma_gemm<EPI_Y_ONLY>;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(prefill gemm)", e);
-  dim3 grid((args.M + BM - 1) / BM, (args.N + BN - 1) / BN);
-  kern<<<grid, THREADS, SMEM_BYTES, stream>>>(a, b0, b1, args);
-  e = cudaGetLastError();
+  // programmatic dependent launch: each GEMM may start (weight tiles in flight) while the previous
+  // kernel of the stream drains; its dependent loads follow griddepcontrol.wait
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((args.M + BM - 1) / BM, (args.N + BN - 1) / BN);
+  cfg.blockDim = dim3(THREADS);
+  cfg.dynamicSmemBytes = SMEM_BYTES;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, kern, a, b0, b1, args);
   if (e != cudaSuccess) return pifa_fail_cuda("prefill gemm launch", e);
   return PIFA_OK;
 }
