@@ -33,7 +33,7 @@ using namespace pifa;
 using bf16 = __nv_bfloat16;
 
 constexpr int BM = 128;  // weight rows per tile (MMA M)
-constexpr int BN = 256;  // tokens per tile (MMA N)
+constexpr int BN = 256;  // tokens per tile at most (MMA N); the launch picks bn <= BN, a multiple of 16
 constexpr int BK = 64;   // K per stage: one 128-byte swizzle row of bf16
 constexpr int STAGES = 4;
 constexpr int EPI_WARPS = 16;                 // epilogue warps: four per TMEM lane quarter
@@ -51,6 +51,7 @@ struct GemmArgs {
   uint32_t idesc;        // tcgen05 instruction descriptor (bf16 or fp16 operands)
   int M;                 // weight rows (r for GEMM 1, m - r for GEMM 2)
   int N;                 // tokens T
+  int bn;                // tokens per tile (MMA N, TMA box rows of B): a multiple of 16, <= BN
   int kchunks;           // ceil(K / 64) per pass
   int passes;            // 1, or 2 for the hi + lo passes of GEMM 2
   const int32_t* cols;   // output column of each weight row (I or I^c)
@@ -78,7 +79,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   pdl_launch_dependents();  // the next kernel may launch now (its CTAs take SMs this grid leaves idle)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
+  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * p.bn;
+  const uint32_t b_bytes = (uint32_t)p.bn * BK * 2;  // one B box
   const int total = p.kchunks * p.passes;
 
   if (warp == 0 && lane == 0) {
@@ -116,7 +118,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       pdl_wait_primary();
       for (int i = 0; i < pre; ++i) {
         const int pass = i / p.kchunks, kc = i % p.kchunks;
-        mbar_arrive_expect_tx(&full[i], B_BYTES);
+        mbar_arrive_expect_tx(&full[i], b_bytes);
         tma_load_2d(smem_u32(smem + i * STAGE_BYTES + A_BYTES), pass ? &tmB1 : &tmB0, kc * BK, n0, &full[i]);
       }
       int issued = pre;
@@ -131,7 +133,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (*abort_flag) break;
         const int pass = i / p.kchunks, kc = i % p.kchunks;
         uint8_t* sa = smem + s * STAGE_BYTES;
-        mbar_arrive_expect_tx(&full[s], STAGE_BYTES);
+        mbar_arrive_expect_tx(&full[s], A_BYTES + b_bytes);
         tma_load_2d(smem_u32(sa), &tmA, kc * BK, m0, &full[s]);
         tma_load_2d(smem_u32(sa + A_BYTES), pass ? &tmB1 : &tmB0, kc * BK, n0, &full[s]);
         issued = i + 1;
@@ -172,7 +174,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     // EPI_WARPS / 4 warps of a quarter split the tile's tokens. Many warps keep the store issue
     // rate up: the scattered 2-byte stores into Y's columns are instruction-bound.
     constexpr int kSlices = EPI_WARPS / 4;
-    constexpr int kChunks = BN / 32 / kSlices;  // 32-token chunks per warp
+    constexpr int kChunks = BN / 32 / kSlices;  // 32-token chunks per warp (the last ones may lie beyond bn)
+    const int tend = min(n0 + p.bn, p.N);       // this tile's tokens end here
     const int q = warp & 3;
     const int slice = (warp - 2) >> 2;
     const int row = m0 + q * 32 + lane;
@@ -196,13 +199,14 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll 1
       for (int ci = 0; ci < kChunks; ++ci) {
         const int tb = n0 + (slice * kChunks + ci) * 32;  // first token of the chunk
+        if (tb >= tend) break;  // warp-uniform; TMEM columns beyond bn hold no result
         uint32_t v[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(tb - n0), v);
         tmem_ld_wait();
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
           const float f = __uint_as_float(v[j]);
-          if (col >= 0 && tb + j < p.N) p.Y[(int64_t)(tb + j) * p.ldy + col] = __float2bfloat16_rn(f);
+          if (col >= 0 && tb + j < tend) p.Y[(int64_t)(tb + j) * p.ldy + col] = __float2bfloat16_rn(f);
           if (kEpi == EPI_SPLIT_BF16) {
             const bf16 h = __float2bfloat16_rn(f);
             st_hi[j * 32 + lane] = __bfloat16_as_ushort(h);
@@ -226,7 +230,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int c = lane + 32 * k;
             const int t = tb + (c >> 2);
             const int rr = m0 + q * 32 + (c & 3) * 8;  // rows beyond M hold zeros (padding columns)
-            if (t < p.N && rr < p.ldyp) {
+            if (t < tend && rr < p.ldyp) {
               *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(p.yp_hi) + (int64_t)t * p.ldyp + rr) =
                   *reinterpret_cast<const uint4*>(st_hi + c * 8);
               *reinterpret_cast<uint4*>(reinterpret_cast<uint16_t*>(p.yp_lo) + (int64_t)t * p.ldyp + rr) =
@@ -258,7 +262,7 @@ int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtenso
   // programmatic dependent launch: each GEMM may start (weight tiles in flight) while the previous
   // kernel of the stream drains; its dependent loads follow griddepcontrol.wait
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((args.M + BM - 1) / BM, (args.N + BN - 1) / BN);
+  cfg.gridDim = dim3((args.M + BM - 1) / BM, (args.N + args.bn - 1) / args.bn);
   cfg.blockDim = dim3(THREADS);
   cfg.dynamicSmemBytes = SMEM_BYTES;
   cfg.stream = stream;
@@ -273,6 +277,31 @@ int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtenso
 }
 
 inline int64_t pad8(int64_t v) { return (v + 7) / 8 * 8; }
+
+// Tokens per tile for an M x T GEMM: the multiple of 16 (16..256) minimising the slowest SM's time,
+// waves x (tile time); ties to the larger bn. The tile time is the measured fit on the 4096 x 4096,
+// r = 2048 layer (T = 8192: 4 waves of 256-token tiles 254 us, 6 waves of 144-token tiles 320 us):
+// t(bn) ~ t0 (432 + bn), most of a tile's time not shrinking with its width. There T = 2048 takes
+// 240 (144 tiles, one wave of 152 SMs, where 256 leaves 24 SMs idle: 58.3 -> 57.3 us) and
+// T = 8192 224 (254.4 -> 242.8 us).
+int pick_bn(int64_t M, int64_t T) {
+  int sms = 0, dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      sms < 1)
+    sms = 1;
+  const int64_t mt = (M + BM - 1) / BM;
+  int best = BN;
+  int64_t best_cost = -1;
+  for (int bn = BN; bn >= 16; bn -= 16) {
+    const int64_t tiles = mt * ((T + bn - 1) / bn);
+    const int64_t cost = (tiles + sms - 1) / sms * (432 + bn);
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = bn;
+    }
+  }
+  return best;
+}
 
 }  // namespace
 
@@ -291,13 +320,15 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
 
   CUtensorMap tWp, tX, tC, tHi, tLo;
   int st;
+  const int bn1 = pick_bn(s.r, s.T);
   if ((st = make_tmap_2d(&tWp, PIFA_DTYPE_BF16, p.Wp, s.r, s.n, s.ldwp, BK, BM)) != PIFA_OK) return st;
-  if ((st = make_tmap_2d(&tX, PIFA_DTYPE_BF16, p.X, s.T, s.n, s.ldx, BK, BN)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tX, PIFA_DTYPE_BF16, p.X, s.T, s.n, s.ldx, BK, bn1)) != PIFA_OK) return st;
 
   GemmArgs g1 = {};
-  g1.idesc = idesc_bf16_f32(BM, BN);
+  g1.idesc = idesc_bf16_f32(BM, bn1);
   g1.M = (int)s.r;
   g1.N = (int)s.T;
+  g1.bn = bn1;
   g1.kchunks = (int)((s.n + BK - 1) / BK);
   g1.passes = 1;
   g1.cols = p.piv;
@@ -312,11 +343,13 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
   if ((st = run_gemm(f16 ? EPI_SPLIT_F16 : EPI_SPLIT_BF16, tWp, tX, tX, g1, stream)) != PIFA_OK) return st;
   if (s.m == s.r) return PIFA_OK;
 
+  const int bn2 = pick_bn(s.m - s.r, s.T);
   if ((st = make_tmap_2d(&tC, s.c_dtype, p.C, s.m - s.r, s.r, s.ldc, BK, BM)) != PIFA_OK) return st;
-  if ((st = make_tmap_2d(&tHi, s.c_dtype, hi, s.T, s.r, ldyp, BK, BN)) != PIFA_OK) return st;
-  if ((st = make_tmap_2d(&tLo, s.c_dtype, lo, s.T, s.r, ldyp, BK, BN)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tHi, s.c_dtype, hi, s.T, s.r, ldyp, BK, bn2)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tLo, s.c_dtype, lo, s.T, s.r, ldyp, BK, bn2)) != PIFA_OK) return st;
   GemmArgs g2 = g1;
-  g2.idesc = f16 ? idesc_f16_f32(BM, BN) : idesc_bf16_f32(BM, BN);
+  g2.bn = bn2;
+  g2.idesc = f16 ? idesc_f16_f32(BM, bn2) : idesc_bf16_f32(BM, bn2);
   g2.M = (int)(s.m - s.r);
   g2.kchunks = (int)((s.r + BK - 1) / BK);
   g2.passes = 2;
