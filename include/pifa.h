@@ -120,6 +120,39 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx,
                          int variant, void* cuda_stream);
 
 /*
+ * pifa_forward_grouped -- Algorithm 2 for `groups` (G) PIFA layers of one shape (m, n, r, c_dtype)
+ * that share their input X, e.g. a transformer MLP's gate and up projections, as one computation:
+ * their pivot rows are stacked into one first contraction Y_p = X [W_p^(0); ...; W_p^(G-1)]^T, and
+ * the second runs over all groups' rows of C at once, group g's rows against y_p's columns
+ * [g r, (g + 1) r) -- in matrix form the layers make one PIFA computation whose C is
+ * block-diagonal. The paper treats one layer at a time (Sec. 3.2); stacking changes no result.
+ *
+ *   X            as pifa_forward (T x n, shared by the groups).
+ *   Wp           G r x n, row-major, leading dimension ldwp >= n: group g's W_p in rows [g r, (g + 1) r).
+ *   C            G (m - r) x r, leading dimension ldc >= r: group g's C in rows [g (m - r), (g + 1) (m - r)).
+ *   pivot_idx    G r int32: group g's pivot indices I^(g) plus g m (columns of Y).
+ *   nonpivot_idx G (m - r) int32: group g's non-pivot indices plus g m.
+ *   Y            T x (G m), leading dimension ldy >= G m: group g's output in columns [g m, (g + 1) m).
+ *   workspace    at least pifa_workspace_size_grouped(G, T, m, n, r, c_dtype) bytes, 256-byte aligned.
+ *   Variant, alignment, aliasing, asynchrony and status codes as pifa_forward (the variant is the
+ *   one pifa_select_variant picks for one layer; the fused prefill does not run grouped layers).
+ *   G in [1, 64]; G > 1 needs m > r, (m - r) % 128 == 0 and r % 8 == 0 (PIFA_ERR_UNSUPPORTED
+ *   otherwise: call pifa_forward per layer), so that no tile spans two groups. G = 1 is
+ *   pifa_forward.
+ */
+int pifa_forward_grouped(int64_t groups, const void* X, int64_t T, int64_t n, int64_t ldx,
+                         const void* Wp, int64_t r, int64_t ldwp,
+                         const void* C, int64_t m, int64_t ldc, int c_dtype,
+                         const int32_t* pivot_idx, const int32_t* nonpivot_idx,
+                         void* Y, int64_t ldy,
+                         void* workspace, int64_t workspace_bytes,
+                         void* cuda_stream);
+
+/* pifa_workspace_size_grouped -- bytes of device scratch pifa_forward_grouped needs (y_p for all
+ * groups); negative pifa_status on bad arguments. Pure host arithmetic. */
+int64_t pifa_workspace_size_grouped(int64_t groups, int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype);
+
+/*
  * pifa_forward_decode_noalloc -- the decode variant of pifa_forward (T <= 16) for callers that
  * cannot allocate device memory, e.g. a runtime that plans all device memory up front and forbids
  * a library's cudaMalloc, or a decode loop where an allocation's implicit synchronization is not

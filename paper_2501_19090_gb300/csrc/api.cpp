@@ -169,19 +169,47 @@ int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dt
   }
 }
 
-int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,
-                         const void* C, int64_t m, int64_t ldc, int c_dtype, const int32_t* pivot_idx,
-                         const int32_t* nonpivot_idx, void* Y, int64_t ldy, void* workspace,
-                         int64_t workspace_bytes, int variant, void* cuda_stream) {
+}  // extern "C"
+
+namespace {
+
+// Extra conditions on G layers sharing X (groups > 1): each group's non-pivot rows a whole number
+// of 128-row tiles and its y_p columns 16-byte aligned. PIFA_OK or the failure.
+int validate_groups(int64_t groups, int64_t m, int64_t r) {
+  if (groups < 1 || groups > 64) return pifa_fail(PIFA_ERR_INVALID_ARG, "groups must be in [1, 64]");
+  if (groups == 1) return PIFA_OK;
+  if (m == r) return pifa_fail(PIFA_ERR_UNSUPPORTED, "grouped layers need m > r");
+  if ((m - r) % 128 != 0 || r % 8 != 0)
+    return pifa_fail(PIFA_ERR_UNSUPPORTED, "grouped layers need (m - r) % 128 == 0 and r % 8 == 0");
+  if (groups * m >= ((int64_t)1 << 30)) return pifa_fail(PIFA_ERR_INVALID_ARG, "groups * m too large (>= 2^30)");
+  return PIFA_OK;
+}
+
+int64_t workspace_bytes_for(const PifaShape& s, int variant) {
+  switch (variant) {
+    case PIFA_VARIANT_DECODE: return kWorkspaceReserve + decode_workspace_bytes(s);
+    case PIFA_VARIANT_PREFILL_SPLIT: return kWorkspaceReserve + prefill_split_workspace_bytes(s);
+    case PIFA_VARIANT_PREFILL_FUSED: return kWorkspaceReserve + prefill_fused_workspace_bytes(s);
+    default: return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
+  }
+}
+
+// Algorithm 2 for `groups` layers of one shape sharing X (groups == 1: one layer).
+int forward_impl(int64_t groups, const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r,
+                 int64_t ldwp, const void* C, int64_t m, int64_t ldc, int c_dtype, const int32_t* pivot_idx,
+                 const int32_t* nonpivot_idx, void* Y, int64_t ldy, void* workspace, int64_t workspace_bytes,
+                 int variant, void* cuda_stream) {
   pifa_clear_error();
   int st = validate_shape(T, m, n, r);
   if (st != PIFA_OK) return st;
+  if ((st = validate_groups(groups, m, r)) != PIFA_OK) return st;
+  const int64_t G = groups;
   const bool has_np = m > r;
   if (c_dtype != PIFA_DTYPE_BF16 && c_dtype != PIFA_DTYPE_FP16) return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown c_dtype");
   if (T == 0) return PIFA_OK;  // no-op: nothing is read or written (X and Y may be null)
   if (!X || !Wp || !pivot_idx || !Y) return pifa_fail(PIFA_ERR_INVALID_ARG, "null X, Wp, pivot_idx or Y");
   if (has_np && (!C || !nonpivot_idx)) return pifa_fail(PIFA_ERR_INVALID_ARG, "null C or nonpivot_idx with m > r");
-  if (ldx < n || ldwp < n || ldy < m || (has_np && ldc < r))
+  if (ldx < n || ldwp < n || ldy < G * m || (has_np && ldc < r))
     return pifa_fail(PIFA_ERR_INVALID_ARG, "leading dimension smaller than the row length");
   if (!aligned16(X) || !aligned16(Wp) || !aligned16(Y) || (has_np && !aligned16(C)))
     return pifa_fail(PIFA_ERR_ALIGNMENT, "X, Wp, C and Y must be 16-byte aligned");
@@ -190,27 +218,19 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const
   if (variant < PIFA_VARIANT_AUTO || variant > PIFA_VARIANT_PREFILL_FUSED)
     return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
   {
-    const Span y = span_of(Y, T, m, ldy, 2);
-    if (overlaps(y, span_of(X, T, n, ldx, 2)) || overlaps(y, span_of(Wp, r, n, ldwp, 2)) ||
-        (has_np && overlaps(y, span_of(C, m - r, r, ldc, 2))))
+    const Span y = span_of(Y, T, G * m, ldy, 2);
+    if (overlaps(y, span_of(X, T, n, ldx, 2)) || overlaps(y, span_of(Wp, G * r, n, ldwp, 2)) ||
+        (has_np && overlaps(y, span_of(C, G * (m - r), r, ldc, 2))))
       return pifa_fail(PIFA_ERR_INVALID_ARG, "Y overlaps an input");
   }
   if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r, c_dtype);
 
   PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy, c_dtype};
-  int64_t need = 0;
-  switch (variant) {
-    case PIFA_VARIANT_DECODE:
-      if (T > 16) return pifa_fail(PIFA_ERR_UNSUPPORTED, "decode variant needs T <= 16");
-      need = decode_workspace_bytes(s);
-      break;
-    case PIFA_VARIANT_PREFILL_SPLIT: need = prefill_split_workspace_bytes(s); break;
-    case PIFA_VARIANT_PREFILL_FUSED:
-      if (!prefill_fused_supported(s)) return pifa_fail(PIFA_ERR_UNSUPPORTED, "fused prefill cannot run this shape");
-      need = prefill_fused_workspace_bytes(s);
-      break;
-  }
-  need += kWorkspaceReserve;
+  s.groups = G;
+  if (variant == PIFA_VARIANT_DECODE && T > 16) return pifa_fail(PIFA_ERR_UNSUPPORTED, "decode variant needs T <= 16");
+  if (variant == PIFA_VARIANT_PREFILL_FUSED && !prefill_fused_supported(s))
+    return pifa_fail(PIFA_ERR_UNSUPPORTED, "fused prefill cannot run this shape");
+  const int64_t need = workspace_bytes_for(s, variant);
   if (!workspace || workspace_bytes < need)
     return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or smaller than pifa_workspace_size()");
   if (reinterpret_cast<uintptr_t>(workspace) & 255u)
@@ -228,6 +248,37 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const
     case PIFA_VARIANT_PREFILL_FUSED: return launch_prefill_fused(s, p, status, pifa_wait_timeout_ns(), stream);
   }
   return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
+}
+
+}  // namespace
+
+extern "C" {
+
+int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,
+                         const void* C, int64_t m, int64_t ldc, int c_dtype, const int32_t* pivot_idx,
+                         const int32_t* nonpivot_idx, void* Y, int64_t ldy, void* workspace,
+                         int64_t workspace_bytes, int variant, void* cuda_stream) {
+  return forward_impl(1, X, T, n, ldx, Wp, r, ldwp, C, m, ldc, c_dtype, pivot_idx, nonpivot_idx, Y, ldy, workspace,
+                      workspace_bytes, variant, cuda_stream);
+}
+
+int pifa_forward_grouped(int64_t groups, const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r,
+                         int64_t ldwp, const void* C, int64_t m, int64_t ldc, int c_dtype, const int32_t* pivot_idx,
+                         const int32_t* nonpivot_idx, void* Y, int64_t ldy, void* workspace, int64_t workspace_bytes,
+                         void* cuda_stream) {
+  return forward_impl(groups, X, T, n, ldx, Wp, r, ldwp, C, m, ldc, c_dtype, pivot_idx, nonpivot_idx, Y, ldy,
+                      workspace, workspace_bytes, PIFA_VARIANT_AUTO, cuda_stream);
+}
+
+int64_t pifa_workspace_size_grouped(int64_t groups, int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype) {
+  int st = validate_shape(T, m, n, r);
+  if (st != PIFA_OK) return st;
+  if ((st = validate_groups(groups, m, r)) != PIFA_OK) return st;
+  if (c_dtype != PIFA_DTYPE_BF16 && c_dtype != PIFA_DTYPE_FP16) return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown c_dtype");
+  if (T == 0) return 0;
+  PifaShape s = {T, m, n, r, n, n, r, groups * m, c_dtype};
+  s.groups = groups;
+  return workspace_bytes_for(s, pifa_select_variant(T, m, n, r, c_dtype));
 }
 
 int pifa_forward(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,

@@ -165,6 +165,10 @@ struct DecodeArgs {
   uint32_t bres_off;    // byte offset of the resident B rows (NB planes x T, pitch row_pitch(kcta))
   uint32_t red_off;     // byte offset of the warps' partial tiles
   int bstaged;          // 1: the chunk's B rows ride in each stage (TMA boxes of tb rows), else resident
+  int gsz;              // grouped layers: weight rows per group (a tile never spans two), else 0
+  int goff;             // B columns between consecutive groups' K ranges (r), when gsz > 0
+  int bcols;            // columns of the B operand (K, or G r when grouped)
+  int ngrp;             // groups whose K range of B a persistent CTA keeps resident (1 when not grouped)
   int tb;               // B box rows: T rounded up to 8
   int* status;
   uint64_t timeout_ns;
@@ -240,13 +244,16 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
   // are computed from a duplicate row and never stored, and so are the output rows of weight
   // rows >= nrows (their stage rows hold stale bytes): an MMA row or column only ever affects
   // itself. Only a K tail beyond the last full step needs masking, and it gets its own step.
+  // grouped layers: this tile's group reads its own K range of B
+  const uint16_t* bp0 = a.B0 + (a.gsz > 0 ? (row0 / a.gsz) * a.goff : 0);
+  const uint16_t* bp1 = NB > 1 ? a.B1 + (a.gsz > 0 ? (row0 / a.gsz) * a.goff : 0) : nullptr;
   const uint16_t* brow[NB][NT];
 #pragma unroll
   for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
       const int t = nt * 8 + g < a.T ? nt * 8 + g : a.T - 1;
-      brow[nb][nt] = (nb == 0 ? a.B0 : a.B1) + (int64_t)t * a.ldb + 8 * c;
+      brow[nb][nt] = (nb == 0 ? bp0 : bp1) + (int64_t)t * a.ldb + 8 * c;
     }
   bool dead = false;
   for (int j = 0; j < nchunks; ++j) {
@@ -301,7 +308,7 @@ __global__ void __launch_bounds__(kWarps * 32, 2) decode_rows(DecodeArgs a) {
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
             const int t = nt * 8 + g < a.T ? nt * 8 + g : a.T - 1;
-            bt[nb][nt] = ldg8_cg(nb == 0 ? a.B0 : a.B1, a.ldb, t, true, kb + kl, a.K);
+            bt[nb][nt] = ldg8_cg(nb == 0 ? bp0 : bp1, a.ldb, t, true, kb + kl, a.K);
           }
 #pragma unroll
         for (int gq = 0; gq < RG; ++gq) {
@@ -484,11 +491,14 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
         if (wa)
           for (int b = 0; b < nblk; ++b)
             tma_load_2d(smem_u32(st + b * kBlk), &tmA, x0 + 64 * b, (int)tile_row0(it / nchunks), &full[s]);
-        if (wb)
+        if (wb) {
+          const int64_t r0 = tile_row0(it / nchunks);
+          const int xb = x0 + (a.gsz > 0 ? (int)(r0 / a.gsz) * a.goff : 0);  // the tile's group's B columns
           for (int nb = 0; nb < NB; ++nb)
             for (int b = 0; b < nblk; ++b)
-              tma_load_2d(smem_u32(st + nblkmax * kBlk + nb * bplane + b * bblk), nb ? &tmB1 : &tmB0, x0 + 64 * b, 0,
+              tma_load_2d(smem_u32(st + nblkmax * kBlk + nb * bplane + b * bblk), nb ? &tmB1 : &tmB0, xb + 64 * b, 0,
                           &full[s]);
+        }
       };
       const int pre = min(a.stages, nitems);
       for (int it = 0; it < pre; ++it) issue(it, true, false);  // weights: before the dependency wait
@@ -526,18 +536,21 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
   const int kbulk = a.bstaged ? 0 : klen & ~7, kpad = a.bstaged ? 0 : (klen + kChunk - 1) / kChunk * kChunk;
   if (warp == 0 && !a.bstaged) {
     const uint32_t bytes = (uint32_t)kbulk * 2u;
-    if (lane == 0) mbar_arrive_expect_tx(&bbar, bytes * (uint32_t)(NB * a.T));
+    if (lane == 0) mbar_arrive_expect_tx(&bbar, bytes * (uint32_t)(a.ngrp * NB * a.T));
     __syncwarp();
+    // row i: group i / (NB T), plane (i / T) % NB, token i % T
     if (bytes)
-      for (int i = lane; i < NB * a.T; i += 32)
-        bulk_copy_g2s(smem_u32(bres + i * bpitch), (i < a.T ? a.B0 : a.B1) + (int64_t)(i % a.T) * a.ldb + k0, bytes, &bbar);
+      for (int i = lane; i < a.ngrp * NB * a.T; i += 32)
+        bulk_copy_g2s(smem_u32(bres + i * bpitch),
+                      ((i / a.T) % NB ? a.B1 : a.B0) + (int64_t)(i % a.T) * a.ldb + (int64_t)(i / (NB * a.T)) * a.goff + k0,
+                      bytes, &bbar);
   }
   const int wtail = kpad - kbulk;
   if (wtail > 0)
-    for (int idx = threadIdx.x; idx < NB * a.T * wtail; idx += kCons) {
+    for (int idx = threadIdx.x; idx < a.ngrp * NB * a.T * wtail; idx += kCons) {
       const int i = idx / wtail, col = kbulk + idx % wtail;
-      const uint16_t v = col < klen ? __ldcg((i < a.T ? a.B0 : a.B1) + (int64_t)(i % a.T) * a.ldb + k0 + col) : (uint16_t)0;
-      reinterpret_cast<uint16_t*>(bres + i * bpitch)[col] = v;
+      const uint16_t* src = ((i / a.T) % NB ? a.B1 : a.B0) + (int64_t)(i % a.T) * a.ldb + (int64_t)(i / (NB * a.T)) * a.goff;
+      reinterpret_cast<uint16_t*>(bres + i * bpitch)[col] = col < klen ? __ldcg(src + k0 + col) : (uint16_t)0;
     }
   bool dead = false;
   if (threadIdx.x == 0 && !a.bstaged && !mbar_wait(&bbar, 0, a.timeout_ns)) {
@@ -567,6 +580,8 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
   for (int tt = 0; tt < ntile; ++tt) {
     const int64_t row0 = tile_row0(tt);
     const int nrows = tile_rows(row0);
+    // grouped layers, resident B: this tile's group's rows of it
+    const uint32_t bgrp = a.gsz > 0 && !a.bstaged ? (uint32_t)((row0 / a.gsz) * NB * a.T) * bpitch : 0u;
     if (tt > 0)  // the columns of this tile's rows, in flight while it computes
       for (int i = threadIdx.x; i < kRows; i += kCons)
         if (i < nrows) cp_async4(smem_u32(&s_cols[i]), a.cols + row0 + i);
@@ -603,7 +618,7 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
 #pragma unroll
               for (int nt = 0; nt < NT; ++nt)
                 bv[nb][nt] = lds128(a.bstaged ? sbase + (uint32_t)(st >> 1) * bblk + (boff[nb][nt] ^ ((uint32_t)(st & 1) << 6))
-                                              : boff[nb][nt] + bj + (uint32_t)st * 64u);
+                                              : boff[nb][nt] + bgrp + bj + (uint32_t)st * 64u);
 #pragma unroll
             for (int gq = 0; gq < RG; ++gq) {
               const uint4 wa = lds128(at + (uint32_t)(16 * gq) * 128u);      // MMA row g
@@ -864,11 +879,11 @@ size_t plan_stream(const void* fn, int kRows, int NT, int NB, DecodeArgs& a, con
   a.tb = (a.T + 7) / 8 * 8;
   int ks = 1;
   while (ks < kMaxCluster && ((int64_t)a.ntiles * ks < sm_count() ||
-                              (!a.bstaged && (size_t)NB * a.T * row_pitch(kcta_of(a.K, ks)) > kStreamBudget / 3)))
+                              (!a.bstaged && (size_t)a.ngrp * NB * a.T * row_pitch(kcta_of(a.K, ks)) > kStreamBudget / 3)))
     ks *= 2;
   a.ks = ks;
   a.kcta = kcta_of(a.K, ks);
-  const size_t bres = a.bstaged ? 0 : round16((size_t)NB * a.T * row_pitch(a.kcta));
+  const size_t bres = a.bstaged ? 0 : round16((size_t)a.ngrp * NB * a.T * row_pitch(a.kcta));
   const size_t side = bres + red + (ks > 1 ? 2 * recv1 : 0);
   const size_t blk = (size_t)kRows * 128 + (a.bstaged ? (size_t)NB * a.tb * 128 : 0);  // one 64-column block
   const size_t ring = kStreamBudget > side + 2 * blk ? kStreamBudget - side : 2 * blk;
@@ -944,29 +959,32 @@ int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, cudaStream_t str
   if (st != PIFA_OK) return st;
   CUtensorMap tm, tb0 = {}, tb1 = {};  // B maps (x, or the y_p planes in C's type): staged B only
   if ((st = make_tmap_2d(&tm, dtype, a.A, a.R, a.K, a.lda, 64, kRowsOf<RGS>)) != PIFA_OK) return st;
-  if (a.bstaged && (st = make_tmap_2d(&tb0, dtype, a.B0, a.T, a.K, a.ldb, 64, a.tb)) != PIFA_OK) return st;
-  if (a.bstaged && PHASE == 2 && (st = make_tmap_2d(&tb1, dtype, a.B1, a.T, a.K, a.ldb, 64, a.tb)) != PIFA_OK)
+  if (a.bstaged && (st = make_tmap_2d(&tb0, dtype, a.B0, a.T, a.bcols, a.ldb, 64, a.tb)) != PIFA_OK) return st;
+  if (a.bstaged && PHASE == 2 && (st = make_tmap_2d(&tb1, dtype, a.B1, a.T, a.bcols, a.ldb, 64, a.tb)) != PIFA_OK)
     return st;
   return launch_stream(ks, tm, tb0, tb1, a, smem_s, stream, what);
 }
 
 template <int NT, bool kF16C, int RG, int RGS>
 int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
-  const int64_t ldyp = (s.r + 7) / 8 * 8;  // 16-byte rows keep the fragment loads aligned
+  const int64_t G = s.groups;                      // layers sharing X (1: one layer)
+  const int64_t ldyp = (G * s.r + 7) / 8 * 8;  // 16-byte rows keep the fragment loads aligned
   uint16_t* yph = reinterpret_cast<uint16_t*>(p.ws);
   uint16_t* ypl = yph + s.T * ldyp;
   DecodeArgs a = {};
   a.A = reinterpret_cast<const uint16_t*>(p.Wp);
   a.lda = s.ldwp;
-  a.R = (int)s.r;
+  a.R = (int)(G * s.r);  // the groups' pivot rows, stacked: phase 1 is one contraction against x
   a.K = (int)s.n;
   a.B0 = reinterpret_cast<const uint16_t*>(p.X);
   a.ldb = s.ldx;
+  a.bcols = (int)s.n;
+  a.ngrp = 1;
   a.yph = s.m > s.r ? yph : nullptr;
   a.ypl = s.m > s.r ? ypl : nullptr;
   a.ldyp = ldyp;
   a.cols = p.piv;
-  a.m = (int)s.m;
+  a.m = (int)(G * s.m);
   a.Y = reinterpret_cast<bf16*>(p.Y);
   a.ldy = s.ldy;
   a.T = (int)s.T;
@@ -977,11 +995,17 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   DecodeArgs b = a;
   b.A = reinterpret_cast<const uint16_t*>(p.C);
   b.lda = s.ldc;
-  b.R = (int)(s.m - s.r);
+  b.R = (int)(G * (s.m - s.r));
   b.K = (int)s.r;
   b.B0 = yph;
   b.B1 = ypl;
   b.ldb = ldyp;
+  b.bcols = (int)(G * s.r);
+  if (G > 1) {  // group g's non-pivot rows (a whole number of tiles) read y_p's columns [g r, (g + 1) r)
+    b.gsz = (int)(s.m - s.r);
+    b.goff = (int)s.r;
+    b.ngrp = (int)G;
+  }
   b.yph = b.ypl = nullptr;
   b.cols = p.nonpiv;
   return launch_one_phase<2, NT, kF16C, RG, RGS>(b, kStageBudget2, (int)s.c_dtype, stream);
@@ -997,9 +1021,9 @@ extern "C" int pifa_set_decode_grid(int mode) {
 }
 
 int64_t decode_workspace_bytes(const PifaShape& s) {
-  // y_p as hi and lo planes of 2-byte elements, T rows of pitch round_up(r, 8) each, rounded up
+  // y_p as hi and lo planes of 2-byte elements, T rows of pitch round_up(G r, 8) each, rounded up
   // to 256 bytes
-  return ((s.T * ((s.r + 7) / 8 * 8) * 4 + 255) / 256) * 256;
+  return ((s.T * ((s.groups * s.r + 7) / 8 * 8) * 4 + 255) / 256) * 256;
 }
 
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {

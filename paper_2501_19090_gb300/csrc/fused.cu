@@ -411,7 +411,8 @@ int64_t prefill_fused_workspace_bytes(const PifaShape& s) {
   return 2 * (((s.T * pad8(s.r) * 2 + 255) / 256) * 256);  // Y_p hi and lo staging, T x pad8(r) each
 }
 
-bool prefill_fused_supported(const PifaShape&) { return query_plan().G >= 2; }
+// (one layer only: grouped layers run the split GEMMs)
+bool prefill_fused_supported(const PifaShape& s) { return s.groups == 1 && query_plan().G >= 2; }
 
 int launch_prefill_fused(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,
                          cudaStream_t stream) {

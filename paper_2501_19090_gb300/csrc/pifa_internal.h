@@ -25,6 +25,12 @@ struct PifaShape {
   int64_t T, m, n, r;
   int64_t ldx, ldwp, ldc, ldy;
   int c_dtype;  // PIFA_DTYPE_BF16 or PIFA_DTYPE_FP16 (storage type of C)
+  // G layers of one shape sharing X (pifa_forward_grouped): W_p holds G r rows, C G (m - r) rows,
+  // Y G m columns (the pivot / non-pivot indices are absolute columns of Y), y_p G r columns; the
+  // non-pivot rows of group g read y_p's columns [g r, (g + 1) r). G > 1 needs (m - r) % 128 == 0
+  // and r % 8 == 0, so that no tile spans two groups and every group's y_p columns start 16-byte
+  // aligned.
+  int64_t groups = 1;
 };
 
 // The first kWorkspaceReserve bytes of every workspace are reserved for library state (no kernel

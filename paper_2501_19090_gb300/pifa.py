@@ -44,7 +44,8 @@ EXPORTS = (
     "pifa_forward", "pifa_forward_variant", "pifa_workspace_size", "pifa_select_variant",
     "pifa_variant_name", "pifa_compress", "pifa_validate_indices", "pifa_device_status",
     "pifa_status_string", "pifa_last_error", "pifa_version", "pifa_forward_decode_noalloc",
-    "pifa_set_wait_timeout", "pifa_selftest_wait_timeout", "pifa_set_decode_grid",
+    "pifa_set_wait_timeout", "pifa_selftest_wait_timeout", "pifa_set_decode_grid", "pifa_forward_grouped",
+    "pifa_workspace_size_grouped",
 )
 
 
@@ -86,6 +87,10 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.pifa_forward_decode_noalloc.restype = ctypes.c_int
         lib.pifa_workspace_size.argtypes = [_I64, _I64, _I64, _I64, ctypes.c_int, ctypes.c_int]
         lib.pifa_workspace_size.restype = _I64
+        lib.pifa_forward_grouped.argtypes = [_I64] + fwd + [ctypes.c_int] + tail + [_VP]
+        lib.pifa_forward_grouped.restype = ctypes.c_int
+        lib.pifa_workspace_size_grouped.argtypes = [_I64, _I64, _I64, _I64, _I64, ctypes.c_int]
+        lib.pifa_workspace_size_grouped.restype = _I64
         lib.pifa_select_variant.argtypes = [_I64, _I64, _I64, _I64, ctypes.c_int]
         lib.pifa_select_variant.restype = ctypes.c_int
         lib.pifa_variant_name.argtypes = [ctypes.c_int]
@@ -273,6 +278,42 @@ def pifa_forward(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, variant: int = PIFA_
         pivot_idx.data_ptr(), nonpivot_idx.data_ptr() if has_np else None,
         Y.data_ptr(), _ld(Y), ws_ptr or None, ws_bytes, variant, _stream_ptr(stream))
     _check(st, "pifa_forward")
+    return Y
+
+
+def pifa_workspace_size_grouped(groups: int, T: int, m: int, n: int, r: int, c_dtype: int = PIFA_DTYPE_BF16) -> int:
+    v = _lib().pifa_workspace_size_grouped(groups, T, m, n, r, c_dtype)
+    if v < 0:
+        _check(int(v), "pifa_workspace_size_grouped")
+    return int(v)
+
+
+def pifa_forward_grouped(groups: int, X, Wp, C, pivot_idx, nonpivot_idx, Y=None, workspace_tensor=None, stream=None):
+    """Y = [PIFA_0(X) | ... | PIFA_{G-1}(X)] for G layers of one shape sharing X, through
+    pifa_forward_grouped: Wp (G r x n) and C (G (m-r) x r) hold the groups' matrices stacked by
+    rows; pivot_idx / nonpivot_idx the groups' indices offset by g m. Allocates Y (T x G m) if not
+    given."""
+    import torch
+    G = int(groups)
+    T, n = X.shape
+    r = Wp.shape[0] // G
+    m = r + nonpivot_idx.numel() // G
+    if Y is None:
+        Y = torch.empty((T, G * m), dtype=torch.bfloat16, device=X.device)
+    cdt = c_dtype_of(C)
+    need = pifa_workspace_size_grouped(G, T, m, n, r, cdt)
+    ws = workspace_tensor
+    if need > 0 and ws is None:
+        ws = workspace(need, X.device, stream)
+    ws_ptr = 0 if ws is None else ws.data_ptr()
+    if ws is not None and ws_ptr % 256:
+        ws_ptr += 256 - ws_ptr % 256
+    ws_bytes = 0 if ws is None else ws.numel() * ws.element_size() - (ws_ptr - ws.data_ptr())
+    st = _lib().pifa_forward_grouped(
+        G, X.data_ptr(), T, n, _ld(X), Wp.data_ptr(), r, _ld(Wp), C.data_ptr(), m, _ld(C), cdt,
+        pivot_idx.data_ptr(), nonpivot_idx.data_ptr(), Y.data_ptr(), _ld(Y), ws_ptr or None, ws_bytes,
+        _stream_ptr(stream))
+    _check(st, "pifa_forward_grouped")
     return Y
 
 

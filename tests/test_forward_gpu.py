@@ -441,3 +441,72 @@ def test_workspace_needs_no_initialisation_and_is_shared():
     ws = torch.full((need,), 0xFF, dtype=torch.uint8, device=DEV)
     for T, v in cases:
         parity(L, T, v, workspace_tensor=ws)
+
+
+# ---------------------------------------------------------------------------------------------
+# grouped layers sharing X (pifa_forward_grouped)
+# ---------------------------------------------------------------------------------------------
+def run_grouped(layers, X32, pad=8):
+    """pifa_forward_grouped over `layers` (one shape) stacked by rows; Y (T x G m) inside a
+    NaN-filled buffer whose padding columns hold a sentinel. Returns Y as float32."""
+    G = len(layers)
+    L0 = layers[0]
+    m, r = L0.m, L0.r
+    Wp = torch.cat([L.dev()[0] for L in layers])
+    C = torch.cat([L.dev()[1] for L in layers])
+    piv = torch.cat([L.dev()[2] + g * m for g, L in enumerate(layers)])
+    nonp = torch.cat([L.dev()[3] + g * m for g, L in enumerate(layers)])
+    T = X32.shape[0]
+    X = _pad_dev(X32)
+    ldy = _round8(G * m + pad)
+    big = torch.full((T, ldy), SENTINEL, dtype=torch.bfloat16, device=DEV)
+    Y = big[:, :G * m]
+    Y.fill_(float("nan"))
+    P.pifa_forward_grouped(G, X, Wp, C, piv, nonp, Y=Y)
+    st = P.pifa_device_status(None)
+    assert st == P.PIFA_OK, P.pifa_status_string(st)
+    host = big.float().cpu().numpy()
+    assert np.all(host[:, G * m:] == SENTINEL), "padding columns of Y were written"
+    out = host[:, :G * m]
+    assert not np.isnan(out).any(), "some output element was never written"
+    return out
+
+
+def grouped_parity(layers, T, sample=None, seed=0):
+    X = acts(T, layers[0].n, seed)
+    Y = run_grouped(layers, X)
+    m = layers[0].m
+    rows = np.arange(T) if (sample is None or sample >= T) else inputs.random_rows(T, sample, seed)
+    for g, L in enumerate(layers):
+        ref = oracle.forward(X[rows], L.Wp, L.C, L.pivots, L.nonpivots)
+        check(Y[rows, g * m:(g + 1) * m], ref, f"group {g} of {len(layers)} ({L.name}) T={T}")
+
+
+@pytest.mark.parametrize("G", [2, 3])
+@pytest.mark.parametrize("T", [1, 3, 8, 16, 100, 300])
+def test_grouped_layers_match_per_layer_oracle(G, T):
+    """G synthetic layers of one shape (m - r = 7 x 128, ragged n) sharing X: each group's block of
+    Y equals the oracle's forward of that layer alone (decode for T <= 16, split prefill above)."""
+    layers = [layer_for(1408, 1000, 512, 10 + g, "synthetic") for g in range(G)]
+    grouped_parity(layers, T)
+
+
+@pytest.mark.parametrize("T", [2, 8, 16])
+@pytest.mark.parametrize("grid", [P.PIFA_DECODE_GRID_PERSISTENT, P.PIFA_DECODE_GRID_WAVES])
+def test_grouped_layers_both_decode_grids(T, grid):
+    """Grouped decode under both layouts; the persistent grid keeps every group's K range of y_p
+    resident (T <= 2) or stages the tile's group's columns (T > 2)."""
+    layers = [layer_for(1408, 1000, 512, 20 + g, "synthetic") for g in range(2)]
+    P.pifa_set_decode_grid(grid)
+    try:
+        grouped_parity(layers, T)
+    finally:
+        P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
+
+
+@pytest.mark.parametrize("T,sample", [(1, None), (8, None), (2048, 256)])
+def test_grouped_mlp7b_gate_up(T, sample):
+    """The 7B MLP's gate and up projections (11008 x 4096, r = 2048, m - r = 70 x 128) as one grouped
+    call on a shared X."""
+    layers = [layer_for(11008, 4096, 2048, 0, "library"), layer_for(11008, 4096, 2048, 1, "library")]
+    grouped_parity(layers, T, sample=sample)

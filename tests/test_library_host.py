@@ -57,6 +57,19 @@ def test_decode_grid_setter(lib):
     assert lib.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO) == P.PIFA_OK
 
 
+def test_grouped_workspace_and_argument_rules(lib):
+    """pifa_workspace_size_grouped: y_p scratch for all groups; the grouped shape rules."""
+    one = P.pifa_workspace_size(8, 1408, 1000, 512)
+    assert P.pifa_workspace_size_grouped(1, 8, 1408, 1000, 512) == one
+    assert P.pifa_workspace_size_grouped(3, 8, 1408, 1000, 512) > one
+    assert P.pifa_workspace_size_grouped(2, 2048, 11008, 4096, 2048) >= 2 * 2048 * 4096 * 2
+    assert lib.pifa_workspace_size_grouped(0, 8, 1408, 1000, 512, P.PIFA_DTYPE_BF16) == P.PIFA_ERR_INVALID_ARG
+    assert lib.pifa_workspace_size_grouped(2, 8, 1400, 1000, 512, P.PIFA_DTYPE_BF16) == P.PIFA_ERR_UNSUPPORTED
+    assert lib.pifa_workspace_size_grouped(2, 8, 1412, 1000, 516, P.PIFA_DTYPE_BF16) == P.PIFA_ERR_UNSUPPORTED
+    assert lib.pifa_workspace_size_grouped(2, 8, 512, 1000, 512, P.PIFA_DTYPE_BF16) == P.PIFA_ERR_UNSUPPORTED
+    assert lib.pifa_workspace_size_grouped(2, 0, 1408, 1000, 512, P.PIFA_DTYPE_BF16) == 0
+
+
 def test_selector(lib):
     assert P.pifa_select_variant(1, 4096, 4096, 2048) == P.PIFA_VARIANT_DECODE
     assert P.pifa_select_variant(16, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE
