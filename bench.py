@@ -296,6 +296,7 @@ def run_ours(args, rank, world, local_rank):
         out["prefill_fused"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src,
                                              variant=P.PIFA_VARIANT_PREFILL_FUSED)
         out["decode_sweep"] = decode_sweep(dev, stream, hbm_peak, peak_src)
+        out["grouped_mlp7b_gate_up"] = grouped_point(dev, stream, hbm_peak, tc_peak, peak_src)
         out["cpu_baseline"] = cpu_baseline(lay, T)
     return out
 
@@ -395,6 +396,72 @@ def decode_sweep(dev, stream, hbm_peak, peak_src):
             del g, g2
         del Wps, Cs, Us, Vs
         torch.cuda.empty_cache()
+    return out
+
+
+def grouped_point(dev, stream, hbm_peak, tc_peak, peak_src):
+    """The 7B MLP's gate and up projections (11008 x 4096, r = 2048) sharing X: one
+    pifa_forward_grouped call against two pifa_forward calls, graph replay, >= 4 rotating weight
+    copies; timing operands as in decode_sweep (seeded N(0, 1) weights, random pivot sets)."""
+    import torch
+    from paper_2501_19090_gb300 import pifa as P
+    shape = inputs.MLP7B_GATE
+    m, n, r, G = shape.m, shape.n, shape.r, 2
+    rng = np.random.default_rng(13)
+    piv_l, nonp_l = [], []
+    for g in range(G):
+        perm = rng.permutation(m)
+        piv_l.append(torch.from_numpy(np.sort(perm[:r]).astype(np.int32)).to(dev))
+        nonp_l.append(torch.from_numpy(np.sort(perm[r:]).astype(np.int32)).to(dev))
+    piv_s = torch.cat([piv_l[g] + g * m for g in range(G)])
+    nonp_s = torch.cat([nonp_l[g] + g * m for g in range(G)])
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(14)
+    copies = 4
+    Wps = [torch.randn((G * r, n), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
+    Cs = [torch.randn((G * (m - r), r), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
+    out = []
+    for T in (1, 8, T_PREFILL):
+        X = torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16)
+        Y = torch.empty((T, G * m), dtype=torch.bfloat16, device=dev)
+        Ys = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(G)]
+        ws1 = P.workspace(P.pifa_workspace_size(T, m, n, r), dev, "grp1")
+        wsg = P.workspace(P.pifa_workspace_size_grouped(G, T, m, n, r), dev, "grpG")
+
+        def sep(i):
+            j = i % copies
+            for g in range(G):
+                P.pifa_forward(X, Wps[j][g * r:(g + 1) * r], Cs[j][g * (m - r):(g + 1) * (m - r)], piv_l[g],
+                               nonp_l[g], Y=Ys[g], workspace_tensor=ws1, stream=stream)
+
+        def grp(i):
+            j = i % copies
+            P.pifa_forward_grouped(G, X, Wps[j], Cs[j], piv_s, nonp_s, Y=Y, workspace_tensor=wsg, stream=stream)
+
+        per_graph = 16 if T <= 16 else 4
+        res = {}
+        for name, fn in (("separate", sep), ("grouped", grp)):
+            with torch.cuda.stream(stream):
+                for i in range(4):
+                    fn(i)
+            g_ = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g_, stream=stream):
+                for i in range(per_graph):
+                    fn(i)
+            res[name] = _graph_ms(g_, stream, replays=5) / per_graph
+            del g_
+        assert P.pifa_device_status(stream) == P.PIFA_OK
+        e = {"workload": f"{shape.name} x2 (gate + up) T={T}", "grouped_us": res["grouped"] * 1e3,
+             "separate_us": res["separate"] * 1e3, "speedup": res["separate"] / res["grouped"]}
+        if T <= 16:
+            gbs = G * decode_bytes(T, m, n, r) / res["grouped"] / 1e6
+            e.update({"hbm_gbs": gbs, "frac": gbs / hbm_peak, "peak_source": f"{peak_src} hbm_gbs"})
+        else:
+            tf = G * pifa_flops(T, m, n, r) / res["grouped"] / 1e9
+            e.update({"tflops": tf, "frac": tf / tc_peak, "peak_source": f"{peak_src} bf16_tflops (burst)"})
+        out.append(e)
+    del Wps, Cs
+    torch.cuda.empty_cache()
     return out
 
 
