@@ -510,3 +510,42 @@ def test_grouped_mlp7b_gate_up(T, sample):
     call on a shared X."""
     layers = [layer_for(11008, 4096, 2048, 0, "library"), layer_for(11008, 4096, 2048, 1, "library")]
     grouped_parity(layers, T, sample=sample)
+
+
+# ---------------------------------------------------------------------------------------------
+# split prefill: many tiles per GEMM
+# ---------------------------------------------------------------------------------------------
+@pytest.mark.parametrize("T", [17, 300, 1000])
+def test_prefill_many_tiles_ragged(T):
+    """Split prefill on a layer whose GEMM 2 spans several waves of tiles (m - r = 39736 rows: 311
+    row tiles, the last one partial); ragged K in both GEMMs (520 and 264)."""
+    L = layer_for(40000, 520, 264, 3, "synthetic")
+    parity(L, T, P.PIFA_VARIANT_PREFILL_SPLIT, sample=192)
+
+
+@pytest.mark.parametrize("T", [40, 700])
+def test_prefill_fp16_c_padding_rank_not_multiple_of_64(T):
+    """Split prefill with C in fp16 (the single fp16 y_p pass, range check in the GEMM 1 epilogue)
+    on padded pitches holding NaN, with a rank (600) that leaves a partial 64-column K chunk."""
+    L = layer_for(3000, 1000, 600, 4, "synthetic", "fp16")
+    parity(L, T, P.PIFA_VARIANT_PREFILL_SPLIT, ldx=1000 + 24, ldwp=1000 + 40, ldc=600 + 16)
+
+
+def test_prefill_two_waves_deterministic():
+    """Bitwise-identical Y over repeated calls where both GEMMs take two waves of tiles (70B q/o
+    layer, T = 2048: 288 tiles each on 152 SMs), with the next GEMM launched programmatically
+    while the previous one drains."""
+    L = layer_for(8192, 8192, 4096, 0, "library")
+    X = acts(2048, 8192, 9)
+    first = run(L, X, P.PIFA_VARIANT_PREFILL_SPLIT)
+    for _ in range(2):
+        assert np.array_equal(run(L, X, P.PIFA_VARIANT_PREFILL_SPLIT), first)
+    rows = inputs.random_rows(2048, 96, 9)
+    check(first[rows], oracle.forward(X[rows], L.Wp, L.C, L.pivots, L.nonpivots), "70B q/o T=2048")
+
+
+@pytest.mark.parametrize("T", [300, 1200])
+def test_grouped_layers_prefill_three_groups(T):
+    """Grouped prefill, three groups: GEMM 2 tiles read their group's hi/lo column range."""
+    layers = [layer_for(1408, 1000, 512, 30 + g, "synthetic") for g in range(3)]
+    grouped_parity(layers, T, sample=160)
