@@ -78,21 +78,40 @@ def pifa_flops(T, m, n, r):
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons sampled every 100 ms while active."""
+    """nvidia-smi clocks, throttle reasons and temperatures sampled every 100 ms while active.
+
+    The temperatures are context for the decode numbers: with the SM clock at its maximum the
+    same decode graph times differently by the GPU's recent load (slower right after a burst of
+    dense GEMMs), so each line carries the GPU and HBM temperatures seen while it was timed."""
 
     Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
          "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
          "clocks_event_reasons.sw_power_cap")
+    EXTRA = ",clocks.mem,temperature.gpu,temperature.memory"
+    _query = None  # Q + EXTRA where this nvidia-smi accepts the extra fields, else Q
 
     def __init__(self, gpu_index: int):
         self.gpu = gpu_index
         self.proc = None
         self.lines = []
 
+    def _pick_query(self):
+        if ClockSampler._query is None:
+            ClockSampler._query = self.Q
+            try:
+                r = subprocess.run(["nvidia-smi", f"--query-gpu={self.Q + self.EXTRA}", "--format=csv,noheader,nounits",
+                                    "-i", str(self.gpu)], capture_output=True, text=True, timeout=20)
+                if r.returncode == 0 and len(r.stdout.strip().split(",")) >= 11:
+                    ClockSampler._query = self.Q + self.EXTRA
+            except Exception:
+                pass
+        return ClockSampler._query
+
     def __enter__(self):
         try:
+            q = self._pick_query()
             self.proc = subprocess.Popen(
-                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits", "-lms", "100",
+                ["nvidia-smi", f"--query-gpu={q}", "--format=csv,noheader,nounits", "-lms", "100",
                  "-i", str(self.gpu)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -114,6 +133,7 @@ class ClockSampler:
 
     def summary(self):
         sm, mx, reasons = [], [], set()
+        extra = {"mem_mhz": [], "gpu_temp_c": [], "hbm_temp_c": []}
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for ln in self.lines:
             parts = [p.strip() for p in ln.split(",")]
@@ -127,10 +147,21 @@ class ClockSampler:
             for nm, val in zip(names, parts[4:8]):
                 if val.lower().startswith("active"):
                     reasons.add(nm)
+            for key, val in zip(("mem_mhz", "gpu_temp_c", "hbm_temp_c"), parts[8:11]):
+                try:
+                    extra[key].append(float(val))
+                except ValueError:
+                    pass
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        out = {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+               "samples": len(sm)}
+        if extra["mem_mhz"]:
+            out["mem_mhz"] = statistics.median(extra["mem_mhz"])
+        for key in ("gpu_temp_c", "hbm_temp_c"):
+            if extra[key]:
+                out[key] = [min(extra[key]), max(extra[key])]
+        return out
 
 
 # ---------------------------------------------------------------------------------------------
