@@ -9,7 +9,9 @@ Printed as one JSON line on rank 0:
              from a CUDA graph; the weights rotate over enough copies that the working set is
              larger than L2 (every step streams its weights from HBM);
   e2e        the same metric through the public API with host buffers: per step, X copied from
-             pinned host memory, pifa_forward, Y copied back to pinned host memory;
+             pinned host memory, pifa_forward, Y copied back to pinned host memory, with the copies
+             of neighbouring steps overlapping the forwards (two copy streams, four buffers in
+             flight); the serial loop (no overlap) is reported beside it;
   roofline   the decode call's achieved HBM GB/s against MEASURED_PEAKS.json (algorithmic bytes:
              2 r(m + n - r) weight bytes + 2 T (n + m) activation bytes + 4 m index bytes);
   cpu_baseline  the fp64 oracle (numpy) on the host cores over a bounded sample of the workload;
@@ -337,6 +339,8 @@ def run_ours(args, rank, world, local_rank):
     stream.synchronize()
     e2e_graph = _job_value(world, T, e2e_replays * per_e2e, _max_over_ranks(e0.elapsed_time(e1)))
     assert np.array_equal(Yhs[(per_e2e - 1) % nh].float().numpy(), Ys[0].cpu().float().numpy())
+    e2e_pipe, e2e_pipe_steps, e2e_pipe_per = e2e_pipelined(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws,
+                                                           stream, world, e2e_steps)
 
     out = {
         "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
@@ -347,17 +351,27 @@ def run_ours(args, rank, world, local_rank):
                    "variant": P.pifa_variant_name(variant), "parallelism": f"replicas{world}",
                    "l2_defeat": f"{copies} rotating weight copies ({copies * wbytes / 1e6:.0f} MB > 3x L2)",
                    "timing": "CUDA graph replay, CUDA events on the launching stream"},
-        "e2e": {"value": e2e_eager, "unit": "tokens/s", "h2d_bytes_per_step": T * n * 2,
+        "e2e": {"value": e2e_pipe, "unit": "tokens/s", "h2d_bytes_per_step": T * n * 2,
                 "d2h_bytes_per_step": T * m * 2,
-                "mode": "per step: X uploaded from pinned host memory, pifa_forward, Y downloaded to pinned host "
-                        "memory, issued call by call",
-                "graph_value": e2e_graph,
-                "graph_mode": "the same loop captured as a CUDA graph and replayed (the two copies, not the host, "
-                              "dominate a step)"},
-        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                     "frac": achieved / hbm_peak, "traffic": _traffic("decode.cu", "decode") if (T, m, n, r) == (8, 4096, 4096, 2048) else None,
-                     "peak_source": f"{peak_src} hbm_gbs", "kernel": "decode_rows phase 1 + phase 2 (one PDL-chained pair per call)",
-                     "algorithmic_bytes_per_launch": decode_bytes(T, m, n, r)},
+                "mode": f"serving loop: per step X uploaded from pinned host memory, pifa_forward, Y downloaded to "
+                        f"pinned host memory; 4 device buffers in flight, uploads and downloads on two copy streams "
+                        f"overlapping the forwards of neighbouring steps; {e2e_pipe_per} steps per CUDA graph, "
+                        f"{e2e_pipe_steps} steps timed; the last step's Y checked against a separate forward",
+                "serial_value": e2e_eager,
+                "serial_mode": "the same steps one after another on one stream, issued call by call (no overlap)",
+                "serial_graph_value": e2e_graph,
+                "serial_graph_mode": "the serial loop captured as a CUDA graph and replayed"},
+        "roofline": ({"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                      "frac": achieved / hbm_peak,
+                      "traffic": _traffic("decode.cu", "decode") if (T, m, n, r) == (8, 4096, 4096, 2048) else None,
+                      "peak_source": f"{peak_src} hbm_gbs",
+                      "kernel": "decode phase 1 + phase 2 (one PDL-chained pair per call)",
+                      "algorithmic_bytes_per_launch": decode_bytes(T, m, n, r)} if T <= 16 else
+                     {"bound": "tensor", "achieved": pifa_flops(T, m, n, r) / (step_ms / 1e3) / 1e12, "peak": tc_peak,
+                      "unit": "TFLOP/s", "frac": pifa_flops(T, m, n, r) / (step_ms / 1e3) / 1e12 / tc_peak,
+                      "traffic": None, "peak_source": f"{peak_src} bf16_tflops (burst)",
+                      "kernel": f"{P.pifa_variant_name(variant)} prefill (GEMM 1 + GEMM 2 per call)",
+                      "algorithmic_flops_per_launch": pifa_flops(T, m, n, r)}),
         "gpu_launches": steps * (2 if m > r else 1),
         "clocks": clk.summary(),
     }
@@ -542,6 +556,93 @@ def grouped_point(dev, stream, hbm_peak, tc_peak, peak_src):
     del Wps, Cs
     torch.cuda.empty_cache()
     return out
+
+
+def e2e_pipelined(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws, stream, world, steps):
+    """End to end through pifa_forward as a serving loop issues it: every step uploads its X from
+    pinned host memory, runs the forward and downloads its Y to pinned host memory, with NB device
+    buffers in flight so that the copies of neighbouring steps overlap the forward (uploads on one
+    copy stream, downloads on another, the forwards in order on the compute stream; events order
+    each buffer's reuse; one copy stream per buffer measured no faster). Captured as one
+    multi-stream CUDA graph of `per` steps and replayed; a replay starts after the previous one has
+    drained, so each replay pays one pipeline fill. Returns (tokens/s over all ranks, steps timed,
+    per)."""
+    import torch
+    NB = 4
+    nh = len(Xhs)
+    copies = len(Wps)
+    Xd = [torch.empty((T, n), dtype=torch.bfloat16, device=dev) for _ in range(NB)]
+    Yd = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(NB)]
+    Yhs = [torch.empty((T, m), dtype=torch.bfloat16).pin_memory() for _ in range(nh)]
+    s_in = torch.cuda.Stream(device=dev)       # uploads, in step order
+    s_out = torch.cuda.Stream(device=dev)      # downloads, in step order
+    per = copies * max(1, 64 // copies)
+
+    def pipeline(k_steps):
+        ev_in = [torch.cuda.Event() for _ in range(NB)]
+        ev_fwd = [torch.cuda.Event() for _ in range(NB)]
+        ev_out = [torch.cuda.Event() for _ in range(NB)]
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        s_in.wait_event(fork)
+        s_out.wait_event(fork)
+        for i in range(k_steps):
+            b = i % NB
+            if i >= NB:
+                s_in.wait_event(ev_fwd[b])        # forward i - NB has read Xd[b]
+            with torch.cuda.stream(s_in):
+                Xd[b].copy_(Xhs[i % nh], non_blocking=True)
+            ev_in[b].record(s_in)
+            stream.wait_event(ev_in[b])
+            if i >= NB:
+                stream.wait_event(ev_out[b])      # download i - NB has read Yd[b]
+            P.pifa_forward(Xd[b], Wps[i % copies], Cs[i % copies], piv, nonp, Y=Yd[b], variant=variant,
+                           workspace_tensor=ws, stream=stream)
+            ev_fwd[b].record(stream)
+            s_out.wait_event(ev_fwd[b])
+            with torch.cuda.stream(s_out):
+                Yhs[i % nh].copy_(Yd[b], non_blocking=True)
+            ev_out[b].record(s_out)
+        join_in, join_out = torch.cuda.Event(), torch.cuda.Event()
+        join_in.record(s_in)
+        join_out.record(s_out)
+        stream.wait_event(join_in)
+        stream.wait_event(join_out)
+
+    with torch.cuda.stream(stream):
+        pipeline(2 * NB)                          # eager warm-up of the same streams and buffers
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        pipeline(per)
+    replays = max(1, steps // per)
+    for _ in range(2):
+        g.replay()
+    stream.synchronize()
+    dist = _dist()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(replays):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    ms = _max_over_ranks(e0.elapsed_time(e1))
+    # the last step's downloaded Y equals a separate forward of the same inputs (decode and prefill
+    # are deterministic)
+    i = per - 1
+    with torch.cuda.stream(stream):
+        Xchk = Xhs[i % nh].to(dev)
+        Ychk = torch.empty((T, m), dtype=torch.bfloat16, device=dev)
+        P.pifa_forward(Xchk, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Ychk, variant=variant,
+                       workspace_tensor=ws, stream=stream)
+    stream.synchronize()
+    assert torch.equal(Yhs[i % nh].view(torch.int16), Ychk.cpu().view(torch.int16)), "pipelined e2e output mismatch"
+    return _job_value(world, T, replays * per, ms), replays * per, per
 
 
 def _graph_ms(g, stream, replays):
