@@ -80,11 +80,8 @@ def pifa_flops(T, m, n, r):
 
 
 class ClockSampler:
-    """nvidia-smi clocks, throttle reasons and temperatures sampled every 100 ms while active.
-
-    The temperatures are context for the decode numbers: with the SM clock at its maximum the
-    same decode graph times differently by the GPU's recent load (slower right after a burst of
-    dense GEMMs), so each line carries the GPU and HBM temperatures seen while it was timed."""
+    """nvidia-smi clocks, throttle reasons, memory clock and GPU / HBM temperatures sampled every
+    100 ms while active (the state each timed region ran in)."""
 
     Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
          "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
@@ -250,8 +247,9 @@ def run_ours(args, rank, world, local_rank):
             step(i)
     replays = max(1, math.ceil(args.steps / per_graph))
     steps = replays * per_graph
-    for _ in range(max(3, args.warmup)):
-        g.replay()
+    with torch.cuda.stream(stream):                # replays launch on the current stream
+        for _ in range(max(3, args.warmup)):
+            g.replay()
     stream.synchronize()
 
     dist = _dist()
@@ -325,8 +323,9 @@ def run_ours(args, rank, world, local_rank):
         for i in range(per_e2e):
             e2e_step(i)
     e2e_replays = max(1, e2e_steps // per_e2e)
-    for _ in range(2):
-        ge.replay()
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            ge.replay()
     stream.synchronize()
     if dist:
         dist.barrier()
@@ -392,7 +391,8 @@ def run_ours(args, rank, world, local_rank):
 
 
 def comparators(dev, lay, T, copies, stream):
-    """Dense X W^T and two-factor low-rank (X V) U^T on the same GPU (torch.matmul, bf16)."""
+    """Dense X W^T and two-factor low-rank (X V) U^T on the same GPU (torch.matmul, bf16), each a
+    CUDA graph over rotating weight copies timed in steady state (_graph_ms)."""
     import torch
     res = {}
     U = torch.from_numpy(lay["U"]).to(dev).to(torch.bfloat16)
@@ -408,15 +408,14 @@ def comparators(dev, lay, T, copies, stream):
             with torch.cuda.stream(stream):
                 for i in range(5):
                     fn(i)
-                e0 = torch.cuda.Event(enable_timing=True)
-                e1 = torch.cuda.Event(enable_timing=True)
-                reps = 200 if Tq <= 16 else 40
-                e0.record(stream)
-                for i in range(reps):
-                    fn(i)
-                e1.record(stream)
             stream.synchronize()
-            ms = e0.elapsed_time(e1) / reps
+            per = nrot * max(1, 64 // nrot) if Tq <= 16 else nrot
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for i in range(per):
+                    fn(i)
+            ms = _graph_ms(g, stream) / per
+            del g
             res[f"{name}_T{Tq}"] = {"tokens_per_s": Tq / (ms / 1e3), "ms": ms}
     return res
 
@@ -616,8 +615,9 @@ def e2e_pipelined(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws, stream,
     with torch.cuda.graph(g, stream=stream):
         pipeline(per)
     replays = max(1, steps // per)
-    for _ in range(2):
-        g.replay()
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            g.replay()
     stream.synchronize()
     dist = _dist()
     if dist:
@@ -645,20 +645,57 @@ def e2e_pipelined(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws, stream,
     return _job_value(world, T, replays * per, ms), replays * per, per
 
 
-def _graph_ms(g, stream, replays):
+def _graph_ms(g, stream, replays=None, warm_s=0.1, timed_s=0.25):
+    """Milliseconds per replay of graph g, every replay on `stream`: about warm_s seconds of
+    replays first, then at least `replays` (or about timed_s seconds of) replays timed with events
+    on the same stream. (CUDAGraph.replay() launches on the current stream; a warm-up replayed on
+    the default stream is not waited for by a side stream's start event, and its tail would be
+    timed as well.)"""
     import torch
-    for _ in range(2):
-        g.replay()
-    stream.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         e0.record(stream)
-        for _ in range(replays):
+        g.replay()
+        e1.record(stream)
+        stream.synchronize()
+        one = max(e0.elapsed_time(e1) / 1e3, 1e-6)       # seconds per replay, first estimate
+        for _ in range(max(2, math.ceil(warm_s / one))):
+            g.replay()
+        stream.synchronize()
+        n_rep = max(replays or 3, math.ceil(timed_s / one))
+        e0.record(stream)
+        for _ in range(n_rep):
             g.replay()
         e1.record(stream)
     stream.synchronize()
-    return e0.elapsed_time(e1) / replays
+    return e0.elapsed_time(e1) / n_rep
+
+
+def _eager_ms(call, stream, warm_s=0.1, timed_s=0.25):
+    """Milliseconds per call(i) issued eagerly on `stream` (calls long enough that the host keeps
+    ahead), in steady state as _graph_ms: about warm_s seconds of calls first, then about timed_s
+    seconds timed."""
+    import torch
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for i in range(4):
+            call(i)
+        e1.record(stream)
+    stream.synchronize()
+    one = max(e0.elapsed_time(e1) / 4e3, 1e-6)
+    with torch.cuda.stream(stream):
+        for i in range(math.ceil(warm_s / one)):
+            call(i)
+        n_call = max(8, math.ceil(timed_s / one))
+        e0.record(stream)
+        for i in range(n_call):
+            call(i)
+        e1.record(stream)
+    stream.synchronize()
+    return e0.elapsed_time(e1) / n_call
 
 
 def prefill_point(dev, lay, copies, stream, tc_peak, peak_src, variant=None):
@@ -685,17 +722,14 @@ def prefill_point(dev, lay, copies, stream, tc_peak, peak_src, variant=None):
         for i in range(5):
             P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,
                            workspace_tensor=ws, stream=stream)
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        reps = 50
-        e0.record(stream)
-        for i in range(reps):
-            P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,
-                           workspace_tensor=ws, stream=stream)
-        e1.record(stream)
     stream.synchronize()
+
+    def call(i):
+        P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,
+                       workspace_tensor=ws, stream=stream)
+
+    ms = _eager_ms(call, stream)
     assert P.pifa_device_status(stream) == P.PIFA_OK
-    ms = e0.elapsed_time(e1) / reps
     tf = pifa_flops(T, m, n, r) / (ms / 1e3) / 1e12
     return {"workload": f"{SHAPE.name} prefill T={T}", "variant": P.pifa_variant_name(variant),
             "tokens_per_s": T / (ms / 1e3), "ms_per_step": ms,
