@@ -9,9 +9,9 @@ Printed as one JSON line on rank 0:
              from a CUDA graph; the weights rotate over enough copies that the working set is
              larger than L2 (every step streams its weights from HBM);
   e2e        the same metric through the public API with host buffers: per step, X copied from
-             pinned host memory, pifa_forward, Y copied back to pinned host memory, with the copies
-             of neighbouring steps overlapping the forwards (two copy streams, four buffers in
-             flight); the serial loop (no overlap) is reported beside it;
+             pinned host memory, pifa_forward, Y copied back to pinned host memory, in groups of
+             four steps whose copies overlap the neighbouring groups' forwards (two copy streams,
+             two groups in flight); the serial loop (no overlap) is reported beside it;
   roofline   the decode call's achieved HBM GB/s against MEASURED_PEAKS.json (algorithmic bytes:
              2 r(m + n - r) weight bytes + 2 T (n + m) activation bytes + 4 m index bytes);
   cpu_baseline  the fp64 oracle (numpy) on the host cores over a bounded sample of the workload;
@@ -352,10 +352,12 @@ def run_ours(args, rank, world, local_rank):
                    "timing": "CUDA graph replay, CUDA events on the launching stream"},
         "e2e": {"value": e2e_pipe, "unit": "tokens/s", "h2d_bytes_per_step": T * n * 2,
                 "d2h_bytes_per_step": T * m * 2,
-                "mode": f"serving loop: per step X uploaded from pinned host memory, pifa_forward, Y downloaded to "
-                        f"pinned host memory; 4 device buffers in flight, uploads and downloads on two copy streams "
-                        f"overlapping the forwards of neighbouring steps; {e2e_pipe_per} steps per CUDA graph, "
-                        f"{e2e_pipe_steps} steps timed; the last step's Y checked against a separate forward",
+                "mode": f"serving loop: per step X uploaded from pinned host memory (one copy per step), "
+                        f"pifa_forward, Y downloaded to pinned host memory (one copy per step); steps in groups of "
+                        f"4 with two groups in flight, uploads and downloads on two copy streams overlapping the "
+                        f"neighbouring groups' forwards, the compute stream waiting on the copies once per group; "
+                        f"{e2e_pipe_per} steps per CUDA graph, {e2e_pipe_steps} steps timed; the last step's Y "
+                        f"checked against a separate forward",
                 "serial_value": e2e_eager,
                 "serial_mode": "the same steps one after another on one stream, issued call by call (no overlap)",
                 "serial_graph_value": e2e_graph,
@@ -558,50 +560,59 @@ def grouped_point(dev, stream, hbm_peak, tc_peak, peak_src):
 
 
 def e2e_pipelined(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws, stream, world, steps):
-    """End to end through pifa_forward as a serving loop issues it: every step uploads its X from
-    pinned host memory, runs the forward and downloads its Y to pinned host memory, with NB device
-    buffers in flight so that the copies of neighbouring steps overlap the forward (uploads on one
-    copy stream, downloads on another, the forwards in order on the compute stream; events order
-    each buffer's reuse; one copy stream per buffer measured no faster). Captured as one
-    multi-stream CUDA graph of `per` steps and replayed; a replay starts after the previous one has
-    drained, so each replay pays one pipeline fill. Returns (tokens/s over all ranks, steps timed,
-    per)."""
+    """End to end through pifa_forward as a serving loop issues it: every step uploads its own X
+    from pinned host memory, runs its forward and downloads its own Y to pinned host memory. Steps
+    go in groups of K: a group's K uploads (one copy per step) on an upload stream, its K forwards
+    back to back on the compute stream, its K downloads (one copy per step) on a download stream,
+    with two groups' buffers in flight so that one group's copies overlap the neighbouring groups'
+    forwards. The compute stream waits on the copies once per group, so that the forwards of a
+    group follow one another with programmatic dependent launch, as in the device-only line (a
+    wait before every forward measured 15.5 µs per step at T = 8 against 8.8 µs of kernel time).
+    Captured as one multi-stream CUDA graph of `per` steps and replayed; a replay starts after the
+    previous one has drained, so each replay pays one pipeline fill. Returns (tokens/s over all
+    ranks, steps timed, per)."""
     import torch
-    NB = 4
+    K, NG = 4, 2                                   # steps per group, groups in flight
     nh = len(Xhs)
     copies = len(Wps)
-    Xd = [torch.empty((T, n), dtype=torch.bfloat16, device=dev) for _ in range(NB)]
-    Yd = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(NB)]
+    Xd = [torch.empty((T, n), dtype=torch.bfloat16, device=dev) for _ in range(K * NG)]
+    Yd = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(K * NG)]
     Yhs = [torch.empty((T, m), dtype=torch.bfloat16).pin_memory() for _ in range(nh)]
-    s_in = torch.cuda.Stream(device=dev)       # uploads, in step order
-    s_out = torch.cuda.Stream(device=dev)      # downloads, in step order
-    per = copies * max(1, 64 // copies)
+    s_in = torch.cuda.Stream(device=dev)
+    s_out = torch.cuda.Stream(device=dev)
+    per = K * math.ceil(copies * max(1, 64 // copies) / K)
 
     def pipeline(k_steps):
-        ev_in = [torch.cuda.Event() for _ in range(NB)]
-        ev_fwd = [torch.cuda.Event() for _ in range(NB)]
-        ev_out = [torch.cuda.Event() for _ in range(NB)]
+        ev_in = [torch.cuda.Event() for _ in range(NG)]
+        ev_fwd = [torch.cuda.Event() for _ in range(NG)]
+        ev_out = [torch.cuda.Event() for _ in range(NG)]
         fork = torch.cuda.Event()
         fork.record(stream)
         s_in.wait_event(fork)
         s_out.wait_event(fork)
-        for i in range(k_steps):
-            b = i % NB
-            if i >= NB:
-                s_in.wait_event(ev_fwd[b])        # forward i - NB has read Xd[b]
+        for j in range(k_steps // K):
+            gb = j % NG                            # the group's buffer set
+            if j >= NG:
+                s_in.wait_event(ev_fwd[gb])        # group j - NG's forwards have read Xd
             with torch.cuda.stream(s_in):
-                Xd[b].copy_(Xhs[i % nh], non_blocking=True)
-            ev_in[b].record(s_in)
-            stream.wait_event(ev_in[b])
-            if i >= NB:
-                stream.wait_event(ev_out[b])      # download i - NB has read Yd[b]
-            P.pifa_forward(Xd[b], Wps[i % copies], Cs[i % copies], piv, nonp, Y=Yd[b], variant=variant,
-                           workspace_tensor=ws, stream=stream)
-            ev_fwd[b].record(stream)
-            s_out.wait_event(ev_fwd[b])
+                for t in range(K):
+                    i = j * K + t
+                    Xd[gb * K + t].copy_(Xhs[i % nh], non_blocking=True)
+            ev_in[gb].record(s_in)
+            stream.wait_event(ev_in[gb])
+            if j >= NG:
+                stream.wait_event(ev_out[gb])      # group j - NG's downloads have read Yd
+            for t in range(K):
+                i = j * K + t
+                P.pifa_forward(Xd[gb * K + t], Wps[i % copies], Cs[i % copies], piv, nonp, Y=Yd[gb * K + t],
+                               variant=variant, workspace_tensor=ws, stream=stream)
+            ev_fwd[gb].record(stream)
+            s_out.wait_event(ev_fwd[gb])
             with torch.cuda.stream(s_out):
-                Yhs[i % nh].copy_(Yd[b], non_blocking=True)
-            ev_out[b].record(s_out)
+                for t in range(K):
+                    i = j * K + t
+                    Yhs[i % nh].copy_(Yd[gb * K + t], non_blocking=True)
+            ev_out[gb].record(s_out)
         join_in, join_out = torch.cuda.Event(), torch.cuda.Event()
         join_in.record(s_in)
         join_out.record(s_out)
@@ -609,7 +620,7 @@ def e2e_pipelined(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws, stream,
         stream.wait_event(join_out)
 
     with torch.cuda.stream(stream):
-        pipeline(2 * NB)                          # eager warm-up of the same streams and buffers
+        pipeline(2 * K * NG)                       # eager warm-up of the same streams and buffers
     stream.synchronize()
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=stream):
