@@ -21,6 +21,8 @@ Functions and the passages they follow:
   compress             Algorithm 1 (Sec. 3.2, Eqs. 1-2): I, I^c, W_p, W_np and C from
                        W_np = C W_p solved by least squares (Householder QR + back substitution).
   forward              Algorithm 2 (Sec. 3.2): Y_p, Y_np and the two index assignments.
+  backward             the gradients of Algorithm 2 w.r.t. X, W_p and C (fine-tuning after
+                       pruning, Sec. 5.1; differentiability, Sec. 6): its steps in reverse.
   storage_count        Sec. 3.3 (memory cost): r(m+n) - r^2 (+ r indices).
   flop_count           Sec. 3.3 (computational cost): 2 b r (m + n - r).
   dense_forward, lowrank_forward  the two comparison layers of Sec. 3.3 (Y = W X, Y = U V^T X).
@@ -223,6 +225,34 @@ def forward(X, Wp, C, pivots, nonpivots) -> np.ndarray:
     Y[:, pivots] = Yp
     Y[:, nonpivots] = Ynp
     return Y
+
+
+def backward(X, Wp, C, pivots, nonpivots, dY):
+    """Gradients of Algorithm 2 with respect to its three real inputs, in float64.
+
+    The paper fine-tunes pruned layers, PIFA layers accelerating the backward pass as well as the
+    forward (Sec. 5.1, fine-tuning after pruning), and calls PIFA fully differentiable (Sec. 6);
+    the trainable inputs are X, W_p and C, the index sets stay fixed. Given dY = dL/dY (T x m), this takes the
+    chain rule back through Algorithm 2's steps in reverse order:
+      steps 5, 4: dY_np = dY[:, I^c], dY_p = dY[:, I]          (the two index assignments)
+      step 3:     Y_np = Y_p C^T  ->  dC = dY_np^T Y_p,  dY_p += dY_np C
+      step 2:     Y_p = X W_p^T   ->  dW_p = dY_p^T X,   dX = dY_p W_p
+    Y_p is recomputed from X and W_p (step 2). Returns (dX (T x n), dW_p (r x n), dC ((m-r) x r)).
+    """
+    X = np.asarray(X, dtype=np.float64)
+    Wp = np.asarray(Wp, dtype=np.float64)
+    C = np.asarray(C, dtype=np.float64)
+    dY = np.asarray(dY, dtype=np.float64)
+    pivots = np.asarray(pivots, dtype=np.int64)
+    nonpivots = np.asarray(nonpivots, dtype=np.int64)
+    Yp = X @ Wp.T                      # step 2, recomputed
+    dYnp = dY[:, nonpivots]            # step 5 reversed
+    dYp = dY[:, pivots].copy()         # step 4 reversed
+    dC = dYnp.T @ Yp                   # step 3 reversed
+    dYp += dYnp @ C
+    dWp = dYp.T @ X                    # step 2 reversed
+    dX = dYp @ Wp
+    return dX, dWp, dC
 
 
 def dense_forward(X, W) -> np.ndarray:

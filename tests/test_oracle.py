@@ -10,7 +10,10 @@ the oracle itself.
 * the closed form C = U_np U_p^{-1} when W' = U V^T;
 * the cost counts of Sec. 3.3 against an instrumented naive loop;
 * LAPACK's pivoted QR picks the same rows as the plain greedy loop;
-* planted mistakes in copies of oracle functions make at least one pin fail.
+* planted mistakes in copies of oracle functions make at least one pin fail;
+* the backward pass: exact central differences (Y is linear in each input), Euler's identity for
+  degree-one homogeneous maps, the chain rule through the dense weight, the r = m linear-layer
+  case, and planted mistakes.
 """
 import itertools
 import math
@@ -448,3 +451,163 @@ def test_planted_pivot_mistakes_are_caught(mutant):
 
 def test_planted_coefficient_mistake_is_caught():
     assert not pin_lossless(_compress_unsorted)
+
+
+# ---------------------------------------------------------------------------------------------
+# the backward pass (gradients of Algorithm 2 w.r.t. X, W_p and C): pins that do not restate the
+# oracle's reverse-order chain rule
+# ---------------------------------------------------------------------------------------------
+BWD_SHAPES = ((11, 7, 4, 5), (9, 12, 6, 3), (16, 16, 5, 8), (7, 5, 7, 4))   # (m, n, r, T); last: r = m
+
+
+def _bwd_case(m, n, r, T, seed):
+    """A random layer (random ascending I, real W_p and C, not compressed: the gradients hold for
+    any operands), X and dY."""
+    rng = np.random.default_rng(500 + seed)
+    pivots = np.sort(rng.choice(m, size=r, replace=False))
+    nonpivots = oracle.complement(pivots, m)
+    Wp = rng.standard_normal((r, n))
+    C = rng.standard_normal((m - r, r))
+    X = rng.standard_normal((T, n))
+    dY = rng.standard_normal((T, m))
+    return X, Wp, C, pivots, nonpivots, dY, rng
+
+
+def _safe(pin):
+    def run(*a, **k):
+        try:
+            return bool(pin(*a, **k))
+        except (ValueError, IndexError):
+            return False
+    return run
+
+
+@_safe
+def pin_backward_central_differences(backward=oracle.backward):
+    """L = <dY, Y> is linear in each of X, W_p and C (the others fixed), so a central difference
+    along any direction E equals <E, dL/d(that input)> up to rounding, whatever the step."""
+    for seed, shape in enumerate(BWD_SHAPES):
+        X, Wp, C, I, Ic, dY, rng = _bwd_case(*shape, seed)
+        dX, dWp, dC = backward(X, Wp, C, I, Ic, dY)
+        L = lambda X_, Wp_, C_: float(np.sum(dY * oracle.forward(X_, Wp_, C_, I, Ic)))
+        for which, grad, base in ((0, dX, X), (1, dWp, Wp), (2, dC, C)):
+            if grad.shape != base.shape:
+                return False
+            if base.size == 0:
+                continue
+            E = rng.standard_normal(base.shape)
+            args_p = [X, Wp, C]
+            args_m = [X, Wp, C]
+            args_p[which] = base + E
+            args_m[which] = base - E
+            fd = (L(*args_p) - L(*args_m)) / 2
+            scale = np.linalg.norm(E) * np.linalg.norm(grad) + abs(L(X, Wp, C)) + 1.0
+            if abs(fd - float(np.sum(E * grad))) > 1e-11 * scale:
+                return False
+    return True
+
+
+@_safe
+def pin_backward_euler(backward=oracle.backward):
+    """Y is homogeneous of degree one in X and in W_p, and Y_np in C (Euler): <dX, X> = <dY, Y>,
+    <dW_p, W_p> = <dY, Y>, <dC, C> = <dY[:, I^c], Y[:, I^c]>."""
+    for seed, shape in enumerate(BWD_SHAPES):
+        X, Wp, C, I, Ic, dY, _ = _bwd_case(*shape, seed + 10)
+        dX, dWp, dC = backward(X, Wp, C, I, Ic, dY)
+        Y = oracle.forward(X, Wp, C, I, Ic)
+        full = float(np.sum(dY * Y))
+        tail = float(np.sum(dY[:, Ic] * Y[:, Ic]))
+        tol = 1e-11 * (np.abs(dY).sum() * np.abs(Y).max() + 1.0)
+        if abs(float(np.sum(dX * X)) - full) > tol or abs(float(np.sum(dWp * Wp)) - full) > tol:
+            return False
+        if abs(float(np.sum(dC * C)) - tail) > tol:
+            return False
+    return True
+
+
+@_safe
+def pin_backward_dense_route(backward=oracle.backward):
+    """The same gradients through the dense weight: W'[I] = W_p, W'[I^c] = C W_p (Eqs. 1-2) and
+    Y = X W'^T give dX = dY W' and dW' = dY^T X; W_p reaches W' directly and through C, so
+    dW_p = dW'[I] + C^T dW'[I^c], and dC = dW'[I^c] W_p^T."""
+    for seed, shape in enumerate(BWD_SHAPES):
+        X, Wp, C, I, Ic, dY, _ = _bwd_case(*shape, seed + 20)
+        m = I.size + Ic.size
+        W = np.empty((m, Wp.shape[1]))
+        W[I] = Wp
+        W[Ic] = C @ Wp
+        dW = dY.T @ X
+        ref = (dY @ W, dW[I] + C.T @ dW[Ic], dW[Ic] @ Wp.T)
+        got = backward(X, Wp, C, I, Ic, dY)
+        for g, r_ in zip(got, ref):
+            if g.shape != r_.shape or np.linalg.norm(g - r_) > 1e-12 * (np.linalg.norm(r_) + 1.0):
+                return False
+    return True
+
+
+def test_backward_central_differences():
+    assert pin_backward_central_differences()
+
+
+def test_backward_euler_identities():
+    assert pin_backward_euler()
+
+
+def test_backward_dense_route():
+    assert pin_backward_dense_route()
+
+
+def test_backward_r_equals_m_is_the_linear_layer_gradient():
+    """r = m (C empty): a row-permuted dense layer, whose gradients are the textbook ones."""
+    X, Wp, C, I, Ic, dY, _ = _bwd_case(6, 5, 6, 4, 99)
+    dX, dWp, dC = oracle.backward(X, Wp, C, I, Ic, dY)
+    assert dC.shape == (0, 6)
+    np.testing.assert_allclose(dX, dY[:, I] @ Wp, rtol=0, atol=1e-13)
+    np.testing.assert_allclose(dWp, dY[:, I].T @ X, rtol=0, atol=1e-13)
+
+
+def test_backward_on_a_compressed_layer_matches_the_dense_input_gradient():
+    """On a layer from Algorithm 1, dX equals the dense layer's input gradient dY W' (lossless)."""
+    U, V, rng = random_layer(40, 30, 12, 3)
+    layer = oracle.compress(U, V, 12)
+    X = rng.standard_normal((6, 30))
+    dY = rng.standard_normal((6, 40))
+    dX, _, _ = oracle.backward(X, layer.Wp, layer.C, layer.pivots, layer.nonpivots, dY)
+    ref = dY @ oracle.form_weight(U, V)
+    assert np.linalg.norm(dX - ref) <= 1e-10 * np.linalg.norm(ref)
+
+
+# planted mistakes in copies of the backward
+def _bwd_parts(X, Wp, C, I, Ic, dY):
+    X, Wp, C, dY = (np.asarray(a, np.float64) for a in (X, Wp, C, dY))
+    return X, Wp, C, dY, X @ Wp.T, dY[:, Ic], dY[:, I].copy()
+
+
+def _backward_dropped_c_path(X, Wp, C, I, Ic, dY):
+    X, Wp, C, dY, Yp, dYnp, dYp = _bwd_parts(X, Wp, C, I, Ic, dY)
+    return dYp @ Wp, dYp.T @ X, dYnp.T @ Yp                        # dY_np C never added
+
+
+def _backward_reversed_c(X, Wp, C, I, Ic, dY):
+    X, Wp, C, dY, Yp, dYnp, dYp = _bwd_parts(X, Wp, C, I, Ic, dY)
+    dYp = dYp + dYnp[:, ::-1] @ C                                  # rows of C paired with the wrong outputs
+    return dYp @ Wp, dYp.T @ X, dYnp.T @ Yp
+
+
+def _backward_stale_wp(X, Wp, C, I, Ic, dY):
+    X, Wp, C, dY, Yp, dYnp, dYp = _bwd_parts(X, Wp, C, I, Ic, dY)
+    full = dYp + dYnp @ C
+    return full @ Wp, dYp.T @ X, dYnp.T @ Yp                       # dW_p from the pivot outputs only
+
+
+def _backward_tokens_misaligned(X, Wp, C, I, Ic, dY):
+    X, Wp, C, dY, Yp, dYnp, dYp = _bwd_parts(X, Wp, C, I, Ic, dY)
+    full = dYp + dYnp @ C
+    return full @ Wp, full.T @ X, dYnp.T @ Yp[::-1]                 # dC pairs token t with token T-1-t
+
+
+@pytest.mark.parametrize("mutant", [_backward_dropped_c_path, _backward_reversed_c, _backward_stale_wp,
+                                    _backward_tokens_misaligned])
+def test_planted_backward_mistakes_are_caught(mutant):
+    assert not (pin_backward_central_differences(mutant) and pin_backward_euler(mutant)
+                and pin_backward_dense_route(mutant))
