@@ -86,8 +86,9 @@ typedef struct {
  *   workspace    DEVICE scratch of at least pifa_workspace_size(T, m, n, r, c_dtype, variant) bytes,
  *                256-byte aligned; it needs no initialisation. Its first 256 bytes are reserved
  *                for library state (no kernel of this version reads or writes them); the rest
- *                holds Y_p between the two contractions. A workspace must not be used by another
- *                call that may run concurrently.
+ *                holds Y_p between the two contractions. It must not overlap Y or an input
+ *                (PIFA_ERR_INVALID_ARG; only the first pifa_workspace_size() bytes are checked),
+ *                nor be used by another call that may run concurrently.
  *   cuda_stream  a cudaStream_t (NULL = legacy default stream).
  *
  *   Every matrix buffer spans rows x pitch elements: kernels may read a row's padding up to the

@@ -235,6 +235,13 @@ int forward_impl(int64_t groups, const void* X, int64_t T, int64_t n, int64_t ld
     return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or smaller than pifa_workspace_size()");
   if (reinterpret_cast<uintptr_t>(workspace) & 255u)
     return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  {
+    // the kernels write y_p into the workspace: it must not share a byte with Y or an input
+    const Span w = {reinterpret_cast<uintptr_t>(workspace), reinterpret_cast<uintptr_t>(workspace) + (uintptr_t)need};
+    if (overlaps(w, span_of(Y, T, G * m, ldy, 2)) || overlaps(w, span_of(X, T, n, ldx, 2)) ||
+        overlaps(w, span_of(Wp, G * r, n, ldwp, 2)) || (has_np && overlaps(w, span_of(C, G * (m - r), r, ldc, 2))))
+      return pifa_fail(PIFA_ERR_INVALID_ARG, "workspace overlaps Y or an input");
+  }
   cudaError_t cerr = cudaSuccess;
   int* status = pifa_status_word(&cerr);
   if (!status) return pifa_fail_cuda("device status word", cerr);

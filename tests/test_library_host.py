@@ -143,6 +143,14 @@ def test_forward_argument_errors(lib):
     assert _fwd_raw(lib, wsb=256) == E.PIFA_ERR_WORKSPACE             # only the reserved head
 
 
+def test_forward_rejects_a_workspace_overlapping_y_or_an_input(lib):
+    """The kernels write y_p into the workspace, so it may share no byte with Y or an input; the
+    check runs on the host before any device access (every call here fails validation)."""
+    for ws in (0x60000, 0x5ff00, 0x10000, 0x20000, 0x30000):        # Y, ends inside Y, X, W_p, C
+        assert _fwd_raw(lib, ws=ws) == P.PIFA_ERR_INVALID_ARG, hex(ws)
+        assert "workspace overlaps" in _last(lib)
+
+
 def _last(lib):
     return lib.pifa_last_error().decode()
 
