@@ -96,11 +96,6 @@ __device__ __forceinline__ void bulk_copy_g2s(uint32_t dst_smem, const void* src
                : "memory");
 }
 
-// Bulk prefetch of [ptr, ptr + bytes) into L2 (16-byte aligned address and size).
-__device__ __forceinline__ void prefetch_l2_bulk(const void* ptr, uint32_t bytes) {
-  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
-}
-
 // ---- thread-block clusters ------------------------------------------------------------------
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
@@ -127,23 +122,11 @@ __device__ __forceinline__ uint32_t nclusters_x() {
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
-// Cluster barrier without memory ordering: for "every peer is done reading my shared memory"
-// (a load that has delivered its value is complete), without waiting for this CTA's own global
-// stores to be performed as a release would.
-__device__ __forceinline__ void cluster_sync_relaxed() {
-  asm volatile("barrier.cluster.arrive.relaxed;\n\tbarrier.cluster.wait;" ::: "memory");
-}
 // shared::cluster address of the same shared-memory offset in CTA `rank` of this cluster.
 __device__ __forceinline__ uint32_t mapa_shared(uint32_t local_saddr, uint32_t rank) {
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local_saddr), "r"(rank));
   return r;
-}
-// 32-bit load from the shared memory of a CTA of this cluster (shared::cluster address).
-__device__ __forceinline__ float ld_dsmem_f32(uint32_t cluster_saddr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(cluster_saddr) : "memory");
-  return v;
 }
 // 4-byte asynchronous copy global -> shared (no register dependency); completes by cp_async_wait_all.
 __device__ __forceinline__ void cp_async4(uint32_t dst_smem, const void* src) {
@@ -340,19 +323,6 @@ __device__ __forceinline__ void mma_m16n8k16_f16(float (&d)[4], uint32_t a0, uin
       "{%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
-// Streaming 16-byte global load that does not allocate in L1.
-__device__ __forceinline__ uint4 ld_stream_16(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
-}
-
-__device__ __forceinline__ uint32_t pack_bf16(__nv_bfloat16 lo, __nv_bfloat16 hi) {
-  return (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
 }
 
 }  // namespace pifa
