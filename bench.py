@@ -38,6 +38,11 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+# BLAS threads of the oracle timings, fixed before numpy loads its BLAS: the host cores this
+# process may run on, unless the caller chose (OpenBLAS reads its own variable first)
+os.environ.setdefault("OPENBLAS_NUM_THREADS", str(len(os.sched_getaffinity(0))))
+BLAS_THREADS = int(os.environ["OPENBLAS_NUM_THREADS"])
+
 import numpy as np  # noqa: E402
 
 from paper_2501_19090_gb300 import inputs  # noqa: E402
@@ -376,8 +381,8 @@ def run_ours(args, rank, world, local_rank):
         "gpu_launches": steps * (2 if m > r else 1),
         "clocks": clk.summary(),
     }
-    if rank == 0 and not args.no_extras and shape is SHAPE:
-        # the HBM-bound points first: the prefill-sized GEMMs after them hold the power cap
+    if rank == 0 and world == 1 and not args.no_extras and shape is SHAPE:
+        # one GPU only (at N > 1 every GPU would wait for rank 0's extras); the HBM-bound points first: the prefill-sized GEMMs after them hold the power cap
         with ClockSampler(local_rank) as clk_x:
             out["decode_sweep"] = decode_sweep(dev, stream, hbm_peak, peak_src)
             out["grouped_mlp7b_gate_up"] = grouped_point(dev, stream, hbm_peak, tc_peak, peak_src)
@@ -749,8 +754,10 @@ def prefill_point(dev, lay, copies, stream, tc_peak, peak_src, variant=None):
                          "algorithmic_flops_per_launch": pifa_flops(T, m, n, r)}}
 
 
-def cpu_baseline(lay, T, budget_s=10.0):
-    """The fp64 oracle forward (numpy) on the host cores over a bounded sample of the workload."""
+def cpu_baseline(lay, T, budget_s=10.0, single_s=5.0):
+    """The fp64 oracle forward (numpy) on the host cores over a bounded sample of the workload,
+    with BLAS_THREADS BLAS threads; the same forward on one thread, timed in a fresh interpreter
+    (numpy's thread count is fixed when it loads), is reported beside it."""
     import oracle
     rng = np.random.default_rng(9)
     X = inputs.make_activations(rng, T, SHAPE.n, "bf16")
@@ -763,9 +770,46 @@ def cpu_baseline(lay, T, budget_s=10.0):
         oracle.forward(X, Wp, C, piv, nonp)
         calls += 1
     dt = time.perf_counter() - t0
-    cores = len(os.sched_getaffinity(0))
-    return {"value": calls * T / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": f"{calls} oracle forwards of T={T} tokens on {SHAPE.name} (fp64 numpy, BLAS threads = cores), {dt:.1f} s"}
+    out = {"value": calls * T / dt, "unit": "tokens/s", "cores": BLAS_THREADS, "kind": "oracle",
+           "sample": f"{calls} oracle forwards of T={T} tokens on {SHAPE.name} (fp64 numpy, "
+                     f"{BLAS_THREADS} BLAS threads), {dt:.1f} s"}
+    try:
+        out["single_thread"] = _oracle_rate_one_thread(X, Wp, C, piv, nonp, T, single_s)
+    except Exception as e:  # reported, never fatal: the main figure stands on its own
+        out["single_thread"] = {"error": f"{type(e).__name__}: {e}"}
+    return out
+
+
+_ONE_THREAD_TIMER = """
+import json, sys, time
+import numpy as np
+sys.path.insert(0, sys.argv[1])
+import oracle
+d = np.load(sys.argv[2])
+args = (d["X"], d["Wp"], d["C"], d["piv"], d["nonp"])
+oracle.forward(*args)
+t0, calls = time.perf_counter(), 0
+while time.perf_counter() - t0 < float(sys.argv[3]):
+    oracle.forward(*args)
+    calls += 1
+print(json.dumps({"calls": calls, "seconds": time.perf_counter() - t0}))
+"""
+
+
+def _oracle_rate_one_thread(X, Wp, C, piv, nonp, T, budget_s):
+    """Tokens/s of the oracle forward with one BLAS thread, in a fresh interpreter."""
+    import tempfile
+    with tempfile.TemporaryDirectory() as d:
+        path = os.path.join(d, "case.npz")
+        np.savez(path, X=X, Wp=Wp, C=C, piv=piv, nonp=nonp)
+        env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+        r = subprocess.run([sys.executable, "-c", _ONE_THREAD_TIMER, ROOT, path, str(budget_s)], env=env,
+                           capture_output=True, text=True, timeout=budget_s + 120)
+    if r.returncode != 0:
+        raise RuntimeError(r.stderr.strip().splitlines()[-1] if r.stderr.strip() else f"exit {r.returncode}")
+    res = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": res["calls"] * T / res["seconds"], "unit": "tokens/s", "cores": 1,
+            "sample": f"{res['calls']} oracle forwards, {res['seconds']:.1f} s, one BLAS thread"}
 
 
 def _traffic(src, key):
@@ -824,7 +868,7 @@ def run_reference(args, rank):
         done += 1
     dt = time.perf_counter() - t0
     v = T * done / dt
-    cores = len(os.sched_getaffinity(0))
+    cores = BLAS_THREADS
     del P
     return {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": done, "requested_steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / done,
@@ -833,7 +877,7 @@ def run_reference(args, rank):
                                             "r": SHAPE.r, "tokens_per_step": T},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                              "sample": f"{done} of {args.steps} requested fp64 oracle forwards of T={T} "
-                                       f"(numpy, host cores; capped at ~60 s)"},
+                                       f"(numpy, {cores} BLAS threads; capped at ~60 s)"},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
