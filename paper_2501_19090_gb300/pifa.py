@@ -251,15 +251,62 @@ def c_dtype_of(C) -> int:
     raise TypeError(f"C must be bfloat16 or float16, got {C.dtype}")
 
 
+def _operands(G: int, X, Wp, C, pivot_idx, nonpivot_idx, Y, workspace_tensor=None, c_fp16_ok=True):
+    """Check what the C ABI cannot see -- tensor type, dtype, shape and device -- before any
+    pointer reaches the library (a host or mistyped buffer would otherwise be read as device
+    bf16). Types and shapes first, then that every tensor sits on X's CUDA device. Returns
+    (T, n, r, m) of one group. Raises ValueError."""
+    import torch
+
+    def fail(msg):
+        raise ValueError(f"pifa: {msg}")
+
+    def tensor(name, t):
+        if not isinstance(t, torch.Tensor):
+            fail(f"{name} must be a torch tensor")
+        return t
+
+    if tensor("X", X).dim() != 2 or X.dtype != torch.bfloat16:
+        fail(f"X must be a 2-D bfloat16 tensor (T x n) (it is {X.dtype} {tuple(X.shape)})")
+    T, n = X.shape
+    if tensor("Wp", Wp).dim() != 2 or Wp.dtype != torch.bfloat16 or Wp.shape[1] != n or Wp.shape[0] % G:
+        fail(f"Wp must be a bfloat16 ({G} r) x {n} tensor (it is {Wp.dtype} {tuple(Wp.shape)})")
+    r = Wp.shape[0] // G
+    for name, t in (("pivot_idx", pivot_idx), ("nonpivot_idx", nonpivot_idx)):
+        if t is not None and (tensor(name, t).dim() != 1 or t.dtype != torch.int32 or not t.is_contiguous()):
+            fail(f"{name} must be a contiguous 1-D int32 tensor (it is {t.dtype} {tuple(t.shape)})")
+    if pivot_idx is None or pivot_idx.numel() != G * r:
+        fail(f"pivot_idx must hold {G * r} indices")
+    nnp = nonpivot_idx.numel() if nonpivot_idx is not None else 0
+    if nnp % G:
+        fail("nonpivot_idx must hold the same number of indices for every group")
+    m = r + nnp // G
+    if m > r:
+        ok = (torch.bfloat16, torch.float16) if c_fp16_ok else (torch.bfloat16,)
+        if tensor("C", C).dim() != 2 or C.dtype not in ok or tuple(C.shape) != (G * (m - r), r):
+            fail(f"C must be a {'bfloat16 or float16' if c_fp16_ok else 'bfloat16'} tensor of shape "
+                 f"{(G * (m - r), r)} (it is {C.dtype} {tuple(C.shape)})")
+    if Y is not None and (tensor("Y", Y).dim() != 2 or Y.dtype != torch.bfloat16 or tuple(Y.shape) != (T, G * m)):
+        fail(f"Y must be a bfloat16 tensor of shape {(T, G * m)} (it is {Y.dtype} {tuple(Y.shape)})")
+    if workspace_tensor is not None:
+        tensor("workspace_tensor", workspace_tensor)
+    dev = X.device
+    if dev.type != "cuda":
+        fail(f"X must be a CUDA tensor (it is on {dev})")
+    for name, t in (("Wp", Wp), ("C", C if m > r else None), ("pivot_idx", pivot_idx),
+                    ("nonpivot_idx", nonpivot_idx), ("Y", Y), ("workspace_tensor", workspace_tensor)):
+        if t is not None and t.device != dev:
+            fail(f"{name} is on {t.device}, X on {dev}")
+    return T, n, r, m
+
+
 def pifa_forward(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, variant: int = PIFA_VARIANT_AUTO,
                  workspace_tensor=None, stream=None):
     """Y = PIFA(X) through pifa_forward_variant. X (T x n), Wp (r x n) bf16 CUDA tensors; C
     ((m-r) x r) bf16 or fp16; pivot_idx / nonpivot_idx int32 CUDA tensors. Allocates Y (T x m)
     if not given."""
     import torch
-    T, n = X.shape
-    r = Wp.shape[0]
-    m = r + (nonpivot_idx.numel() if nonpivot_idx is not None else 0)
+    T, n, r, m = _operands(1, X, Wp, C, pivot_idx, nonpivot_idx, Y, workspace_tensor)
     if Y is None:
         Y = torch.empty((T, m), dtype=torch.bfloat16, device=X.device)
     has_np = m > r
@@ -295,9 +342,9 @@ def pifa_forward_grouped(groups: int, X, Wp, C, pivot_idx, nonpivot_idx, Y=None,
     given."""
     import torch
     G = int(groups)
-    T, n = X.shape
-    r = Wp.shape[0] // G
-    m = r + nonpivot_idx.numel() // G
+    if G < 1:
+        raise ValueError("pifa: groups must be >= 1")
+    T, n, r, m = _operands(G, X, Wp, C, pivot_idx, nonpivot_idx, Y, workspace_tensor)
     if Y is None:
         Y = torch.empty((T, G * m), dtype=torch.bfloat16, device=X.device)
     cdt = c_dtype_of(C)
@@ -321,9 +368,7 @@ def pifa_forward_decode_noalloc(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, strea
     """Decode forward (T <= 16) without a workspace: the library's static 1 MiB device scratch
     is used instead (see include/pifa.h). Allocates Y here only if the caller passes none."""
     import torch
-    T, n = X.shape
-    r = Wp.shape[0]
-    m = r + (nonpivot_idx.numel() if nonpivot_idx is not None else 0)
+    T, n, r, m = _operands(1, X, Wp, C, pivot_idx, nonpivot_idx, Y, c_fp16_ok=False)
     if Y is None:
         Y = torch.empty((T, m), dtype=torch.bfloat16, device=X.device)
     has_np = m > r
