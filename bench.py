@@ -461,7 +461,7 @@ def decode_sweep(dev, stream, hbm_peak, peak_src):
             Yc = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(copies)]
             X = Xc[0]
             variant = P.pifa_select_variant(T, m, n, r, P.PIFA_DTYPE_BF16)
-            ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant), dev, "sweep")
+            ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant), dev, tag="sweep")
 
             def step(i):
                 j = i % copies
@@ -524,8 +524,8 @@ def grouped_point(dev, stream, hbm_peak, tc_peak, peak_src):
         X = torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16)
         Y = torch.empty((T, G * m), dtype=torch.bfloat16, device=dev)
         Ys = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(G)]
-        ws1 = P.workspace(P.pifa_workspace_size(T, m, n, r), dev, "grp1")
-        wsg = P.workspace(P.pifa_workspace_size_grouped(G, T, m, n, r), dev, "grpG")
+        ws1 = P.workspace(P.pifa_workspace_size(T, m, n, r), dev, tag="grp1")
+        wsg = P.workspace(P.pifa_workspace_size_grouped(G, T, m, n, r), dev, tag="grpG")
 
         def sep(i):
             j = i % copies
@@ -733,7 +733,7 @@ def prefill_point(dev, lay, copies, stream, tc_peak, peak_src, variant=None):
     Y = torch.empty((T, m), dtype=torch.bfloat16, device=dev)
     if variant is None:
         variant = P.pifa_select_variant(T, m, n, r, cdt)
-    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant, cdt), dev, "prefill")
+    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant, cdt), dev, tag="prefill")
     with torch.cuda.stream(stream):
         for i in range(5):
             P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,

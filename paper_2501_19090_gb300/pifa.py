@@ -221,13 +221,14 @@ def _stream_ptr(stream):
 _workspaces: dict = {}
 
 
-def workspace(nbytes: int, device, stream=None):
+def workspace(nbytes: int, device, stream=None, tag: str = ""):
     """A cached device scratch tensor of at least nbytes on `device` (grown, never shrunk).
 
-    The cache is keyed by device and stream, so calls on different streams never share scratch.
+    The cache is keyed by device, stream and `tag`, so calls on different streams never share
+    scratch, and a caller that keeps several calls' scratch apart on one stream tags them.
     """
     import torch
-    key = (str(device), 0 if stream is None else getattr(stream, "cuda_stream", stream))
+    key = (str(device), 0 if stream is None else getattr(stream, "cuda_stream", stream), str(tag))
     buf = _workspaces.get(key)
     if buf is None or buf.numel() < nbytes:
         buf = torch.empty(max(nbytes, 256) + 256, dtype=torch.uint8, device=device)
