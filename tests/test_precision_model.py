@@ -1,8 +1,8 @@
 """Why every variant carries Y_p into the second contraction as a hi + lo pair of C's type (the
 reading of Algorithm 2's step 3 taken for precision): on a layer from Algorithm 1, rounding Y_p
-once to bf16 already breaks the tolerance the GPU path is held to, while the pair keeps the error
-more than two orders of magnitude inside it. The emulation uses the oracle's steps on the same rounded
-operands the kernels get; only the rounding of Y_p differs between the two arms."""
+once to bf16 already breaks the tolerance the GPU path is held to, while the pair keeps the
+error more than two orders of magnitude inside it. The emulation uses the oracle's steps on the
+same rounded operands the kernels get; only the rounding of Y_p differs between the two arms."""
 import numpy as np
 
 import oracle
