@@ -116,3 +116,24 @@ def test_reading_token_rho_removes_the_b_conflict():
             row, chunk = unswizzle(addrs[lane])
             assert row == rho8(lane >> 2) < 8 and chunk == 4 * (st & 1) + (lane & 3)
     assert _worst_phase_conflict([b_address(lane, 0, 3, rho8)[1] for lane in range(32)]) == 2
+
+
+def row_pitch(kc):
+    """decode.cu row_pitch: a row's bytes, plus 64 when they are a multiple of 128."""
+    return kc * 2 + (64 if (kc * 2) % 128 == 0 else 0)
+
+
+def test_padded_rows_are_conflict_free():
+    """decode_rows' weight rows (lane (g, c) reads row 16 gq + g [+ 8] at step * 64 + 16 c) and
+    decode_stream's resident B rows (token t = g, same column offset) use row_pitch: rows g and
+    g + 1 start 64 bytes apart in the bank window, so each phase covers all 8 bank groups."""
+    for kc in range(32, 2048 + 1, 32):
+        pitch = row_pitch(kc)
+        assert pitch % 128 == 64 and pitch >= 2 * kc
+        for step in range(kc // 32):
+            for gq, half in itertools.product(range(4), range(2)):
+                addrs = [(16 * gq + 8 * half + (lane >> 2)) * pitch + step * 64 + 16 * (lane & 3) for lane in range(32)]
+                assert _worst_phase_conflict(addrs) == 1
+            for T in (1, 2):                      # resident B at T <= 2 (tokens clamped to T - 1)
+                addrs = [min(lane >> 2, T - 1) * pitch + step * 64 + 16 * (lane & 3) for lane in range(32)]
+                assert _worst_phase_conflict(addrs) == 1
