@@ -208,3 +208,58 @@ def test_compress_matches_oracle_lapack_attention_shape(lib):
     """4096 x 4096, r = 2048 (LLaMA-2-7B attention projection): pivots bit-exact with the oracle's
     LAPACK route (skipped unless -m slow)."""
     _compare_with_oracle(4096, 4096, 2048, 0, "lapack")
+
+
+def _header_prototypes():
+    """name -> (return category, [parameter categories]) for every pifa_* function in pifa.h."""
+    import re
+    src = open(os.path.join(ROOT, "include", "pifa.h")).read()
+    src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", " ", src)
+    src = re.sub(r"#[^\n]*", " ", src)
+    src = re.sub(r"\s+", " ", src)
+
+    def cat(decl):
+        decl = decl.strip()
+        if "*" in decl:
+            return "ptr"
+        words = set(re.findall(r"\w+", decl))
+        if "int64_t" in words:
+            return "i64"
+        if words & {"int", "int32_t"}:
+            return "i32"
+        if "double" in words:
+            return "f64"
+        raise AssertionError(f"unmapped C type: {decl!r}")
+
+    out = {}
+    for ret, name, params in re.findall(r"([\w\s\*]+?)\b(pifa_\w+)\s*\(([^;{()]*)\)\s*;", src):
+        params = params.strip()
+        plist = [] if params in ("", "void") else [cat(p) for p in params.split(",")]
+        out[name] = (cat(ret), plist)
+    return out
+
+
+def test_binding_argtypes_match_the_header(lib):
+    """Every declared function's ctypes prototype in the binding matches pifa.h in arity and in
+    each argument's width (pointer / int64_t / int): a mismatch would corrupt arguments silently."""
+    import ctypes
+    protos = _header_prototypes()
+    assert set(P.EXPORTS) <= set(protos), sorted(set(P.EXPORTS) - set(protos))
+
+    def cat(t):
+        if t is ctypes.c_int64 or t is ctypes.c_longlong or t is ctypes.c_long:
+            return "i64"
+        if t is ctypes.c_int or t is ctypes.c_int32:
+            return "i32"
+        if t is ctypes.c_double:
+            return "f64"
+        if t in (ctypes.c_void_p, ctypes.c_char_p) or (isinstance(t, type) and issubclass(t, ctypes._Pointer)):
+            return "ptr"
+        raise AssertionError(f"unmapped ctypes type {t}")
+
+    for name in P.EXPORTS:
+        fn = getattr(lib, name)
+        ret, params = protos[name]
+        assert [cat(t) for t in fn.argtypes] == params, name
+        assert cat(fn.restype) == ret, name
