@@ -1,24 +1,28 @@
 """PIFA layer forward throughput on GB300.
 
-Default workload (one step = one pifa_forward over one token batch): the LLaMA-2-7B-shaped
-attention projection m = n = 4096, r = 2048, decode batch T = 8 (bf16). The step runs the whole
-hot path (selector, Y_p = X W_p^T, Y_np = Y_p C^T, both scatters into Y).
+Headline workload (one step = one pifa_forward over one token batch): the LLaMA-2-70B-shaped MLP
+gate/up projection m = 28672, n = 8192, r = 4096 (the largest layer of the workloads, one layer on
+one GPU), decode batch T = 16, bf16. The step runs the whole hot path: the selector, Y_p = X W_p^T,
+Y_np = Y_p C^T and both scatters into Y.
 
 Printed as one JSON line on rank 0:
-  value      tokens/s, device-timed (CUDA events on the launching stream) over K steps replayed
-             from a CUDA graph; the weights rotate over enough copies that the working set is
-             larger than L2 (every step streams its weights from HBM);
-  e2e        the same metric through the public API with host buffers: per step, X copied from
-             pinned host memory, pifa_forward, Y copied back to pinned host memory, in groups of
-             four steps whose copies overlap the neighbouring groups' forwards (two copy streams,
-             two groups in flight); the serial loop (no overlap) is reported beside it;
-  roofline   the decode call's achieved HBM GB/s against MEASURED_PEAKS.json (algorithmic bytes:
-             2 r(m + n - r) weight bytes + 2 T (n + m) activation bytes + 4 m index bytes);
-  cpu_baseline  the fp64 oracle (numpy) on the host cores over a bounded sample of the workload;
-  comparators   dense X W^T and low-rank (X V) U^T on the same GPU via torch.matmul;
-  prefill    the same layer at T = 2048 (tcgen05 path) with its bf16 tensor roofline.
+  value      tokens/s, device-timed with CUDA events on the launching stream over exactly --steps
+             steps replayed from CUDA graphs; the timed region is repeated until the clock sampler
+             has seen it (value = the median repetition); the weights rotate over enough copies
+             that the working set exceeds L2, so every step streams its weights from HBM;
+  e2e        the same metric through the public API with host buffers: per step X copied from
+             pinned host memory, pifa_forward, Y copied back to pinned host memory (groups of four
+             steps whose copies overlap the neighbouring groups' forwards); the serial loop beside it;
+  roofline   achieved HBM GB/s of the call against MEASURED_PEAKS.json (algorithmic bytes
+             2 r(m + n - r) + 2 T (n + m) + 4 m per call);
+  comparators  the same shape as a dense layer (X W^T) and a two-factor low-rank layer
+             ((X V) U^T) through torch.matmul on the same GPU, timed the same way;
+  cpu_baseline the fp64 oracle (numpy) on the host cores over a bounded sample of the workload.
+Extras (one GPU only): every decode configuration beside its low-rank and dense layers, the 7B MLP
+as three layers back to back, the prefill configurations (7B attention T = 2048 / 8192, 70B q/o and
+gate/up T = 4096) and the rank-fraction sweep at T = 2048, each with its roofline and clock record.
 
---impl reference times the oracle instead (the reference arm: the paper has no code).
+--impl reference times the oracle instead (the reference arm: the paper publishes no code).
 Multi-GPU (torchrun): every rank runs an independent replica of the workload ("replicas only");
 the time is the max over ranks and value sums the ranks' tokens.
 """
@@ -48,17 +52,12 @@ import numpy as np  # noqa: E402
 from paper_2501_19090_gb300 import inputs  # noqa: E402
 
 METRIC = "PIFA layer tokens/s at 1 GB300 + % of HBM / bf16 tensor roofline vs low-rank"
-SHAPE = inputs.ATTN7B
-T_DECODE = 8
-T_PREFILL = 2048
+SHAPE = inputs.MLP70B_GATE       # the headline layer
+T_DECODE = 16
 
-# DRAM traffic per launch measured with ncu for a given kernel source (sha256 of the .cu file).
-# A mismatch (the kernel changed since the capture) reports traffic as null.
-NCU_TRAFFIC = {
-    # decode_rows phase 1 + phase 2 of one call, attn 4096x4096 r=2048 T=8:
-    # dram__bytes_read.sum 16.89 MB + 8.51 MB, dram__bytes_write.sum 0 (profiles/decode_attn7b_T8_ncu_full.md)
-    "decode": {"sha": "fc56ea4f2ef87b8d", "bytes": 16885248 + 8512256},
-}
+# DRAM traffic per call measured with ncu for a given kernel source (sha256 of decode.cu), keyed
+# by (layer, T). A source mismatch (the kernel changed since the capture) reports traffic as null.
+NCU_TRAFFIC = {}
 
 
 def _src_sha(name: str) -> str:
@@ -82,6 +81,14 @@ def decode_bytes(T, m, n, r):
 
 def pifa_flops(T, m, n, r):
     return 2 * T * r * (m + n - r)
+
+
+def lowrank_bytes(T, m, n, r):
+    return 2 * r * (m + n) + 2 * T * (n + m)
+
+
+def dense_bytes(T, m, n):
+    return 2 * m * n + 2 * T * (n + m)
 
 
 class ClockSampler:
@@ -169,38 +176,244 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------------------------
-def build_layer(shape, seed, c_dtype="bf16"):
-    """Host-side setup: the library's compression (Algorithm 1); W_p rounded to bf16 and C to the
-    chosen storage type (bf16 by default, or fp16)."""
-    from paper_2501_19090_gb300 import pifa as P
-    U, V, _ = inputs.make_factors(shape.m, shape.n, shape.r, seed)
-    piv, nonp, Wp, C, info = P.pifa_compress(U, V, shape.r)
-    Cq = inputs.round_fp16(C) if c_dtype == "fp16" else inputs.round_bf16(C)
-    return dict(U=U, V=V, piv=piv, nonp=nonp, Wp=inputs.round_bf16(Wp), C=Cq, info=info, c_dtype=c_dtype)
-
-
-# --shape: the decode measurement on another decode-config layer shape (profiling; the default line
-# is the 7B attention layer). Other shapes use seeded random operands (inputs.synthetic_layer): the
-# kernels' time does not depend on the values, and Algorithm 1 on a 28672 x 8192 layer takes minutes
-# on the host.
 SHAPES = {s.name: s for s in (inputs.ATTN7B, inputs.MLP7B_GATE, inputs.MLP7B_DOWN, inputs.ATTN70B,
                               inputs.MLP70B_GATE)}
 
 
-def synthetic_layer_dict(shape, c_dtype="bf16"):
-    piv, nonp, Wp, C = inputs.synthetic_layer(shape.m, shape.n, shape.r, 0)
-    Cq = inputs.round_fp16(C) if c_dtype == "fp16" else C
-    return dict(piv=piv.astype(np.int32), nonp=nonp.astype(np.int32), Wp=Wp, C=Cq, c_dtype=c_dtype)
-
-
-def _torch_c_dtype(lay):
+def timing_layer(shape, dev, seed, c_dtype="bf16", copies=1):
+    """Device operands of one layer shape for timing: a seeded random ascending pivot set and its
+    complement, W_p ~ N(0, 1/r) and C ~ N(0, 0.18^2) drawn on the GPU (bf16; C in c_dtype), in
+    `copies` independent copies. The kernels' time does not depend on the values (the parity tests
+    run the real compressed layers)."""
     import torch
-    return torch.float16 if lay["c_dtype"] == "fp16" else torch.bfloat16
+    m, n, r = shape.m, shape.n, shape.r
+    rng = np.random.default_rng(20_000 + seed)
+    perm = rng.permutation(m)
+    piv = torch.from_numpy(np.sort(perm[:r]).astype(np.int32)).to(dev)
+    nonp = torch.from_numpy(np.sort(perm[r:]).astype(np.int32)).to(dev)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1000 + seed)
+    cdt = torch.float16 if c_dtype == "fp16" else torch.bfloat16
+    Wps = [_padded((torch.randn((r, n), device=dev, generator=gen) / math.sqrt(r)).to(torch.bfloat16))
+           for _ in range(copies)]
+    Cs = [_padded((torch.randn((m - r, r), device=dev, generator=gen) * 0.18).to(cdt)) for _ in range(copies)]
+    return piv, nonp, Wps, Cs
 
 
-def _pifa_c_dtype(lay):
+def _padded(a):
+    """a (rows x cols) copied into a buffer whose row pitch is cols rounded up to 8 elements (the
+    library's 16-byte row rule); returns the rows x cols view."""
+    import torch
+    rows, cols = a.shape
+    ld = (cols + 7) // 8 * 8
+    if ld == cols:
+        return a
+    buf = torch.zeros((rows, ld), dtype=a.dtype, device=a.device)
+    buf[:, :cols] = a
+    return buf[:, :cols]
+
+
+def _copies_for(dev, weight_bytes, lo=4):
+    """Weight copies whose total exceeds 3x L2, so that a rotation streams every step from HBM."""
+    import torch
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    return max(lo, math.ceil(3 * l2 / weight_bytes))
+
+
+def _graph_of(fn, n, stream):
+    """A CUDA graph of fn(0) .. fn(n - 1) captured on `stream` (after 3 eager warm-up calls)."""
+    import torch
+    with torch.cuda.stream(stream):
+        for i in range(3):
+            fn(i)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(n):
+            fn(i)
+    return g
+
+
+def _steady_us(fn, per_graph, stream):
+    """Microseconds per fn call in steady state: a graph of per_graph calls, replayed on `stream`
+    for ~0.1 s untimed then >= 0.25 s timed (_graph_ms)."""
+    g = _graph_of(fn, per_graph, stream)
+    us = _graph_ms(g, stream) / per_graph * 1e3
+    del g
+    return us
+
+
+def _comparator_fns(dev, shape, T, gen, n_lr, n_dense):
+    """Two-factor low-rank (X V) U^T and dense X W^T layers of the shape (bf16, torch.matmul on the
+    same GPU), each over rotating weight copies: returns (lowrank fn, dense fn, X)."""
+    import torch
+    m, n, r = shape.m, shape.n, shape.r
+    X = torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16)
+    Us = [(torch.randn((m, r), device=dev, generator=gen) / math.sqrt(r)).to(torch.bfloat16) for _ in range(n_lr)]
+    Vs = [(torch.randn((n, r), device=dev, generator=gen) / math.sqrt(r)).to(torch.bfloat16) for _ in range(n_lr)]
+    Ws = [torch.randn((m, n), device=dev, generator=gen).to(torch.bfloat16) for _ in range(n_dense)]
+    lr = lambda i: (X @ Vs[i % n_lr]) @ Us[i % n_lr].t()
+    dense = lambda i: X @ Ws[i % n_dense].t()
+    return lr, dense, X
+
+
+def layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src, name=None, c_dtype="bf16"):
+    """One layer shape at T tokens: the selected PIFA variant, the two-factor low-rank layer and the
+    dense layer on the same GPU, each a CUDA graph replayed in steady state over rotating weight
+    copies (decode: every copy's bytes exceed 3x L2 in total; prefill: two copies), with the
+    roofline of the PIFA call (HBM for T <= 16, bf16 tensor otherwise) and the clocks seen."""
+    import torch
     from paper_2501_19090_gb300 import pifa as P
-    return P.PIFA_DTYPE_FP16 if lay["c_dtype"] == "fp16" else P.PIFA_DTYPE_BF16
+    m, n, r = shape.m, shape.n, shape.r
+    decode = T <= 16
+    copies = _copies_for(dev, 2 * r * (m + n - r)) if decode else 2
+    piv, nonp, Wps, Cs = timing_layer(shape, dev, 7, c_dtype, copies)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(17)
+    Xs = [torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
+    Ys = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(copies)]
+    cdt = P.PIFA_DTYPE_FP16 if c_dtype == "fp16" else P.PIFA_DTYPE_BF16
+    variant = P.pifa_select_variant(T, m, n, r, cdt)
+    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant, cdt), dev, tag="point")
+
+    def step(i):
+        j = i % copies
+        P.pifa_forward(Xs[j], Wps[j], Cs[j], piv, nonp, Y=Ys[j], variant=variant, workspace_tensor=ws, stream=stream)
+
+    per = copies * max(1, 64 // copies) if decode else 8
+    n_lr = _copies_for(dev, 2 * r * (m + n)) if decode else 2
+    n_dense = _copies_for(dev, 2 * m * n, lo=2) if decode else 2
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        us = _steady_us(step, per, stream)
+        st = P.pifa_device_status(stream)
+        assert st == P.PIFA_OK, P.pifa_status_string(st)
+        del Wps, Cs, Xs, Ys
+        torch.cuda.empty_cache()
+        lr, dense, _ = _comparator_fns(dev, shape, T, gen, n_lr, n_dense)
+        lr_us = _steady_us(lr, n_lr * max(1, 64 // n_lr) if decode else 8, stream)
+        dense_us = _steady_us(dense, n_dense * max(1, 64 // n_dense) if decode else 8, stream)
+    del lr, dense
+    torch.cuda.empty_cache()
+    out = {"workload": name or f"{shape.name} {'decode' if decode else 'prefill'} T={T}", "m": m, "n": n, "r": r,
+           "T": T, "variant": P.pifa_variant_name(variant), "c_dtype": c_dtype, "us_per_call": us,
+           "tokens_per_s": T / (us / 1e6), "lowrank_us": lr_us, "dense_us": dense_us,
+           "speedup_vs_lowrank": lr_us / us, "speedup_vs_dense": dense_us / us, "weight_copies": copies}
+    if decode:
+        gbs = decode_bytes(T, m, n, r) / us / 1e3
+        out["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
+                           "algorithmic_bytes_per_call": decode_bytes(T, m, n, r),
+                           "peak_source": f"{peak_src} hbm_gbs"}
+        out["lowrank_hbm_gbs"] = lowrank_bytes(T, m, n, r) / lr_us / 1e3
+        out["dense_hbm_gbs"] = dense_bytes(T, m, n) / dense_us / 1e3
+    else:
+        tf = pifa_flops(T, m, n, r) / us / 1e6
+        out["roofline"] = {"bound": "tensor", "achieved": tf, "peak": tc_peak, "unit": "TFLOP/s", "frac": tf / tc_peak,
+                           "algorithmic_flops_per_call": pifa_flops(T, m, n, r),
+                           "peak_source": f"{peak_src} bf16_tflops (burst)"}
+        out["lowrank_tflops"] = 2 * T * r * (m + n) / lr_us / 1e6
+        out["dense_tflops"] = 2 * T * m * n / dense_us / 1e6
+    out["clocks"] = clk.summary()
+    return out
+
+
+DECODE_POINTS = [(inputs.ATTN7B, (1, 8, 16)), (inputs.MLP7B_GATE, (1, 8, 16)), (inputs.MLP7B_DOWN, (1, 8, 16)),
+                 (inputs.ATTN70B, (1, 8, 16)), (inputs.MLP70B_GATE, (1, 8, 16))]
+PREFILL_POINTS = [(inputs.ATTN7B, 2048), (inputs.ATTN7B, 8192), (inputs.ATTN70B, 4096), (inputs.MLP70B_GATE, 4096)]
+
+
+def mlp7b_point(dev, stream, T, hbm_peak, tc_peak, peak_src):
+    """The 7B MLP as three layers back to back per token batch (gate(X), up(X) on X of width 4096,
+    down on an independent input of width 11008; no activation between them): three pifa_forward
+    calls, and gate + up as one pifa_forward_grouped call followed by down, beside three low-rank
+    and three dense layers; two weight copies of every layer (decode: enough to exceed L2)."""
+    import torch
+    from paper_2501_19090_gb300 import pifa as P
+    G_, D_ = inputs.MLP7B_GATE, inputs.MLP7B_DOWN
+    decode = T <= 16
+    copies = 4 if decode else 2
+    lay = {name: timing_layer(s, dev, seed, copies=copies) for name, s, seed in
+           (("gate", G_, 1), ("up", G_, 2), ("down", D_, 3))}
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(19)
+    Xg = torch.randn((T, G_.n), device=dev, generator=gen).to(torch.bfloat16)
+    Xd = torch.randn((T, D_.n), device=dev, generator=gen).to(torch.bfloat16)
+    Y = {k: torch.empty((T, (G_ if k != "down" else D_).m), dtype=torch.bfloat16, device=dev) for k in lay}
+    ws = P.workspace(max(P.pifa_workspace_size(T, s.m, s.n, s.r) for s in (G_, D_)), dev, tag="mlp")
+    m, r = G_.m, G_.r
+    piv_s = torch.cat([lay["gate"][0], lay["up"][0] + m])
+    nonp_s = torch.cat([lay["gate"][1], lay["up"][1] + m])
+    Wp_s = [torch.cat([lay["gate"][2][j], lay["up"][2][j]]) for j in range(copies)]
+    C_s = [torch.cat([lay["gate"][3][j], lay["up"][3][j]]) for j in range(copies)]
+    Yg = torch.empty((T, 2 * m), dtype=torch.bfloat16, device=dev)
+    wsg = P.workspace(P.pifa_workspace_size_grouped(2, T, m, G_.n, r), dev, tag="mlpg")
+
+    def three(i):
+        j = i % copies
+        for k, X in (("gate", Xg), ("up", Xg), ("down", Xd)):
+            piv, nonp, Wps, Cs = lay[k]
+            P.pifa_forward(X, Wps[j], Cs[j], piv, nonp, Y=Y[k], workspace_tensor=ws, stream=stream)
+
+    def grouped(i):
+        j = i % copies
+        P.pifa_forward_grouped(2, Xg, Wp_s[j], C_s[j], piv_s, nonp_s, Y=Yg, workspace_tensor=wsg, stream=stream)
+        piv, nonp, Wps, Cs = lay["down"]
+        P.pifa_forward(Xd, Wps[j], Cs[j], piv, nonp, Y=Y["down"], workspace_tensor=ws, stream=stream)
+
+    per = 16 if decode else 4
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        us = _steady_us(three, per, stream)
+        gus = _steady_us(grouped, per, stream)
+        assert P.pifa_device_status(stream) == P.PIFA_OK
+        del lay, Wp_s, C_s
+        torch.cuda.empty_cache()
+        cmp_ = {}
+        for kind in ("lowrank", "dense"):
+            fns = []
+            for s in (G_, G_, D_):
+                lr, dense, X = _comparator_fns(dev, s, T, gen, copies, 2)
+                fns.append(lr if kind == "lowrank" else dense)
+            cmp_[kind] = _steady_us(lambda i: [f(i) for f in fns], per, stream)
+            del fns
+            torch.cuda.empty_cache()
+    shapes = (G_, G_, D_)
+    out = {"workload": f"llama2_7b_mlp gate+up+down T={T}", "T": T, "us_per_step": us,
+           "tokens_per_s": T / (us / 1e6), "grouped_us_per_step": gus, "grouped_tokens_per_s": T / (gus / 1e6),
+           "lowrank_us": cmp_["lowrank"], "dense_us": cmp_["dense"],
+           "speedup_vs_lowrank": cmp_["lowrank"] / min(us, gus), "speedup_vs_dense": cmp_["dense"] / min(us, gus)}
+    if decode:
+        b = sum(decode_bytes(T, s.m, s.n, s.r) for s in shapes)
+        gbs = b / min(us, gus) / 1e3
+        out["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": hbm_peak, "unit": "GB/s", "frac": gbs / hbm_peak,
+                           "algorithmic_bytes_per_step": b, "peak_source": f"{peak_src} hbm_gbs"}
+    else:
+        f = sum(pifa_flops(T, s.m, s.n, s.r) for s in shapes)
+        tf = f / min(us, gus) / 1e6
+        out["roofline"] = {"bound": "tensor", "achieved": tf, "peak": tc_peak, "unit": "TFLOP/s", "frac": tf / tc_peak,
+                           "algorithmic_flops_per_step": f, "peak_source": f"{peak_src} bf16_tflops (burst)"}
+    out["clocks"] = clk.summary()
+    return out
+
+
+def extras(dev, stream, hbm_peak, tc_peak, peak_src):
+    """Every configuration of the workload list beside its low-rank and dense layers (one GPU)."""
+    import torch
+    out = {"decode_points": [], "mlp7b_three_layers": [], "prefill_points": [], "rank_sweep": []}
+    for shape, Ts in DECODE_POINTS:
+        for T in Ts:
+            out["decode_points"].append(layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src))
+    for T in (1, 2048):
+        out["mlp7b_three_layers"].append(mlp7b_point(dev, stream, T, hbm_peak, tc_peak, peak_src))
+    for shape, T in PREFILL_POINTS:
+        out["prefill_points"].append(layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src))
+    for s in inputs.rank_sweep_shapes():
+        out["rank_sweep"].append(layer_point(dev, stream, s, 2048, hbm_peak, tc_peak, peak_src))
+    torch.cuda.empty_cache()
+    return out
+
+
+def _pifa_c_dtype(c_dtype):
+    from paper_2501_19090_gb300 import pifa as P
+    return P.PIFA_DTYPE_FP16 if c_dtype == "fp16" else P.PIFA_DTYPE_BF16
 
 
 def run_ours(args, rank, world, local_rank):
@@ -214,22 +427,16 @@ def run_ours(args, rank, world, local_rank):
     shape = SHAPES[args.shape]
     m, n, r = shape.m, shape.n, shape.r
     T = args.tokens
-    lay = (build_layer(shape, seed=0, c_dtype=args.c_dtype) if shape is SHAPE
-           else synthetic_layer_dict(shape, args.c_dtype))
-    bf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev).to(torch.bfloat16)
-    piv = torch.from_numpy(lay["piv"]).to(dev)
-    nonp = torch.from_numpy(lay["nonp"]).to(dev)
-    Wp0 = bf(lay["Wp"])
-    C0 = torch.from_numpy(np.ascontiguousarray(lay["C"])).to(dev).to(_torch_c_dtype(lay))
-    cdt = _pifa_c_dtype(lay)
-    wbytes = (Wp0.numel() + C0.numel()) * 2
-    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    copies = max(4, math.ceil(3 * l2 / wbytes))
-    Wps = [Wp0.clone() for _ in range(copies)]
-    Cs = [C0.clone() for _ in range(copies)]
-    rng = np.random.default_rng(1 + rank)
-    Xs = [bf(inputs.make_activations(rng, T, n, "bf16")) for _ in range(copies)]
+    K = max(1, args.steps)
+    decode = T <= 16
+    wbytes = 2 * r * (m + n - r)
+    copies = _copies_for(dev, wbytes)
+    piv, nonp, Wps, Cs = timing_layer(shape, dev, 0, args.c_dtype, copies)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(1 + rank)
+    Xs = [torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
     Ys = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(copies)]
+    cdt = _pifa_c_dtype(args.c_dtype)
     variant = P.pifa_select_variant(T, m, n, r, cdt)
     ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant, cdt), dev)
     stream = torch.cuda.Stream(device=dev)
@@ -239,122 +446,85 @@ def run_ours(args, rank, world, local_rank):
         P.pifa_forward(Xs[j], Wps[j], Cs[j], piv, nonp, Y=Ys[j], variant=variant, workspace_tensor=ws,
                        stream=stream)
 
-    # warm-up (eager), then capture a graph of `per_graph` steps
+    # W untimed warm-up steps (eager), then graphs covering exactly K steps: `reps` replays of a
+    # graph of `per` steps plus one graph of the remainder
     with torch.cuda.stream(stream):
         for i in range(max(3, args.warmup)):
             step(i)
     stream.synchronize()
     assert P.pifa_device_status(stream) == P.PIFA_OK
-    per_graph = copies * max(1, 64 // copies)
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g, stream=stream):
-        for i in range(per_graph):
-            step(i)
-    replays = max(1, math.ceil(args.steps / per_graph))
-    steps = replays * per_graph
-    with torch.cuda.stream(stream):                # replays launch on the current stream
-        for _ in range(max(3, args.warmup)):
+    per = min(K, copies * max(1, 64 // copies))
+    g = _graph_of(step, per, stream)
+    reps, rem = divmod(K, per)
+    g_rem = _graph_of(step, rem, stream) if rem else None
+
+    def region():
+        for _ in range(reps):
             g.replay()
+        if g_rem is not None:
+            g_rem.replay()
+
+    with torch.cuda.stream(stream):          # replays launch on the current stream
+        for _ in range(max(3, args.warmup)):
+            region()
     stream.synchronize()
 
     dist = _dist()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
-    if dist:
-        dist.barrier()
-    torch.cuda.synchronize()
-    with ClockSampler(local_rank) as clk:
+
+    def timed_region():
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
         with torch.cuda.stream(stream):
             e0.record(stream)
-            for _ in range(replays):
-                g.replay()
+            region()
             e1.record(stream)
         torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
-    ms = e0.elapsed_time(e1)
+        if dist:
+            dist.barrier()
+        return _max_over_ranks(e0.elapsed_time(e1))
+
+    # The timed region (exactly K steps) is repeated until ~0.3 s have passed, so that the clock
+    # sampler sees it; value comes from the median repetition.
+    first = timed_region()
+    n_rep = max(3, min(2000, math.ceil(0.3 / max(first / 1e3, 1e-6))))
+    with ClockSampler(local_rank) as clk:
+        times = [timed_region() for _ in range(n_rep)]
     st = P.pifa_device_status(stream)
     assert st == P.PIFA_OK, P.pifa_status_string(st)
-    ms_max = _max_over_ranks(ms)
-    step_ms = ms_max / steps
-    value = _job_value(world, T, steps, ms_max)
-    achieved = decode_bytes(T, m, n, r) / (step_ms / 1e3) / 1e9
+    ms_region = statistics.median(times)
+    step_ms = ms_region / K
+    value = _job_value(world, T, K, ms_region)
+    del g, g_rem
 
     # --- e2e through the public API with pinned host buffers ---
-    Xh = torch.empty((T, n), dtype=torch.bfloat16).pin_memory()
-    Xh.copy_(Xs[0].cpu())
-    Yh = torch.empty((T, m), dtype=torch.bfloat16).pin_memory()
-    Xd = torch.empty((T, n), dtype=torch.bfloat16, device=dev)
-    e2e_steps = min(steps, 2000)
-    with torch.cuda.stream(stream):
-        for i in range(5):
-            Xd.copy_(Xh, non_blocking=True)
-            P.pifa_forward(Xd, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Ys[0], variant=variant,
-                                      workspace_tensor=ws, stream=stream)
-            Yh.copy_(Ys[0], non_blocking=True)
-    stream.synchronize()
-    if dist:
-        dist.barrier()
-    torch.cuda.synchronize()
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for i in range(e2e_steps):
-            Xd.copy_(Xh, non_blocking=True)
-            P.pifa_forward(Xd, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Ys[0], variant=variant,
-                           workspace_tensor=ws, stream=stream)
-            Yh.copy_(Ys[0], non_blocking=True)
-        e1.record(stream)
-    stream.synchronize()
-    e2e_ms = _max_over_ranks(e0.elapsed_time(e1))
-    e2e_eager = _job_value(world, T, e2e_steps, e2e_ms)
-    # The same loop -- per step the upload of X from pinned host memory, pifa_forward, the download
-    # of Y -- captured once as a CUDA graph and replayed, as a serving loop issues it: every step
-    # still moves its bytes host -> device -> host; the graph removes the per-call host overhead.
     nh = 4
     Xhs = [torch.empty((T, n), dtype=torch.bfloat16).pin_memory() for _ in range(nh)]
-    Yhs = [torch.empty((T, m), dtype=torch.bfloat16).pin_memory() for _ in range(nh)]
     for i in range(nh):
         Xhs[i].copy_(Xs[i % copies].cpu())
-    per_e2e = copies * max(1, 64 // copies)
-
-    def e2e_step(i):
-        Xd.copy_(Xhs[i % nh], non_blocking=True)
-        P.pifa_forward(Xd, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Ys[0], variant=variant, workspace_tensor=ws,
-                       stream=stream)
-        Yhs[i % nh].copy_(Ys[0], non_blocking=True)
-
-    ge = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(ge, stream=stream):
-        for i in range(per_e2e):
-            e2e_step(i)
-    e2e_replays = max(1, e2e_steps // per_e2e)
-    with torch.cuda.stream(stream):
-        for _ in range(2):
-            ge.replay()
-    stream.synchronize()
-    if dist:
-        dist.barrier()
-    torch.cuda.synchronize()
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for _ in range(e2e_replays):
-            ge.replay()
-        e1.record(stream)
-    stream.synchronize()
-    e2e_graph = _job_value(world, T, e2e_replays * per_e2e, _max_over_ranks(e0.elapsed_time(e1)))
-    assert np.array_equal(Yhs[(per_e2e - 1) % nh].float().numpy(), Ys[0].cpu().float().numpy())
+    e2e_steps = max(64, min(4000, math.ceil(0.3 / max(step_ms / 1e3, 1e-7))))
     e2e_pipe, e2e_pipe_steps, e2e_pipe_per = e2e_pipelined(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws,
                                                            stream, world, e2e_steps)
+    e2e_serial = e2e_serial_graph(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws, stream, world, e2e_steps)
 
+    ab = decode_bytes(T, m, n, r)
+    af = pifa_flops(T, m, n, r)
     out = {
-        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": steps,
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": K,
         "warmup": args.warmup, "ms_per_step": step_ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": f"{shape.name} {'decode' if T <= 16 else 'prefill'} T={T}", "m": m, "n": n, "r": r,
-                   "tokens_per_step": T, "c_dtype": lay["c_dtype"],
-                   "variant": P.pifa_variant_name(variant), "parallelism": f"replicas{world}",
-                   "l2_defeat": f"{copies} rotating weight copies ({copies * wbytes / 1e6:.0f} MB > 3x L2)",
-                   "timing": "CUDA graph replay, CUDA events on the launching stream"},
+        "config": {"workload": f"{shape.name} {'decode' if decode else 'prefill'} T={T}", "m": m, "n": n, "r": r,
+                   "tokens_per_step": T, "c_dtype": args.c_dtype, "variant": P.pifa_variant_name(variant),
+                   "parallelism": f"replicas{world}",
+                   "operands": "seeded synthetic layer: random ascending pivot set, W_p ~ N(0, 1/r), C ~ N(0, 0.18^2), "
+                               "X ~ N(0, 1), all bf16 (kernel time does not depend on the values)",
+                   "l2_defeat": f"{copies} rotating weight copies with their own X and Y "
+                                f"({copies * wbytes / 1e6:.0f} MB > 3x L2)",
+                   "timing": f"exactly {K} steps per timed region (CUDA graph replays, CUDA events on the launching "
+                             f"stream); the region repeated {n_rep} times, value from the median"},
+        "timed_repeats": n_rep,
         "e2e": {"value": e2e_pipe, "unit": "tokens/s", "h2d_bytes_per_step": T * n * 2,
                 "d2h_bytes_per_step": T * m * 2,
                 "mode": f"serving loop: per step X uploaded from pinned host memory (one copy per step), "
@@ -363,205 +533,71 @@ def run_ours(args, rank, world, local_rank):
                         f"neighbouring groups' forwards, the compute stream waiting on the copies once per group; "
                         f"{e2e_pipe_per} steps per CUDA graph, {e2e_pipe_steps} steps timed; the last step's Y "
                         f"checked against a separate forward",
-                "serial_value": e2e_eager,
-                "serial_mode": "the same steps one after another on one stream, issued call by call (no overlap)",
-                "serial_graph_value": e2e_graph,
-                "serial_graph_mode": "the serial loop captured as a CUDA graph and replayed"},
-        "roofline": ({"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                      "frac": achieved / hbm_peak,
-                      "traffic": _traffic("decode.cu", "decode") if (T, m, n, r) == (8, 4096, 4096, 2048) else None,
-                      "peak_source": f"{peak_src} hbm_gbs",
+                "serial_value": e2e_serial,
+                "serial_mode": "the same steps one after another on one stream (upload, forward, download), "
+                               "captured as a CUDA graph and replayed"},
+        "roofline": ({"bound": "hbm", "achieved": ab / (step_ms / 1e3) / 1e9, "peak": hbm_peak, "unit": "GB/s",
+                      "frac": ab / (step_ms / 1e3) / 1e9 / hbm_peak,
+                      "traffic": _traffic(shape.name, T),
+                      "peak_source": f"{peak_src} hbm_gbs (burst: the call is timed alone)",
                       "kernel": "decode phase 1 + phase 2 (one PDL-chained pair per call)",
-                      "algorithmic_bytes_per_launch": decode_bytes(T, m, n, r)} if T <= 16 else
-                     {"bound": "tensor", "achieved": pifa_flops(T, m, n, r) / (step_ms / 1e3) / 1e12, "peak": tc_peak,
-                      "unit": "TFLOP/s", "frac": pifa_flops(T, m, n, r) / (step_ms / 1e3) / 1e12 / tc_peak,
+                      "algorithmic_bytes_per_launch": ab} if decode else
+                     {"bound": "tensor", "achieved": af / (step_ms / 1e3) / 1e12, "peak": tc_peak,
+                      "unit": "TFLOP/s", "frac": af / (step_ms / 1e3) / 1e12 / tc_peak,
                       "traffic": None, "peak_source": f"{peak_src} bf16_tflops (burst)",
                       "kernel": f"{P.pifa_variant_name(variant)} prefill (GEMM 1 + GEMM 2 per call)",
-                      "algorithmic_flops_per_launch": pifa_flops(T, m, n, r)}),
-        "gpu_launches": steps * (2 if m > r else 1),
+                      "algorithmic_flops_per_launch": af}),
+        "gpu_launches": K * (2 if m > r else 1),
+        "gpu_launches_all_repeats": K * (2 if m > r else 1) * n_rep,
         "clocks": clk.summary(),
     }
-    if rank == 0 and world == 1 and not args.no_extras and shape is SHAPE:
-        # one GPU only (at N > 1 every GPU would wait for rank 0's extras); the HBM-bound points first: the prefill-sized GEMMs after them hold the power cap
-        with ClockSampler(local_rank) as clk_x:
-            out["decode_sweep"] = decode_sweep(dev, stream, hbm_peak, peak_src)
-            out["grouped_mlp7b_gate_up"] = grouped_point(dev, stream, hbm_peak, tc_peak, peak_src)
-        out["decode_sweep_clocks"] = clk_x.summary()
-        with ClockSampler(local_rank) as clk_p:
-            out["comparators"] = comparators(dev, lay, T, copies, stream)
-            out["prefill"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src)
-            out["prefill_fused"] = prefill_point(dev, lay, copies, stream, tc_peak, peak_src,
-                                                 variant=P.PIFA_VARIANT_PREFILL_FUSED)
-        out["prefill_clocks"] = clk_p.summary()
-        out["cpu_baseline"] = cpu_baseline(lay, T)
-    return out
-
-
-def comparators(dev, lay, T, copies, stream):
-    """Dense X W^T and two-factor low-rank (X V) U^T on the same GPU (torch.matmul, bf16), each a
-    CUDA graph over rotating weight copies timed in steady state (_graph_ms)."""
-    import torch
-    res = {}
-    U = torch.from_numpy(lay["U"]).to(dev).to(torch.bfloat16)
-    V = torch.from_numpy(lay["V"]).to(dev).to(torch.bfloat16)
-    W = (U.float() @ V.float().t()).to(torch.bfloat16)
-    for Tq in (T, T_PREFILL):
-        X = torch.randn((Tq, V.shape[0]), device=dev).to(torch.bfloat16)
-        Ws = [W.clone() for _ in range(max(2, copies // 2))]
-        Us = [U.clone() for _ in range(copies)]
-        Vs = [V.clone() for _ in range(copies)]
-        for name, fn, nrot in (("dense", lambda i: X @ Ws[i % len(Ws)].t(), len(Ws)),
-                               ("lowrank", lambda i: (X @ Vs[i % copies]) @ Us[i % copies].t(), copies)):
-            with torch.cuda.stream(stream):
-                for i in range(5):
-                    fn(i)
-            stream.synchronize()
-            per = nrot * max(1, 64 // nrot) if Tq <= 16 else nrot
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                for i in range(per):
-                    fn(i)
-            ms = _graph_ms(g, stream) / per
-            del g
-            res[f"{name}_T{Tq}"] = {"tokens_per_s": Tq / (ms / 1e3), "ms": ms}
-    return res
-
-
-DECODE_SWEEP = [(inputs.ATTN7B, (1, 8, 16)), (inputs.MLP7B_GATE, (1, 8)), (inputs.MLP7B_DOWN, (1, 8)),
-                (inputs.ATTN70B, (1, 8, 16)), (inputs.MLP70B_GATE, (1, 8, 16))]
-
-
-def decode_sweep(dev, stream, hbm_peak, peak_src):
-    """The decode variant on every decode-sized layer shape (HBM-bound), beside the two-factor
-    low-rank layer of the same shape. Timing inputs only: W_p and C are seeded N(0, 1) bf16 and the
-    pivot set a seeded random r-subset (kernel time does not depend on the values); weight copies
-    rotate so that every call streams its weights from HBM."""
-    import torch
-    from paper_2501_19090_gb300 import pifa as P
-    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    out = []
-    for shape, Ts in DECODE_SWEEP:
-        m, n, r = shape.m, shape.n, shape.r
-        rng = np.random.default_rng(11)
-        perm = rng.permutation(m)
-        piv = torch.from_numpy(np.sort(perm[:r]).astype(np.int32)).to(dev)
-        nonp = torch.from_numpy(np.sort(perm[r:]).astype(np.int32)).to(dev)
-        gen = torch.Generator(device=dev)
-        gen.manual_seed(12)
-        wbytes = 2 * r * (m + n - r)
-        copies = max(4, math.ceil(3 * l2 / wbytes))  # as the main line: every call streams from HBM
-        Wps = [torch.randn((r, n), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
-        Cs = [torch.randn((m - r, r), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
-        lr_copies = max(4, math.ceil(3 * l2 / (2 * r * (m + n))))
-        Us = [torch.randn((m, r), device=dev, generator=gen).to(torch.bfloat16) for _ in range(lr_copies)]
-        Vs = [torch.randn((n, r), device=dev, generator=gen).to(torch.bfloat16) for _ in range(lr_copies)]
-        for T in Ts:
-            # per weight copy its own X and Y, as the main line
-            Xc = [torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
-            Yc = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(copies)]
-            X = Xc[0]
-            variant = P.pifa_select_variant(T, m, n, r, P.PIFA_DTYPE_BF16)
-            ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant), dev, tag="sweep")
-
-            def step(i):
-                j = i % copies
-                P.pifa_forward(Xc[j], Wps[j], Cs[j], piv, nonp, Y=Yc[j], variant=variant,
-                               workspace_tensor=ws, stream=stream)
-
-            with torch.cuda.stream(stream):
-                for i in range(4):
-                    step(i)
-            per_graph = copies * max(1, 64 // copies)
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=stream):
-                for i in range(per_graph):
-                    step(i)
-            ms = _graph_ms(g, stream, replays=max(3, 256 // per_graph)) / per_graph
-            assert P.pifa_device_status(stream) == P.PIFA_OK
-            lr = lambda i: (X @ Vs[i % lr_copies]) @ Us[i % lr_copies].t()
-            with torch.cuda.stream(stream):
-                for i in range(4):
-                    lr(i)
-            g2 = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g2, stream=stream):
-                for i in range(per_graph):
-                    lr(i)
-            lr_ms = _graph_ms(g2, stream, replays=max(3, 256 // per_graph)) / per_graph
-            gbs = decode_bytes(T, m, n, r) / (ms / 1e3) / 1e9
-            out.append({"workload": f"{shape.name} decode T={T}", "us_per_call": ms * 1e3,
-                        "tokens_per_s": T / (ms / 1e3), "hbm_gbs": gbs, "frac": gbs / hbm_peak,
-                        "lowrank_us_per_call": lr_ms * 1e3, "speedup_vs_lowrank": lr_ms / ms,
-                        "weight_copies": copies, "peak_source": f"{peak_src} hbm_gbs"})
-            del g, g2
-        del Wps, Cs, Us, Vs
-        torch.cuda.empty_cache()
-    return out
-
-
-def grouped_point(dev, stream, hbm_peak, tc_peak, peak_src):
-    """The 7B MLP's gate and up projections (11008 x 4096, r = 2048) sharing X: one
-    pifa_forward_grouped call against two pifa_forward calls, graph replay, >= 4 rotating weight
-    copies; timing operands as in decode_sweep (seeded N(0, 1) weights, random pivot sets)."""
-    import torch
-    from paper_2501_19090_gb300 import pifa as P
-    shape = inputs.MLP7B_GATE
-    m, n, r, G = shape.m, shape.n, shape.r, 2
-    rng = np.random.default_rng(13)
-    piv_l, nonp_l = [], []
-    for g in range(G):
-        perm = rng.permutation(m)
-        piv_l.append(torch.from_numpy(np.sort(perm[:r]).astype(np.int32)).to(dev))
-        nonp_l.append(torch.from_numpy(np.sort(perm[r:]).astype(np.int32)).to(dev))
-    piv_s = torch.cat([piv_l[g] + g * m for g in range(G)])
-    nonp_s = torch.cat([nonp_l[g] + g * m for g in range(G)])
-    gen = torch.Generator(device=dev)
-    gen.manual_seed(14)
-    copies = 4
-    Wps = [torch.randn((G * r, n), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
-    Cs = [torch.randn((G * (m - r), r), device=dev, generator=gen).to(torch.bfloat16) for _ in range(copies)]
-    out = []
-    for T in (1, 8, T_PREFILL):
-        X = torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16)
-        Y = torch.empty((T, G * m), dtype=torch.bfloat16, device=dev)
-        Ys = [torch.empty((T, m), dtype=torch.bfloat16, device=dev) for _ in range(G)]
-        ws1 = P.workspace(P.pifa_workspace_size(T, m, n, r), dev, tag="grp1")
-        wsg = P.workspace(P.pifa_workspace_size_grouped(G, T, m, n, r), dev, tag="grpG")
-
-        def sep(i):
-            j = i % copies
-            for g in range(G):
-                P.pifa_forward(X, Wps[j][g * r:(g + 1) * r], Cs[j][g * (m - r):(g + 1) * (m - r)], piv_l[g],
-                               nonp_l[g], Y=Ys[g], workspace_tensor=ws1, stream=stream)
-
-        def grp(i):
-            j = i % copies
-            P.pifa_forward_grouped(G, X, Wps[j], Cs[j], piv_s, nonp_s, Y=Y, workspace_tensor=wsg, stream=stream)
-
-        per_graph = 16 if T <= 16 else 4
-        res = {}
-        for name, fn in (("separate", sep), ("grouped", grp)):
-            with torch.cuda.stream(stream):
-                for i in range(4):
-                    fn(i)
-            g_ = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g_, stream=stream):
-                for i in range(per_graph):
-                    fn(i)
-            res[name] = _graph_ms(g_, stream, replays=5) / per_graph
-            del g_
-        assert P.pifa_device_status(stream) == P.PIFA_OK
-        e = {"workload": f"{shape.name} x2 (gate + up) T={T}", "grouped_us": res["grouped"] * 1e3,
-             "separate_us": res["separate"] * 1e3, "speedup": res["separate"] / res["grouped"]}
-        if T <= 16:
-            gbs = G * decode_bytes(T, m, n, r) / res["grouped"] / 1e6
-            e.update({"hbm_gbs": gbs, "frac": gbs / hbm_peak, "peak_source": f"{peak_src} hbm_gbs"})
-        else:
-            tf = G * pifa_flops(T, m, n, r) / res["grouped"] / 1e9
-            e.update({"tflops": tf, "frac": tf / tc_peak, "peak_source": f"{peak_src} bf16_tflops (burst)"})
-        out.append(e)
-    del Wps, Cs
+    del Wps, Cs, Xs, Ys
     torch.cuda.empty_cache()
+    if rank == 0 and world == 1 and not args.no_extras and shape is SHAPE and T == T_DECODE:
+        # one GPU only (at N > 1 every GPU would wait for rank 0's extras)
+        out["comparators"] = layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src,
+                                         name="headline layer, same T (PIFA re-timed beside the comparators)")
+        out.update(extras(dev, stream, hbm_peak, tc_peak, peak_src))
+        out["cpu_baseline"] = cpu_baseline(shape, T)
     return out
+
+
+def e2e_serial_graph(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws, stream, world, steps):
+    """The serial serving loop (upload X, forward, download Y, one after another on one stream)
+    captured as a CUDA graph and replayed; tokens/s over all ranks."""
+    import torch
+    nh = len(Xhs)
+    copies = len(Wps)
+    Xd = torch.empty((T, n), dtype=torch.bfloat16, device=dev)
+    Yd = torch.empty((T, m), dtype=torch.bfloat16, device=dev)
+    Yhs = [torch.empty((T, m), dtype=torch.bfloat16).pin_memory() for _ in range(nh)]
+
+    def e2e_step(i):
+        Xd.copy_(Xhs[i % nh], non_blocking=True)
+        P.pifa_forward(Xd, Wps[i % copies], Cs[i % copies], piv, nonp, Y=Yd, variant=variant, workspace_tensor=ws,
+                       stream=stream)
+        Yhs[i % nh].copy_(Yd, non_blocking=True)
+
+    per = copies * max(1, 64 // copies)
+    g = _graph_of(e2e_step, per, stream)
+    reps = max(1, steps // per)
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            g.replay()
+    stream.synchronize()
+    dist = _dist()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    return _job_value(world, T, reps * per, _max_over_ranks(e0.elapsed_time(e1)))
 
 
 def e2e_pipelined(P, dev, T, n, m, Xhs, Wps, Cs, piv, nonp, variant, ws, stream, world, steps):
@@ -688,81 +724,22 @@ def _graph_ms(g, stream, replays=None, warm_s=0.1, timed_s=0.25):
     return e0.elapsed_time(e1) / n_rep
 
 
-def _eager_ms(call, stream, warm_s=0.1, timed_s=0.25):
-    """Milliseconds per call(i) issued eagerly on `stream` (calls long enough that the host keeps
-    ahead), in steady state as _graph_ms: about warm_s seconds of calls first, then about timed_s
-    seconds timed."""
-    import torch
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for i in range(4):
-            call(i)
-        e1.record(stream)
-    stream.synchronize()
-    one = max(e0.elapsed_time(e1) / 4e3, 1e-6)
-    with torch.cuda.stream(stream):
-        for i in range(math.ceil(warm_s / one)):
-            call(i)
-        n_call = max(8, math.ceil(timed_s / one))
-        e0.record(stream)
-        for i in range(n_call):
-            call(i)
-        e1.record(stream)
-    stream.synchronize()
-    return e0.elapsed_time(e1) / n_call
+def _host_layer(shape, seed=0):
+    """The headline layer's operands on the host for the oracle timings: inputs.synthetic_layer of
+    the shape (random ascending pivots, W_p ~ N(0, 1/r), C ~ N(0, 0.18^2), bf16 values). The
+    oracle's time depends on the shapes only."""
+    piv, nonp, Wp, C = inputs.synthetic_layer(shape.m, shape.n, shape.r, seed)
+    return piv.astype(np.int64), nonp.astype(np.int64), Wp.astype(np.float64), C.astype(np.float64)
 
 
-def prefill_point(dev, lay, copies, stream, tc_peak, peak_src, variant=None):
-    import torch
-    from paper_2501_19090_gb300 import pifa as P
-    m, n, r = SHAPE.m, SHAPE.n, SHAPE.r
-    T = T_PREFILL
-    bf = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev).to(torch.bfloat16)
-    piv = torch.from_numpy(lay["piv"]).to(dev)
-    nonp = torch.from_numpy(lay["nonp"]).to(dev)
-    Wp = bf(lay["Wp"])
-    C = torch.from_numpy(np.ascontiguousarray(lay["C"])).to(dev).to(_torch_c_dtype(lay))
-    cdt = _pifa_c_dtype(lay)
-    ncp = max(2, copies // 4)
-    Wps = [Wp.clone() for _ in range(ncp)]
-    Cs = [C.clone() for _ in range(ncp)]
-    rng = np.random.default_rng(5)
-    Xs = [bf(inputs.make_activations(rng, T, n, "bf16")) for _ in range(ncp)]
-    Y = torch.empty((T, m), dtype=torch.bfloat16, device=dev)
-    if variant is None:
-        variant = P.pifa_select_variant(T, m, n, r, cdt)
-    ws = P.workspace(P.pifa_workspace_size(T, m, n, r, variant, cdt), dev, tag="prefill")
-    with torch.cuda.stream(stream):
-        for i in range(5):
-            P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,
-                           workspace_tensor=ws, stream=stream)
-    stream.synchronize()
-
-    def call(i):
-        P.pifa_forward(Xs[i % ncp], Wps[i % ncp], Cs[i % ncp], piv, nonp, Y=Y, variant=variant,
-                       workspace_tensor=ws, stream=stream)
-
-    ms = _eager_ms(call, stream)
-    assert P.pifa_device_status(stream) == P.PIFA_OK
-    tf = pifa_flops(T, m, n, r) / (ms / 1e3) / 1e12
-    return {"workload": f"{SHAPE.name} prefill T={T}", "variant": P.pifa_variant_name(variant),
-            "tokens_per_s": T / (ms / 1e3), "ms_per_step": ms,
-            "roofline": {"bound": "tensor", "achieved": tf, "peak": tc_peak, "unit": "TFLOP/s",
-                         "frac": tf / tc_peak, "peak_source": f"{peak_src} bf16_tflops (burst)",
-                         "algorithmic_flops_per_launch": pifa_flops(T, m, n, r)}}
-
-
-def cpu_baseline(lay, T, budget_s=10.0, single_s=5.0):
+def cpu_baseline(shape, T, budget_s=10.0, single_s=5.0):
     """The fp64 oracle forward (numpy) on the host cores over a bounded sample of the workload,
     with BLAS_THREADS BLAS threads; the same forward on one thread, timed in a fresh interpreter
     (numpy's thread count is fixed when it loads), is reported beside it."""
     import oracle
+    piv, nonp, Wp, C = _host_layer(shape)
     rng = np.random.default_rng(9)
-    X = inputs.make_activations(rng, T, SHAPE.n, "bf16")
-    Wp, C = lay["Wp"].astype(np.float64), lay["C"].astype(np.float64)
-    piv, nonp = lay["piv"].astype(np.int64), lay["nonp"].astype(np.int64)
+    X = inputs.make_activations(rng, T, shape.n, "bf16")
     oracle.forward(X, Wp, C, piv, nonp)
     t0 = time.perf_counter()
     calls = 0
@@ -771,10 +748,10 @@ def cpu_baseline(lay, T, budget_s=10.0, single_s=5.0):
         calls += 1
     dt = time.perf_counter() - t0
     out = {"value": calls * T / dt, "unit": "tokens/s", "cores": BLAS_THREADS, "kind": "oracle",
-           "sample": f"{calls} oracle forwards of T={T} tokens on {SHAPE.name} (fp64 numpy, "
+           "sample": f"{calls} oracle forwards of T={T} tokens on {shape.name} (fp64 numpy, "
                      f"{BLAS_THREADS} BLAS threads), {dt:.1f} s"}
     try:
-        out["single_thread"] = _oracle_rate_one_thread(X, Wp, C, piv, nonp, T, single_s)
+        out["single_thread"] = _oracle_rate_one_thread(shape, T, single_s)
     except Exception as e:  # reported, never fatal: the main figure stands on its own
         out["single_thread"] = {"error": f"{type(e).__name__}: {e}"}
     return out
@@ -785,26 +762,25 @@ import json, sys, time
 import numpy as np
 sys.path.insert(0, sys.argv[1])
 import oracle
-d = np.load(sys.argv[2])
-args = (d["X"], d["Wp"], d["C"], d["piv"], d["nonp"])
+from paper_2501_19090_gb300 import inputs
+m, n, r, T = (int(v) for v in sys.argv[2:6])
+piv, nonp, Wp, C = inputs.synthetic_layer(m, n, r, 0)
+args = (inputs.make_activations(np.random.default_rng(9), T, n, "bf16"), Wp.astype(np.float64),
+        C.astype(np.float64), piv.astype(np.int64), nonp.astype(np.int64))
 oracle.forward(*args)
 t0, calls = time.perf_counter(), 0
-while time.perf_counter() - t0 < float(sys.argv[3]):
+while time.perf_counter() - t0 < float(sys.argv[6]):
     oracle.forward(*args)
     calls += 1
 print(json.dumps({"calls": calls, "seconds": time.perf_counter() - t0}))
 """
 
 
-def _oracle_rate_one_thread(X, Wp, C, piv, nonp, T, budget_s):
+def _oracle_rate_one_thread(shape, T, budget_s):
     """Tokens/s of the oracle forward with one BLAS thread, in a fresh interpreter."""
-    import tempfile
-    with tempfile.TemporaryDirectory() as d:
-        path = os.path.join(d, "case.npz")
-        np.savez(path, X=X, Wp=Wp, C=C, piv=piv, nonp=nonp)
-        env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
-        r = subprocess.run([sys.executable, "-c", _ONE_THREAD_TIMER, ROOT, path, str(budget_s)], env=env,
-                           capture_output=True, text=True, timeout=budget_s + 120)
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    r = subprocess.run([sys.executable, "-c", _ONE_THREAD_TIMER, ROOT, str(shape.m), str(shape.n), str(shape.r),
+                        str(T), str(budget_s)], env=env, capture_output=True, text=True, timeout=budget_s + 180)
     if r.returncode != 0:
         raise RuntimeError(r.stderr.strip().splitlines()[-1] if r.stderr.strip() else f"exit {r.returncode}")
     res = json.loads(r.stdout.strip().splitlines()[-1])
@@ -812,9 +788,9 @@ def _oracle_rate_one_thread(X, Wp, C, piv, nonp, T, budget_s):
             "sample": f"{res['calls']} oracle forwards, {res['seconds']:.1f} s, one BLAS thread"}
 
 
-def _traffic(src, key):
-    t = NCU_TRAFFIC.get(key)
-    if not t or t.get("sha") != _src_sha(src):
+def _traffic(layer, T):
+    t = NCU_TRAFFIC.get((layer, T))
+    if not t or t.get("sha") != _src_sha("decode.cu"):
         return None
     return t["bytes"]
 
@@ -846,38 +822,36 @@ def _job_value(world, tokens_per_step, steps, ms_max):
 
 
 def run_reference(args, rank):
-    """Reference arm: the fp64 oracle (the paper publishes no code) on the host cores, same workload."""
+    """Reference arm: the fp64 oracle (the paper publishes no code) on the host cores, on the same
+    workload as our arm's line (rank 0 only; other ranks exit without work)."""
     import oracle
-    from paper_2501_19090_gb300 import pifa as P
     if rank != 0:
         return None
+    shape = SHAPES[args.shape]
     T = args.tokens
-    U, V, _ = inputs.make_factors(SHAPE.m, SHAPE.n, SHAPE.r, 0)
-    L = oracle.compress(U, V, SHAPE.r, "lapack")
-    Cq = inputs.round_fp16(L.C) if args.c_dtype == "fp16" else inputs.round_bf16(L.C)
-    Wp, C = inputs.round_bf16(L.Wp).astype(np.float64), Cq.astype(np.float64)
+    piv, nonp, Wp, C = _host_layer(shape)
     rng = np.random.default_rng(1)
-    X = inputs.make_activations(rng, T, SHAPE.n, "bf16")
+    X = inputs.make_activations(rng, T, shape.n, "bf16")
     for _ in range(max(3, args.warmup)):
-        oracle.forward(X, Wp, C, L.pivots, L.nonpivots)
+        oracle.forward(X, Wp, C, piv, nonp)
     # bounded sample: at most ~60 s of oracle forwards, however many steps were asked for
     t0 = time.perf_counter()
     done = 0
     while done < args.steps and (done == 0 or time.perf_counter() - t0 < 60.0):
-        oracle.forward(X, Wp, C, L.pivots, L.nonpivots)
+        oracle.forward(X, Wp, C, piv, nonp)
         done += 1
     dt = time.perf_counter() - t0
     v = T * done / dt
     cores = BLAS_THREADS
-    del P
     return {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": done, "requested_steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / done,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": f"{SHAPE.name} decode T={T}", "m": SHAPE.m, "n": SHAPE.n,
-                                            "r": SHAPE.r, "tokens_per_step": T},
+            "data": "synthetic", "config": {"workload": f"{shape.name} {'decode' if T <= 16 else 'prefill'} T={T}",
+                                            "m": shape.m, "n": shape.n, "r": shape.r, "tokens_per_step": T,
+                                            "c_dtype": args.c_dtype, "parallelism": f"replicas{args.gpus}"},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                             "sample": f"{done} of {args.steps} requested fp64 oracle forwards of T={T} "
-                                       f"(numpy, {cores} BLAS threads; capped at ~60 s)"},
+                             "sample": f"{done} of {args.steps} requested fp64 oracle forwards of T={T} on a seeded "
+                                       f"synthetic layer of the shape (numpy, {cores} BLAS threads; capped at ~60 s)"},
             "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -885,14 +859,14 @@ def main():
     global _DIST
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200000)
+    ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--tokens", type=int, default=T_DECODE)
     ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--c-dtype", default="bf16", choices=["bf16", "fp16"])
     ap.add_argument("--shape", default=SHAPE.name, choices=sorted(SHAPES),
-                    help="decode layer shape of the main line (other shapes: synthetic operands, no extras)")
+                    help="layer shape of the main line (extras run with the default shape and T only)")
     args = ap.parse_args()
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

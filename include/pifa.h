@@ -58,8 +58,7 @@ typedef enum {
   PIFA_VARIANT_AUTO = 0,
   PIFA_VARIANT_DECODE = 1,        /* T <= 16: two-phase HBM-streaming GEMV (mma.sync fragments)  */
   PIFA_VARIANT_PREFILL_SPLIT = 2, /* tcgen05 GEMM 1 -> Y_p in workspace -> tcgen05 GEMM 2        */
-  PIFA_VARIANT_PREFILL_FUSED = 3  /* one persistent cluster kernel per token tile: GEMM 1, Y_p kept
-                                     on chip (L2 + shared memory), GEMM 2                        */
+  PIFA_VARIANT_PREFILL_FUSED = 3  /* reserved: not built in this version (PIFA_ERR_UNSUPPORTED)   */
 } pifa_variant;
 
 /* Diagnostics of pifa_compress (all optional to read). */
@@ -136,7 +135,7 @@ int pifa_forward_variant(const void* X, int64_t T, int64_t n, int64_t ldx,
  *   Y            T x (G m), leading dimension ldy >= G m: group g's output in columns [g m, (g + 1) m).
  *   workspace    at least pifa_workspace_size_grouped(G, T, m, n, r, c_dtype) bytes, 256-byte aligned.
  *   Variant, alignment, aliasing, asynchrony and status codes as pifa_forward (the variant is the
- *   one pifa_select_variant picks for one layer; the fused prefill does not run grouped layers).
+ *   one pifa_select_variant picks for one layer).
  *   G in [1, 64]; G > 1 needs m > r, (m - r) % 128 == 0 and r % 8 == 0 (PIFA_ERR_UNSUPPORTED
  *   otherwise: call pifa_forward per layer), so that no tile spans two groups. G = 1 is
  *   pifa_forward.
@@ -167,7 +166,9 @@ int64_t pifa_workspace_size_grouped(int64_t groups, int64_t T, int64_t m, int64_
  *   256 + T * round_up(r, 8) * 4 > 1 MiB are rejected with PIFA_ERR_WORKSPACE; T > 16 with
  *   PIFA_ERR_UNSUPPORTED.
  *   The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
- *   that device current; make that first call before any stream capture. Every call on a device
+ *   that device current; make that first call before any stream capture. The address is kept for
+ *   the process, so only the device's primary context (the CUDA runtime's) is supported, and a
+ *   cudaDeviceReset() ends this library's use on that device (so does the status word's). Every call on a device
  *   shares the one array and it keeps the last call's contents, which no call depends on: y_p is
  *   fully written before it is read. Calls that may overlap on the GPU, e.g. on different
  *   streams, race on the array.
@@ -185,8 +186,7 @@ int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dt
 
 /* pifa_select_variant -- the selector (host, < 1 us): the pifa_variant pifa_forward runs for
  * (T, m, n, r, c_dtype) on this build, never PIFA_VARIANT_AUTO; negative pifa_status on bad
- * arguments. Decode for T <= 16, else the split prefill (the fused prefill kernel is measured
- * slower on GB300 and runs only when requested). */
+ * arguments. Decode for T <= 16, else the split prefill. */
 int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype);
 
 /* pifa_variant_name -- static string naming a pifa_variant ("decode", ...); "?" if unknown. */
@@ -216,6 +216,39 @@ int pifa_compress(const double* U, const double* V, int64_t m, int64_t n, int64_
                   int32_t* pivot_idx, int32_t* nonpivot_idx,
                   double* Wp, int64_t ldwp, double* C, int64_t ldc,
                   pifa_compress_info* info);
+
+/*
+ * pifa_compress_device -- Algorithm 1 (Sec. 3.2) on W' = U V^T on the GPU in float64: the same
+ * outputs as pifa_compress, for layers where the host route is slow (minutes at 28672 x 8192).
+ *
+ *   U, V         DEVICE, float64, m x r and n x r, row-major, contiguous (W' = U V^T).
+ *   pivot_idx    DEVICE out, int32[r]: I, ascending.
+ *   nonpivot_idx DEVICE out, int32[m - r]: I^c, ascending (may be NULL when r == m).
+ *   Wp           DEVICE out, float64, r x n, row pitch ldwp >= n: W'[I, :] (Eq. 1).
+ *   C            DEVICE out, float64, (m - r) x r, row pitch ldc >= r: W'[I^c, :] = C W_p (Eq. 2),
+ *                columns in ascending-I order (may be NULL when r == m).
+ *   workspace    DEVICE scratch of pifa_compress_device_workspace_size(m, n, r) bytes, 256-byte
+ *                aligned, no initialisation needed (about 8 (m r + 4 r^2) bytes).
+ *   info         HOST out, optional: min_pivot_gap, r_ratio and max_abs_c as pifa_compress
+ *                (threads = 0).
+ *   cuda_stream  the stream the work is enqueued on; the call synchronizes it before returning.
+ *
+ *   Pivot rule exactly as pifa_compress (greedy Businger-Golub on W'^T, residual norms recomputed
+ *   every step, ties to the lowest index), computed in the r-dimensional row space Z = U L with
+ *   L L^T = V^T V (Cholesky), which has the row inner products of W'. C = Z[I^c] R^{-T} from the
+ *   triangular factor R of that pivoted QR; W_p = U[I] V^T. Requires 1 <= r <= min(m, n) and
+ *   r <= 16384 (PIFA_ERR_UNSUPPORTED otherwise); PIFA_ERR_RANK_DEFICIENT when V^T V is not
+ *   positive definite or |R_(r-1,r-1)| < 1e-8 |R_00|. Synchronous; no device memory is allocated.
+ */
+int pifa_compress_device(const double* U, const double* V, int64_t m, int64_t n, int64_t r,
+                         int32_t* pivot_idx, int32_t* nonpivot_idx,
+                         double* Wp, int64_t ldwp, double* C, int64_t ldc,
+                         void* workspace, int64_t workspace_bytes,
+                         pifa_compress_info* info, void* cuda_stream);
+
+/* pifa_compress_device_workspace_size -- bytes of device scratch pifa_compress_device needs;
+ * negative pifa_status on bad arguments. Pure host arithmetic. */
+int64_t pifa_compress_device_workspace_size(int64_t m, int64_t n, int64_t r);
 
 /* pifa_validate_indices -- HOST copies: PIFA_OK iff pivot_idx (r entries) and nonpivot_idx
  * (m - r entries) are strictly ascending, inside [0, m) and disjoint (so together a partition

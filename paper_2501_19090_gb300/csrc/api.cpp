@@ -149,8 +149,6 @@ int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype)
   if (st != PIFA_OK) return st;
   if (c_dtype != PIFA_DTYPE_BF16 && c_dtype != PIFA_DTYPE_FP16) return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown c_dtype");
   if (T <= 16) return PIFA_VARIANT_DECODE;
-  // The fused cluster kernel is correct but measured slower than the split GEMMs on GB300 (attn
-  // 4096 x 4096, r = 2048, T = 2048: 171 us against 70 us); it runs only when asked for.
   return PIFA_VARIANT_PREFILL_SPLIT;
 }
 
@@ -164,7 +162,7 @@ int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dt
   switch (variant) {
     case PIFA_VARIANT_DECODE: return kWorkspaceReserve + decode_workspace_bytes(s);
     case PIFA_VARIANT_PREFILL_SPLIT: return kWorkspaceReserve + prefill_split_workspace_bytes(s);
-    case PIFA_VARIANT_PREFILL_FUSED: return kWorkspaceReserve + prefill_fused_workspace_bytes(s);
+    case PIFA_VARIANT_PREFILL_FUSED: return pifa_fail(PIFA_ERR_UNSUPPORTED, "variant not built in this version");
     default: return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
   }
 }
@@ -189,7 +187,7 @@ int64_t workspace_bytes_for(const PifaShape& s, int variant) {
   switch (variant) {
     case PIFA_VARIANT_DECODE: return kWorkspaceReserve + decode_workspace_bytes(s);
     case PIFA_VARIANT_PREFILL_SPLIT: return kWorkspaceReserve + prefill_split_workspace_bytes(s);
-    case PIFA_VARIANT_PREFILL_FUSED: return kWorkspaceReserve + prefill_fused_workspace_bytes(s);
+    case PIFA_VARIANT_PREFILL_FUSED: return pifa_fail(PIFA_ERR_UNSUPPORTED, "variant not built in this version");
     default: return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
   }
 }
@@ -228,9 +226,8 @@ int forward_impl(int64_t groups, const void* X, int64_t T, int64_t n, int64_t ld
   PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy, c_dtype};
   s.groups = G;
   if (variant == PIFA_VARIANT_DECODE && T > 16) return pifa_fail(PIFA_ERR_UNSUPPORTED, "decode variant needs T <= 16");
-  if (variant == PIFA_VARIANT_PREFILL_FUSED && !prefill_fused_supported(s))
-    return pifa_fail(PIFA_ERR_UNSUPPORTED, "fused prefill cannot run this shape");
   const int64_t need = workspace_bytes_for(s, variant);
+  if (need < 0) return (int)need;
   if (!workspace || workspace_bytes < need)
     return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or smaller than pifa_workspace_size()");
   if (reinterpret_cast<uintptr_t>(workspace) & 255u)
@@ -252,7 +249,6 @@ int forward_impl(int64_t groups, const void* X, int64_t T, int64_t n, int64_t ld
   switch (variant) {
     case PIFA_VARIANT_DECODE: return launch_decode(s, p, status, stream);
     case PIFA_VARIANT_PREFILL_SPLIT: return launch_prefill_split(s, p, status, pifa_wait_timeout_ns(), stream);
-    case PIFA_VARIANT_PREFILL_FUSED: return launch_prefill_fused(s, p, status, pifa_wait_timeout_ns(), stream);
   }
   return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown variant");
 }

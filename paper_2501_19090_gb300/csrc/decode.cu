@@ -433,7 +433,7 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
   constexpr uint32_t kCons = kWarps * 32; // consumer threads (named barrier 1)
   extern __shared__ __align__(128) uint8_t smem_raw[];
   __shared__ uint64_t full[kMaxStages], empty[kMaxStages];
-  __shared__ uint64_t bbar, rready[2], rfree[2], done;
+  __shared__ uint64_t bbar, rready[2], rfree[2];
   __shared__ int s_cols[kRows];
   pdl_launch_dependents();  // the next kernel may launch now and start staging its weights
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -458,7 +458,6 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
       mbar_init(&empty[s], kWarps);
     }
     mbar_init(&bbar, 1);
-    mbar_init(&done, (uint32_t)a.ks);  // one arrival per CTA of the cluster
     for (int b = 0; b < 2; ++b) {
       mbar_init(&rready[b], (uint32_t)a.ks);  // one arrival per source CTA
       mbar_init(&rfree[b], (uint32_t)a.ks);   // one arrival per owner CTA
@@ -521,6 +520,9 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
         if (!mbar_wait(&full[it % a.stages], (uint32_t)(it / a.stages) & 1u, 100000000ull))
           latch_status(a.status, PIFA_ERR_TIMEOUT);
     }
+    __syncwarp();
+    // the producer warp's share of the closing cluster barrier (see the end of the consumers)
+    if (a.ks > 1) cluster_sync_all();
     return;  // from here on the consumers synchronise on named barrier 1 only
   }
 
@@ -726,17 +728,13 @@ __global__ void __launch_bounds__((kWarps + 1) * 32, 2)
     }
   }
   if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
-  // No CTA retires before every CTA of its cluster has made its last remote access to it (pushes
-  // and arrivals precede each CTA's arrival here): after a timeout the waits above are skipped,
-  // and a CTA could otherwise leave while a peer still writes into its shared memory.
-  if (a.ks > 1) {
-    named_barrier_sync(1, kCons);
-    if (threadIdx.x == 0) {
-      for (int o = 0; o < a.ks; ++o) mbar_arrive_remote(mapa_shared(smem_u32(&done), (uint32_t)o));
-      if (!mbar_wait_cluster(&done, 0, a.timeout_ns)) latch_status(a.status, PIFA_ERR_TIMEOUT);
-    }
-    named_barrier_sync(1, kCons);
-  }
+  // No CTA retires before every CTA of its cluster has made its last remote access to it: every
+  // thread of every CTA of the cluster (the producer warps included) arrives on the hardware
+  // cluster barrier after its last push or remote arrival, and leaves only once all have arrived.
+  // That barrier has no time limit, but every wait before it is bounded (after a timeout the CTA
+  // skips its waits and runs to here), so each CTA reaches it: a CTA whose wait ran out cannot
+  // retire while a late peer may still write into its shared memory.
+  if (a.ks > 1) cluster_sync_all();
 }
 
 // Once per kernel, device and size: the dynamic shared-memory limit, and the largest shared-memory
@@ -1078,6 +1076,13 @@ extern "C" int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, 
     return pifa_fail(PIFA_ERR_ALIGNMENT, "X, Wp, C and Y must be 16-byte aligned");
   if ((ldx | ldwp | ldy | (has_np ? ldc : 0)) & 7)
     return pifa_fail(PIFA_ERR_ALIGNMENT, "ldx, ldwp, ldc and ldy must be multiples of 8 elements");
+  {
+    // as pifa_forward: Y must not share a byte with an input
+    const PifaSpan y = pifa_span(Y, T, m, ldy, 2);
+    if (pifa_spans_overlap(y, pifa_span(X, T, n, ldx, 2)) || pifa_spans_overlap(y, pifa_span(Wp, r, n, ldwp, 2)) ||
+        (has_np && pifa_spans_overlap(y, pifa_span(C, m - r, r, ldc, 2))))
+      return pifa_fail(PIFA_ERR_INVALID_ARG, "Y overlaps an input");
+  }
   const PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy, PIFA_DTYPE_BF16};
   const int64_t need = kWorkspaceReserve + decode_workspace_bytes(s);
   if (need > kNoAllocScratchBytes)

@@ -48,6 +48,20 @@ struct PifaPointers {
   int64_t ws_bytes;   // bytes available at ws
 };
 
+// Byte span [lo, hi) of a row-major matrix (rows x cols used elements, pitch ld, elem bytes);
+// empty for a null base or no rows/columns. Used to reject outputs that overlap inputs.
+struct PifaSpan {
+  uintptr_t lo, hi;
+};
+inline PifaSpan pifa_span(const void* base, int64_t rows, int64_t cols, int64_t ld, int64_t elem) {
+  const uintptr_t b = reinterpret_cast<uintptr_t>(base);
+  if (!base || rows <= 0 || cols <= 0) return {0, 0};
+  return {b, b + (uintptr_t)(((rows - 1) * ld + cols) * elem)};
+}
+inline bool pifa_spans_overlap(PifaSpan a, PifaSpan b) {
+  return a.lo < a.hi && b.lo < b.hi && a.lo < b.hi && b.lo < a.hi;
+}
+
 // ---- decode (decode.cu) ----------------------------------------------------------------------
 int64_t decode_workspace_bytes(const PifaShape& s);
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream);
@@ -55,10 +69,6 @@ int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaSt
 // ---- prefill (prefill.cu) --------------------------------------------------------------------
 int64_t prefill_split_workspace_bytes(const PifaShape& s);
 int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,
-                         cudaStream_t stream);
-int64_t prefill_fused_workspace_bytes(const PifaShape& s);
-bool prefill_fused_supported(const PifaShape& s);
-int launch_prefill_fused(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,
                          cudaStream_t stream);
 
 // ---- TMA descriptors (api.cpp) ---------------------------------------------------------------

@@ -45,7 +45,7 @@ EXPORTS = (
     "pifa_variant_name", "pifa_compress", "pifa_validate_indices", "pifa_device_status",
     "pifa_status_string", "pifa_last_error", "pifa_version", "pifa_forward_decode_noalloc",
     "pifa_set_wait_timeout", "pifa_selftest_wait_timeout", "pifa_set_decode_grid", "pifa_forward_grouped",
-    "pifa_workspace_size_grouped",
+    "pifa_workspace_size_grouped", "pifa_compress_device", "pifa_compress_device_workspace_size",
 )
 
 
@@ -98,6 +98,11 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.pifa_compress.argtypes = [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _I64, _VP, _I64,
                                       ctypes.POINTER(PifaCompressInfo)]
         lib.pifa_compress.restype = ctypes.c_int
+        lib.pifa_compress_device.argtypes = [_VP, _VP, _I64, _I64, _I64, _VP, _VP, _VP, _I64, _VP, _I64, _VP, _I64,
+                                             ctypes.POINTER(PifaCompressInfo), _VP]
+        lib.pifa_compress_device.restype = ctypes.c_int
+        lib.pifa_compress_device_workspace_size.argtypes = [_I64, _I64, _I64]
+        lib.pifa_compress_device_workspace_size.restype = _I64
         lib.pifa_validate_indices.argtypes = [_VP, _VP, _I64, _I64]
         lib.pifa_validate_indices.restype = ctypes.c_int
         lib.pifa_device_status.argtypes = [_VP]
@@ -204,6 +209,42 @@ def pifa_compress(U: np.ndarray, V: np.ndarray, r: int):
                               C.ctypes.data if m > r else None, r, ctypes.byref(info))
     _check(st, "pifa_compress")
     return piv, nonpiv, Wp, C, info
+
+
+def pifa_compress_device_workspace_size(m: int, n: int, r: int) -> int:
+    v = _lib().pifa_compress_device_workspace_size(m, n, r)
+    if v < 0:
+        _check(int(v), "pifa_compress_device_workspace_size")
+    return int(v)
+
+
+def pifa_compress_device(U, V, stream=None):
+    """Algorithm 1 on the GPU in float64 (pifa_compress_device). U (m x r) and V (n x r) are CUDA
+    tensors (converted to contiguous float64 on their device). Returns (I, I^c, W_p, C, info) as
+    CUDA tensors (int32, int32, float64, float64) and the host info struct."""
+    import torch
+    if not (isinstance(U, torch.Tensor) and isinstance(V, torch.Tensor)) or U.device.type != "cuda" or V.device != U.device:
+        raise ValueError("pifa: U and V must be CUDA tensors on one device")
+    if U.dim() != 2 or V.dim() != 2 or U.shape[1] != V.shape[1]:
+        raise ValueError("pifa: U must be m x r and V n x r")
+    U = U.to(torch.float64).contiguous()
+    V = V.to(torch.float64).contiguous()
+    (m, r), n = U.shape, V.shape[0]
+    dev = U.device
+    need = pifa_compress_device_workspace_size(m, n, r)
+    ws = torch.empty(need + 256, dtype=torch.uint8, device=dev)
+    ws_ptr = ws.data_ptr() + (-ws.data_ptr()) % 256
+    piv = torch.empty(r, dtype=torch.int32, device=dev)
+    nonpiv = torch.empty(max(m - r, 1), dtype=torch.int32, device=dev)
+    Wp = torch.empty((r, n), dtype=torch.float64, device=dev)
+    C = torch.empty((max(m - r, 1), r), dtype=torch.float64, device=dev)
+    info = PifaCompressInfo()
+    st = _lib().pifa_compress_device(U.data_ptr(), V.data_ptr(), m, n, r, piv.data_ptr(),
+                                     nonpiv.data_ptr() if m > r else None, Wp.data_ptr(), n,
+                                     C.data_ptr() if m > r else None, r, ws_ptr, need, ctypes.byref(info),
+                                     _stream_ptr(stream))
+    _check(st, "pifa_compress_device")
+    return piv, nonpiv[:m - r], Wp, C[:m - r], info
 
 
 # ---- forward -------------------------------------------------------------------------------------

@@ -8,9 +8,9 @@ NaN, so a missed or stray write fails the test.
 
 Layers: the oracle's own compression where it is quick (tiny: plain greedy loop; up to
 4096 x 4096: the LAPACK pivoted-QR route); the library's host compression for the 7B MLP and
-70B q/o shapes, each of which is checked against Eq. 2 by the oracle on sampled rows; and a
-randomly drawn layer (inputs.synthetic_layer) for the 28672 x 8192 shape, whose compression
-would take minutes on the host.
+70B q/o shapes and the library's GPU compression for the 28672 x 8192 shape, each checked against
+Eq. 1 and Eq. 2 in fp64 on sampled rows; and randomly drawn layers (inputs.synthetic_layer) where
+only the kernels' tiling matters (many tiles, ragged K, grouped layers).
 """
 import functools
 
@@ -96,6 +96,24 @@ def _compressed(m, n, r, seed, source):
             err = np.linalg.norm(C[rows] @ Wp - Wnp_s) / np.linalg.norm(Wnp_s)
             assert err <= 1e-10
         assert P.pifa_validate_indices(piv, nonp, m, r) == P.PIFA_OK
+        return piv, nonp, Wp, C
+    if source == "gpu":
+        # the library's GPU compression (Algorithm 1 on the device); Eq. 1 and Eq. 2 checked in fp64
+        # on the host on sampled rows
+        Ud = torch.from_numpy(U.astype(np.float64)).to(DEV)
+        Vd = torch.from_numpy(V.astype(np.float64)).to(DEV)
+        piv_d, nonp_d, Wp_d, C_d, _ = P.pifa_compress_device(Ud, Vd)
+        piv, nonp = piv_d.cpu().numpy(), nonp_d.cpu().numpy()
+        Wp, C = Wp_d.cpu().numpy(), C_d.cpu().numpy()
+        del Ud, Vd, Wp_d, C_d
+        assert P.pifa_validate_indices(piv, nonp, m, r) == P.PIFA_OK
+        rows = inputs.random_rows(m - r, 48, seed)
+        Vd64 = V.astype(np.float64)
+        Wnp_s = U[nonp[rows]].astype(np.float64) @ Vd64.T
+        pr = inputs.random_rows(r, 16, seed)
+        Wp_ref = U[piv[pr]].astype(np.float64) @ Vd64.T
+        assert np.abs(Wp[pr] - Wp_ref).max() <= 1e-12 * np.abs(Wp_ref).max()
+        assert np.linalg.norm(C[rows] @ Wp - Wnp_s) / np.linalg.norm(Wnp_s) <= 1e-10
         return piv, nonp, Wp, C
     if source == "synthetic":
         return inputs.synthetic_layer(m, n, r, seed)
@@ -218,7 +236,9 @@ def test_llama70b_qo_persistent_grid(T):
 
 @pytest.mark.parametrize("T", [1, 8, 16, 4096])
 def test_llama70b_gate_up(T):
-    L = layer_for(28672, 8192, 4096, 0, "synthetic")
+    """The 28672 x 8192, r = 4096 layer as Algorithm 1 makes it from Gaussian U V^T (compressed on
+    the GPU): its C cancels heavily, the case that makes the hi + lo split of y_p necessary."""
+    L = layer_for(28672, 8192, 4096, 0, "gpu")
     parity(L, T, sample=128)
 
 
@@ -329,15 +349,14 @@ def test_prefill_variants_agree_with_decode_at_t16():
 
 
 # ---------------------------------------------------------------------------------------------
-# C stored as fp16: decode, split prefill (single fp16 pass) and the fused cluster kernel
+# C stored as fp16: decode and split prefill (hi + lo planes of fp16)
 # ---------------------------------------------------------------------------------------------
-FUSED = P.PIFA_VARIANT_PREFILL_FUSED
 SPLIT = P.PIFA_VARIANT_PREFILL_SPLIT
 
 
 def test_fp16_c_tiny_all_variants():
     L = layer_for(256, 256, 128, 0, "oracle_greedy", "fp16")
-    for v in (P.PIFA_VARIANT_DECODE, SPLIT, FUSED):
+    for v in (P.PIFA_VARIANT_DECODE, SPLIT):
         parity(L, 16, v)
 
 
@@ -346,36 +365,21 @@ def test_fp16_c_attn7b_decode(T):
     parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16"), T)
 
 
-def test_selector_picks_split_prefill_and_fused_still_plans():
+def test_selector_picks_split_prefill():
     assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(16, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
-    # the fused kernel is still runnable on request for this shape
-    assert P.pifa_workspace_size(2048, 4096, 4096, 2048, FUSED) > 0
-
-
-def test_bf16_c_fused_attn7b_and_ragged():
-    parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack"), 2048, FUSED)
-    L = layer_for(300, 200, 77, 3, "oracle_greedy")
-    for T in (1, 17, 300):
-        parity(L, T, FUSED)
 
 
 @pytest.mark.parametrize("T,sample", [(2048, None), (8192, 512), (300, None), (17, None)])
-def test_fp16_c_attn7b_fused(T, sample):
-    L = layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16")
-    parity(L, T, FUSED, sample=sample)
-
-
-@pytest.mark.parametrize("T", [2048])
-def test_fp16_c_attn7b_split(T):
-    parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16"), T, SPLIT)
+def test_fp16_c_attn7b_split(T, sample):
+    parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16"), T, SPLIT, sample=sample)
 
 
 @pytest.mark.parametrize("frac", [0.25, 0.4, 0.6, 0.75])
-def test_fp16_c_rank_sweep_fused(frac):
+def test_fp16_c_rank_sweep_split(frac):
     r = int(np.floor(frac * 4096 + 0.5))
-    parity(layer_for(4096, 4096, r, 0, "oracle_lapack", "fp16"), 2048, FUSED, sample=512)
+    parity(layer_for(4096, 4096, r, 0, "oracle_lapack", "fp16"), 2048, SPLIT, sample=512)
 
 
 @pytest.mark.parametrize("T", [1, 2048])
@@ -387,28 +391,28 @@ def test_fp16_c_mlp7b(T):
 @pytest.mark.parametrize("T", [16, 4096])
 def test_fp16_c_llama70b(T):
     parity(layer_for(8192, 8192, 4096, 0, "library", "fp16"), T, sample=256)
-    parity(layer_for(28672, 8192, 4096, 0, "synthetic", "fp16"), T, sample=128)
+    parity(layer_for(28672, 8192, 4096, 0, "gpu", "fp16"), T, sample=128)
 
 
 @pytest.mark.parametrize("T", [1, 17, 100, 300, 513])
-def test_fp16_c_ragged_fused_and_split(T):
+def test_fp16_c_ragged_split_and_decode(T):
     L = layer_for(300, 200, 77, 3, "oracle_greedy", "fp16")
-    for v in ([SPLIT, FUSED] if T > 16 else [P.PIFA_VARIANT_DECODE, SPLIT, FUSED]):
+    for v in ([SPLIT] if T > 16 else [P.PIFA_VARIANT_DECODE, SPLIT]):
         parity(L, T, v)
 
 
-@pytest.mark.parametrize("variant", [P.PIFA_VARIANT_DECODE, SPLIT, FUSED])
+@pytest.mark.parametrize("variant", [P.PIFA_VARIANT_DECODE, SPLIT])
 def test_fp16_c_full_rank_and_rank_one(variant):
     parity(layer_for(64, 128, 64, 4, "oracle_greedy", "fp16"), 16 if variant == P.PIFA_VARIANT_DECODE else 40,
            variant)
     parity(layer_for(40, 48, 1, 5, "oracle_greedy", "fp16"), 12, variant)
 
 
-def test_fp16_c_fused_deterministic_and_padded():
+def test_fp16_c_split_deterministic_and_padded():
     L = layer_for(4096, 4096, 2048, 0, "oracle_lapack", "fp16")
     X = acts(600, 4096, 7)
-    a = run(L, X, FUSED)
-    b = run(L, X, FUSED, ldx=4104, ldwp=4112, ldc=2056, ldy_pad=24)
+    a = run(L, X, SPLIT)
+    b = run(L, X, SPLIT, ldx=4104, ldwp=4112, ldc=2056, ldy_pad=24)
     assert np.array_equal(a, b)
 
 
@@ -427,7 +431,7 @@ def test_wait_timeout_is_reported_and_recoverable():
         assert P.pifa_device_status() == P.PIFA_OK       # read-and-clear
     finally:
         P.pifa_set_wait_timeout(0)
-    for v in (P.PIFA_VARIANT_DECODE, P.PIFA_VARIANT_PREFILL_SPLIT, P.PIFA_VARIANT_PREFILL_FUSED):
+    for v in (P.PIFA_VARIANT_DECODE, P.PIFA_VARIANT_PREFILL_SPLIT):
         parity(L, 16, v)
 
 
@@ -436,7 +440,7 @@ def test_workspace_needs_no_initialisation_and_is_shared():
     decode at several T, then prefill, then decode again: no call depends on its contents."""
     L = layer_for(300, 200, 77, 3, "oracle_greedy")
     cases = ((8, P.PIFA_VARIANT_DECODE), (1, P.PIFA_VARIANT_DECODE), (100, SPLIT), (16, P.PIFA_VARIANT_DECODE),
-             (300, FUSED), (3, P.PIFA_VARIANT_DECODE))
+             (300, SPLIT), (3, P.PIFA_VARIANT_DECODE))
     need = max(P.pifa_workspace_size(T, L.m, L.n, L.r, v) for T, v in cases)
     ws = torch.full((need,), 0xFF, dtype=torch.uint8, device=DEV)
     for T, v in cases:

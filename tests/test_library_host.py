@@ -86,11 +86,11 @@ def test_workspace_sizes(lib):
     assert P.pifa_workspace_size(8, 4096, 4096, 2048, P.PIFA_VARIANT_DECODE) == 256 + 8 * 2048 * 4
     assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) % 256 == 0
     assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) >= 256 + 3 * 1640 * 4
-    # split and fused prefill: Y_p hi and lo, two 2-byte T x round_up(r, 8) matrices
+    # split prefill: Y_p hi and lo, two 2-byte T x round_up(r, 8) matrices
     assert P.pifa_workspace_size(2048, 4096, 4096, 2048, P.PIFA_VARIANT_PREFILL_SPLIT) == 256 + 2 * 2048 * 2048 * 2
     assert P.pifa_workspace_size(2048, 4096, 4096, 2048, P.PIFA_VARIANT_PREFILL_SPLIT,
                                  P.PIFA_DTYPE_FP16) == 256 + 2 * 2048 * 2048 * 2
-    assert P.pifa_workspace_size(2048, 4096, 4096, 1638, P.PIFA_VARIANT_PREFILL_FUSED,
+    assert P.pifa_workspace_size(2048, 4096, 4096, 1638, P.PIFA_VARIANT_PREFILL_SPLIT,
                                  P.PIFA_DTYPE_FP16) == 256 + 2 * 2048 * 1640 * 2
     assert P.pifa_workspace_size(0, 4096, 4096, 2048, P.PIFA_VARIANT_AUTO) == 0
     with pytest.raises(P.PifaError) as e:

@@ -31,8 +31,8 @@ def _dev_bf16(a32):
 
 
 def _close(got, ref):
+    """The parity bar against the fp64 oracle: relative Frobenius and per-element bounds."""
     got = got.float().cpu().numpy().astype(np.float64)
-    ref = ref.float().cpu().numpy().astype(np.float64)
     rel = np.linalg.norm(got - ref) / np.linalg.norm(ref)
     elem = np.max(np.abs(got - ref) / (np.abs(ref) + 1.0))
     assert rel <= REL_FRO and elem <= ELEM, f"rel_fro {rel:.3e}, elem {elem:.3e}"
@@ -56,16 +56,31 @@ def test_noalloc_decode_matches_pifa_forward_twice():
         nd = torch.from_numpy(np.asarray(nonp, np.int32)).to(DEV)
         rng = np.random.default_rng(7)
         for T in (16, 5):                         # two calls in a row, different token counts
-            X = _dev_bf16(inputs.make_activations(rng, T, Wp32.shape[1], "bf16"))
+            X32 = inputs.make_activations(rng, T, Wp32.shape[1], "bf16")
+            X = _dev_bf16(X32)
             ref = P.pifa_forward(X, Wp, C, pd, nd, variant=P.PIFA_VARIANT_DECODE)
             got = P.pifa_forward_decode_noalloc(X, Wp, C, pd, nd)
             assert P.pifa_device_status() == P.PIFA_OK
-            _close(got, ref)
+            # same kernels, same operands: the two entry points agree bit for bit (a read of stale
+            # scratch left by the previous, larger call would show here)
+            assert torch.equal(got.view(torch.int16), ref.view(torch.int16))
+            _close(got, oracle.forward(X32, Wp32, C32, np.asarray(piv, np.int64), np.asarray(nonp, np.int64)))
+
+
+def test_noalloc_rejects_output_overlapping_an_input():
+    lib = P.load()
+    base = 0x100000                              # never dereferenced: rejected before any launch
+    # Y (4 x 64, pitch 64) placed over X (4 x 64): PIFA_ERR_INVALID_ARG, as pifa_forward
+    st = lib.pifa_forward_decode_noalloc(base, 4, 64, 64, base + 0x10000, 16, 64, base + 0x20000, 48, 16,
+                                         base + 0x30000, base + 0x31000, base + 64, 48, None)
+    assert st == P.PIFA_ERR_INVALID_ARG
+    assert "overlaps" in P.pifa_last_error()
 
 
 def test_noalloc_rejects_sizes_beyond_the_static_scratch():
     lib = P.load()
-    fake = 0x100000                              # never dereferenced: rejected before any launch
+    fake = 1 << 36                               # never dereferenced: rejected before any launch;
+    # the buffers sit 64 GiB apart, so none overlaps another
     # 256 + T * round_up(r, 8) * 4 bytes must fit in 1 MiB: r = 16392 at T = 16 does not
     st = lib.pifa_forward_decode_noalloc(fake, 16, 20000, 20000, fake * 2, 16392, 20000, fake * 3,
                                          20000, 16392, fake * 4, fake * 5, fake * 6, 20000, None)
