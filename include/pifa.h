@@ -277,6 +277,7 @@ int pifa_set_wait_timeout(int64_t ns);
 #define PIFA_DECODE_GRID_AUTO 0
 #define PIFA_DECODE_GRID_WAVES 1
 #define PIFA_DECODE_GRID_PERSISTENT 2
+#define PIFA_DECODE_GRID_SPLITK 3
 int pifa_set_decode_grid(int mode);
 
 /* pifa_selftest_wait_timeout -- enqueues on `cuda_stream` a one-CTA kernel that waits, with the

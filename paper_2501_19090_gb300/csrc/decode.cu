@@ -935,10 +935,58 @@ int launch_stream(Kern kernel, const CUtensorMap& tm, const CUtensorMap& tb0, co
 // the weights in their storage type `dtype`). The stream reads its B operand once per CTA, so its
 // tiles can be taller than decode_rows': 32 rows make 4 KB TMA boxes (2 KB boxes of 16 rows
 // issue too many copies per byte).
+// Scratch of the split-K tensor-core form (decode_tc.cu): where its partial sums go, and how many
+// bytes are available there.
+struct SplitKScratch {
+  float* P;
+  int64_t bytes;
+};
+
+// The split-K tensor-core form of one phase (decode_tc.cu) on the same operands.
+template <int PHASE, bool kF16C>
+int launch_phase_tc(const DecodeArgs& a, int dtype, const SplitKScratch& sk, cudaStream_t stream) {
+  DecodeTcPhase ph = {};
+  ph.A = a.A;
+  ph.lda = a.lda;
+  ph.R = a.R;
+  ph.K = a.K;
+  ph.dtype = dtype;
+  ph.B0 = a.B0;
+  ph.B1 = a.B1;
+  ph.ldb = a.ldb;
+  ph.bcols = a.bcols;
+  ph.T = a.T;
+  ph.planes = PHASE == 1 ? 1 : 2;
+  ph.gsz = a.gsz;
+  ph.goff = a.goff;
+  ph.mma_f16 = PHASE == 2 && kF16C;
+  ph.split_f16 = kF16C;
+  ph.P = sk.P;
+  ph.cols = a.cols;
+  ph.m = a.m;
+  ph.Y = a.Y;
+  ph.ldy = a.ldy;
+  ph.yph = a.yph;
+  ph.ypl = a.ypl;
+  ph.ldyp = a.ldyp;
+  return launch_decode_tc(ph, a.status, a.timeout_ns, stream);
+}
+
 template <int PHASE, int NT, bool kF16C, int RG, int RGS>
-int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, cudaStream_t stream) {
+int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, const SplitKScratch& sk, bool large,
+                     cudaStream_t stream) {
   constexpr int kRows = kRowsOf<RG>;
   const char* what = PHASE == 1 ? "decode phase 1 launch" : "decode phase 2 launch";
+  const int mode = g_decode_grid.load(std::memory_order_relaxed);
+  const bool tc_fits = sk.P != nullptr && decode_tc_partial_bytes(a.R, a.K, a.T, PHASE == 1 ? 1 : 2) <= sk.bytes;
+  if (mode == PIFA_DECODE_GRID_SPLITK && tc_fits) return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
+  // Auto, layers of >= 64 MiB of weights at T > 2: both phases split-K on the tensor cores
+  // (measured, 70B q/o T = 16: 27.4 us against 31.2 with phase 1 in waves).
+  if (mode == PIFA_DECODE_GRID_AUTO && large && a.T > 2 && tc_fits) return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
+  // Auto: a phase beyond two waves of decode_rows runs split-K on the tensor cores (decode_tc.cu)
+  // for T > 2, and decode_stream for T <= 2, where its resident x / y_p and short loop win
+  // (measured, 70B gate/up: T = 1 46.9 against 51.7 us; T = 8 73.3 against 54.9; T = 16 105.6
+  // against 59.6; 70B q/o T = 16 36.5 against 27.4).
   const auto kr = decode_rows<PHASE, NT, kF16C, RG>;
   plan_phase(kRows, budget, a);
   const size_t smem = smem_bytes(kRows, a, NT);
@@ -947,10 +995,10 @@ int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, cudaStream_t str
   // decode_rows in waves while a phase takes at most two of them (its weights staged at launch,
   // before the dependency wait, outweigh the persistent grid's streaming); else decode_stream
   const int tiles = (a.R + kRows - 1) / kRows;
-  const int mode = g_decode_grid.load(std::memory_order_relaxed);
   if (mode == PIFA_DECODE_GRID_WAVES ||
       (mode == PIFA_DECODE_GRID_AUTO && tiles <= 2 * max_clusters(reinterpret_cast<const void*>(kr), a.ks, smem)))
     return launch_phase(kr, kRows, a, smem, stream, what);
+  if (mode == PIFA_DECODE_GRID_AUTO && a.T > 2 && tc_fits) return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
   const auto ks = decode_stream<PHASE, NT, kF16C, RGS>;
   const size_t smem_s =
       plan_stream(reinterpret_cast<const void*>(ks), kRowsOf<RGS>, NT, PHASE == 1 ? 1 : 2, a, what, &st);
@@ -963,12 +1011,24 @@ int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, cudaStream_t str
   return launch_stream(ks, tm, tb0, tb1, a, smem_s, stream, what);
 }
 
+int64_t decode_planes_bytes(const PifaShape& s) {
+  // y_p as hi and lo planes of 2-byte elements, T rows of pitch round_up(G r, 8) each, rounded up
+  // to 256 bytes
+  return ((s.T * ((s.groups * s.r + 7) / 8 * 8) * 4 + 255) / 256) * 256;
+}
+
 template <int NT, bool kF16C, int RG, int RGS>
 int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
   const int64_t G = s.groups;                      // layers sharing X (1: one layer)
   const int64_t ldyp = (G * s.r + 7) / 8 * 8;  // 16-byte rows keep the fragment loads aligned
   uint16_t* yph = reinterpret_cast<uint16_t*>(p.ws);
   uint16_t* ypl = yph + s.T * ldyp;
+  // the split-K form's partial sums follow the planes (phase 2 reuses phase 1's: the reduction of
+  // phase 1 has completed before phase 2 writes)
+  const int64_t planes = decode_planes_bytes(s);
+  const SplitKScratch sk = {p.ws_bytes > planes ? reinterpret_cast<float*>(static_cast<uint8_t*>(p.ws) + planes) : nullptr,
+                            p.ws_bytes - planes};
+  const bool large = 2 * G * s.r * (s.n + s.m - s.r) >= ((int64_t)64 << 20);  // weight bytes of the call
   DecodeArgs a = {};
   a.A = reinterpret_cast<const uint16_t*>(p.Wp);
   a.lda = s.ldwp;
@@ -988,7 +1048,7 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   a.T = (int)s.T;
   a.status = status;
   a.timeout_ns = pifa_wait_timeout_ns();
-  int st = launch_one_phase<1, NT, kF16C, RG, RGS>(a, kStageBudget1, PIFA_DTYPE_BF16, stream);
+  int st = launch_one_phase<1, NT, kF16C, RG, RGS>(a, kStageBudget1, PIFA_DTYPE_BF16, sk, large, stream);
   if (st != PIFA_OK || s.m == s.r) return st;
   DecodeArgs b = a;
   b.A = reinterpret_cast<const uint16_t*>(p.C);
@@ -1006,22 +1066,29 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   }
   b.yph = b.ypl = nullptr;
   b.cols = p.nonpiv;
-  return launch_one_phase<2, NT, kF16C, RG, RGS>(b, kStageBudget2, (int)s.c_dtype, stream);
+  return launch_one_phase<2, NT, kF16C, RG, RGS>(b, kStageBudget2, (int)s.c_dtype, sk, large, stream);
 }
 
 }  // namespace
 
 extern "C" int pifa_set_decode_grid(int mode) {
-  if (mode != PIFA_DECODE_GRID_AUTO && mode != PIFA_DECODE_GRID_WAVES && mode != PIFA_DECODE_GRID_PERSISTENT)
-    return pifa_fail(PIFA_ERR_INVALID_ARG, "decode grid mode must be 0 (auto), 1 (waves) or 2 (persistent)");
+  if (mode != PIFA_DECODE_GRID_AUTO && mode != PIFA_DECODE_GRID_WAVES && mode != PIFA_DECODE_GRID_PERSISTENT &&
+      mode != PIFA_DECODE_GRID_SPLITK)
+    return pifa_fail(PIFA_ERR_INVALID_ARG,
+                     "decode grid mode must be 0 (auto), 1 (waves), 2 (persistent) or 3 (split-K tensor cores)");
   g_decode_grid.store(mode, std::memory_order_relaxed);
   return PIFA_OK;
 }
 
 int64_t decode_workspace_bytes(const PifaShape& s) {
-  // y_p as hi and lo planes of 2-byte elements, T rows of pitch round_up(G r, 8) each, rounded up
-  // to 256 bytes
-  return ((s.T * ((s.groups * s.r + 7) / 8 * 8) * 4 + 255) / 256) * 256;
+  // the y_p planes, then room for the split-K form's partial sums of either phase
+  const int64_t G = s.groups;
+  int64_t part = decode_tc_partial_bytes(G * s.r, s.n, s.T, 1);
+  if (s.m > s.r) {
+    const int64_t p2 = decode_tc_partial_bytes(G * (s.m - s.r), s.r, s.T, 2);
+    part = p2 > part ? p2 : part;
+  }
+  return decode_planes_bytes(s) + (part + 255) / 256 * 256;
 }
 
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream) {
@@ -1084,7 +1151,7 @@ extern "C" int pifa_forward_decode_noalloc(const void* X, int64_t T, int64_t n, 
       return pifa_fail(PIFA_ERR_INVALID_ARG, "Y overlaps an input");
   }
   const PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy, PIFA_DTYPE_BF16};
-  const int64_t need = kWorkspaceReserve + decode_workspace_bytes(s);
+  const int64_t need = kWorkspaceReserve + decode_planes_bytes(s);
   if (need > kNoAllocScratchBytes)
     return pifa_fail(PIFA_ERR_WORKSPACE,
                      "256 + T * round_up(r, 8) * 4 bytes exceeds the 1 MiB static scratch of "

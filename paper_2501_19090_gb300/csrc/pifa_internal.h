@@ -66,6 +66,33 @@ inline bool pifa_spans_overlap(PifaSpan a, PifaSpan b) {
 int64_t decode_workspace_bytes(const PifaShape& s);
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream);
 
+// ---- decode on the tensor cores, split over K (decode_tc.cu) ------------------------------------
+// One decode phase D = A B^T (A: R x K weight rows, B: T <= 16 token rows of K columns, NB = planes
+// 1 or 2) as a persistent split-K tcgen05 kernel writing fp32 partial sums P, then a reduction
+// that writes Y[t, cols[j]] (and, for phase 1, the y_p hi/lo planes).
+struct DecodeTcPhase {
+  const void* A;
+  int64_t lda, R, K;
+  int dtype;            // storage type of A and B (PIFA_DTYPE_*)
+  const void* B0;       // first (or only) B plane: T x bcols, pitch ldb
+  const void* B1;       // second plane (planes == 2)
+  int64_t ldb, bcols, T;
+  int planes;
+  int64_t gsz, goff;    // grouped layers: rows per group and B columns per group (0: one layer)
+  bool mma_f16;         // A and B fp16 (else bf16)
+  bool split_f16;       // phase 1: split y_p into fp16 hi/lo (else bf16)
+  float* P;             // partial sums, decode_tc_partial_bytes(R, K, T, planes) bytes
+  const int32_t* cols;  // output column of each weight row
+  int64_t m;            // columns of Y (index bound)
+  void* Y;
+  int64_t ldy;
+  uint16_t* yph;        // phase 1 with m > r: y_p planes (T x ldyp), else null
+  uint16_t* ypl;
+  int64_t ldyp;
+};
+int64_t decode_tc_partial_bytes(int64_t R, int64_t K, int64_t T, int NB);
+int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, cudaStream_t stream);
+
 // ---- prefill (prefill.cu) --------------------------------------------------------------------
 int64_t prefill_split_workspace_bytes(const PifaShape& s);
 int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,

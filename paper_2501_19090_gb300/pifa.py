@@ -38,6 +38,7 @@ PIFA_VARIANT_PREFILL_FUSED = 3
 PIFA_DECODE_GRID_AUTO = 0
 PIFA_DECODE_GRID_WAVES = 1
 PIFA_DECODE_GRID_PERSISTENT = 2
+PIFA_DECODE_GRID_SPLITK = 3
 
 # every symbol include/pifa.h declares
 EXPORTS = (

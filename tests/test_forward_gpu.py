@@ -269,6 +269,45 @@ def test_decode_persistent_grid_fp16_c_and_padding(T):
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
+@pytest.mark.parametrize("T", [1, 3, 8, 16])
+def test_decode_splitk_tensor_cores_ragged(T):
+    """The split-K tensor-core decode form forced on a layer with ragged K in both phases (520 and
+    264 columns: partial 64-column chunks and K-slices), a partial last 128-row block in phase 1
+    (264 rows) and many units per CTA in phase 2 (39736 rows)."""
+    L = layer_for(40000, 520, 264, 3, "synthetic")
+    P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_SPLITK)
+    try:
+        parity(L, T, P.PIFA_VARIANT_DECODE)
+    finally:
+        P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
+
+
+@pytest.mark.parametrize("T", [1, 8, 16])
+def test_decode_splitk_tensor_cores_compressed_layers(T):
+    """The split-K form on compressed layers (C that cancels): 7B attention and the 70B gate/up
+    layer, and C stored as fp16 (fp16 MMAs in phase 2, fp16 hi/lo planes) on padded pitches."""
+    P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_SPLITK)
+    try:
+        parity(layer_for(4096, 4096, 2048, 0, "oracle_lapack"), T, P.PIFA_VARIANT_DECODE)
+        parity(layer_for(28672, 8192, 4096, 0, "gpu"), T, P.PIFA_VARIANT_DECODE, sample=128)
+        parity(layer_for(3000, 1000, 600, 4, "synthetic", "fp16"), T, P.PIFA_VARIANT_DECODE,
+               ldx=1000 + 24, ldwp=1000 + 40, ldc=600 + 16)
+    finally:
+        P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
+
+
+def test_decode_splitk_deterministic_and_r_equals_m():
+    L = layer_for(4096, 4096, 2048, 0, "oracle_lapack")
+    P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_SPLITK)
+    try:
+        X = acts(16, 4096, 5)
+        assert np.array_equal(run(L, X, P.PIFA_VARIANT_DECODE), run(L, X, P.PIFA_VARIANT_DECODE))
+        parity(layer_for(64, 128, 64, 4, "oracle_greedy"), 9, P.PIFA_VARIANT_DECODE)
+        parity(layer_for(40, 48, 1, 5, "oracle_greedy"), 12, P.PIFA_VARIANT_DECODE)
+    finally:
+        P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
+
+
 # ---------------------------------------------------------------------------------------------
 # edge cases
 # ---------------------------------------------------------------------------------------------
@@ -496,7 +535,8 @@ def test_grouped_layers_match_per_layer_oracle(G, T):
 
 
 @pytest.mark.parametrize("T", [2, 8, 16])
-@pytest.mark.parametrize("grid", [P.PIFA_DECODE_GRID_PERSISTENT, P.PIFA_DECODE_GRID_WAVES])
+@pytest.mark.parametrize("grid", [P.PIFA_DECODE_GRID_PERSISTENT, P.PIFA_DECODE_GRID_WAVES,
+                                  P.PIFA_DECODE_GRID_SPLITK])
 def test_grouped_layers_both_decode_grids(T, grid):
     """Grouped decode under both layouts; the persistent grid keeps every group's K range of y_p
     resident (T <= 2) or stages the tile's group's columns (T > 2)."""
@@ -553,3 +593,54 @@ def test_grouped_layers_prefill_three_groups(T):
     """Grouped prefill, three groups: GEMM 2 tiles read their group's hi/lo column range."""
     layers = [layer_for(1408, 1000, 512, 30 + g, "synthetic") for g in range(3)]
     grouped_parity(layers, T, sample=160)
+
+
+# ---------------------------------------------------------------------------------------------
+# back-to-back calls in a CUDA graph (the chained kernels of one call overlap the next call's)
+# ---------------------------------------------------------------------------------------------
+@pytest.mark.parametrize("m,n,r,T", [(4096, 4096, 2048, 8), (8192, 8192, 4096, 1), (8192, 8192, 4096, 16),
+                                     (28672, 8192, 4096, 16), (4096, 4096, 2048, 300)])
+def test_graph_replay_back_to_back_matches_single_calls(m, n, r, T):
+    """64 calls captured in one CUDA graph and replayed, on four rotating (X, Y) pairs that share one
+    workspace: every call's kernels launch while the previous call's still run (programmatic
+    dependent launch), so a call that read the shared y_p planes or partial sums too early, or
+    wrote them too late, would change some output. Each Y must equal, bit for bit, the same call
+    made alone. Covers the wave, split-K tensor-core and persistent decode forms and the prefill."""
+    piv, nonp, Wp32, C32 = inputs.synthetic_layer(m, n, r, 40)
+    L = Layer(piv, nonp, Wp32, C32, f"{m}x{n}r{r}/graph")
+    Wp, C, pd, nd = L.dev()
+    copies = 4
+    Xs = [_pad_dev(acts(T, n, 50 + j)) for j in range(copies)]
+    Ys = [torch.full((T, m), float("nan"), dtype=torch.bfloat16, device=DEV) for _ in range(copies)]
+    ws = torch.empty(P.pifa_workspace_size(T, m, n, r) + 512, dtype=torch.uint8, device=DEV)
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    ref = []
+    for j in range(copies):
+        Yj = torch.empty((T, m), dtype=torch.bfloat16, device=DEV)
+        P.pifa_forward(Xs[j], Wp, C, pd, nd, Y=Yj, workspace_tensor=ws, stream=stream)
+        stream.synchronize()
+        ref.append(Yj)
+
+    def step(i):
+        P.pifa_forward(Xs[i % copies], Wp, C, pd, nd, Y=Ys[i % copies], workspace_tensor=ws, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for i in range(4):
+            step(i)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for i in range(64):
+            step(i)
+    for _ in range(2):
+        for Y in Ys:
+            Y.fill_(float("nan"))
+        torch.cuda.synchronize()
+        with torch.cuda.stream(stream):
+            g.replay()
+        stream.synchronize()
+        assert P.pifa_device_status(stream) == P.PIFA_OK
+        for j in range(copies):
+            assert torch.equal(Ys[j].view(torch.int16), ref[j].view(torch.int16)), f"copy {j} differs"
+    del g

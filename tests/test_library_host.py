@@ -48,11 +48,12 @@ def test_status_and_variant_strings(lib):
 
 
 def test_decode_grid_setter(lib):
-    """The decode layout knob takes the three declared modes and rejects anything else (no GPU
+    """The decode layout knob takes the four declared modes and rejects anything else (no GPU
     work: the mode only steers later launches)."""
-    for mode in (P.PIFA_DECODE_GRID_WAVES, P.PIFA_DECODE_GRID_PERSISTENT, P.PIFA_DECODE_GRID_AUTO):
+    for mode in (P.PIFA_DECODE_GRID_WAVES, P.PIFA_DECODE_GRID_PERSISTENT, P.PIFA_DECODE_GRID_SPLITK,
+                 P.PIFA_DECODE_GRID_AUTO):
         assert lib.pifa_set_decode_grid(mode) == P.PIFA_OK
-    for bad in (-1, 3, 99):
+    for bad in (-1, 4, 99):
         assert lib.pifa_set_decode_grid(bad) == P.PIFA_ERR_INVALID_ARG
     assert lib.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO) == P.PIFA_OK
 
@@ -83,9 +84,11 @@ def test_selector(lib):
 def test_workspace_sizes(lib):
     # decode: fp32 y_p, T rows of pitch round_up(r, 8)
     # every size includes the 256 reserved bytes at the head of the workspace
-    assert P.pifa_workspace_size(8, 4096, 4096, 2048, P.PIFA_VARIANT_DECODE) == 256 + 8 * 2048 * 4
+    # decode: the y_p planes (two 2-byte T x round_up(r, 8) matrices), then room for the split-K
+    # form's fp32 partial sums: at least one T x rows block per phase
+    assert P.pifa_workspace_size(8, 4096, 4096, 2048, P.PIFA_VARIANT_DECODE) >= 256 + 8 * 2048 * 4 + 8 * 2048 * 4
     assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) % 256 == 0
-    assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) >= 256 + 3 * 1640 * 4
+    assert P.pifa_workspace_size(3, 4096, 4096, 1638, P.PIFA_VARIANT_DECODE) >= 256 + 3 * 1640 * 4 + 3 * 2458 * 4
     # split prefill: Y_p hi and lo, two 2-byte T x round_up(r, 8) matrices
     assert P.pifa_workspace_size(2048, 4096, 4096, 2048, P.PIFA_VARIANT_PREFILL_SPLIT) == 256 + 2 * 2048 * 2048 * 2
     assert P.pifa_workspace_size(2048, 4096, 4096, 2048, P.PIFA_VARIANT_PREFILL_SPLIT,
