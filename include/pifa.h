@@ -250,6 +250,63 @@ int pifa_compress_device(const double* U, const double* V, int64_t m, int64_t n,
  * negative pifa_status on bad arguments. Pure host arithmetic. */
 int64_t pifa_compress_device_workspace_size(int64_t m, int64_t n, int64_t r);
 
+/*
+ * pifa_backward -- the gradients of Algorithm 2 with respect to X, W_p and C, for fine-tuning a
+ * compressed model (Sec. 5.1; the PIFA layer is differentiable, Sec. 6). With tokens as rows and
+ * dY = dL/dY (T x m): dY_p = dY[:, I] + dY[:, I^c] C, dX = dY_p W_p, dW_p = dY_p^T X,
+ * dC = dY[:, I^c]^T Y_p with Y_p = X W_p^T recomputed. The index sets are not trained.
+ *
+ *   X, Wp, C, pivot_idx, nonpivot_idx   as pifa_forward (DEVICE; C bf16).
+ *   dY           DEVICE, bf16, T x m, row pitch lddy >= m.
+ *   dX           DEVICE out, bf16, T x n, pitch lddx >= n (NULL: not computed).
+ *   dWp          DEVICE out, fp32, r x n, pitch lddwp >= n (NULL: not computed).
+ *   dC           DEVICE out, fp32, (m - r) x r, pitch lddc >= r (NULL: not computed).
+ *   workspace    DEVICE scratch of pifa_backward_workspace_size(T, m, n, r) bytes, 256-byte
+ *                aligned, no initialisation needed (dY_np, Y_p and dY_p in bf16).
+ *   Numerics: bf16 operands, fp32 accumulation; dY_p and Y_p are rounded to bf16 between the
+ *   contractions. Alignment as pifa_forward (fp32 pitches multiples of 4 elements). T == 0 writes
+ *   zero dW_p and dC. Asynchronous on cuda_stream; out-of-range indices latch
+ *   PIFA_ERR_DEVICE_INDEX (read with pifa_device_status()).
+ */
+int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx,
+                  const void* Wp, int64_t r, int64_t ldwp,
+                  const void* C, int64_t m, int64_t ldc,
+                  const int32_t* pivot_idx, const int32_t* nonpivot_idx,
+                  const void* dY, int64_t lddy,
+                  void* dX, int64_t lddx, float* dWp, int64_t lddwp, float* dC, int64_t lddc,
+                  void* workspace, int64_t workspace_bytes, void* cuda_stream);
+
+/* pifa_backward_workspace_size -- bytes of device scratch pifa_backward needs; negative pifa_status
+ * on bad arguments. Pure host arithmetic. */
+int64_t pifa_backward_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r);
+
+/*
+ * pifa_m_accumulate -- one calibration batch into the online accumulators of the M reconstruction
+ * (Sec. 4, the accumulation steps of Algorithm 3): with the dense-flow inputs X_o and the
+ * low-rank-flow inputs X_u of a layer W (m x n), tokens as rows,
+ *   XXt  += X_u^T X_u                                      (n x n: the sum of x_u x_u^T)
+ *   YtXt += Y_t^T X_u,  Y_t = (lambda X_o + (1 - lambda) X_u) W^T   (m x n: the sum of y_t x_u^T)
+ * so that any number of batches can be folded in with constant memory.
+ *
+ *   Xo, Xu       DEVICE, bf16, T x n, common row pitch ldx >= n (Xo may be NULL when YtXt is).
+ *   W            DEVICE, bf16, m x n, pitch ldw >= n (the dense weight; may be NULL when YtXt is).
+ *   lambda       mix ratio in [0, 1] (Eq. 6; the paper uses 0.25).
+ *   XXt          DEVICE in/out, fp32, n x n, pitch ldxx >= n.
+ *   YtXt         DEVICE in/out, fp32, m x n, pitch ldyx >= n (NULL: only XXt is accumulated).
+ *   workspace    DEVICE scratch of pifa_m_accumulate_workspace_size(T, m, n) bytes, 256-byte
+ *                aligned (the mixed input and Y_t in bf16); unused when YtXt is NULL.
+ *   Numerics: bf16 operands, fp32 accumulation; the mixed input and Y_t are rounded to bf16.
+ *   T == 0 is a no-op. Asynchronous on cuda_stream.
+ */
+int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int64_t n, int64_t ldx,
+                      const void* W, int64_t m, int64_t ldw, float lambda,
+                      float* XXt, int64_t ldxx, float* YtXt, int64_t ldyx,
+                      void* workspace, int64_t workspace_bytes, void* cuda_stream);
+
+/* pifa_m_accumulate_workspace_size -- bytes of device scratch pifa_m_accumulate needs; negative
+ * pifa_status on bad arguments. Pure host arithmetic. */
+int64_t pifa_m_accumulate_workspace_size(int64_t T, int64_t m, int64_t n);
+
 /* pifa_validate_indices -- HOST copies: PIFA_OK iff pivot_idx (r entries) and nonpivot_idx
  * (m - r entries) are strictly ascending, inside [0, m) and disjoint (so together a partition
  * of [0, m), as Algorithm 1 step 2 defines I^c); else PIFA_ERR_INVALID_ARG. */

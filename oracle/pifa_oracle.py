@@ -23,6 +23,11 @@ Functions and the passages they follow:
   forward              Algorithm 2 (Sec. 3.2): Y_p, Y_np and the two index assignments.
   backward             the gradients of Algorithm 2 w.r.t. X, W_p and C (fine-tuning after
                        pruning, Sec. 5.1; differentiability, Sec. 6): its steps in reverse.
+  m_accumulate         Algorithm 3 (MPIFA), part 1, the two accumulation steps (Sec. 4): the sums
+                       of x_u x_u^T and of y_t x_u^T over calibration samples, y_t the mixed target
+                       of Eq. 6 (lambda W x_o + (1 - lambda) W x_u), one sample at a time.
+  m_reconstruct        Algorithm 3, part 1, the two reconstruction steps: U_r by Eq. 4 (the online
+                       form of Eq. 3) and V_r^T by Eq. 8 (Eq. 7 with the alpha regulariser).
   storage_count        Sec. 3.3 (memory cost): r(m+n) - r^2 (+ r indices).
   flop_count           Sec. 3.3 (computational cost): 2 b r (m + n - r).
   dense_forward, lowrank_forward  the two comparison layers of Sec. 3.3 (Y = W X, Y = U V^T X).
@@ -253,6 +258,58 @@ def backward(X, Wp, C, pivots, nonpivots, dY):
     dWp = dYp.T @ X                    # step 2 reversed
     dX = dYp @ Wp
     return dX, dWp, dC
+
+
+# ---------------------------------------------------------------------------------------------
+# Sec. 4 / Algorithm 3: the online accumulators of the M reconstruction and its two solves
+# ---------------------------------------------------------------------------------------------
+def m_accumulate(Xo, Xu, W, lam, XXt=None, YtXt=None, rows=None):
+    """The accumulation steps of Algorithm 3 over one calibration batch, in float64.
+
+    Rows of Xo and Xu are samples (the paper's columns x_o^i, x_u^i of X_o, X_u); W is the dense
+    m x n weight. For every sample i, in order:
+      XXt  += x_u^i (x_u^i)^T                                        (n x n)
+      YtXt += (lambda W x_o^i + (1 - lambda) W x_u^i) (x_u^i)^T      (m x n; Eq. 6 target)
+    Existing accumulators are continued (the online form: memory independent of the sample count).
+    `rows` restricts both accumulators to those rows (for large shapes); the result then has
+    len(rows) rows. Returns (XXt, YtXt).
+    """
+    Xo = np.asarray(Xo, dtype=np.float64)
+    Xu = np.asarray(Xu, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    n, m = Xu.shape[1], W.shape[0]
+    rx = np.arange(n) if rows is None else np.asarray(rows[0])
+    ry = np.arange(m) if rows is None else np.asarray(rows[1])
+    XXt = np.zeros((rx.size, n)) if XXt is None else np.array(XXt, dtype=np.float64, copy=True)
+    YtXt = np.zeros((ry.size, n)) if YtXt is None else np.array(YtXt, dtype=np.float64, copy=True)
+    for i in range(Xu.shape[0]):
+        xu, xo = Xu[i], Xo[i]
+        XXt += np.outer(xu[rx], xu)
+        yt = lam * (W[ry] @ xo) + (1.0 - lam) * (W[ry] @ xu)
+        YtXt += np.outer(yt, xu)
+    return XXt, YtXt
+
+
+def m_reconstruct(XXt, YtXt, V, W=None, alpha=0.0):
+    """The reconstruction steps of Algorithm 3 from the accumulators, in float64.
+
+    U_r = (Y_t X^T) V (V^T (X X^T) V)^{-1}                                      (Eq. 4)
+    V_r^T = (U_r^T U_r)^{-1} U_r^T (Y_t X^T + alpha W) (X X^T + alpha I)^{-1}   (Eq. 8; alpha = 0
+                                                                                  gives Eq. 7)
+    V is n x r (the paper's V, W ~ U V^T). Returns (U_r (m x r), V_r (n x r)); linear solves, no
+    explicit inverses.
+    """
+    XXt = np.asarray(XXt, dtype=np.float64)
+    YtXt = np.asarray(YtXt, dtype=np.float64)
+    V = np.asarray(V, dtype=np.float64)
+    S = V.T @ XXt @ V                                  # r x r
+    U_r = np.linalg.solve(S.T, (YtXt @ V).T).T        # (Y_t X^T V) S^{-1}
+    n = XXt.shape[0]
+    rhs = YtXt + (alpha * np.asarray(W, dtype=np.float64) if alpha else 0.0)
+    G = XXt + alpha * np.eye(n)
+    left = np.linalg.solve(U_r.T @ U_r, U_r.T @ rhs)   # (U_r^T U_r)^{-1} U_r^T (...)   r x n
+    Vt = np.linalg.solve(G.T, left.T).T                 # (...) (X X^T + alpha I)^{-1}
+    return U_r, Vt.T
 
 
 def dense_forward(X, W) -> np.ndarray:

@@ -1,0 +1,275 @@
+// backward.cu -- the gradients of a PIFA layer (fine-tuning after compression, Sec. 5.1; the layer
+// is differentiable, Sec. 6) and the online accumulators of the M reconstruction (Sec. 4; the
+// accumulation steps of Algorithm 3), as tensor-core contractions (gemm_tc.cu) plus a column gather.
+//
+// Backward, tokens as rows (Y = X W'^T, Y_p = X W_p^T, Y_np = Y_p C^T), given dY = dL/dY:
+//   dY_np = dY[:, I^c]                       gather                 (Algorithm 2, step 5, reversed)
+//   dY_p  = dY[:, I] + dY_np C               T x r,  K = m - r      (steps 4 and 3, reversed)
+//   dX    = dY_p W_p                         T x n,  K = r          (step 2, reversed)
+// dY_p and Y_p are kept as hi + lo pairs of bf16 planes: in exact arithmetic dX = dY W', and the
+// route through dY_p (amplified by C, then contracted with W_p) would otherwise lose the bits that
+// cancel -- the same effect that makes the forward pass carry Y_p as hi + lo; dW_p and dC show it
+// in their small entries.
+//   dW_p  = dY_p^T X                         r x n,  K = T
+//   dC    = dY_np^T Y_p,  Y_p = X W_p^T      (m - r) x r,  K = T    (step 3, reversed)
+// M accumulators for one calibration batch (X_o the dense data flow, X_u the low-rank one):
+//   Y_t  = (lambda X_o + (1 - lambda) X_u) W^T          T x m   (the mixed target, Eq. 6)
+// The mixed input and Y_t are carried as hi + lo bf16 pairs: each feeds a contraction whose sums
+// cancel, and a single bf16 rounding of them shows in Y_t X^T's small entries.
+//   XXt += X_u^T X_u                                    n x n   (x x^T summed over the batch)
+//   YtXt += Y_t^T X_u                                   m x n   (Y_t X^T summed over the batch)
+#include <cuda_bf16.h>
+
+#include "pifa.h"
+#include "pifa_internal.h"
+#include "ptx.cuh"
+
+namespace {
+
+using namespace pifa;
+using bf16 = __nv_bfloat16;
+
+int64_t pad8(int64_t v) { return (v + 7) / 8 * 8; }
+int64_t a256(int64_t b) { return (b + 255) / 256 * 256; }
+
+// out[t][i] = in[t][idx[i]] for t < T, i < cnt (bf16); an index outside [0, bound) writes 0 and
+// latches PIFA_ERR_DEVICE_INDEX.
+__global__ void gather_cols(const bf16* in, int64_t ldin, const int32_t* idx, int cnt, int bound, int T, bf16* out,
+                            int64_t ldout, int* status) {
+  pdl_launch_dependents();
+  pdl_wait_primary();
+  const int64_t n = (int64_t)T * cnt;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+    const int t = (int)(e / cnt), i = (int)(e % cnt);
+    const int c = idx[i];
+    bf16 v = __float2bfloat16_rn(0.0f);
+    if ((unsigned)c < (unsigned)bound)
+      v = in[(int64_t)t * ldin + c];
+    else
+      latch_status(status, PIFA_ERR_DEVICE_INDEX);
+    out[(int64_t)t * ldout + i] = v;
+  }
+}
+
+// out = a * x + b * y elementwise over T rows of n (bf16 in, fp32 arithmetic), written as a hi +
+// lo pair of bf16 planes.
+__global__ void axpby_rows(const bf16* x, const bf16* y, int64_t ld, int T, int n, float a, float b, bf16* out,
+                           bf16* out_lo, int64_t ldout) {
+  pdl_launch_dependents();
+  pdl_wait_primary();
+  const int64_t tot = (int64_t)T * n;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < tot; e += (int64_t)gridDim.x * blockDim.x) {
+    const int t = (int)(e / n), c = (int)(e % n);
+    const float v = a * __bfloat162float(x[(int64_t)t * ld + c]) + b * __bfloat162float(y[(int64_t)t * ld + c]);
+    const bf16 h = __float2bfloat16_rn(v);
+    out[(int64_t)t * ldout + c] = h;
+    out_lo[(int64_t)t * ldout + c] = __float2bfloat16_rn(v - __bfloat162float(h));
+  }
+}
+
+int launch_small(const void* fn, void** args, int64_t work, cudaStream_t stream, const char* what) {
+  cudaLaunchConfig_t cfg = {};
+  const int64_t blocks = (work + 255) / 256;
+  cfg.gridDim = dim3((unsigned)(blocks < 4 * 152 ? (blocks > 0 ? blocks : 1) : 4 * 152));
+  cfg.blockDim = dim3(256);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelExC(&cfg, fn, args);
+  return e == cudaSuccess ? PIFA_OK : pifa_fail_cuda(what, e);
+}
+
+bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+struct BwdLayout {
+  int64_t dynp, yp, yp_lo, dyp, dyp_lo, total;
+};
+
+BwdLayout bwd_layout(int64_t T, int64_t m, int64_t r) {
+  BwdLayout L;
+  int64_t o = 0;
+  L.dynp = o;
+  o += a256(T * pad8(m - r > 0 ? m - r : 1) * 2);
+  L.yp = o;
+  o += a256(T * pad8(r) * 2);
+  L.yp_lo = o;
+  o += a256(T * pad8(r) * 2);
+  L.dyp = o;
+  o += a256(T * pad8(r) * 2);
+  L.dyp_lo = o;
+  o += a256(T * pad8(r) * 2);
+  L.total = o;
+  return L;
+}
+
+struct MaccLayout {
+  int64_t xmix, xmix_lo, yt, yt_lo, total;
+};
+
+MaccLayout macc_layout(int64_t T, int64_t m, int64_t n) {
+  MaccLayout L;
+  L.xmix = 0;
+  L.xmix_lo = a256(T * pad8(n) * 2);
+  L.yt = 2 * L.xmix_lo;
+  L.yt_lo = L.yt + a256(T * pad8(m) * 2);
+  L.total = L.yt_lo + a256(T * pad8(m) * 2);
+  return L;
+}
+
+}  // namespace
+
+extern "C" int64_t pifa_backward_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r) {
+  pifa_clear_error();
+  if (T < 0 || m < 1 || n < 1 || r < 1 || r > m || r > n) return pifa_fail(PIFA_ERR_INVALID_ARG, "need T >= 0 and 1 <= r <= min(m, n)");
+  return bwd_layout(T, m, r).total;
+}
+
+extern "C" int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,
+                             const void* C, int64_t m, int64_t ldc, const int32_t* pivot_idx,
+                             const int32_t* nonpivot_idx, const void* dY, int64_t lddy, void* dX, int64_t lddx,
+                             float* dWp, int64_t lddwp, float* dC, int64_t lddc, void* workspace,
+                             int64_t workspace_bytes, void* cuda_stream) {
+  pifa_clear_error();
+  if (T < 0 || m < 1 || n < 1 || r < 1 || r > m || r > n || T >= (1 << 30) || m >= (1 << 30) || n >= (1 << 30))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "need T >= 0 and 1 <= r <= min(m, n) < 2^30");
+  const bool has_np = m > r;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(cuda_stream);
+  if (!Wp || !pivot_idx || (has_np && (!C || !nonpivot_idx)))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "null Wp, C, pivot_idx or nonpivot_idx");
+  if (ldwp < n || (has_np && ldc < r)) return pifa_fail(PIFA_ERR_INVALID_ARG, "leading dimension smaller than the row");
+  if ((dX && lddx < n) || (dWp && lddwp < n) || (dC && lddc < r))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "output leading dimension smaller than the row");
+  if (T == 0) {  // no tokens: zero weight gradients
+    cudaError_t e = cudaSuccess;
+    if (dWp) e = cudaMemset2DAsync(dWp, lddwp * 4, 0, n * 4, r, s);
+    if (e == cudaSuccess && dC && has_np) e = cudaMemset2DAsync(dC, lddc * 4, 0, r * 4, m - r, s);
+    return e == cudaSuccess ? PIFA_OK : pifa_fail_cuda("backward: zero gradients", e);
+  }
+  if (!X || !dY) return pifa_fail(PIFA_ERR_INVALID_ARG, "null X or dY");
+  if (ldx < n || lddy < m) return pifa_fail(PIFA_ERR_INVALID_ARG, "leading dimension smaller than the row");
+  if (!al16(X) || !al16(Wp) || !al16(dY) || (has_np && !al16(C)) || (dX && !al16(dX)) || (dWp && !al16(dWp)) ||
+      (dC && !al16(dC)) || ((ldx | ldwp | lddy | (has_np ? ldc : 0) | (dX ? lddx : 0)) & 7) ||
+      ((dWp ? lddwp : 0) & 3) || ((dC ? lddc : 0) & 3))
+    return pifa_fail(PIFA_ERR_ALIGNMENT, "16-byte aligned buffers and 16-byte row pitches required");
+  const BwdLayout Ly = bwd_layout(T, m, r);
+  if (!workspace || workspace_bytes < Ly.total) return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or too small");
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u) return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  cudaError_t ce = cudaSuccess;
+  int* status = pifa_status_word(&ce);
+  if (!status) return pifa_fail_cuda("device status word", ce);
+  const uint64_t tmo = pifa_wait_timeout_ns();
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  bf16* dYnp = reinterpret_cast<bf16*>(ws + Ly.dynp);
+  bf16* Yp = reinterpret_cast<bf16*>(ws + Ly.yp);
+  bf16* Yp_lo = reinterpret_cast<bf16*>(ws + Ly.yp_lo);
+  bf16* dYp = reinterpret_cast<bf16*>(ws + Ly.dyp);
+  bf16* dYp_lo = reinterpret_cast<bf16*>(ws + Ly.dyp_lo);
+  const int64_t ldnp = pad8(m - r > 0 ? m - r : 1), ldr = pad8(r);
+  int st;
+  int Ti = (int)T, mi = (int)m;
+  // dY_np = dY[:, I^c]
+  if (has_np) {
+    int cnt = (int)(m - r);
+    void* args[] = {(void*)&dY, (void*)&lddy, (void*)&nonpivot_idx, (void*)&cnt, (void*)&mi, (void*)&Ti,
+                    (void*)&dYnp, (void*)&ldnp, (void*)&status};
+    if ((st = launch_small((const void*)gather_cols, args, T * (m - r), s, "backward: gather")) != PIFA_OK) return st;
+  }
+  // Y_p = X W_p^T as hi + lo planes (only dC needs it)
+  if (dC && has_np) {
+    GemmTc g = {T, r, n, X, ldx, false, Wp, ldwp, false, Yp, ldr, 3, 1.0f, nullptr, nullptr, 0, 0};
+    g.D2 = Yp_lo;
+    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+  }
+  // dY_p = dY[:, I] + dY_np C, as hi + lo planes
+  if (has_np) {
+    GemmTc g = {T, r, m - r, dYnp, ldnp, false, C, ldc, true, dYp, ldr, 3, 1.0f, dY, pivot_idx, lddy, m};
+    g.D2 = dYp_lo;
+    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+  } else {
+    int cnt = (int)r;
+    void* args[] = {(void*)&dY, (void*)&lddy, (void*)&pivot_idx, (void*)&cnt, (void*)&mi, (void*)&Ti,
+                    (void*)&dYp, (void*)&ldr, (void*)&status};
+    if ((st = launch_small((const void*)gather_cols, args, T * r, s, "backward: gather")) != PIFA_OK) return st;
+  }
+  if (dX) {  // dX = (dY_p,hi + dY_p,lo) W_p  (dY_p exact in bf16 when r == m)
+    GemmTc g = {T, n, r, dYp, ldr, false, Wp, ldwp, true, dX, lddx, 0, 1.0f, nullptr, nullptr, 0, 0};
+    if (has_np) g.A2 = dYp_lo;
+    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+  }
+  if (dWp) {  // dW_p = (dY_p,hi + dY_p,lo)^T X
+    GemmTc g = {r, n, T, dYp, ldr, true, X, ldx, true, dWp, lddwp, 1, 1.0f, nullptr, nullptr, 0, 0};
+    if (has_np) g.A2 = dYp_lo;
+    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+  }
+  if (dC && has_np) {  // dC = dY_np^T (Y_p,hi + Y_p,lo)
+    GemmTc g = {m - r, r, T, dYnp, ldnp, true, Yp, ldr, true, dC, lddc, 1, 1.0f, nullptr, nullptr, 0, 0};
+    g.B2 = Yp_lo;
+    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+  }
+  return PIFA_OK;
+}
+
+extern "C" int64_t pifa_m_accumulate_workspace_size(int64_t T, int64_t m, int64_t n) {
+  pifa_clear_error();
+  if (T < 0 || m < 1 || n < 1) return pifa_fail(PIFA_ERR_INVALID_ARG, "need T >= 0, m >= 1, n >= 1");
+  return macc_layout(T, m, n).total;
+}
+
+extern "C" int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int64_t n, int64_t ldx, const void* W,
+                                 int64_t m, int64_t ldw, float lambda, float* XXt, int64_t ldxx, float* YtXt,
+                                 int64_t ldyx, void* workspace, int64_t workspace_bytes, void* cuda_stream) {
+  pifa_clear_error();
+  if (T < 0 || m < 1 || n < 1 || T >= (1 << 30) || m >= (1 << 30) || n >= (1 << 30))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "need T >= 0 and 1 <= m, n < 2^30");
+  if (!(lambda >= 0.0f && lambda <= 1.0f)) return pifa_fail(PIFA_ERR_INVALID_ARG, "lambda must be in [0, 1]");
+  if (T == 0) return PIFA_OK;  // nothing to accumulate
+  if (!Xu || !XXt || (YtXt && (!W || !Xo))) return pifa_fail(PIFA_ERR_INVALID_ARG, "null Xu, XXt, or W / Xo with YtXt");
+  if (ldx < n || ldxx < n || (YtXt && (ldw < n || ldyx < n)))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "leading dimension smaller than the row");
+  if (!al16(Xu) || !al16(XXt) || (YtXt && (!al16(Xo) || !al16(W) || !al16(YtXt))) || (ldx & 7) || (ldxx & 3) ||
+      (YtXt && ((ldw & 7) || (ldyx & 3))))
+    return pifa_fail(PIFA_ERR_ALIGNMENT, "16-byte aligned buffers and 16-byte row pitches required");
+  const MaccLayout Ly = macc_layout(T, m, n);
+  if (YtXt && (!workspace || workspace_bytes < Ly.total)) return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or too small");
+  if (YtXt && (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  cudaError_t ce = cudaSuccess;
+  int* status = pifa_status_word(&ce);
+  if (!status) return pifa_fail_cuda("device status word", ce);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(cuda_stream);
+  const uint64_t tmo = pifa_wait_timeout_ns();
+  int st;
+  {  // XXt += X_u^T X_u
+    GemmTc g = {n, n, T, Xu, ldx, true, Xu, ldx, true, XXt, ldxx, 2, 1.0f, nullptr, nullptr, 0, 0};
+    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+  }
+  if (!YtXt) return PIFA_OK;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  bf16* Xmix = reinterpret_cast<bf16*>(ws + Ly.xmix);
+  bf16* Xmix_lo = reinterpret_cast<bf16*>(ws + Ly.xmix_lo);
+  bf16* Yt = reinterpret_cast<bf16*>(ws + Ly.yt);
+  bf16* Yt_lo = reinterpret_cast<bf16*>(ws + Ly.yt_lo);
+  const int64_t ldn = pad8(n), ldm = pad8(m);
+  {  // X_mix = lambda X_o + (1 - lambda) X_u
+    int Ti = (int)T, ni = (int)n;
+    float a = lambda, b = 1.0f - lambda;
+    void* args[] = {(void*)&Xo, (void*)&Xu, (void*)&ldx, (void*)&Ti, (void*)&ni, (void*)&a, (void*)&b, (void*)&Xmix,
+                    (void*)&Xmix_lo, (void*)&ldn};
+    if ((st = launch_small((const void*)axpby_rows, args, T * n, s, "m_accumulate: mix")) != PIFA_OK) return st;
+  }
+  {  // Y_t = (X_mix,hi + X_mix,lo) W^T, as hi + lo planes
+    GemmTc g = {T, m, n, Xmix, ldn, false, W, ldw, false, Yt, ldm, 3, 1.0f, nullptr, nullptr, 0, 0};
+    g.A2 = Xmix_lo;
+    g.D2 = Yt_lo;
+    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+  }
+  {  // YtXt += (Y_t,hi + Y_t,lo)^T X_u
+    GemmTc g = {m, n, T, Yt, ldm, true, Xu, ldx, true, YtXt, ldyx, 2, 1.0f, nullptr, nullptr, 0, 0};
+    g.A2 = Yt_lo;
+    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+  }
+  return PIFA_OK;
+}

@@ -93,6 +93,37 @@ struct DecodeTcPhase {
 int64_t decode_tc_partial_bytes(int64_t R, int64_t K, int64_t T, int NB);
 int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, cudaStream_t stream);
 
+// ---- general tensor-core contraction (gemm_tc.cu) ------------------------------------------------
+// D (M x N) = alpha A B^T (+ addend), bf16 operands, fp32 accumulation. A is M x K, B is N x K; each
+// is K-major (a_mn = false: element (i, k) at [i * ld + k]) or MN-major (true: at [k * ld + i]).
+// out_mode 0: D bf16; 1: D fp32; 2: D fp32 += result; 3: D = bf16 hi, D2 = bf16 lo of the result.
+// A2 / B2 (optional, A's / B's layout and pitch): a second K pass with A2 for A and / or B2 for B,
+// D = (A + A2) B^T or A (B + B2)^T. Optional addend:
+// D[i][j] += add[i * ldadd + (add_idx ? add_idx[j] : j)] (bf16; add_idx values must lie in
+// [0, add_bound)). Pointers 16-byte aligned, leading dimensions multiples of 8 elements (the caller
+// checks).
+struct GemmTc {
+  int64_t M, N, K;
+  const void* A;
+  int64_t lda;
+  bool a_mn;
+  const void* B;
+  int64_t ldb;
+  bool b_mn;
+  void* D;
+  int64_t ldd;
+  int out_mode;
+  float alpha;
+  const void* add;
+  const int32_t* add_idx;
+  int64_t ldadd;
+  int64_t add_bound;
+  const void* A2 = nullptr;
+  const void* B2 = nullptr;
+  void* D2 = nullptr;
+};
+int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stream);
+
 // ---- prefill (prefill.cu) --------------------------------------------------------------------
 int64_t prefill_split_workspace_bytes(const PifaShape& s);
 int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status, uint64_t timeout_ns,

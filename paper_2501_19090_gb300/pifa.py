@@ -47,6 +47,7 @@ EXPORTS = (
     "pifa_status_string", "pifa_last_error", "pifa_version", "pifa_forward_decode_noalloc",
     "pifa_set_wait_timeout", "pifa_selftest_wait_timeout", "pifa_set_decode_grid", "pifa_forward_grouped",
     "pifa_workspace_size_grouped", "pifa_compress_device", "pifa_compress_device_workspace_size",
+    "pifa_backward", "pifa_backward_workspace_size", "pifa_m_accumulate", "pifa_m_accumulate_workspace_size",
 )
 
 
@@ -104,6 +105,16 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.pifa_compress_device.restype = ctypes.c_int
         lib.pifa_compress_device_workspace_size.argtypes = [_I64, _I64, _I64]
         lib.pifa_compress_device_workspace_size.restype = _I64
+        lib.pifa_backward.argtypes = [_VP, _I64, _I64, _I64, _VP, _I64, _I64, _VP, _I64, _I64, _VP, _VP, _VP, _I64,
+                                      _VP, _I64, _VP, _I64, _VP, _I64, _VP, _I64, _VP]
+        lib.pifa_backward.restype = ctypes.c_int
+        lib.pifa_backward_workspace_size.argtypes = [_I64, _I64, _I64, _I64]
+        lib.pifa_backward_workspace_size.restype = _I64
+        lib.pifa_m_accumulate.argtypes = [_VP, _VP, _I64, _I64, _I64, _VP, _I64, _I64, ctypes.c_float, _VP, _I64,
+                                          _VP, _I64, _VP, _I64, _VP]
+        lib.pifa_m_accumulate.restype = ctypes.c_int
+        lib.pifa_m_accumulate_workspace_size.argtypes = [_I64, _I64, _I64]
+        lib.pifa_m_accumulate_workspace_size.restype = _I64
         lib.pifa_validate_indices.argtypes = [_VP, _VP, _I64, _I64]
         lib.pifa_validate_indices.restype = ctypes.c_int
         lib.pifa_device_status.argtypes = [_VP]
@@ -422,3 +433,79 @@ def pifa_forward_decode_noalloc(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, strea
         Y.data_ptr(), _ld(Y), _stream_ptr(stream))
     _check(st, "pifa_forward_decode_noalloc")
     return Y
+
+
+def pifa_backward(X, Wp, C, pivot_idx, nonpivot_idx, dY, want=("dX", "dWp", "dC"), workspace_tensor=None,
+                  stream=None):
+    """Gradients of the forward pass through pifa_backward: returns (dX bf16 T x n, dW_p fp32 r x n,
+    dC fp32 (m-r) x r), each None unless named in `want`. Tensors as pifa_forward (C bf16); dY is
+    a bf16 CUDA tensor T x m."""
+    import torch
+    T, n, r, m = _operands(1, X, Wp, C, pivot_idx, nonpivot_idx, None, workspace_tensor, c_fp16_ok=False)
+    if not isinstance(dY, torch.Tensor) or dY.dtype != torch.bfloat16 or tuple(dY.shape) != (T, m) or dY.device != X.device:
+        raise ValueError(f"pifa: dY must be a bfloat16 tensor of shape {(T, m)} on {X.device}")
+    dev = X.device
+    has_np = m > r
+    def out(rows, cols, dtype, per16):  # row pitch a multiple of 16 bytes; returns the rows x cols view
+        ld = (cols + per16 - 1) // per16 * per16
+        return torch.empty((rows, ld), dtype=dtype, device=dev)[:, :cols]
+
+    dX = out(T, n, torch.bfloat16, 8) if "dX" in want else None
+    dWp = out(r, n, torch.float32, 4) if "dWp" in want else None
+    dC = out(m - r, r, torch.float32, 4) if ("dC" in want and has_np) else None
+    need = int(_lib().pifa_backward_workspace_size(T, m, n, r))
+    if need < 0:
+        _check(need, "pifa_backward_workspace_size")
+    ws = workspace_tensor if workspace_tensor is not None else workspace(need, dev, stream, tag="backward")
+    ws_ptr = ws.data_ptr() + (-ws.data_ptr()) % 256
+    ws_bytes = ws.numel() * ws.element_size() - (ws_ptr - ws.data_ptr())
+    st = _lib().pifa_backward(
+        X.data_ptr(), T, n, _ld(X), Wp.data_ptr(), r, _ld(Wp), C.data_ptr() if has_np else None, m,
+        _ld(C) if has_np else r, pivot_idx.data_ptr(), nonpivot_idx.data_ptr() if has_np else None,
+        dY.data_ptr(), _ld(dY), dX.data_ptr() if dX is not None else None, _ld(dX) if dX is not None else n,
+        dWp.data_ptr() if dWp is not None else None, _ld(dWp) if dWp is not None else n,
+        dC.data_ptr() if dC is not None else None, _ld(dC) if dC is not None else r,
+        ws_ptr, ws_bytes, _stream_ptr(stream))
+    _check(st, "pifa_backward")
+    return dX, dWp, dC
+
+
+def pifa_m_accumulate(Xo, Xu, W, lam, XXt, YtXt=None, workspace_tensor=None, stream=None):
+    """One calibration batch into the M accumulators (pifa_m_accumulate): XXt (fp32 n x n) and
+    YtXt (fp32 m x n, optional) are updated in place. Xo, Xu bf16 T x n; W bf16 m x n."""
+    import torch
+    for name, t in (("Xu", Xu), ("XXt", XXt)):
+        if not isinstance(t, torch.Tensor) or t.device.type != "cuda":
+            raise ValueError(f"pifa: {name} must be a CUDA tensor")
+    if Xu.dtype != torch.bfloat16 or Xu.dim() != 2:
+        raise ValueError("pifa: Xu must be a 2-D bfloat16 tensor")
+    T, n = Xu.shape
+    if XXt.dtype != torch.float32 or tuple(XXt.shape) != (n, n):
+        raise ValueError(f"pifa: XXt must be a float32 tensor of shape {(n, n)}")
+    m = 1
+    if YtXt is not None:
+        if Xo is None or W is None or Xo.dtype != torch.bfloat16 or tuple(Xo.shape) != (T, n) or _ld(Xo) != _ld(Xu):
+            raise ValueError("pifa: Xo must be a bfloat16 tensor shaped and strided like Xu")
+        if W.dtype != torch.bfloat16 or W.dim() != 2 or W.shape[1] != n:
+            raise ValueError("pifa: W must be a bfloat16 m x n tensor")
+        m = W.shape[0]
+        if YtXt.dtype != torch.float32 or tuple(YtXt.shape) != (m, n):
+            raise ValueError(f"pifa: YtXt must be a float32 tensor of shape {(m, n)}")
+        for name, t in (("Xo", Xo), ("W", W), ("YtXt", YtXt)):
+            if t.device != Xu.device:
+                raise ValueError(f"pifa: {name} is on {t.device}, Xu on {Xu.device}")
+    if XXt.device != Xu.device:
+        raise ValueError("pifa: XXt must be on Xu's device")
+    need = int(_lib().pifa_m_accumulate_workspace_size(T, m, n))
+    if need < 0:
+        _check(need, "pifa_m_accumulate_workspace_size")
+    ws = workspace_tensor if workspace_tensor is not None else workspace(need, Xu.device, stream, tag="macc")
+    ws_ptr = ws.data_ptr() + (-ws.data_ptr()) % 256
+    ws_bytes = ws.numel() * ws.element_size() - (ws_ptr - ws.data_ptr())
+    st = _lib().pifa_m_accumulate(
+        Xo.data_ptr() if YtXt is not None else None, Xu.data_ptr(), T, n, _ld(Xu),
+        W.data_ptr() if YtXt is not None else None, m, _ld(W) if YtXt is not None else n, float(lam),
+        XXt.data_ptr(), _ld(XXt), YtXt.data_ptr() if YtXt is not None else None,
+        _ld(YtXt) if YtXt is not None else n, ws_ptr, ws_bytes, _stream_ptr(stream))
+    _check(st, "pifa_m_accumulate")
+    return XXt, YtXt

@@ -233,6 +233,8 @@ def _header_prototypes():
             return "i32"
         if "double" in words:
             return "f64"
+        if "float" in words:
+            return "f32"
         raise AssertionError(f"unmapped C type: {decl!r}")
 
     out = {}
@@ -257,6 +259,8 @@ def test_binding_argtypes_match_the_header(lib):
             return "i32"
         if t is ctypes.c_double:
             return "f64"
+        if t is ctypes.c_float:
+            return "f32"
         if t in (ctypes.c_void_p, ctypes.c_char_p) or (isinstance(t, type) and issubclass(t, ctypes._Pointer)):
             return "ptr"
         raise AssertionError(f"unmapped ctypes type {t}")

@@ -1,0 +1,146 @@
+"""GPU parity of the training-side paths through the C ABI, against the fp64 oracle:
+
+* pifa_backward -- the gradients of Algorithm 2 (fine-tuning, Sec. 5.1; Sec. 6): dX, dW_p, dC
+  against oracle.backward on the same bf16 operands;
+* pifa_m_accumulate -- the online accumulators of the M reconstruction (Sec. 4, Algorithm 3):
+  X X^T and Y_t X^T against oracle.m_accumulate, over two batches in a row (the online form).
+
+Tolerance as the forward pass: relative Frobenius error <= 5e-3 and |err| <= 2e-2 (|ref| + 1) per
+element (bf16 operands, fp32 accumulation, bf16 intermediates).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2501_19090_gb300 import inputs
+from paper_2501_19090_gb300 import pifa as P
+
+pytestmark = pytest.mark.gpu
+DEV = torch.device("cuda:0")
+REL_FRO = 5e-3
+ELEM = 2e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    P.load()
+
+
+def check(got, ref, what):
+    got = np.asarray(got, dtype=np.float64)
+    rel = np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-300)
+    elem = np.max(np.abs(got - ref) / (np.abs(ref) + 1.0)) if ref.size else 0.0
+    assert rel <= REL_FRO and elem <= ELEM, f"{what}: rel_fro {rel:.3e}, elem {elem:.3e}"
+
+
+def dev_bf16(a32):
+    rows, cols = a32.shape
+    ld = (cols + 7) // 8 * 8
+    buf = torch.full((rows, ld), float("nan"), dtype=torch.bfloat16, device=DEV)
+    buf[:, :cols] = torch.from_numpy(np.ascontiguousarray(a32, dtype=np.float32)).to(DEV).to(torch.bfloat16)
+    return buf[:, :cols]
+
+
+def compressed(m, n, r, seed, route):
+    U, V, _ = inputs.make_factors(m, n, r, seed)
+    L = oracle.compress(U, V, r, route)
+    return L.pivots, L.nonpivots, inputs.round_bf16(L.Wp), inputs.round_bf16(L.C)
+
+
+CASES = [
+    ("tiny 256x256 r128", (256, 256, 128, 0, "greedy"), 64),
+    ("ragged 300x200 r77", (300, 200, 77, 3, "greedy"), 37),
+    ("r = m 64x128", (64, 128, 64, 4, "greedy"), 20),
+    ("rank one 40x48", (40, 48, 1, 5, "greedy"), 13),
+    ("7B attention 4096x4096 r2048", (4096, 4096, 2048, 0, "lapack"), 512),
+]
+
+
+@pytest.mark.parametrize("name,layer,T", CASES, ids=[c[0] for c in CASES])
+def test_backward_matches_the_oracle(name, layer, T):
+    piv, nonp, Wp32, C32 = compressed(*layer)
+    m, n, r = piv.size + nonp.size, Wp32.shape[1], Wp32.shape[0]
+    rng = np.random.default_rng(11)
+    X32 = inputs.make_activations(rng, T, n, "bf16")
+    dY32 = inputs.make_activations(rng, T, m, "bf16")
+    X, Wp, dY = dev_bf16(X32), dev_bf16(Wp32), dev_bf16(dY32)
+    C = dev_bf16(C32) if m > r else torch.empty((0, r), dtype=torch.bfloat16, device=DEV)
+    pd = torch.from_numpy(piv.astype(np.int32)).to(DEV)
+    nd = torch.from_numpy(nonp.astype(np.int32)).to(DEV)
+    dX, dWp, dC = P.pifa_backward(X, Wp, C, pd, nd, dY)
+    assert P.pifa_device_status() == P.PIFA_OK
+    rX, rWp, rC = oracle.backward(X32, Wp32, C32, piv, nonp, dY32)
+    check(dX.float().cpu().numpy(), rX, f"{name} dX")
+    check(dWp.cpu().numpy(), rWp, f"{name} dW_p")
+    if m > r:
+        check(dC.cpu().numpy(), rC, f"{name} dC")
+    else:
+        assert dC is None
+
+
+def test_backward_zero_tokens_gives_zero_weight_gradients():
+    piv, nonp, Wp32, C32 = compressed(256, 256, 128, 0, "greedy")
+    Wp, C = dev_bf16(Wp32), dev_bf16(C32)
+    pd = torch.from_numpy(piv.astype(np.int32)).to(DEV)
+    nd = torch.from_numpy(nonp.astype(np.int32)).to(DEV)
+    X = torch.empty((0, 256), dtype=torch.bfloat16, device=DEV)
+    dY = torch.empty((0, 256), dtype=torch.bfloat16, device=DEV)
+    _, dWp, dC = P.pifa_backward(X, Wp, C, pd, nd, dY)
+    assert P.pifa_device_status() == P.PIFA_OK
+    assert torch.count_nonzero(dWp) == 0 and torch.count_nonzero(dC) == 0
+
+
+def _macc_inputs(T, n, m, seed):
+    rng = np.random.default_rng(seed)
+    Xu = inputs.round_bf16(rng.standard_normal((T, n)))
+    Xo = inputs.round_bf16(Xu + 0.1 * rng.standard_normal((T, n)))
+    W = inputs.round_bf16(rng.standard_normal((m, n)) / np.sqrt(n))
+    return Xo, Xu, W
+
+
+def test_m_accumulate_two_batches_match_the_oracle():
+    n, m, lam = 520, 1000, 0.25
+    XXt = torch.zeros((n, n), dtype=torch.float32, device=DEV)
+    YtXt = torch.zeros((m, n), dtype=torch.float32, device=DEV)
+    ref = (None, None)
+    for T, seed in ((300, 1), (77, 2)):
+        Xo, Xu, W = _macc_inputs(T, n, m, seed)
+        # one W for both batches (the same layer): the second draw's W is replaced by the first's
+        if seed == 1:
+            W0 = W
+        P.pifa_m_accumulate(dev_bf16(Xo), dev_bf16(Xu), dev_bf16(W0), lam, XXt, YtXt)
+        ref = oracle.m_accumulate(Xo, Xu, W0, lam, *ref)
+    assert P.pifa_device_status() == P.PIFA_OK
+    check(XXt.cpu().numpy(), ref[0], "X X^T")
+    check(YtXt.cpu().numpy(), ref[1], "Y_t X^T")
+
+
+def test_m_accumulate_xxt_only_and_lambda_edges():
+    n = 256
+    Xo, Xu, W = _macc_inputs(100, n, 128, 3)
+    XXt = torch.zeros((n, n), dtype=torch.float32, device=DEV)
+    P.pifa_m_accumulate(None, dev_bf16(Xu), None, 0.5, XXt)
+    check(XXt.cpu().numpy(), oracle.m_accumulate(Xo, Xu, W, 0.5)[0], "X X^T alone")
+    for lam in (0.0, 1.0):
+        XXt.zero_()
+        Y = torch.zeros((128, n), dtype=torch.float32, device=DEV)
+        P.pifa_m_accumulate(dev_bf16(Xo), dev_bf16(Xu), dev_bf16(W), lam, XXt, Y)
+        check(Y.cpu().numpy(), oracle.m_accumulate(Xo, Xu, W, lam)[1], f"Y_t X^T lambda={lam}")
+    assert P.pifa_device_status() == P.PIFA_OK
+
+
+def test_m_accumulate_llama_shape_sampled_rows():
+    """7B attention shape (n = m = 4096) with T = 512 samples; 48 sampled rows of each
+    accumulator against the oracle restricted to those rows."""
+    n = m = 4096
+    Xo, Xu, W = _macc_inputs(512, n, m, 4)
+    XXt = torch.zeros((n, n), dtype=torch.float32, device=DEV)
+    YtXt = torch.zeros((m, n), dtype=torch.float32, device=DEV)
+    P.pifa_m_accumulate(dev_bf16(Xo), dev_bf16(Xu), dev_bf16(W), 0.25, XXt, YtXt)
+    assert P.pifa_device_status() == P.PIFA_OK
+    rx, ry = inputs.random_rows(n, 48, 5), inputs.random_rows(m, 48, 6)
+    a, b = oracle.m_accumulate(Xo, Xu, W, 0.25, rows=(rx, ry))
+    check(XXt[torch.from_numpy(rx)].cpu().numpy(), a, "X X^T rows")
+    check(YtXt[torch.from_numpy(ry)].cpu().numpy(), b, "Y_t X^T rows")
