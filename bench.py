@@ -394,6 +394,96 @@ def mlp7b_point(dev, stream, T, hbm_peak, tc_peak, peak_src):
     return out
 
 
+def backward_point(dev, stream, shape, T, tc_peak, peak_src):
+    """pifa_backward (dX, dW_p, dC) at T tokens beside the same shape's dense backward (dX = dY W,
+    dW = dY^T X) and two-factor low-rank backward (H = X V: dU = dY^T H, dH = dY U, dV = X^T dH,
+    dX = dH V^T) through torch.matmul; tensor roofline on the PIFA backward's algorithmic FLOPs,
+    2 T r (2 (m - r) + 2 n) (the Y_p recompute and the lo passes are not counted)."""
+    import torch
+    from paper_2501_19090_gb300 import pifa as P
+    m, n, r = shape.m, shape.n, shape.r
+    piv, nonp, Wps, Cs = timing_layer(shape, dev, 9, "bf16", 2)
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(23)
+    X = torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16)
+    dY = torch.randn((T, m), device=dev, generator=gen).to(torch.bfloat16)
+    ws = P.workspace(P.pifa_backward_workspace_size(T, m, n, r), dev, tag="bwd")
+    torch.cuda.synchronize()
+
+    def bwd(i):
+        P.pifa_backward(X, Wps[i % 2], Cs[i % 2], piv, nonp, dY, workspace_tensor=ws, stream=stream)
+
+    U = (torch.randn((m, r), device=dev, generator=gen) / math.sqrt(r)).to(torch.bfloat16)
+    V = (torch.randn((n, r), device=dev, generator=gen) / math.sqrt(r)).to(torch.bfloat16)
+    W = torch.randn((m, n), device=dev, generator=gen).to(torch.bfloat16)
+
+    def dense(i):
+        dY @ W
+        dY.t() @ X
+
+    def lowrank(i):
+        H = X @ V
+        dY.t() @ H
+        dH = dY @ U
+        X.t() @ dH
+        dH @ V.t()
+
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        us = _steady_us(bwd, 4, stream)
+        assert P.pifa_device_status(stream) == P.PIFA_OK
+        d_us = _steady_us(dense, 4, stream)
+        l_us = _steady_us(lowrank, 4, stream)
+    flops = 2 * T * r * (2 * (m - r) + 2 * n)
+    tf = flops / us / 1e6
+    del Wps, Cs, X, dY, U, V, W
+    torch.cuda.empty_cache()
+    return {"workload": f"{shape.name} backward T={T}", "us_per_call": us, "tokens_per_s": T / (us / 1e6),
+            "dense_us": d_us, "lowrank_us": l_us, "speedup_vs_dense": d_us / us, "speedup_vs_lowrank": l_us / us,
+            "roofline": {"bound": "tensor", "achieved": tf, "peak": tc_peak, "unit": "TFLOP/s", "frac": tf / tc_peak,
+                         "algorithmic_flops_per_call": flops, "peak_source": f"{peak_src} bf16_tflops (burst)"},
+            "clocks": clk.summary()}
+
+
+def m_accumulate_point(dev, stream, shape, T, tc_peak, peak_src):
+    """pifa_m_accumulate (X X^T and Y_t X^T of one calibration batch, lambda = 0.25) beside the same
+    products through torch.matmul (bf16 in, fp32 out); tensor roofline on 2 T (n^2 + 2 m n)."""
+    import torch
+    from paper_2501_19090_gb300 import pifa as P
+    m, n = shape.m, shape.n
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(29)
+    Xu = torch.randn((T, n), device=dev, generator=gen).to(torch.bfloat16)
+    Xo = (Xu.float() + 0.1 * torch.randn((T, n), device=dev, generator=gen)).to(torch.bfloat16)
+    W = (torch.randn((m, n), device=dev, generator=gen) / math.sqrt(n)).to(torch.bfloat16)
+    XXt = torch.zeros((n, n), dtype=torch.float32, device=dev)
+    YtXt = torch.zeros((m, n), dtype=torch.float32, device=dev)
+    ws = P.workspace(P.pifa_m_accumulate_workspace_size(T, m, n), dev, tag="macc")
+    torch.cuda.synchronize()
+
+    def macc(i):
+        P.pifa_m_accumulate(Xo, Xu, W, 0.25, XXt, YtXt, workspace_tensor=ws, stream=stream)
+
+    def ref(i):
+        XXt.add_((Xu.t() @ Xu).float())
+        Yt = (0.25 * Xo.float() + 0.75 * Xu.float()).to(torch.bfloat16) @ W.t()
+        YtXt.add_((Yt.t() @ Xu).float())
+
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        us = _steady_us(macc, 4, stream)
+        assert P.pifa_device_status(stream) == P.PIFA_OK
+        t_us = _steady_us(ref, 4, stream)
+    flops = 2 * T * (n * n + 2 * m * n)
+    tf = flops / us / 1e6
+    del Xu, Xo, W, XXt, YtXt
+    torch.cuda.empty_cache()
+    return {"workload": f"{shape.name} M accumulators T={T}", "us_per_call": us, "tokens_per_s": T / (us / 1e6),
+            "torch_us": t_us, "speedup_vs_torch": t_us / us,
+            "torch_note": "single bf16 roundings of the mixed input and Y_t (the library carries them as hi + lo pairs)",
+            "roofline": {"bound": "tensor", "achieved": tf, "peak": tc_peak, "unit": "TFLOP/s", "frac": tf / tc_peak,
+                         "algorithmic_flops_per_call": flops, "peak_source": f"{peak_src} bf16_tflops (burst)"},
+            "clocks": clk.summary()}
+
+
 def extras(dev, stream, hbm_peak, tc_peak, peak_src):
     """Every configuration of the workload list beside its low-rank and dense layers (one GPU)."""
     import torch
@@ -407,6 +497,9 @@ def extras(dev, stream, hbm_peak, tc_peak, peak_src):
         out["prefill_points"].append(layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src))
     for s in inputs.rank_sweep_shapes():
         out["rank_sweep"].append(layer_point(dev, stream, s, 2048, hbm_peak, tc_peak, peak_src))
+    out["backward"] = [backward_point(dev, stream, sh, 2048, tc_peak, peak_src)
+                       for sh in (inputs.ATTN7B, inputs.MLP7B_GATE)]
+    out["m_accumulate"] = [m_accumulate_point(dev, stream, inputs.ATTN7B, 2048, tc_peak, peak_src)]
     torch.cuda.empty_cache()
     return out
 

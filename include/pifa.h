@@ -294,7 +294,7 @@ int64_t pifa_backward_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r)
  *   XXt          DEVICE in/out, fp32, n x n, pitch ldxx >= n.
  *   YtXt         DEVICE in/out, fp32, m x n, pitch ldyx >= n (NULL: only XXt is accumulated).
  *   workspace    DEVICE scratch of pifa_m_accumulate_workspace_size(T, m, n) bytes, 256-byte
- *                aligned (the mixed input and Y_t in bf16); unused when YtXt is NULL.
+ *                aligned (X_u^T, the mixed input and Y_t^T in bf16).
  *   Numerics: bf16 operands, fp32 accumulation; the mixed input and Y_t are rounded to bf16.
  *   T == 0 is a no-op. Asynchronous on cuda_stream.
  */

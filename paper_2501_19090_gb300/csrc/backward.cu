@@ -33,44 +33,62 @@ int64_t pad8(int64_t v) { return (v + 7) / 8 * 8; }
 int64_t a256(int64_t b) { return (b + 255) / 256 * 256; }
 
 // out[t][i] = in[t][idx[i]] for t < T, i < cnt (bf16); an index outside [0, bound) writes 0 and
-// latches PIFA_ERR_DEVICE_INDEX.
+// latches PIFA_ERR_DEVICE_INDEX. Row t = blockIdx.y (grid-stride), columns across the x grid.
 __global__ void gather_cols(const bf16* in, int64_t ldin, const int32_t* idx, int cnt, int bound, int T, bf16* out,
                             int64_t ldout, int* status) {
   pdl_launch_dependents();
   pdl_wait_primary();
-  const int64_t n = (int64_t)T * cnt;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
-    const int t = (int)(e / cnt), i = (int)(e % cnt);
-    const int c = idx[i];
-    bf16 v = __float2bfloat16_rn(0.0f);
-    if ((unsigned)c < (unsigned)bound)
-      v = in[(int64_t)t * ldin + c];
-    else
-      latch_status(status, PIFA_ERR_DEVICE_INDEX);
-    out[(int64_t)t * ldout + i] = v;
-  }
+  for (int t = blockIdx.y; t < T; t += gridDim.y)
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < cnt; i += gridDim.x * blockDim.x) {
+      const int c = __ldg(idx + i);
+      bf16 v = __float2bfloat16_rn(0.0f);
+      if ((unsigned)c < (unsigned)bound)
+        v = in[(int64_t)t * ldin + c];
+      else
+        latch_status(status, PIFA_ERR_DEVICE_INDEX);
+      out[(int64_t)t * ldout + i] = v;
+    }
 }
 
 // out = a * x + b * y elementwise over T rows of n (bf16 in, fp32 arithmetic), written as a hi +
-// lo pair of bf16 planes.
+// lo pair of bf16 planes. Rows across the y grid, columns across x.
 __global__ void axpby_rows(const bf16* x, const bf16* y, int64_t ld, int T, int n, float a, float b, bf16* out,
                            bf16* out_lo, int64_t ldout) {
   pdl_launch_dependents();
   pdl_wait_primary();
-  const int64_t tot = (int64_t)T * n;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < tot; e += (int64_t)gridDim.x * blockDim.x) {
-    const int t = (int)(e / n), c = (int)(e % n);
-    const float v = a * __bfloat162float(x[(int64_t)t * ld + c]) + b * __bfloat162float(y[(int64_t)t * ld + c]);
-    const bf16 h = __float2bfloat16_rn(v);
-    out[(int64_t)t * ldout + c] = h;
-    out_lo[(int64_t)t * ldout + c] = __float2bfloat16_rn(v - __bfloat162float(h));
+  for (int t = blockIdx.y; t < T; t += gridDim.y)
+    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < n; c += gridDim.x * blockDim.x) {
+      const float v = a * __bfloat162float(x[(int64_t)t * ld + c]) + b * __bfloat162float(y[(int64_t)t * ld + c]);
+      const bf16 h = __float2bfloat16_rn(v);
+      out[(int64_t)t * ldout + c] = h;
+      out_lo[(int64_t)t * ldout + c] = __float2bfloat16_rn(v - __bfloat162float(h));
+    }
+}
+
+// out (cols x rows) = in (rows x cols)^T, bf16, through 32 x 32 shared-memory tiles (coalesced
+// reads and writes). Block (32, 8); grid (ceil(cols / 32), ceil(rows / 32)).
+__global__ void transpose_bf16(const bf16* in, int64_t ldin, int rows, int cols, bf16* out, int64_t ldout) {
+  __shared__ bf16 t[32][34];
+  pdl_launch_dependents();
+  pdl_wait_primary();
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  for (int k = threadIdx.y; k < 32; k += 8) {
+    const int r = r0 + k, c = c0 + threadIdx.x;
+    t[k][threadIdx.x] = (r < rows && c < cols) ? in[(int64_t)r * ldin + c] : __float2bfloat16_rn(0.0f);
+  }
+  __syncthreads();
+  for (int k = threadIdx.y; k < 32; k += 8) {
+    const int c = c0 + k, r = r0 + threadIdx.x;
+    if (c < cols && r < rows) out[(int64_t)c * ldout + r] = t[threadIdx.x][k];
   }
 }
 
-int launch_small(const void* fn, void** args, int64_t work, cudaStream_t stream, const char* what) {
+// A row-wise elementwise kernel over `rows` rows of `cols` columns: rows on the y grid (at most
+// 65535, the kernel loops beyond), columns on x.
+int launch_small(const void* fn, void** args, int64_t rows, int64_t cols, cudaStream_t stream, const char* what) {
   cudaLaunchConfig_t cfg = {};
-  const int64_t blocks = (work + 255) / 256;
-  cfg.gridDim = dim3((unsigned)(blocks < 4 * 152 ? (blocks > 0 ? blocks : 1) : 4 * 152));
+  const int64_t bx = (cols + 255) / 256;
+  cfg.gridDim = dim3((unsigned)(bx < 8 ? (bx > 0 ? bx : 1) : 8), (unsigned)(rows < 65535 ? (rows > 0 ? rows : 1) : 65535));
   cfg.blockDim = dim3(256);
   cfg.stream = stream;
   cudaLaunchAttribute attr;
@@ -106,16 +124,25 @@ BwdLayout bwd_layout(int64_t T, int64_t m, int64_t r) {
 }
 
 struct MaccLayout {
-  int64_t xmix, xmix_lo, yt, yt_lo, total;
+  int64_t xut, xmix, xmix_lo, ytt, ytt_lo, total;
 };
 
+// X_u^T (n x pad8(T)), the mixed input's hi and lo planes (T x pad8(n)), Y_t^T's hi and lo planes
+// (m x pad8(T)), all bf16
 MaccLayout macc_layout(int64_t T, int64_t m, int64_t n) {
   MaccLayout L;
-  L.xmix = 0;
-  L.xmix_lo = a256(T * pad8(n) * 2);
-  L.yt = 2 * L.xmix_lo;
-  L.yt_lo = L.yt + a256(T * pad8(m) * 2);
-  L.total = L.yt_lo + a256(T * pad8(m) * 2);
+  int64_t o = 0;
+  L.xut = o;
+  o += a256(n * pad8(T) * 2);
+  L.xmix = o;
+  o += a256(T * pad8(n) * 2);
+  L.xmix_lo = o;
+  o += a256(T * pad8(n) * 2);
+  L.ytt = o;
+  o += a256(m * pad8(T) * 2);
+  L.ytt_lo = o;
+  o += a256(m * pad8(T) * 2);
+  L.total = o;
   return L;
 }
 
@@ -175,7 +202,7 @@ extern "C" int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx, c
     int cnt = (int)(m - r);
     void* args[] = {(void*)&dY, (void*)&lddy, (void*)&nonpivot_idx, (void*)&cnt, (void*)&mi, (void*)&Ti,
                     (void*)&dYnp, (void*)&ldnp, (void*)&status};
-    if ((st = launch_small((const void*)gather_cols, args, T * (m - r), s, "backward: gather")) != PIFA_OK) return st;
+    if ((st = launch_small((const void*)gather_cols, args, T, m - r, s, "backward: gather")) != PIFA_OK) return st;
   }
   // Y_p = X W_p^T as hi + lo planes (only dC needs it)
   if (dC && has_np) {
@@ -192,7 +219,7 @@ extern "C" int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx, c
     int cnt = (int)r;
     void* args[] = {(void*)&dY, (void*)&lddy, (void*)&pivot_idx, (void*)&cnt, (void*)&mi, (void*)&Ti,
                     (void*)&dYp, (void*)&ldr, (void*)&status};
-    if ((st = launch_small((const void*)gather_cols, args, T * r, s, "backward: gather")) != PIFA_OK) return st;
+    if ((st = launch_small((const void*)gather_cols, args, T, r, s, "backward: gather")) != PIFA_OK) return st;
   }
   if (dX) {  // dX = (dY_p,hi + dY_p,lo) W_p  (dY_p exact in bf16 when r == m)
     GemmTc g = {T, n, r, dYp, ldr, false, Wp, ldwp, true, dX, lddx, 0, 1.0f, nullptr, nullptr, 0, 0};
@@ -233,42 +260,58 @@ extern "C" int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int6
       (YtXt && ((ldw & 7) || (ldyx & 3))))
     return pifa_fail(PIFA_ERR_ALIGNMENT, "16-byte aligned buffers and 16-byte row pitches required");
   const MaccLayout Ly = macc_layout(T, m, n);
-  if (YtXt && (!workspace || workspace_bytes < Ly.total)) return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or too small");
-  if (YtXt && (reinterpret_cast<uintptr_t>(workspace) & 255u))
-    return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  if (!workspace || workspace_bytes < Ly.total) return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or too small");
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u) return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
   cudaError_t ce = cudaSuccess;
   int* status = pifa_status_word(&ce);
   if (!status) return pifa_fail_cuda("device status word", ce);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(cuda_stream);
   const uint64_t tmo = pifa_wait_timeout_ns();
   int st;
+  // Every product runs with both operands K-major (measured twice as fast as the transposed forms):
+  // X_u^T is formed once, and Y_t^T comes out of W X_mix^T directly.
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  bf16* XuT = reinterpret_cast<bf16*>(ws + Ly.xut);
+  const int64_t ldT = pad8(T), ldn = pad8(n);
+  {  // X_u^T
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((n + 31) / 32), (unsigned)((T + 31) / 32));
+    cfg.blockDim = dim3(32, 8);
+    cfg.stream = s;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, transpose_bf16, reinterpret_cast<const bf16*>(Xu), ldx, (int)T,
+                                             (int)n, XuT, ldT);
+    if (e != cudaSuccess) return pifa_fail_cuda("m_accumulate: transpose", e);
+  }
   {  // XXt += X_u^T X_u
-    GemmTc g = {n, n, T, Xu, ldx, true, Xu, ldx, true, XXt, ldxx, 2, 1.0f, nullptr, nullptr, 0, 0};
+    GemmTc g = {n, n, T, XuT, ldT, false, XuT, ldT, false, XXt, ldxx, 2, 1.0f, nullptr, nullptr, 0, 0};
     if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
   }
   if (!YtXt) return PIFA_OK;
-  uint8_t* ws = static_cast<uint8_t*>(workspace);
   bf16* Xmix = reinterpret_cast<bf16*>(ws + Ly.xmix);
   bf16* Xmix_lo = reinterpret_cast<bf16*>(ws + Ly.xmix_lo);
-  bf16* Yt = reinterpret_cast<bf16*>(ws + Ly.yt);
-  bf16* Yt_lo = reinterpret_cast<bf16*>(ws + Ly.yt_lo);
-  const int64_t ldn = pad8(n), ldm = pad8(m);
-  {  // X_mix = lambda X_o + (1 - lambda) X_u
+  bf16* YtT = reinterpret_cast<bf16*>(ws + Ly.ytt);
+  bf16* YtT_lo = reinterpret_cast<bf16*>(ws + Ly.ytt_lo);
+  {  // X_mix = lambda X_o + (1 - lambda) X_u, as hi + lo planes
     int Ti = (int)T, ni = (int)n;
     float a = lambda, b = 1.0f - lambda;
     void* args[] = {(void*)&Xo, (void*)&Xu, (void*)&ldx, (void*)&Ti, (void*)&ni, (void*)&a, (void*)&b, (void*)&Xmix,
                     (void*)&Xmix_lo, (void*)&ldn};
-    if ((st = launch_small((const void*)axpby_rows, args, T * n, s, "m_accumulate: mix")) != PIFA_OK) return st;
+    if ((st = launch_small((const void*)axpby_rows, args, T, n, s, "m_accumulate: mix")) != PIFA_OK) return st;
   }
-  {  // Y_t = (X_mix,hi + X_mix,lo) W^T, as hi + lo planes
-    GemmTc g = {T, m, n, Xmix, ldn, false, W, ldw, false, Yt, ldm, 3, 1.0f, nullptr, nullptr, 0, 0};
-    g.A2 = Xmix_lo;
-    g.D2 = Yt_lo;
+  {  // Y_t^T = W (X_mix,hi + X_mix,lo)^T, as hi + lo planes (m x T)
+    GemmTc g = {m, T, n, W, ldw, false, Xmix, ldn, false, YtT, ldT, 3, 1.0f, nullptr, nullptr, 0, 0};
+    g.B2 = Xmix_lo;
+    g.D2 = YtT_lo;
     if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
   }
-  {  // YtXt += (Y_t,hi + Y_t,lo)^T X_u
-    GemmTc g = {m, n, T, Yt, ldm, true, Xu, ldx, true, YtXt, ldyx, 2, 1.0f, nullptr, nullptr, 0, 0};
-    g.A2 = Yt_lo;
+  {  // YtXt += (Y_t^T,hi + Y_t^T,lo) X_u
+    GemmTc g = {m, n, T, YtT, ldT, false, XuT, ldT, false, YtXt, ldyx, 2, 1.0f, nullptr, nullptr, 0, 0};
+    g.A2 = YtT_lo;
     if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
   }
   return PIFA_OK;

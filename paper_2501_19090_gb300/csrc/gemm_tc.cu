@@ -39,6 +39,9 @@ constexpr uint32_t MN_BOX = 64 * BK * 2;      // one MN-major box: 64 (MN) x 64 
 struct GemmTcArgs {
   int M, N, K;
   int bn;             // N per tile
+  int d_trans;        // 1: store D^T (element (i, j) at D[j * ldd + i]); no accumulation or addend
+  int prefetch;       // 1: the epilogue adds values read from global memory (D itself or the addend),
+                      //    staged into shared memory while the MMAs run
   uint32_t idesc;
   int passes;         // 1, or 2 (the second pass reads tmA2 and tmB2)
   void* D;            // M x N, pitch ldd: bf16 (out_mode 0) or fp32 (1: store, 2: add into), or
@@ -74,8 +77,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t b_bytes = (uint32_t)p.bn * BK * 2;
-  const uint32_t stage_bytes = A_BYTES + B_MAX;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * stage_bytes);
+  const uint32_t stage_bytes = A_BYTES + b_bytes;
+  // the epilogue's staged addends: 4 warps x 32 rows x (bn + 1) fp32, after the stages
+  float* ext_sm = reinterpret_cast<float*>(smem + STAGES * stage_bytes);
+  const uint32_t ext_bytes = p.prefetch ? 4u * 32u * (uint32_t)(p.bn + 1) * 4u : 0u;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * stage_bytes + ((ext_bytes + 15) & ~15u));
   uint64_t* empty = full + STAGES;
   uint64_t* accf = empty + STAGES;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accf + 1);
@@ -175,42 +181,98 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
   } else {
     // ---------------- epilogue: warps 2..5, TMEM lane quarter warp % 4 ----------------
+    // Each 32 x 32 block (32 rows of this quarter, 32 columns) goes through this warp's 4 KB of the
+    // stage memory (free once every MMA has completed): read from TMEM one row per lane, written to
+    // global memory one row per store instruction, the lanes covering 32 consecutive columns.
     const int q = warp & 3;
-    const int row = m0 + q * 32 + lane;
+    float* ext = ext_sm + (warp - 2) * 32 * (p.bn + 1);  // this warp's rows: [32][bn + 1]
+    if (p.prefetch) {
+      // while the MMAs run: the old D (accumulation) plus the addend. The lanes cover consecutive
+      // columns (coalesced); each thread issues the loads of 8 rows x 4 columns before storing any
+      // of them to shared memory, so that many loads are in flight at once.
+      for (int r0 = 0; r0 < 32; r0 += 8) {
+        float v[8][4];
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int row = m0 + q * 32 + r0 + i, c = lane + 32 * j, col = n0 + c;
+            float e = 0.0f;
+            if (c < p.bn && row < p.M && col < p.N) {
+              if (p.out_mode == 2) e = __ldcg(reinterpret_cast<const float*>(p.D) + (int64_t)row * p.ldd + col);
+              if (p.add) {
+                const int ac = p.add_idx ? __ldg(p.add_idx + col) : col;
+                if ((unsigned)ac < (unsigned)p.add_bound)
+                  e += __bfloat162float(p.add[(int64_t)row * p.ldadd + ac]);
+                else
+                  latch_status(p.status, PIFA_ERR_DEVICE_INDEX);
+              }
+            }
+            v[i][j] = e;
+          }
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            if (lane + 32 * j < p.bn) ext[(r0 + i) * (p.bn + 1) + lane + 32 * j] = v[i][j];
+      }
+      __syncwarp();
+    }
     const bool ok = mbar_wait(accf, 0, p.timeout_ns) && !*abort_flag;
     if (!ok) latch_status(p.status, PIFA_ERR_TIMEOUT);
     tc_fence_after();
     if (ok) {
+      float* tile = reinterpret_cast<float*>(smem) + (warp - 2) * (32 * 33);
       const int ncols = min(p.bn, p.N - n0);
       for (int c0 = 0; c0 < ncols; c0 += 32) {
         uint32_t v[32];
         tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c0, v);
         tmem_ld_wait();
-        if (row >= p.M) continue;
-        for (int j = 0; j < 32; ++j) {
-          const int col = n0 + c0 + j;
-          if (col >= p.N) break;
-          float f = p.alpha * __uint_as_float(v[j]);
-          if (p.add) {
-            const int ac = p.add_idx ? p.add_idx[col] : col;
-            if ((unsigned)ac >= (unsigned)p.add_bound) {
-              latch_status(p.status, PIFA_ERR_DEVICE_INDEX);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) tile[lane * 33 + j] = __uint_as_float(v[j]);
+        __syncwarp();
+        const int nrows = min(32, p.M - (m0 + q * 32));
+        if (p.d_trans) {
+          // D^T: one column of the block per step, the lanes covering consecutive rows (coalesced)
+          const int row = m0 + q * 32 + lane;
+          for (int cc = 0; cc < 32; ++cc) {
+            const int col = n0 + c0 + cc;
+            if (col >= p.N) break;
+            if (lane >= nrows) continue;
+            float f = p.alpha * tile[lane * 33 + cc];
+            if (p.prefetch) f += ext[lane * (p.bn + 1) + c0 + cc];
+            const int64_t o = (int64_t)col * p.ldd + row;
+            if (p.out_mode == 3) {
+              const bf16 h = __float2bfloat16_rn(f);
+              reinterpret_cast<bf16*>(p.D)[o] = h;
+              reinterpret_cast<bf16*>(p.D2)[o] = __float2bfloat16_rn(f - __bfloat162float(h));
+            } else if (p.out_mode == 0) {
+              reinterpret_cast<bf16*>(p.D)[o] = __float2bfloat16_rn(f);
             } else {
-              f += __bfloat162float(p.add[(int64_t)row * p.ldadd + ac]);
+              reinterpret_cast<float*>(p.D)[o] = f;
             }
           }
-          if (p.out_mode == 3) {
-            const bf16 h = __float2bfloat16_rn(f);
-            reinterpret_cast<bf16*>(p.D)[(int64_t)row * p.ldd + col] = h;
-            reinterpret_cast<bf16*>(p.D2)[(int64_t)row * p.ldd + col] = __float2bfloat16_rn(f - __bfloat162float(h));
-          } else if (p.out_mode == 0) {
-            reinterpret_cast<bf16*>(p.D)[(int64_t)row * p.ldd + col] = __float2bfloat16_rn(f);
-          } else if (p.out_mode == 1) {
-            reinterpret_cast<float*>(p.D)[(int64_t)row * p.ldd + col] = f;
-          } else {
-            reinterpret_cast<float*>(p.D)[(int64_t)row * p.ldd + col] += f;
+        } else {
+          // D: one row of the block per step, the lanes covering consecutive columns (coalesced)
+          const int col = n0 + c0 + lane;
+          for (int rr = 0; rr < nrows; ++rr) {
+            const int row = m0 + q * 32 + rr;
+            if (col >= p.N) break;
+            float f = p.alpha * tile[rr * 33 + lane];
+            if (p.prefetch) f += ext[rr * (p.bn + 1) + c0 + lane];
+            const int64_t o = (int64_t)row * p.ldd + col;
+            if (p.out_mode == 3) {
+              const bf16 h = __float2bfloat16_rn(f);
+              reinterpret_cast<bf16*>(p.D)[o] = h;
+              reinterpret_cast<bf16*>(p.D2)[o] = __float2bfloat16_rn(f - __bfloat162float(h));
+            } else if (p.out_mode == 0) {
+              reinterpret_cast<bf16*>(p.D)[o] = __float2bfloat16_rn(f);
+            } else {
+              reinterpret_cast<float*>(p.D)[o] = f;
+            }
           }
         }
+        __syncwarp();  // the next block reuses the tile
       }
     }
   }
@@ -236,7 +298,12 @@ int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stre
   a.K = (int)g.K;
   // tile width: MN-major B tiles come in 64-column boxes, K-major ones in multiples of 16
   const int64_t unit = g.b_mn ? 64 : 16;
-  a.bn = (int)(g.N >= BNMAX ? BNMAX : (g.N + unit - 1) / unit * unit);
+  // with values to add in, the tile is at most 128 wide so that their staging fits beside the ring
+  a.prefetch = (g.out_mode == 2 || g.add) ? 1 : 0;
+  const int64_t bnmax = a.prefetch ? 128 : BNMAX;
+  a.bn = (int)(g.N >= bnmax ? bnmax : (g.N + unit - 1) / unit * unit);
+  a.d_trans = g.d_trans ? 1 : 0;
+  if (a.d_trans && a.prefetch) return pifa_fail(PIFA_ERR_UNSUPPORTED, "gemm_tc: transposed store with an addend");
   a.idesc = idesc_bf16_f32(BM, (uint32_t)a.bn) | (g.a_mn ? (1u << 15) : 0u) | (g.b_mn ? (1u << 16) : 0u);
   a.passes = (g.A2 || g.B2) ? 2 : 1;
   a.D = g.D;
@@ -280,7 +347,8 @@ int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stre
   }
   auto kern = g.a_mn ? (g.b_mn ? gemm_tc_kernel<true, true> : gemm_tc_kernel<true, false>)
                      : (g.b_mn ? gemm_tc_kernel<false, true> : gemm_tc_kernel<false, false>);
-  const size_t smem = 1024 + (size_t)STAGES * (A_BYTES + B_MAX) + 256;
+  const size_t ext_bytes = a.prefetch ? (size_t)4 * 32 * (a.bn + 1) * 4 : 0;
+  const size_t smem = 1024 + (size_t)STAGES * (A_BYTES + (size_t)a.bn * BK * 2) + (ext_bytes + 15) / 16 * 16 + 256;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(gemm_tc)", e);
   const unsigned nt = (unsigned)((g.N + a.bn - 1) / a.bn), mt = (unsigned)((g.M + BM - 1) / BM);

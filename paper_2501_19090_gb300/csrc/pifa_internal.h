@@ -121,6 +121,7 @@ struct GemmTc {
   const void* A2 = nullptr;
   const void* B2 = nullptr;
   void* D2 = nullptr;
+  bool d_trans = false;  // store D^T: element (i, j) at D[j * ldd + i] (out_mode 0, 1 or 3 only)
 };
 int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stream);
 

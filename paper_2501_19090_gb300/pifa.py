@@ -435,6 +435,20 @@ def pifa_forward_decode_noalloc(X, Wp, C, pivot_idx, nonpivot_idx, Y=None, strea
     return Y
 
 
+def pifa_backward_workspace_size(T: int, m: int, n: int, r: int) -> int:
+    v = int(_lib().pifa_backward_workspace_size(T, m, n, r))
+    if v < 0:
+        _check(v, "pifa_backward_workspace_size")
+    return v
+
+
+def pifa_m_accumulate_workspace_size(T: int, m: int, n: int) -> int:
+    v = int(_lib().pifa_m_accumulate_workspace_size(T, m, n))
+    if v < 0:
+        _check(v, "pifa_m_accumulate_workspace_size")
+    return v
+
+
 def pifa_backward(X, Wp, C, pivot_idx, nonpivot_idx, dY, want=("dX", "dWp", "dC"), workspace_tensor=None,
                   stream=None):
     """Gradients of the forward pass through pifa_backward: returns (dX bf16 T x n, dW_p fp32 r x n,
@@ -453,9 +467,7 @@ def pifa_backward(X, Wp, C, pivot_idx, nonpivot_idx, dY, want=("dX", "dWp", "dC"
     dX = out(T, n, torch.bfloat16, 8) if "dX" in want else None
     dWp = out(r, n, torch.float32, 4) if "dWp" in want else None
     dC = out(m - r, r, torch.float32, 4) if ("dC" in want and has_np) else None
-    need = int(_lib().pifa_backward_workspace_size(T, m, n, r))
-    if need < 0:
-        _check(need, "pifa_backward_workspace_size")
+    need = pifa_backward_workspace_size(T, m, n, r)
     ws = workspace_tensor if workspace_tensor is not None else workspace(need, dev, stream, tag="backward")
     ws_ptr = ws.data_ptr() + (-ws.data_ptr()) % 256
     ws_bytes = ws.numel() * ws.element_size() - (ws_ptr - ws.data_ptr())
@@ -496,9 +508,7 @@ def pifa_m_accumulate(Xo, Xu, W, lam, XXt, YtXt=None, workspace_tensor=None, str
                 raise ValueError(f"pifa: {name} is on {t.device}, Xu on {Xu.device}")
     if XXt.device != Xu.device:
         raise ValueError("pifa: XXt must be on Xu's device")
-    need = int(_lib().pifa_m_accumulate_workspace_size(T, m, n))
-    if need < 0:
-        _check(need, "pifa_m_accumulate_workspace_size")
+    need = pifa_m_accumulate_workspace_size(T, m, n)
     ws = workspace_tensor if workspace_tensor is not None else workspace(need, Xu.device, stream, tag="macc")
     ws_ptr = ws.data_ptr() + (-ws.data_ptr()) % 256
     ws_bytes = ws.numel() * ws.element_size() - (ws_ptr - ws.data_ptr())
