@@ -307,6 +307,37 @@ int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int64_t n, int6
  * pifa_status on bad arguments. Pure host arithmetic. */
 int64_t pifa_m_accumulate_workspace_size(int64_t T, int64_t m, int64_t n);
 
+/*
+ * pifa_m_reconstruct -- the two reconstruction steps of the M method (Sec. 4; Algorithm 3, part 1)
+ * from the accumulators pifa_m_accumulate builds, in float64 on the GPU:
+ *   U_r   = (Y_t X^T) V (V^T (X X^T) V)^{-1}                                       (Eq. 4)
+ *   V_r^T = (U_r^T U_r)^{-1} U_r^T (Y_t X^T + alpha W) (X X^T + alpha I)^{-1}        (Eq. 8)
+ * whose product U_r V_r^T is the low-rank weight that Algorithm 1 (pifa_compress_device) turns
+ * into a PIFA layer.
+ *
+ *   XXt          DEVICE, fp32, n x n, pitch ldxx >= n (X X^T).
+ *   YtXt         DEVICE, fp32, m x n, pitch ldyx >= n (Y_t X^T).
+ *   V            DEVICE, float64, n x r, contiguous (the pruned layer's right factor).
+ *   W            DEVICE, bf16, m x n, pitch ldw >= n (the dense weight; used when alpha > 0).
+ *   alpha        the regulariser of Eq. 8 (>= 0; the paper uses 0.001; 0 gives Eq. 7).
+ *   U_r, V_r     DEVICE out, float64, m x r and n x r, contiguous.
+ *   workspace    DEVICE scratch of pifa_m_reconstruct_workspace_size(m, n, r) bytes, 256-byte
+ *                aligned (about 8 (2 n^2 + m n + 4 r n + 4 r^2 + 2.25 p^2) bytes, p = n rounded up
+ *                to 32 * 2^k).
+ *   The symmetric positive definite matrices are inverted by Cholesky factorisation and the
+ *   inverse of the triangular factor. Requires 1 <= r <= min(m, n) and n <= 16384;
+ *   PIFA_ERR_RANK_DEFICIENT when a matrix to invert is not positive definite. Synchronous.
+ */
+int pifa_m_reconstruct(const float* XXt, int64_t ldxx, const float* YtXt, int64_t ldyx,
+                       const double* V, const void* W, int64_t ldw,
+                       int64_t m, int64_t n, int64_t r, double alpha,
+                       double* U_r, double* V_r, void* workspace, int64_t workspace_bytes,
+                       void* cuda_stream);
+
+/* pifa_m_reconstruct_workspace_size -- bytes of device scratch pifa_m_reconstruct needs; negative
+ * pifa_status on bad arguments. Pure host arithmetic. */
+int64_t pifa_m_reconstruct_workspace_size(int64_t m, int64_t n, int64_t r);
+
 /* pifa_validate_indices -- HOST copies: PIFA_OK iff pivot_idx (r entries) and nonpivot_idx
  * (m - r entries) are strictly ascending, inside [0, m) and disjoint (so together a partition
  * of [0, m), as Algorithm 1 step 2 defines I^c); else PIFA_ERR_INVALID_ARG. */

@@ -1,4 +1,5 @@
-// compress_gpu.cu -- pifa_compress_device: Algorithm 1 (Sec. 3.2) on the GPU in float64.
+// compress_gpu.cu -- the float64 set-up steps on the GPU: pifa_compress_device (Algorithm 1,
+// Sec. 3.2) and pifa_m_reconstruct (the two solves of the M reconstruction, Sec. 4, at the end).
 //
 // Route (all device-resident, float64; the caller's workspace holds every temporary):
 //   1. G = V^T V (r x r) and its Cholesky factor L (G = L L^T). Then Z = U L (m x r) has the row
@@ -20,6 +21,7 @@
 #include <cmath>
 #include <cstdio>
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "pifa.h"
@@ -386,6 +388,38 @@ __global__ void max_abs(const double* C, int64_t rows, int64_t cols, int64_t ldc
   if ((threadIdx.x & 31) == 0) atomicMax(out, (unsigned long long)__double_as_longlong(mx));
 }
 
+// Rinv = R^{-1} for an upper-triangular R (rp x rp, rp = 32 * 2^k; identity on any padding), by
+// doubling: the 32 x 32 diagonal blocks inverted directly, then, level by level, for every pair
+// of sz-blocks [[A, B], [0, D]] along the diagonal the off-diagonal block -A^{-1} (B D^{-1}).
+// Tt: scratch of rp * rp / 4 doubles.
+int upper_inverse(const double* R, double* Rinv, double* Tt, int rp, cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(Rinv, 0, (size_t)rp * rp * 8, s);
+  if (e != cudaSuccess) return pifa_fail_cuda("upper inverse: memset", e);
+  inv_diag32<<<rp / 32, 32, 0, s>>>(R, Rinv, rp);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return pifa_fail_cuda("upper inverse: launch", e);
+  int st;
+  for (int sz = 32; sz < rp; sz *= 2) {
+    const int pairs = rp / (2 * sz);
+    const int64_t step = (int64_t)2 * sz * rp + 2 * sz;  // next pair along the diagonal
+    GemmF64 a = {};
+    a.M = sz; a.N = sz; a.K = sz;
+    a.A = R + sz; a.sa_i = rp; a.sa_k = 1;                        // B block
+    a.B = Rinv + (int64_t)sz * rp + sz; a.sb_k = rp; a.sb_j = 1;  // D^{-1}
+    a.C = Tt; a.ldc = sz; a.alpha = 1.0; a.beta = 0.0;
+    a.za = step; a.zb = step; a.zc = (int64_t)sz * sz;
+    if ((st = run_gemm_f64(a, pairs, s)) != PIFA_OK) return st;
+    GemmF64 b = {};
+    b.M = sz; b.N = sz; b.K = sz;
+    b.A = Rinv; b.sa_i = rp; b.sa_k = 1;                          // A^{-1}
+    b.B = Tt; b.sb_k = sz; b.sb_j = 1;
+    b.C = Rinv + sz; b.ldc = rp; b.alpha = -1.0; b.beta = 0.0;
+    b.za = step; b.zb = (int64_t)sz * sz; b.zc = step;
+    if ((st = run_gemm_f64(b, pairs, s)) != PIFA_OK) return st;
+  }
+  return PIFA_OK;
+}
+
 // Workspace layout (bytes, each part 256-aligned).
 struct Layout {
   int64_t G, L, Z, R, Rinv, T, blk, order, rdiag, gap, sel, pos, asc, flags, total;
@@ -520,29 +554,7 @@ extern "C" int pifa_compress_device(const double* U, const double* V, int64_t m,
   {
     const int64_t tot = (int64_t)rp * rp;
     build_r<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(g, R, rp);
-    PIFA_CK(cudaMemsetAsync(Rinv, 0, tot * 8, s), "compress: memset");
-    inv_diag32<<<rp / 32, 32, 0, s>>>(R, Rinv, rp);
-    PIFA_CK(cudaGetLastError(), "compress: inverse launch");
-    for (int sz = 32; sz < rp; sz *= 2) {
-      // for every pair of sz-blocks [[A, B], [0, D]] along the diagonal: T = B D^{-1}, then
-      // the off-diagonal block of the inverse -A^{-1} T
-      const int pairs = rp / (2 * sz);
-      const int64_t step = (int64_t)2 * sz * rp + 2 * sz;  // next pair along the diagonal
-      GemmF64 a = {};
-      a.M = sz; a.N = sz; a.K = sz;
-      a.A = R + sz; a.sa_i = rp; a.sa_k = 1;                     // B block
-      a.B = Rinv + (int64_t)sz * rp + sz; a.sb_k = rp; a.sb_j = 1;  // D^{-1}
-      a.C = Tt; a.ldc = sz; a.alpha = 1.0; a.beta = 0.0;
-      a.za = step; a.zb = step; a.zc = (int64_t)sz * sz;
-      if ((st = run_gemm_f64(a, pairs, s)) != PIFA_OK) return st;
-      GemmF64 b = {};
-      b.M = sz; b.N = sz; b.K = sz;
-      b.A = Rinv; b.sa_i = rp; b.sa_k = 1;                        // A^{-1}
-      b.B = Tt; b.sb_k = sz; b.sb_j = 1;
-      b.C = Rinv + sz; b.ldc = rp; b.alpha = -1.0; b.beta = 0.0;
-      b.za = step; b.zb = (int64_t)sz * sz; b.zc = step;
-      if ((st = run_gemm_f64(b, pairs, s)) != PIFA_OK) return st;
-    }
+    if ((st = upper_inverse(R, Rinv, Tt, rp, s)) != PIFA_OK) return st;
   }
   if (has_np) {
     // C[a][asc[j]] = sum_{k >= j} Z[I^c[a]][k] Rinv[j][k]
@@ -594,5 +606,168 @@ extern "C" int pifa_compress_device(const double* U, const double* V, int64_t m,
   }
   if (hflags[0] || !(std::fabs(rdl) >= 1e-8 * std::fabs(rd0)) || rd0 == 0.0)
     return pifa_fail(PIFA_ERR_RANK_DEFICIENT, "W' = U V^T has fewer than r independent rows (|R_rr| < 1e-8 |R_00|)");
+  return PIFA_OK;
+}
+
+// ---- the M reconstruction solves (Sec. 4, Eqs. 4 and 8; Algorithm 3, part 1) ------------------
+namespace {
+
+// dst (rows x cols, pitch lddst, fp64) = src (fp32, pitch ldsrc)
+__global__ void f32_to_f64(const float* src, int64_t ldsrc, int64_t rows, int64_t cols, double* dst, int64_t lddst) {
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < rows * cols; e += (int64_t)gridDim.x * blockDim.x)
+    dst[(e / cols) * lddst + e % cols] = (double)src[(e / cols) * ldsrc + e % cols];
+}
+
+// dst (rows x cols, fp64) += alpha * W (bf16, pitch ldw)
+__global__ void add_scaled_bf16(const __nv_bfloat16* W, int64_t ldw, int64_t rows, int64_t cols, double alpha,
+                                double* dst, int64_t lddst) {
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < rows * cols; e += (int64_t)gridDim.x * blockDim.x)
+    dst[(e / cols) * lddst + e % cols] += alpha * (double)__bfloat162float(W[(e / cols) * ldw + e % cols]);
+}
+
+__global__ void add_diag(double* A, int64_t k, int64_t lda, double alpha) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < k; i += (int64_t)gridDim.x * blockDim.x)
+    A[i * lda + i] += alpha;
+}
+
+// R (rp x rp) = L^T for a lower-triangular L (k x k, pitch k), identity on the padding i >= k.
+__global__ void transpose_pad_lower(const double* L, int64_t k, double* R, int rp) {
+  const int64_t tot = (int64_t)rp * rp;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < tot; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = e / rp, j = e % rp;
+    double v = 0.0;
+    if (i < k && j < k)
+      v = i <= j ? L[j * k + i] : 0.0;
+    else if (i == j)
+      v = 1.0;
+    R[e] = v;
+  }
+}
+
+int grid_for(int64_t work) {
+  const int64_t b = (work + 255) / 256;
+  return (int)(b < 4 * 152 ? (b > 0 ? b : 1) : 4 * 152);
+}
+
+int pad_pow2_32(int64_t k) {
+  int rp = 32;
+  while (rp < k) rp *= 2;
+  return rp;
+}
+
+// Scratch of spd_inverse for k: a copy of S, L, R and R^{-1} (rp x rp), and the doubling's T.
+int64_t spd_scratch_doubles(int64_t k) {
+  const int64_t rp = pad_pow2_32(k);
+  return 2 * k * k + 2 * rp * rp + rp * rp / 4 + 64;
+}
+
+// Sinv = S^{-1} for a symmetric positive definite S (k x k, pitch k): S = L L^T (Cholesky, one
+// column per launch), R = L^T, S^{-1} = R^{-1} R^{-T}. `bad` is set when a pivot is not positive.
+int spd_inverse(const double* S, int64_t k, double* Sinv, double* scratch, int* bad, cudaStream_t s) {
+  const int rp = pad_pow2_32(k);
+  double* G = scratch;
+  double* L = G + k * k;
+  double* R = L + k * k;
+  double* Rinv = R + (int64_t)rp * rp;
+  double* Tt = Rinv + (int64_t)rp * rp;
+  cudaError_t e = cudaMemcpyAsync(G, S, (size_t)k * k * 8, cudaMemcpyDeviceToDevice, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L, 0, (size_t)k * k * 8, s);
+  if (e != cudaSuccess) return pifa_fail_cuda("spd inverse: copy", e);
+  for (int j = 0; j < (int)k; ++j) {
+    const int t = ((int)k - j + 15) / 16;
+    chol_step<<<dim3(t, t), 256, 0, s>>>(G, L, (int)k, j, bad);
+  }
+  transpose_pad_lower<<<grid_for((int64_t)rp * rp), 256, 0, s>>>(L, k, R, rp);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return pifa_fail_cuda("spd inverse: launch", e);
+  int st = upper_inverse(R, Rinv, Tt, rp, s);
+  if (st != PIFA_OK) return st;
+  GemmF64 g = {};  // Sinv[i][j] = sum_t Rinv[i][t] Rinv[j][t]
+  g.M = (int)k; g.N = (int)k; g.K = (int)k;
+  g.A = Rinv; g.sa_i = rp; g.sa_k = 1;
+  g.B = Rinv; g.sb_k = 1; g.sb_j = rp;
+  g.C = Sinv; g.ldc = k; g.alpha = 1.0; g.beta = 0.0;
+  return run_gemm_f64(g, 1, s);
+}
+
+}  // namespace
+
+extern "C" int64_t pifa_m_reconstruct_workspace_size(int64_t m, int64_t n, int64_t r) {
+  pifa_clear_error();
+  if (m < 1 || n < 1 || r < 1 || r > n || r > m) return pifa_fail(PIFA_ERR_INVALID_ARG, "need 1 <= r <= min(m, n)");
+  if (n > 16384 || m >= ((int64_t)1 << 30)) return pifa_fail(PIFA_ERR_UNSUPPORTED, "pifa_m_reconstruct needs n <= 16384");
+  const int64_t d = 2 * n * n + m * n + n * r + m * r + 4 * r * r + 2 * r * n + spd_scratch_doubles(n > r ? n : r) + 64;
+  return d * 8 + 256;
+}
+
+extern "C" int pifa_m_reconstruct(const float* XXt, int64_t ldxx, const float* YtXt, int64_t ldyx, const double* V,
+                                  const void* W, int64_t ldw, int64_t m, int64_t n, int64_t r, double alpha,
+                                  double* U_r, double* V_r, void* workspace, int64_t workspace_bytes,
+                                  void* cuda_stream) {
+  const int64_t need = pifa_m_reconstruct_workspace_size(m, n, r);
+  if (need < 0) return (int)need;
+  pifa_clear_error();
+  if (!XXt || !YtXt || !V || !U_r || !V_r || (alpha != 0.0 && !W))
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "null XXt, YtXt, V, U_r, V_r, or W with alpha != 0");
+  if (!(alpha >= 0.0)) return pifa_fail(PIFA_ERR_INVALID_ARG, "alpha must be >= 0");
+  if (ldxx < n || ldyx < n || (W && ldw < n)) return pifa_fail(PIFA_ERR_INVALID_ARG, "leading dimension smaller than the row");
+  if (!workspace || workspace_bytes < need) return pifa_fail(PIFA_ERR_WORKSPACE, "workspace missing or too small");
+  if (reinterpret_cast<uintptr_t>(workspace) & 255u) return pifa_fail(PIFA_ERR_ALIGNMENT, "workspace must be 256-byte aligned");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(cuda_stream);
+  double* A = static_cast<double*>(workspace);  // X X^T (n x n), later X X^T + alpha I
+  double* B = A + n * n;                         // Y_t X^T (m x n), later + alpha W
+  double* T1 = B + m * n;                        // X X^T V (n x r)
+  double* Sm = T1 + n * r;                       // V^T X X^T V (r x r)
+  double* B1 = Sm + r * r;                       // Y_t X^T V (m x r)
+  double* Sinv = B1 + m * r;
+  double* Pm = Sinv + r * r;                     // U_r^T U_r
+  double* Pinv = Pm + r * r;
+  double* Rhs = Pinv + r * r;                    // U_r^T (Y_t X^T + alpha W) (r x n)
+  double* Q = Rhs + r * n;                       // (U_r^T U_r)^{-1} Rhs (r x n)
+  double* Ginv = Q + r * n;                      // (X X^T + alpha I)^{-1}
+  int* bad = reinterpret_cast<int*>(Ginv + n * n);
+  double* scratch = reinterpret_cast<double*>(bad) + 8;
+  cudaError_t e = cudaMemsetAsync(bad, 0, 8, s);
+  if (e != cudaSuccess) return pifa_fail_cuda("reconstruct: memset", e);
+  f32_to_f64<<<grid_for(n * n), 256, 0, s>>>(XXt, ldxx, n, n, A, n);
+  f32_to_f64<<<grid_for(m * n), 256, 0, s>>>(YtXt, ldyx, m, n, B, n);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return pifa_fail_cuda("reconstruct: launch", e);
+  const int ni = (int)n, mi = (int)m, ri = (int)r;
+  int st;
+  auto gemm = [&](int M, int N, int K, const double* Ap, int64_t sai, int64_t sak, const double* Bp, int64_t sbk,
+                  int64_t sbj, double* Cp, int64_t ldc) {
+    GemmF64 g = {};
+    g.M = M; g.N = N; g.K = K;
+    g.A = Ap; g.sa_i = sai; g.sa_k = sak;
+    g.B = Bp; g.sb_k = sbk; g.sb_j = sbj;
+    g.C = Cp; g.ldc = ldc; g.alpha = 1.0; g.beta = 0.0;
+    return run_gemm_f64(g, 1, s);
+  };
+  // Eq. 4: U_r = (Y_t X^T) V (V^T (X X^T) V)^{-1}
+  if ((st = gemm(ni, ri, ni, A, n, 1, V, r, 1, T1, r)) != PIFA_OK) return st;
+  if ((st = gemm(ri, ri, ni, V, 1, r, T1, r, 1, Sm, r)) != PIFA_OK) return st;   // V^T T1
+  if ((st = gemm(mi, ri, ni, B, n, 1, V, r, 1, B1, r)) != PIFA_OK) return st;
+  if ((st = spd_inverse(Sm, r, Sinv, scratch, bad, s)) != PIFA_OK) return st;
+  if ((st = gemm(mi, ri, ri, B1, r, 1, Sinv, r, 1, U_r, r)) != PIFA_OK) return st;
+  // Eq. 8: V_r^T = (U_r^T U_r)^{-1} U_r^T (Y_t X^T + alpha W) (X X^T + alpha I)^{-1}
+  if ((st = gemm(ri, ri, mi, U_r, 1, r, U_r, r, 1, Pm, r)) != PIFA_OK) return st;   // U_r^T U_r
+  if ((st = spd_inverse(Pm, r, Pinv, scratch, bad, s)) != PIFA_OK) return st;
+  if (alpha != 0.0) {
+    add_scaled_bf16<<<grid_for(m * n), 256, 0, s>>>(static_cast<const __nv_bfloat16*>(W), ldw, m, n, alpha, B, n);
+    add_diag<<<grid_for(n), 256, 0, s>>>(A, n, n, alpha);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return pifa_fail_cuda("reconstruct: launch", e);
+  }
+  if ((st = gemm(ri, ni, mi, U_r, 1, r, B, n, 1, Rhs, n)) != PIFA_OK) return st;   // U_r^T B
+  if ((st = gemm(ri, ni, ri, Pinv, r, 1, Rhs, n, 1, Q, n)) != PIFA_OK) return st;
+  if ((st = spd_inverse(A, n, Ginv, scratch, bad, s)) != PIFA_OK) return st;
+  // V_r = (Q Ginv)^T = Ginv Q^T (Ginv symmetric)
+  if ((st = gemm(ni, ri, ni, Ginv, n, 1, Q, 1, n, V_r, r)) != PIFA_OK) return st;
+  int hbad = 0;
+  e = cudaMemcpyAsync(&hbad, bad, sizeof(int), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return pifa_fail_cuda("reconstruct: synchronize", e);
+  if (hbad) return pifa_fail(PIFA_ERR_RANK_DEFICIENT, "a matrix of the reconstruction is not positive definite");
   return PIFA_OK;
 }

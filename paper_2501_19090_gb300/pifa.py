@@ -48,6 +48,7 @@ EXPORTS = (
     "pifa_set_wait_timeout", "pifa_selftest_wait_timeout", "pifa_set_decode_grid", "pifa_forward_grouped",
     "pifa_workspace_size_grouped", "pifa_compress_device", "pifa_compress_device_workspace_size",
     "pifa_backward", "pifa_backward_workspace_size", "pifa_m_accumulate", "pifa_m_accumulate_workspace_size",
+    "pifa_m_reconstruct", "pifa_m_reconstruct_workspace_size",
 )
 
 
@@ -115,6 +116,11 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.pifa_m_accumulate.restype = ctypes.c_int
         lib.pifa_m_accumulate_workspace_size.argtypes = [_I64, _I64, _I64]
         lib.pifa_m_accumulate_workspace_size.restype = _I64
+        lib.pifa_m_reconstruct.argtypes = [_VP, _I64, _VP, _I64, _VP, _VP, _I64, _I64, _I64, _I64, ctypes.c_double,
+                                           _VP, _VP, _VP, _I64, _VP]
+        lib.pifa_m_reconstruct.restype = ctypes.c_int
+        lib.pifa_m_reconstruct_workspace_size.argtypes = [_I64, _I64, _I64]
+        lib.pifa_m_reconstruct_workspace_size.restype = _I64
         lib.pifa_validate_indices.argtypes = [_VP, _VP, _I64, _I64]
         lib.pifa_validate_indices.restype = ctypes.c_int
         lib.pifa_device_status.argtypes = [_VP]
@@ -519,3 +525,36 @@ def pifa_m_accumulate(Xo, Xu, W, lam, XXt, YtXt=None, workspace_tensor=None, str
         _ld(YtXt) if YtXt is not None else n, ws_ptr, ws_bytes, _stream_ptr(stream))
     _check(st, "pifa_m_accumulate")
     return XXt, YtXt
+
+
+def pifa_m_reconstruct(XXt, YtXt, V, W=None, alpha=0.0, stream=None):
+    """The M reconstruction (pifa_m_reconstruct): U_r (Eq. 4) and V_r (Eq. 8) in float64 from the
+    fp32 accumulators XXt (n x n) and YtXt (m x n), V (n x r, converted to float64) and, for
+    alpha > 0, the dense W (bf16 m x n). Returns (U_r, V_r) as float64 CUDA tensors."""
+    import torch
+    n = XXt.shape[0]
+    m = YtXt.shape[0]
+    for name, t in (("XXt", XXt), ("YtXt", YtXt)):
+        if not isinstance(t, torch.Tensor) or t.dtype != torch.float32 or t.dim() != 2 or t.device.type != "cuda":
+            raise ValueError(f"pifa: {name} must be a 2-D float32 CUDA tensor")
+    if tuple(XXt.shape) != (n, n) or YtXt.shape[1] != n:
+        raise ValueError("pifa: XXt must be n x n and YtXt m x n")
+    V = V.to(device=XXt.device, dtype=torch.float64).contiguous()
+    if V.dim() != 2 or V.shape[0] != n:
+        raise ValueError("pifa: V must be n x r")
+    r = V.shape[1]
+    if alpha and (W is None or W.dtype != torch.bfloat16 or tuple(W.shape) != (m, n)):
+        raise ValueError("pifa: alpha > 0 needs W, a bfloat16 m x n tensor")
+    need = int(_lib().pifa_m_reconstruct_workspace_size(m, n, r))
+    if need < 0:
+        _check(need, "pifa_m_reconstruct_workspace_size")
+    ws = torch.empty(need + 256, dtype=torch.uint8, device=XXt.device)
+    ws_ptr = ws.data_ptr() + (-ws.data_ptr()) % 256
+    U_r = torch.empty((m, r), dtype=torch.float64, device=XXt.device)
+    V_r = torch.empty((n, r), dtype=torch.float64, device=XXt.device)
+    st = _lib().pifa_m_reconstruct(XXt.data_ptr(), _ld(XXt), YtXt.data_ptr(), _ld(YtXt), V.data_ptr(),
+                                   W.data_ptr() if (alpha and W is not None) else None, _ld(W) if (alpha and W is not None) else n,
+                                   m, n, r, float(alpha), U_r.data_ptr(), V_r.data_ptr(), ws_ptr, need,
+                                   _stream_ptr(stream))
+    _check(st, "pifa_m_reconstruct")
+    return U_r, V_r

@@ -144,3 +144,54 @@ def test_m_accumulate_llama_shape_sampled_rows():
     a, b = oracle.m_accumulate(Xo, Xu, W, 0.25, rows=(rx, ry))
     check(XXt[torch.from_numpy(rx)].cpu().numpy(), a, "X X^T rows")
     check(YtXt[torch.from_numpy(ry)].cpu().numpy(), b, "Y_t X^T rows")
+
+
+# ---------------------------------------------------------------------------------------------
+# pifa_m_reconstruct: U_r (Eq. 4) and V_r (Eq. 8) from the accumulators, float64
+# ---------------------------------------------------------------------------------------------
+def _accumulated(T, n, m, r, seed):
+    Xo, Xu, W = _macc_inputs(T, n, m, seed)
+    XXt = torch.zeros((n, n), dtype=torch.float32, device=DEV)
+    YtXt = torch.zeros((m, n), dtype=torch.float32, device=DEV)
+    P.pifa_m_accumulate(dev_bf16(Xo), dev_bf16(Xu), dev_bf16(W), 0.25, XXt, YtXt)
+    V = np.random.default_rng(seed + 100).standard_normal((n, r)) / np.sqrt(n)
+    return Xo, Xu, W, XXt, YtXt, V
+
+
+@pytest.mark.parametrize("m,n,r,T,alpha", [(300, 256, 64, 1000, 0.0), (300, 256, 64, 1000, 1e-3),
+                                           (1024, 1024, 256, 3000, 1e-3)])
+def test_m_reconstruct_matches_the_oracle_on_the_same_accumulators(m, n, r, T, alpha):
+    """Same fp32 accumulators on both sides; both solve in float64 (the library by Cholesky and
+    triangular inverses, the oracle by LAPACK solves): agreement to 1e-8 relative."""
+    Xo, Xu, W, XXt, YtXt, V = _accumulated(T, n, m, r, 7)
+    Wd = dev_bf16(W)
+    U_r, V_r = P.pifa_m_reconstruct(XXt, YtXt, torch.from_numpy(V).to(DEV), W=Wd, alpha=alpha)
+    A, B = XXt.double().cpu().numpy(), YtXt.double().cpu().numpy()
+    rU, rV = oracle.m_reconstruct(A, B, V, W=W.astype(np.float64), alpha=alpha)
+    for got, ref, what in ((U_r, rU, "U_r"), (V_r, rV, "V_r")):
+        got = got.cpu().numpy()
+        rel = np.linalg.norm(got - ref) / np.linalg.norm(ref)
+        assert rel <= 1e-8, f"{what}: rel {rel:.3e}"
+
+
+def test_m_path_end_to_end_against_the_oracle():
+    """GPU accumulation then GPU reconstruction against the oracle's accumulation and
+    reconstruction from the same bf16 samples: within the bf16 tolerance."""
+    m, n, r, T = 300, 256, 64, 1000
+    Xo, Xu, W, XXt, YtXt, V = _accumulated(T, n, m, r, 8)
+    U_r, V_r = P.pifa_m_reconstruct(XXt, YtXt, torch.from_numpy(V).to(DEV), W=dev_bf16(W), alpha=1e-3)
+    A, B = oracle.m_accumulate(Xo, Xu, W, 0.25)
+    rU, rV = oracle.m_reconstruct(A, B, V, W=W.astype(np.float64), alpha=1e-3)
+    check(U_r.cpu().numpy(), rU, "U_r")
+    # the reconstructed layer U_r V_r^T is the product that matters downstream
+    check((U_r @ V_r.t()).cpu().numpy(), rU @ rV.T, "U_r V_r^T")
+
+
+def test_m_reconstruct_reports_a_singular_system():
+    """Fewer samples than inputs (T < n) leave X X^T singular; without the regulariser
+    (alpha = 0) Eq. 7 has no unique solution: PIFA_ERR_RANK_DEFICIENT."""
+    m, n, r, T = 128, 256, 32, 100
+    _, _, _, XXt, YtXt, V = _accumulated(T, n, m, r, 9)
+    with pytest.raises(P.PifaError) as e:
+        P.pifa_m_reconstruct(XXt, YtXt, torch.from_numpy(V).to(DEV), alpha=0.0)
+    assert e.value.status == P.PIFA_ERR_RANK_DEFICIENT
