@@ -3,23 +3,28 @@
 //
 // A phase is a skinny product D = A B^T: A the weight rows (W_p for Y_p = X W_p^T, Algorithm 2
 // step 2; C for Y_np = Y_p C^T, step 3), B the T token rows (x, or y_p as its hi and lo planes).
-// The weight matrix is cut into units of 128 rows x one K-slice; units are numbered slice-major
-// (u = s nrb + rb) and dealt to the CTAs in equal contiguous ranges, so every SM streams the same
-// number of weight bytes and a CTA meets few distinct K-slices of B.
+// The weight matrix is cut into units of 128 rows x one K-slice, and a unit into chunks of 64
+// columns (one 16 KB weight tile). Units are numbered slice-major (u = s nrb + rb) and the chunks
+// of all units, in that order, are dealt to the CTAs in equal contiguous ranges: every CTA streams
+// the same number of weight bytes to within one tile, whatever the unit count. The slice width is
+// the largest multiple of 64 that keeps a unit no longer than a CTA's range, so a unit is split
+// between at most two CTAs: its head (chunk 0 on) goes to P, its tail (if split) to P2.
 //
 // Partial kernel (two CTAs per SM, 192 threads each):
-//   warp 0     TMA producer: the weight tiles (128 rows x 64 columns, 16 KB, 128-byte swizzle)
-//              through a ring of stages, the first ones before the dependency wait (the weights
-//              do not depend on the previous kernel); the unit's K-slice of B into one of two
-//              buffers (16 token rows x 64 columns per box; rows >= T zero-filled), after the wait.
-//   warp 1     owns 256 TMEM columns (two units in flight) and issues tcgen05.mma.kind::f16
+//   warp 0     TMA producer: per chunk, the weight tile (128 rows x 64 columns, 128-byte swizzle)
+//              and the matching 64 columns of B (16 token rows per plane; rows >= T zero-filled)
+//              into one stage of a ring; the first weight tiles go out before the dependency wait
+//              (the weights do not depend on the previous kernel), their B boxes after it.
+//   warp 1     owns 256 TMEM columns (two segments in flight) and issues tcgen05.mma.kind::f16
 //              M = 128, K = 16, N = 16 (one B plane) or 32 (the y_p hi and lo planes as one
-//              operand) from one thread, dealing a unit's MMAs round-robin over independent
+//              operand) from one thread, dealing a segment's MMAs round-robin over independent
 //              accumulators so that consecutive MMAs do not wait for each other.
-//   warps 2-5  sum a unit's accumulators (TMEM lane quarter each) while the next unit fills the
-//              other set, and store its partial sums P[s][t][row] (fp32, coalesced over rows).
-// Reduce kernel: Y[t, cols[j]] = bf16(sum_s P[s][t][j]) in slice order (deterministic); phase 1
-// also writes y_p as the hi + lo planes of C's dtype that phase 2 reads.
+//   warps 2-5  sum a segment's accumulators (TMEM lane quarter each) while the next segment fills
+//              the other set, and store its partial sums P[s][t][row] (fp32, coalesced over rows).
+// A unit's head CTA writes zeros to P2 when it holds the whole unit, so P2 is defined everywhere.
+// Reduce kernel: Y[t, cols[j]] = bf16(sum_s (P[s][t][j] + P2[s][t][j])) in slice order
+// (deterministic for a given grid); phase 1 also writes y_p as the hi + lo planes of C's dtype
+// that phase 2 reads.
 // Every wait is bounded (globaltimer); on timeout the CTA latches PIFA_ERR_TIMEOUT, drains what
 // it has in flight and returns.
 #include <cuda_bf16.h>
@@ -41,11 +46,11 @@ constexpr uint32_t A_BYTES = TM * KB * 2;       // one weight tile
 constexpr uint32_t BOX_BYTES = TN * KB * 2;     // one B box
 constexpr int MAX_STAGES = 10;
 constexpr int THREADS = 192;
-// A unit's MMAs are dealt round-robin over NACC independent accumulators (summed in the
+// A segment's MMAs are dealt round-robin over NACC independent accumulators (summed in the
 // epilogue), so that consecutive MMAs do not wait for each other. With two B planes (y_p hi and
 // lo) one MMA of N = 32 covers both: the lo box follows the hi box in shared memory, making one
-// 32-row operand, and accumulator columns t and 16 + t are added in the epilogue. Per unit
-// NACC * 16 * NB columns; two units in flight: 256 TMEM columns either way.
+// 32-row operand, and accumulator columns t and 16 + t are added in the epilogue. Per segment
+// NACC * 16 * NB columns; two segments in flight: 256 TMEM columns either way.
 template <int NB>
 constexpr int kNacc = NB == 1 ? 8 : 4;
 constexpr uint32_t TMEM_COLS = 256;
@@ -54,44 +59,93 @@ constexpr uint32_t TMEM_COLS = 256;
 // four, 73 us with three of two), so a CTA keeps to half an SM's shared memory and TMEM.
 constexpr int CTAS_PER_SM = 2;
 constexpr size_t SMEM_PER_CTA = 112 * 1024;
+// The grid never exceeds GRID_MAX CTAs: the slice plan made for GRID_MAX bounds the partial-sum
+// bytes of every smaller grid (a smaller grid gives longer ranges, wider slices, fewer of them).
+constexpr int GRID_MAX = 512;
+constexpr int MIN_CHUNKS_PER_CTA = 4;
+
+// How one phase is cut: slice width, slice count and grid.
+struct Plan {
+  int nrb, nck;   // 128-row blocks; 64-column chunks over K
+  int64_t total;  // chunks over all units (nrb * nck)
+  int grid;       // CTAs
+  int ncf;        // chunks per full slice
+  int ns;         // slices
+  int nclast;     // chunks in the last slice
+};
+
+Plan make_plan(int64_t R, int64_t K, int grid_cap) {
+  Plan p;
+  p.nrb = (int)((R + TM - 1) / TM);
+  p.nck = (int)((K + KB - 1) / KB);
+  p.total = (int64_t)p.nrb * p.nck;
+  int64_t g = p.total / MIN_CHUNKS_PER_CTA;
+  if (g > grid_cap) g = grid_cap;
+  if (g < 1) g = 1;
+  p.grid = (int)g;
+  int64_t u = p.total / p.grid;  // every CTA range holds at least u chunks
+  if (u > p.nck) u = p.nck;
+  if (u < 1) u = 1;
+  p.ncf = (int)u;
+  p.ns = (p.nck + p.ncf - 1) / p.ncf;
+  p.nclast = p.nck - (p.ns - 1) * p.ncf;
+  return p;
+}
 
 struct TcArgs {
   int R, K, T;
-  int nrb, ns, KS;  // 128-row blocks, K-slices, slice width (a multiple of 64)
-  int units;        // ns * nrb
-  int gsz, goff;    // grouped layers: rows per group (a multiple of 128) and B columns per group
+  int nrb, ns, ncf, nclast;  // 128-row blocks, K-slices, chunks per full / last slice
+  int64_t total;             // chunks over all units
+  int grid;
+  int gsz, goff;  // grouped layers: rows per group (a multiple of 128) and B columns per group
   int stages;
-  uint32_t chunk_bytes;  // B bytes per 64-column chunk of a slice: NB boxes (hi, then lo)
+  uint32_t stage_bytes;  // one weight tile and NB B boxes (hi, then lo)
   uint32_t idesc;
-  float* P;              // partial sums [ns][T][R]
+  float* P;   // partial sums of unit heads [ns][T][R]
+  float* P2;  // partial sums of the tails of split units [ns][T][R]
   int* status;
   uint64_t timeout_ns;
 };
 
-__device__ __forceinline__ int unit_key(const TcArgs& a, int u) {
-  const int s = u / a.nrb, rb = u % a.nrb;
-  const int g = a.gsz > 0 ? (rb * TM) / a.gsz : 0;
-  return g * a.ns + s;
+// A CTA's run of chunks inside one unit.
+struct Seg {
+  int s, rb;  // the unit
+  int c0;     // its first chunk within the unit
+  int nc;     // chunks
+};
+
+// The segment that starts at chunk g of the global order and ends at the unit's end or at e.
+__host__ __device__ __forceinline__ Seg seg_at(int nrb, int ns, int ncf, int nclast, int64_t g, int64_t e) {
+  const int64_t per = (int64_t)nrb * ncf;
+  int s = (int)(g / per);
+  if (s > ns - 1) s = ns - 1;
+  const int64_t rem = g - (int64_t)s * per;
+  const int n = s < ns - 1 ? ncf : nclast;
+  Seg q;
+  q.s = s;
+  q.rb = (int)(rem / n);
+  q.c0 = (int)(rem % n);
+  const int64_t uend = g - q.c0 + n;
+  q.nc = (int)((uend < e ? uend : e) - g);
+  return q;
 }
-__device__ __forceinline__ int unit_chunks(const TcArgs& a, int u) {
-  const int s = u / a.nrb;
-  return (min(a.KS, a.K - s * a.KS) + KB - 1) / KB;
+
+__device__ __forceinline__ Seg seg_at(const TcArgs& a, int64_t g, int64_t e) {
+  return seg_at(a.nrb, a.ns, a.ncf, a.nclast, g, e);
 }
+
+// Column (within the unit's K-slice) of the c-th chunk a CTA loads for segment q.
+__device__ __forceinline__ int seg_col(const Seg& q, int c) { return (q.c0 + c) * KB; }
 
 template <int NB>
 __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
     decode_tc_partial(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                       const __grid_constant__ CUtensorMap tmB1, TcArgs a) {
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t bbuf = (uint32_t)(a.KS / KB) * a.chunk_bytes;  // one B buffer (both planes)
-  uint8_t* bsm = smem;                                  // two B buffers
-  uint8_t* ring = smem + 2 * bbuf;                      // weight stages (1024-aligned: bbuf % 2048 == 0)
-  uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)a.stages * A_BYTES);
+  uint8_t* ring = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(ring + (size_t)a.stages * a.stage_bytes);
   uint64_t* empty = full + MAX_STAGES;
-  uint64_t* bfull = empty + MAX_STAGES;
-  uint64_t* bempty = bfull + 2;
-  uint64_t* accf = bempty + 2;
+  uint64_t* accf = empty + MAX_STAGES;
   uint64_t* acce = accf + 2;
   uint64_t* drain = acce + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -99,8 +153,8 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
 
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int u0 = (int)(((int64_t)blockIdx.x * a.units) / gridDim.x);
-  const int u1 = (int)(((int64_t)(blockIdx.x + 1) * a.units) / gridDim.x);
+  const int64_t g0 = ((int64_t)blockIdx.x * a.total) / a.grid;
+  const int64_t g1 = ((int64_t)(blockIdx.x + 1) * a.total) / a.grid;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < a.stages; ++s) {
@@ -108,8 +162,6 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&bfull[b], 1);
-      mbar_init(&bempty[b], 1);
       mbar_init(&accf[b], 1);
       mbar_init(&acce[b], 4);
     }
@@ -132,109 +184,85 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- producer ----------------
-      int total = 0;
-      for (int u = u0; u < u1; ++u) total += unit_chunks(a, u);
+      const int total = (int)(g1 - g0);
       const int pre = min(total, a.stages);
-      {  // weight tiles of the first stages, before the dependency wait
+      {  // weight tiles of the first stages, before the dependency wait; their B boxes follow it
         int it = 0;
-        for (int u = u0; u < u1 && it < pre; ++u) {
-          const int s = u / a.nrb, rb = u % a.nrb, nck = unit_chunks(a, u);
-          for (int c = 0; c < nck && it < pre; ++c, ++it) {
-            mbar_arrive_expect_tx(&full[it], A_BYTES);
-            tma_load_2d(smem_u32(ring + (size_t)it * A_BYTES), &tmA, s * a.KS + c * KB, rb * TM, &full[it]);
+        for (int64_t g = g0; it < pre;) {
+          const Seg q = seg_at(a, g, g1);
+          for (int c = 0; c < q.nc && it < pre; ++c, ++it) {
+            mbar_arrive_expect_tx(&full[it], a.stage_bytes);
+            tma_load_2d(smem_u32(ring + (size_t)it * a.stage_bytes), &tmA, q.s * a.ncf * KB + seg_col(q, c),
+                        q.rb * TM, &full[it]);
           }
+          g += q.nc;
         }
       }
       pdl_wait_primary();
-      int it = 0, kb = -1, cur = -1, issued = 0;
+      int it = 0;
       bool dead = false;
-      for (int u = u0; u < u1 && !dead; ++u) {
-        const int s = u / a.nrb, rb = u % a.nrb, nck = unit_chunks(a, u);
-        const int key = unit_key(a, u);
-        if (key != cur) {  // the unit's K-slice of B into the next buffer
-          ++kb;
-          cur = key;
-          const int b = kb & 1;
-          if (kb >= 2 && !mbar_wait(&bempty[b], (uint32_t)((kb >> 1) - 1) & 1u, a.timeout_ns)) {
-            latch_status(a.status, PIFA_ERR_TIMEOUT);
-            *abort_flag = 1;
-            dead = true;
-            break;
-          }
-          const int x0 = (a.gsz > 0 ? ((rb * TM) / a.gsz) * a.goff : 0) + s * a.KS;
-          mbar_arrive_expect_tx(&bfull[b], (uint32_t)(NB * nck) * BOX_BYTES);
-          uint8_t* dst = bsm + b * bbuf;
-          for (int c = 0; c < nck; ++c) {
-            tma_load_2d(smem_u32(dst + c * a.chunk_bytes), &tmB0, x0 + c * KB, 0, &bfull[b]);
-            if (NB > 1) tma_load_2d(smem_u32(dst + c * a.chunk_bytes + BOX_BYTES), &tmB1, x0 + c * KB, 0, &bfull[b]);
-          }
-        }
-        for (int c = 0; c < nck; ++c, ++it) {
-          if (it < pre) continue;  // issued before the wait
+      for (int64_t g = g0; g < g1 && !dead;) {
+        const Seg q = seg_at(a, g, g1);
+        g += q.nc;
+        const int x0 = (a.gsz > 0 ? ((q.rb * TM) / a.gsz) * a.goff : 0) + q.s * a.ncf * KB;
+        for (int c = 0; c < q.nc; ++c, ++it) {
           const int st = it % a.stages;
-          if (!mbar_wait(&empty[st], (uint32_t)((it / a.stages) - 1) & 1u, a.timeout_ns) || *abort_flag) {
-            latch_status(a.status, PIFA_ERR_TIMEOUT);
-            *abort_flag = 1;
-            dead = true;
-            break;
+          uint8_t* stage = ring + (size_t)st * a.stage_bytes;
+          const int kx = seg_col(q, c);
+          if (it >= pre) {
+            if (!mbar_wait(&empty[st], (uint32_t)((it / a.stages) - 1) & 1u, a.timeout_ns) || *abort_flag) {
+              latch_status(a.status, PIFA_ERR_TIMEOUT);
+              *abort_flag = 1;
+              dead = true;
+              break;
+            }
+            mbar_arrive_expect_tx(&full[st], a.stage_bytes);
+            tma_load_2d(smem_u32(stage), &tmA, q.s * a.ncf * KB + kx, q.rb * TM, &full[st]);
           }
-          mbar_arrive_expect_tx(&full[st], A_BYTES);
-          tma_load_2d(smem_u32(ring + (size_t)st * A_BYTES), &tmA, s * a.KS + c * KB, rb * TM, &full[st]);
+          tma_load_2d(smem_u32(stage + A_BYTES), &tmB0, x0 + kx, 0, &full[st]);
+          if (NB > 1) tma_load_2d(smem_u32(stage + A_BYTES + BOX_BYTES), &tmB1, x0 + kx, 0, &full[st]);
         }
       }
-      issued = dead ? it : total;
+      int issued = dead ? it : total;
       if (issued < pre) issued = pre;
-      // nothing may land in shared memory once the CTA has left: the last use of every stage and
-      // of both B buffers
+      // nothing may land in shared memory once the CTA has left: the last use of every stage
       for (int j = issued > a.stages ? issued - a.stages : 0; j < issued; ++j)
         if (!mbar_wait(&full[j % a.stages], (uint32_t)(j / a.stages) & 1u, 100000000ull))
-          latch_status(a.status, PIFA_ERR_TIMEOUT);
-      for (int k = kb > 1 ? kb - 1 : 0; k <= kb; ++k)
-        if (k >= 0 && !mbar_wait(&bfull[k & 1], (uint32_t)(k >> 1) & 1u, 100000000ull))
           latch_status(a.status, PIFA_ERR_TIMEOUT);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
-      int it = 0, kb = -1, cur = -1;
+      int it = 0, j = 0;
       bool dead = false;
-      for (int u = u0; u < u1 && !dead; ++u) {
-        const int j = u - u0, acc = j & 1, nck = unit_chunks(a, u);
-        const int key = unit_key(a, u);
-        if (key != cur) {
-          ++kb;
-          cur = key;
-          if (!mbar_wait(&bfull[kb & 1], (uint32_t)(kb >> 1) & 1u, a.timeout_ns)) {
-            dead = true;
-            break;
-          }
-        }
+      for (int64_t g = g0; g < g1; ++j) {
+        const Seg q = seg_at(a, g, g1);
+        g += q.nc;
+        const int acc = j & 1;
         if (j >= 2 && !mbar_wait(&acce[acc], (uint32_t)((j >> 1) - 1) & 1u, a.timeout_ns)) {
           dead = true;
           break;
         }
         tc_fence_after();
-        const uint32_t bbase = smem_u32(bsm + (kb & 1) * bbuf);
         constexpr int NACC = kNacc<NB>;
         const uint32_t dacc = tmem + (uint32_t)(acc * NACC * TN * NB);
-        int e = 0;  // MMAs of this unit so far: accumulator e % NACC, first use overwrites
-        for (int c = 0; c < nck; ++c, ++it) {
+        int e = 0;  // MMAs of this segment so far: accumulator e % NACC, first use overwrites
+        for (int c = 0; c < q.nc; ++c, ++it) {
           const int st = it % a.stages;
           if (!mbar_wait(&full[st], (uint32_t)(it / a.stages) & 1u, a.timeout_ns) || *abort_flag) {
             dead = true;
             break;
           }
           tc_fence_after();
-          const uint32_t at = smem_u32(ring + (size_t)st * A_BYTES);
+          const uint32_t at = smem_u32(ring + (size_t)st * a.stage_bytes);
 #pragma unroll
           for (int kk = 0; kk < KB / 16; ++kk, ++e)
             mma_bf16_ss(dacc + (uint32_t)((e % NACC) * TN * NB), sw128_desc(at + kk * 32),
-                        sw128_desc(bbase + c * a.chunk_bytes + kk * 32), a.idesc, e >= NACC ? 1u : 0u);
+                        sw128_desc(at + A_BYTES + kk * 32), a.idesc, e >= NACC ? 1u : 0u);
           mma_commit(&empty[st]);  // the stage is free once these MMAs have read it
         }
         if (dead) break;
         mma_commit(&accf[acc]);
-        if (u + 1 == u1 || unit_key(a, u + 1) != cur) mma_commit(&bempty[kb & 1]);
       }
       if (dead) {
         latch_status(a.status, PIFA_ERR_TIMEOUT);
@@ -245,46 +273,54 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
     }
   } else {
     // ---------------- epilogue: warps 2..5, TMEM lane quarter warp % 4 ----------------
-    const int q = warp & 3;
-    for (int u = u0; u < u1; ++u) {
-      const int j = u - u0, acc = j & 1;
-      const int s = u / a.nrb, rb = u % a.nrb;
+    const int q4 = warp & 3;
+    int j = 0;
+    for (int64_t g = g0; g < g1; ++j) {
+      const Seg q = seg_at(a, g, g1);
+      g += q.nc;
+      const int acc = j & 1;
       if (!mbar_wait(&accf[acc], (uint32_t)(j >> 1) & 1u, a.timeout_ns) || *abort_flag) {
         latch_status(a.status, PIFA_ERR_TIMEOUT);
         *abort_flag = 1;
         break;
       }
       tc_fence_after();
-      // the accumulators this unit wrote (fewer than NACC only when it has fewer MMAs), summed in
-      // a fixed order
+      // the accumulators this segment wrote (fewer than NACC only when it has fewer MMAs), summed
+      // in a fixed order
       constexpr int NACC = kNacc<NB>;
-      const int used = min(NACC, unit_chunks(a, u) * (KB / 16));
-      const uint32_t base = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * NACC * TN * NB);
+      const int used = min(NACC, q.nc * (KB / 16));
+      const uint32_t base = tmem + ((uint32_t)(q4 * 32) << 16) + (uint32_t)(acc * NACC * TN * NB);
       float sum[TN];
 #pragma unroll
       for (int t = 0; t < TN; ++t) sum[t] = 0.0f;
       // column groups of 16: accumulator a, plane nb at (a NB + nb) 16
-      for (int g0 = 0; g0 < used * NB; g0 += 4) {
+      for (int c0 = 0; c0 < used * NB; c0 += 4) {
         uint32_t v[4][16];
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          if (g0 + k < used * NB) tmem_ld_32x32b_x16(base + (uint32_t)((g0 + k) * TN), v[k]);
+          if (c0 + k < used * NB) tmem_ld_32x32b_x16(base + (uint32_t)((c0 + k) * TN), v[k]);
         tmem_ld_wait();
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          if (g0 + k < used * NB)
+          if (c0 + k < used * NB)
 #pragma unroll
             for (int t = 0; t < TN; ++t) sum[t] += __uint_as_float(v[k][t]);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acce[acc]);  // this quarter of the accumulators may be refilled
-      const int row = rb * TM + q * 32 + lane;
+      // the head of a unit goes to P and, when the unit was not split, zeros to P2; a tail to P2
+      const int row = q.rb * TM + q4 * 32 + lane;
       if (row < a.R) {
-        float* dst = a.P + (size_t)s * a.T * a.R + row;
+        const size_t off = (size_t)q.s * a.T * a.R + row;
+        const bool whole = q.c0 == 0 && q.nc == (q.s < a.ns - 1 ? a.ncf : a.nclast);
+        float* dst = (q.c0 == 0 ? a.P : a.P2) + off;
 #pragma unroll
         for (int t = 0; t < TN; ++t)
-          if (t < a.T) dst[(size_t)t * a.R] = sum[t];
+          if (t < a.T) {
+            dst[(size_t)t * a.R] = sum[t];
+            if (whole) a.P2[off + (size_t)t * a.R] = 0.0f;
+          }
       }
     }
   }
@@ -318,6 +354,7 @@ __device__ __forceinline__ void split_hi_lo(float f, uint16_t& h, uint16_t& l, b
 
 struct ReduceArgs {
   const float* P;
+  const float* P2;
   int ns, T, R;
   const int32_t* cols;  // output column of each row (I or I^c)
   int m;                // columns of Y (index bound)
@@ -329,8 +366,11 @@ struct ReduceArgs {
   int* status;
 };
 
-// Y[t, cols[j]] = bf16(sum_s P[s][t][j]), slices summed in order; phase 1 also splits y_p.
-template <bool kF16>
+// One row j of one token t per thread: Y[t, cols[j]] = bf16 of sum_s (P[s][t][j] + P2[s][t][j])
+// in slice order. The loads of G slices (G >= ns up to 16) are all in flight at once (no load
+// depends on another), so the kernel takes about one memory round trip; G is no larger than the
+// slice count needs, which keeps registers low and the grid resident. Phase 1 also splits y_p.
+template <bool kF16, int G>
 __global__ void __launch_bounds__(256) decode_tc_reduce(ReduceArgs a) {
   pdl_launch_dependents();
   pdl_wait_primary();
@@ -339,13 +379,24 @@ __global__ void __launch_bounds__(256) decode_tc_reduce(ReduceArgs a) {
   if (i >= n) return;
   const int t = (int)(i / a.R), j = (int)(i % a.R);
   float sum = 0.0f;
-  for (int s = 0; s < a.ns; ++s) sum += __ldcg(a.P + (size_t)s * n + i);
+  for (int s0 = 0; s0 < a.ns; s0 += G) {
+    float h[G], w[G];
+#pragma unroll
+    for (int k = 0; k < G; ++k)
+      if (s0 + k < a.ns) {
+        h[k] = __ldcg(a.P + (size_t)(s0 + k) * n + i);
+        w[k] = __ldcg(a.P2 + (size_t)(s0 + k) * n + i);
+      }
+#pragma unroll
+    for (int k = 0; k < G; ++k)
+      if (s0 + k < a.ns) sum += h[k] + w[k];
+  }
   bool range_err = false;
   if (a.yph) {
-    uint16_t h, l;
-    split_hi_lo<kF16>(sum, h, l, range_err);
-    a.yph[(int64_t)t * a.ldyp + j] = h;
-    a.ypl[(int64_t)t * a.ldyp + j] = l;
+    uint16_t hi, lo;
+    split_hi_lo<kF16>(sum, hi, lo, range_err);
+    a.yph[(int64_t)t * a.ldyp + j] = hi;
+    a.ypl[(int64_t)t * a.ldyp + j] = lo;
   }
   if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
   const int col = __ldg(a.cols + j);
@@ -366,45 +417,46 @@ int sm_count_tc() {
   return n;
 }
 
-int pick_ks(int R, int K, int NB) {
-  // 256 columns: a K-slice of B (16 token rows, hi and lo) is 16 KB, so two buffers and a four-stage
-  // ring of weight tiles fit half an SM; the partial sums are K / 256 fp32 values per output
-  (void)R;
-  (void)K;
-  (void)NB;
-  return 256;
+int grid_cap() {
+  const int g = CTAS_PER_SM * sm_count_tc();
+  return g < GRID_MAX ? g : GRID_MAX;
 }
 
 }  // namespace
 
 int64_t decode_tc_partial_bytes(int64_t R, int64_t K, int64_t T, int NB) {
-  const int ks = pick_ks((int)R, (int)K, NB);
-  return ((K + ks - 1) / ks) * T * R * 4;
+  (void)NB;
+  const Plan p = make_plan(R, K, GRID_MAX);  // the most slices any grid can give
+  return 2 * (int64_t)p.ns * T * R * 4;      // P and P2
 }
 
 int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, cudaStream_t stream) {
   const int NB = ph.planes;
+  if (ph.R < 1 || ph.K < 1 || ph.T < 1 || ph.T > TN) return pifa_fail(PIFA_ERR_INVALID_ARG, "decode_tc: empty or oversized phase");
+  const Plan p = make_plan(ph.R, ph.K, grid_cap());
   TcArgs a = {};
   a.R = (int)ph.R;
   a.K = (int)ph.K;
   a.T = (int)ph.T;
-  a.nrb = (a.R + TM - 1) / TM;
-  a.KS = pick_ks(a.R, a.K, NB);
-  a.ns = (a.K + a.KS - 1) / a.KS;
-  a.units = a.ns * a.nrb;
+  a.nrb = p.nrb;
+  a.ns = p.ns;
+  a.ncf = p.ncf;
+  a.nclast = p.nclast;
+  a.total = p.total;
+  a.grid = p.grid;
   a.gsz = (int)ph.gsz;
   a.goff = (int)ph.goff;
-  a.chunk_bytes = (uint32_t)NB * BOX_BYTES;
+  a.stage_bytes = A_BYTES + (uint32_t)NB * BOX_BYTES;
   const bool f16 = ph.mma_f16;
   a.idesc = f16 ? idesc_f16_f32(TM, TN * NB) : idesc_bf16_f32(TM, TN * NB);
   a.P = ph.P;
+  a.P2 = ph.P + (size_t)p.ns * ph.T * ph.R;
   a.status = status;
   a.timeout_ns = timeout_ns;
-  const size_t fixed = 1024 + 2 * (size_t)(a.KS / KB) * a.chunk_bytes + 512;
-  int stages = (int)((SMEM_PER_CTA - fixed) / A_BYTES);
+  const size_t fixed = 1024 + 512;  // alignment slack; barriers and the TMEM slot
+  const int stages = (int)((SMEM_PER_CTA - fixed) / a.stage_bytes);
   a.stages = stages > MAX_STAGES ? MAX_STAGES : stages;
-  if (a.stages < 2) return pifa_fail(PIFA_ERR_UNSUPPORTED, "decode_tc: shared memory too small");
-  const size_t smem = fixed + (size_t)a.stages * A_BYTES;
+  const size_t smem = fixed + (size_t)a.stages * a.stage_bytes;
 
   CUtensorMap tA, tB0, tB1;
   int st;
@@ -417,8 +469,7 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(decode_tc)", e);
   cudaLaunchConfig_t cfg = {};
-  const int nsm = sm_count_tc();
-  cfg.gridDim = dim3((unsigned)(a.units < CTAS_PER_SM * nsm ? a.units : CTAS_PER_SM * nsm));
+  cfg.gridDim = dim3((unsigned)p.grid);
   cfg.blockDim = dim3(THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
@@ -431,7 +482,8 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   if (e != cudaSuccess) return pifa_fail_cuda("decode_tc partial launch", e);
 
   ReduceArgs r = {};
-  r.P = ph.P;
+  r.P = a.P;
+  r.P2 = a.P2;
   r.ns = a.ns;
   r.T = a.T;
   r.R = a.R;
@@ -448,7 +500,16 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   rc.gridDim = dim3((unsigned)((n + 255) / 256));
   rc.blockDim = dim3(256);
   rc.dynamicSmemBytes = 0;
-  e = ph.split_f16 ? cudaLaunchKernelEx(&rc, decode_tc_reduce<true>, r) : cudaLaunchKernelEx(&rc, decode_tc_reduce<false>, r);
+  void (*red)(ReduceArgs);
+  if (a.ns <= 2)
+    red = ph.split_f16 ? decode_tc_reduce<true, 2> : decode_tc_reduce<false, 2>;
+  else if (a.ns <= 4)
+    red = ph.split_f16 ? decode_tc_reduce<true, 4> : decode_tc_reduce<false, 4>;
+  else if (a.ns <= 8)
+    red = ph.split_f16 ? decode_tc_reduce<true, 8> : decode_tc_reduce<false, 8>;
+  else
+    red = ph.split_f16 ? decode_tc_reduce<true, 16> : decode_tc_reduce<false, 16>;
+  e = cudaLaunchKernelEx(&rc, red, r);
   if (e != cudaSuccess) return pifa_fail_cuda("decode_tc reduce launch", e);
   return PIFA_OK;
 }
