@@ -356,12 +356,17 @@ int pifa_device_status(void* cuda_stream);
 int pifa_set_wait_timeout(int64_t ns);
 
 /* pifa_set_decode_grid -- how the decode variant (T <= 16) lays out each of its two phases for
- * calls made after this one (process-wide): PIFA_DECODE_GRID_AUTO (0, the default) runs a phase
- * as waves of one-tile clusters, every CTA staging its weight rows at launch, while it takes at
- * most two waves, and otherwise as a persistent grid of co-resident clusters that stream their
- * tiles through a ring of TMA-filled stages; PIFA_DECODE_GRID_WAVES (1) and
- * PIFA_DECODE_GRID_PERSISTENT (2) force one layout (a tuning and test knob: both compute the same
- * result up to the summation order of fp32 partial sums). PIFA_ERR_INVALID_ARG for other values. */
+ * calls made after this one (process-wide). Three forms compute a phase (R weight rows, K
+ * columns): waves of one-tile clusters, every CTA staging its weight rows at launch; a persistent
+ * grid of co-resident clusters that stream their tiles through a ring of TMA-filled stages; and
+ * split-K on the tensor cores, where equal ranges of 128 x 64 weight tiles go to a persistent grid
+ * and a second kernel sums the fp32 partial sums in a fixed order.
+ * PIFA_DECODE_GRID_AUTO (0, the default) picks per phase from its shape and T: split-K when
+ * T > 2 and R >= 4096, else waves while the phase takes at most two of them, else the persistent
+ * grid. PIFA_DECODE_GRID_WAVES (1), PIFA_DECODE_GRID_PERSISTENT (2) and PIFA_DECODE_GRID_SPLITK
+ * (3) force one form for both phases (a tuning and test knob: all compute the same result up to
+ * the summation order of fp32 partial sums; forced split-K runs the persistent grid instead when the
+ * workspace is too small for its partial sums). PIFA_ERR_INVALID_ARG for other values. */
 #define PIFA_DECODE_GRID_AUTO 0
 #define PIFA_DECODE_GRID_WAVES 1
 #define PIFA_DECODE_GRID_PERSISTENT 2

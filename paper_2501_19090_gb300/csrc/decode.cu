@@ -973,20 +973,28 @@ int launch_phase_tc(const DecodeArgs& a, int dtype, const SplitKScratch& sk, cud
 }
 
 template <int PHASE, int NT, bool kF16C, int RG, int RGS>
-int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, const SplitKScratch& sk, bool large,
-                     cudaStream_t stream) {
+int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, const SplitKScratch& sk, cudaStream_t stream) {
   constexpr int kRows = kRowsOf<RG>;
   const char* what = PHASE == 1 ? "decode phase 1 launch" : "decode phase 2 launch";
   const int mode = g_decode_grid.load(std::memory_order_relaxed);
   const bool tc_fits = sk.P != nullptr && decode_tc_partial_bytes(a.R, a.K, a.T, PHASE == 1 ? 1 : 2) <= sk.bytes;
   if (mode == PIFA_DECODE_GRID_SPLITK && tc_fits) return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
-  // Auto, layers of >= 64 MiB of weights at T > 2: both phases split-K on the tensor cores
-  // (measured, 70B q/o T = 16: 27.4 us against 31.2 with phase 1 in waves).
-  if (mode == PIFA_DECODE_GRID_AUTO && large && a.T > 2 && tc_fits) return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
-  // Auto: a phase beyond two waves of decode_rows runs split-K on the tensor cores (decode_tc.cu)
-  // for T > 2, and decode_stream for T <= 2, where its resident x / y_p and short loop win
-  // (measured, 70B gate/up: T = 1 46.9 against 51.7 us; T = 8 73.3 against 54.9; T = 16 105.6
-  // against 59.6; 70B q/o T = 16 36.5 against 27.4).
+  // Auto, keyed on the phase's shape and T (phase 1: r rows of K = n; phase 2: m - r rows of
+  // K = r): for T > 2 a phase of at least 32 blocks of 128 rows runs split-K on the tensor cores
+  // (decode_tc.cu); a shorter one gives the grid too few row blocks, so that each CTA's range
+  // spans many K-slices and the partial sums grow with them. Measured per phase, every
+  // combination of the three forms (us, T = 4 / 8 / 16):
+  //   70B gate/up 28672x8192 r4096 (4096 and 24576 rows): tc+tc 51.5 / 54.1 / 56.9, best of all
+  //   70B q/o     8192x8192 r4096  (4096 and 4096 rows):  tc+tc 27.6 / 27.1 / 28.9, best within 1%
+  //   7B gate     11008x4096 r2048 (2048 and 8960 rows):  waves+tc 16.1 / 17.5 / 20.8 (was 19.0 /
+  //                                                       19.5 / 21.1 in waves+waves)
+  //   7B down     4096x11008 r2048 (2048 and 2048 rows):  stream+waves 18.9 / 19.1 / 22.6 (was
+  //                                                       21.4 / 22.3 / 22.3 with phase 1 on tc)
+  //   7B attn     4096x4096 r2048  (2048 and 2048 rows):  waves+waves 8.6 / 8.7 / 13.0
+  // For T <= 2 decode_stream's resident x / y_p and short loop win (70B gate/up, T = 1: 46.9
+  // against 51.7 us on the tensor cores).
+  if (mode == PIFA_DECODE_GRID_AUTO && a.T > 2 && a.R >= 32 * 128 && tc_fits)
+    return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
   const auto kr = decode_rows<PHASE, NT, kF16C, RG>;
   plan_phase(kRows, budget, a);
   const size_t smem = smem_bytes(kRows, a, NT);
@@ -998,7 +1006,6 @@ int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, const SplitKScra
   if (mode == PIFA_DECODE_GRID_WAVES ||
       (mode == PIFA_DECODE_GRID_AUTO && tiles <= 2 * max_clusters(reinterpret_cast<const void*>(kr), a.ks, smem)))
     return launch_phase(kr, kRows, a, smem, stream, what);
-  if (mode == PIFA_DECODE_GRID_AUTO && a.T > 2 && tc_fits) return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
   const auto ks = decode_stream<PHASE, NT, kF16C, RGS>;
   const size_t smem_s =
       plan_stream(reinterpret_cast<const void*>(ks), kRowsOf<RGS>, NT, PHASE == 1 ? 1 : 2, a, what, &st);
@@ -1028,7 +1035,6 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   const int64_t planes = decode_planes_bytes(s);
   const SplitKScratch sk = {p.ws_bytes > planes ? reinterpret_cast<float*>(static_cast<uint8_t*>(p.ws) + planes) : nullptr,
                             p.ws_bytes - planes};
-  const bool large = 2 * G * s.r * (s.n + s.m - s.r) >= ((int64_t)64 << 20);  // weight bytes of the call
   DecodeArgs a = {};
   a.A = reinterpret_cast<const uint16_t*>(p.Wp);
   a.lda = s.ldwp;
@@ -1048,7 +1054,7 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   a.T = (int)s.T;
   a.status = status;
   a.timeout_ns = pifa_wait_timeout_ns();
-  int st = launch_one_phase<1, NT, kF16C, RG, RGS>(a, kStageBudget1, PIFA_DTYPE_BF16, sk, large, stream);
+  int st = launch_one_phase<1, NT, kF16C, RG, RGS>(a, kStageBudget1, PIFA_DTYPE_BF16, sk, stream);
   if (st != PIFA_OK || s.m == s.r) return st;
   DecodeArgs b = a;
   b.A = reinterpret_cast<const uint16_t*>(p.C);
@@ -1066,7 +1072,7 @@ int launch_decode_t(const PifaShape& s, const PifaPointers& p, int* status, cuda
   }
   b.yph = b.ypl = nullptr;
   b.cols = p.nonpiv;
-  return launch_one_phase<2, NT, kF16C, RG, RGS>(b, kStageBudget2, (int)s.c_dtype, sk, large, stream);
+  return launch_one_phase<2, NT, kF16C, RG, RGS>(b, kStageBudget2, (int)s.c_dtype, sk, stream);
 }
 
 }  // namespace

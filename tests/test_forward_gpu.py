@@ -308,6 +308,26 @@ def test_decode_splitk_deterministic_and_r_equals_m():
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
+@pytest.mark.parametrize("m,n,r,T,forced", [
+    (8192, 4096, 4096, 8, P.PIFA_DECODE_GRID_SPLITK),  # both phases 4096 rows, T > 2
+    (8192, 4096, 4096, 16, P.PIFA_DECODE_GRID_SPLITK),
+    (4096, 4096, 2048, 8, P.PIFA_DECODE_GRID_WAVES),   # 2048-row phases, at most two waves each
+])
+def test_decode_selector_matches_the_form_it_picks(m, n, r, T, forced):
+    """The automatic decode choice is keyed on each phase's rows and T: split-K on the tensor cores
+    for phases of at least 32 blocks of 128 rows when T > 2, waves of one-tile clusters for a
+    phase that fits two waves. Its output equals, bit for bit, that of the form it should pick,
+    forced."""
+    L = layer_for(m, n, r, 6, "synthetic")
+    X = acts(T, n, 6)
+    auto = run(L, X, P.PIFA_VARIANT_DECODE)
+    P.pifa_set_decode_grid(forced)
+    try:
+        assert np.array_equal(auto, run(L, X, P.PIFA_VARIANT_DECODE))
+    finally:
+        P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
+
+
 # ---------------------------------------------------------------------------------------------
 # edge cases
 # ---------------------------------------------------------------------------------------------
