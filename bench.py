@@ -55,9 +55,16 @@ METRIC = "PIFA layer tokens/s at 1 GB300 + % of HBM / bf16 tensor roofline vs lo
 SHAPE = inputs.MLP70B_GATE       # the headline layer
 T_DECODE = 16
 
-# DRAM traffic per call measured with ncu for a given kernel source (sha256 of decode.cu), keyed
-# by (layer, T). A source mismatch (the kernel changed since the capture) reports traffic as null.
-NCU_TRAFFIC = {}
+# DRAM traffic per call (dram__bytes_read.sum + dram__bytes_write.sum over the call's kernels)
+# measured with ncu, keyed by (layer, T), with the sha256 prefixes of the kernel sources it was
+# taken on. A source mismatch (a kernel changed since the capture) reports traffic as null.
+NCU_TRAFFIC = {
+    # profiles/decode_tc_gateup70b_T16_traffic.md: split-K partial + reduce, both phases
+    ("llama2_70b_gate_up_28672x8192_r4096", 16): {
+        "sha": {"decode_tc.cu": "df2f3ae613e49c89", "decode.cu": "0d83c7d91223b49c"},
+        "bytes": 285136896,
+    },
+}
 
 
 def _src_sha(name: str) -> str:
@@ -546,6 +553,12 @@ def run_ours(args, rank, world, local_rank):
             step(i)
     stream.synchronize()
     assert P.pifa_device_status(stream) == P.PIFA_OK
+    # kernels one step enqueues, counted by the library itself
+    c0 = P.pifa_launch_count()
+    with torch.cuda.stream(stream):
+        step(0)
+    launches_per_step = P.pifa_launch_count() - c0
+    stream.synchronize()
     per = min(K, copies * max(1, 64 // copies))
     g = _graph_of(step, per, stream)
     reps, rem = divmod(K, per)
@@ -633,15 +646,16 @@ def run_ours(args, rank, world, local_rank):
                       "frac": ab / (step_ms / 1e3) / 1e9 / hbm_peak,
                       "traffic": _traffic(shape.name, T),
                       "peak_source": f"{peak_src} hbm_gbs (burst: the call is timed alone)",
-                      "kernel": "decode phase 1 + phase 2 (one PDL-chained pair per call)",
+                      "kernel": f"decode phase 1 + phase 2 ({launches_per_step} PDL-chained kernels per call)",
                       "algorithmic_bytes_per_launch": ab} if decode else
                      {"bound": "tensor", "achieved": af / (step_ms / 1e3) / 1e12, "peak": tc_peak,
                       "unit": "TFLOP/s", "frac": af / (step_ms / 1e3) / 1e12 / tc_peak,
                       "traffic": None, "peak_source": f"{peak_src} bf16_tflops (burst)",
                       "kernel": f"{P.pifa_variant_name(variant)} prefill (GEMM 1 + GEMM 2 per call)",
                       "algorithmic_flops_per_launch": af}),
-        "gpu_launches": K * (2 if m > r else 1),
-        "gpu_launches_all_repeats": K * (2 if m > r else 1) * n_rep,
+        "gpu_launches": K * launches_per_step,
+        "gpu_launches_per_step": launches_per_step,
+        "gpu_launches_all_repeats": K * launches_per_step * n_rep,
         "clocks": clk.summary(),
     }
     del Wps, Cs, Xs, Ys
@@ -883,7 +897,7 @@ def _oracle_rate_one_thread(shape, T, budget_s):
 
 def _traffic(layer, T):
     t = NCU_TRAFFIC.get((layer, T))
-    if not t or t.get("sha") != _src_sha("decode.cu"):
+    if not t or any(_src_sha(f) != h for f, h in t["sha"].items()):
         return None
     return t["bytes"]
 

@@ -373,6 +373,12 @@ int pifa_set_wait_timeout(int64_t ns);
 #define PIFA_DECODE_GRID_SPLITK 3
 int pifa_set_decode_grid(int mode);
 
+/* pifa_launch_count -- how many kernels this library has enqueued since it was loaded, over all
+ * threads, devices and entry points (a launch captured into a CUDA graph counts once, at capture;
+ * its replays do not). The difference across one call is the number of kernels that call runs.
+ * Not part of the paper. */
+int64_t pifa_launch_count(void);
+
 /* pifa_selftest_wait_timeout -- enqueues on `cuda_stream` a one-CTA kernel that waits, with the
  * current bound (pifa_set_wait_timeout), on an mbarrier that nothing arrives on, so the wait runs
  * out and PIFA_ERR_TIMEOUT is latched for pifa_device_status(). Checks the failure-detection path

@@ -97,6 +97,7 @@ int launch_small(const void* fn, void** args, int64_t rows, int64_t cols, cudaSt
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   const cudaError_t e = cudaLaunchKernelExC(&cfg, fn, args);
+  if (e == cudaSuccess) pifa_count_launch();
   return e == cudaSuccess ? PIFA_OK : pifa_fail_cuda(what, e);
 }
 
@@ -283,7 +284,7 @@ extern "C" int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int6
     attr.val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, transpose_bf16, reinterpret_cast<const bf16*>(Xu), ldx, (int)T,
+    const cudaError_t e = pifa_launch_ex(&cfg, transpose_bf16, reinterpret_cast<const bf16*>(Xu), ldx, (int)T,
                                              (int)n, XuT, ldT);
     if (e != cudaSuccess) return pifa_fail_cuda("m_accumulate: transpose", e);
   }

@@ -115,6 +115,7 @@ int run_gemm_f64(const GemmF64& p, int batch, cudaStream_t s) {
   if (p.M <= 0 || p.N <= 0 || batch <= 0) return PIFA_OK;
   dim3 grid((unsigned)((p.N + GT - 1) / GT), (unsigned)((p.M + GT - 1) / GT), (unsigned)batch);
   gemm_f64<<<grid, 256, 0, s>>>(p);
+  pifa_count_launch();
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? PIFA_OK : pifa_fail_cuda("compress: gemm launch", e);
 }
@@ -396,6 +397,7 @@ int upper_inverse(const double* R, double* Rinv, double* Tt, int rp, cudaStream_
   cudaError_t e = cudaMemsetAsync(Rinv, 0, (size_t)rp * rp * 8, s);
   if (e != cudaSuccess) return pifa_fail_cuda("upper inverse: memset", e);
   inv_diag32<<<rp / 32, 32, 0, s>>>(R, Rinv, rp);
+  pifa_count_launch();
   e = cudaGetLastError();
   if (e != cudaSuccess) return pifa_fail_cuda("upper inverse: launch", e);
   int st;
@@ -530,6 +532,7 @@ extern "C" int pifa_compress_device(const double* U, const double* V, int64_t m,
   for (int j = 0; j < ri; ++j) {
     const int t = (ri - j + 15) / 16;
     chol_step<<<dim3(t, t), 256, 0, s>>>(G, L, ri, j, flags);
+    pifa_count_launch();
   }
   PIFA_CK(cudaGetLastError(), "compress: cholesky launch");
   q = GemmF64{};
@@ -541,19 +544,25 @@ extern "C" int pifa_compress_device(const double* U, const double* V, int64_t m,
 
   // 2. r greedy steps
   greedy_init<<<Ly.nblk, 256, 0, s>>>(g);
+  pifa_count_launch();
   PIFA_CK(cudaGetLastError(), "compress: greedy init launch");
   const size_t vsm = (size_t)r * 8;
   PIFA_CK(cudaFuncSetAttribute(greedy_step, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)vsm),
           "compress: greedy smem attribute");
-  for (int k = 0; k < ri; ++k) greedy_step<<<Ly.nblk, 256, (size_t)(r - k) * 8, s>>>(g, k);
+  for (int k = 0; k < ri; ++k) {
+    greedy_step<<<Ly.nblk, 256, (size_t)(r - k) * 8, s>>>(g, k);
+    pifa_count_launch();
+  }
   PIFA_CK(cudaGetLastError(), "compress: greedy step launch");
 
   // 3. index sets, R, R^{-1}, C = Z[I^c] R^{-T} in ascending-I columns
   index_sets<<<1, 1024, 0, s>>>(g.sel, mi, g.order, ri, pivot_idx, has_np ? nonpivot_idx : pos, pos, asc);
+  pifa_count_launch();
   PIFA_CK(cudaGetLastError(), "compress: index sets launch");
   {
     const int64_t tot = (int64_t)rp * rp;
     build_r<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(g, R, rp);
+    pifa_count_launch();
     if ((st = upper_inverse(R, Rinv, Tt, rp, s)) != PIFA_OK) return st;
   }
   if (has_np) {
@@ -565,6 +574,7 @@ extern "C" int pifa_compress_device(const double* U, const double* V, int64_t m,
     c.C = C; c.cidx = asc; c.ldc = ldc; c.alpha = 1.0; c.beta = 0.0; c.tri = 1;
     if ((st = run_gemm_f64(c, 1, s)) != PIFA_OK) return st;
     max_abs<<<4 * 152, 256, 0, s>>>(C, m - r, r, ldc, reinterpret_cast<unsigned long long*>(flags + 2));
+    pifa_count_launch();
     PIFA_CK(cudaGetLastError(), "compress: max launch");
   }
   // 4. W_p = U[I] V^T
@@ -676,8 +686,10 @@ int spd_inverse(const double* S, int64_t k, double* Sinv, double* scratch, int* 
   for (int j = 0; j < (int)k; ++j) {
     const int t = ((int)k - j + 15) / 16;
     chol_step<<<dim3(t, t), 256, 0, s>>>(G, L, (int)k, j, bad);
+    pifa_count_launch();
   }
   transpose_pad_lower<<<grid_for((int64_t)rp * rp), 256, 0, s>>>(L, k, R, rp);
+  pifa_count_launch();
   e = cudaGetLastError();
   if (e != cudaSuccess) return pifa_fail_cuda("spd inverse: launch", e);
   int st = upper_inverse(R, Rinv, Tt, rp, s);
@@ -730,7 +742,9 @@ extern "C" int pifa_m_reconstruct(const float* XXt, int64_t ldxx, const float* Y
   cudaError_t e = cudaMemsetAsync(bad, 0, 8, s);
   if (e != cudaSuccess) return pifa_fail_cuda("reconstruct: memset", e);
   f32_to_f64<<<grid_for(n * n), 256, 0, s>>>(XXt, ldxx, n, n, A, n);
+  pifa_count_launch();
   f32_to_f64<<<grid_for(m * n), 256, 0, s>>>(YtXt, ldyx, m, n, B, n);
+  pifa_count_launch();
   e = cudaGetLastError();
   if (e != cudaSuccess) return pifa_fail_cuda("reconstruct: launch", e);
   const int ni = (int)n, mi = (int)m, ri = (int)r;
@@ -755,7 +769,9 @@ extern "C" int pifa_m_reconstruct(const float* XXt, int64_t ldxx, const float* Y
   if ((st = spd_inverse(Pm, r, Pinv, scratch, bad, s)) != PIFA_OK) return st;
   if (alpha != 0.0) {
     add_scaled_bf16<<<grid_for(m * n), 256, 0, s>>>(static_cast<const __nv_bfloat16*>(W), ldw, m, n, alpha, B, n);
+    pifa_count_launch();
     add_diag<<<grid_for(n), 256, 0, s>>>(A, n, n, alpha);
+    pifa_count_launch();
     e = cudaGetLastError();
     if (e != cudaSuccess) return pifa_fail_cuda("reconstruct: launch", e);
   }

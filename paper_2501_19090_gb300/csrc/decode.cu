@@ -776,7 +776,7 @@ int launch_phase(Kern kernel, int rows, const DecodeArgs& args, size_t smem, cud
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, args);
+  cudaError_t e = pifa_launch_ex(&cfg, kernel, args);
   if (e != cudaSuccess) return pifa_fail_cuda(what, e);
   return PIFA_OK;
 }
@@ -926,7 +926,7 @@ int launch_stream(Kern kernel, const CUtensorMap& tm, const CUtensorMap& tb0, co
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, tm, tb0, tb1, args);
+  cudaError_t e = pifa_launch_ex(&cfg, kernel, tm, tb0, tb1, args);
   if (e != cudaSuccess) return pifa_fail_cuda(what, e);
   return PIFA_OK;
 }

@@ -478,7 +478,7 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   attr.val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, kern, tA, tB0, tB1, a);
+  e = pifa_launch_ex(&cfg, kern, tA, tB0, tB1, a);
   if (e != cudaSuccess) return pifa_fail_cuda("decode_tc partial launch", e);
 
   ReduceArgs r = {};
@@ -509,7 +509,7 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
     red = ph.split_f16 ? decode_tc_reduce<true, 8> : decode_tc_reduce<false, 8>;
   else
     red = ph.split_f16 ? decode_tc_reduce<true, 16> : decode_tc_reduce<false, 16>;
-  e = cudaLaunchKernelEx(&rc, red, r);
+  e = pifa_launch_ex(&rc, red, r);
   if (e != cudaSuccess) return pifa_fail_cuda("decode_tc reduce launch", e);
   return PIFA_OK;
 }

@@ -363,7 +363,7 @@ int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stre
   attr.val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, kern, tA, tA2, tB, tB2, a);
+  e = pifa_launch_ex(&cfg, kern, tA, tA2, tB, tB2, a);
   if (e != cudaSuccess) return pifa_fail_cuda("gemm_tc launch", e);
   return PIFA_OK;
 }

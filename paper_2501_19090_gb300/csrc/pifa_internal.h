@@ -20,6 +20,21 @@ int* pifa_status_word(cudaError_t* err);
 // Default bound of every device-side wait, nanoseconds (env PIFA_WAIT_TIMEOUT_NS overrides).
 uint64_t pifa_wait_timeout_ns();
 
+// Kernels this library has enqueued (status.cu): every launch site calls pifa_count_launch() once
+// per successful launch; pifa_launch_count() reads the total.
+void pifa_count_launch();
+
+#ifdef __CUDACC__
+#include <utility>
+// cudaLaunchKernelEx, counted.
+template <typename... K, typename... A>
+inline cudaError_t pifa_launch_ex(const cudaLaunchConfig_t* cfg, void (*kernel)(K...), A&&... args) {
+  const cudaError_t e = cudaLaunchKernelEx(cfg, kernel, std::forward<A>(args)...);
+  if (e == cudaSuccess) pifa_count_launch();
+  return e;
+}
+#endif
+
 // Shape of one forward call after validation (element counts and pitches).
 struct PifaShape {
   int64_t T, m, n, r;

@@ -288,7 +288,7 @@ int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtenso
   attr.val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, kern, a, b0, b1, g);
+  e = pifa_launch_ex(&cfg, kern, a, b0, b1, g);
   if (e != cudaSuccess) return pifa_fail_cuda("prefill gemm launch", e);
   return PIFA_OK;
 }

@@ -1,5 +1,6 @@
 // status.cu -- the device-side error word that kernels latch (first error wins) and
 // pifa_device_status() reads and clears. One int per device, in this library's static device data.
+#include <atomic>
 #include <mutex>
 
 #include <cuda_runtime.h>
@@ -11,10 +12,16 @@
 namespace {
 __device__ int g_pifa_status_word = 0;
 
+std::atomic<int64_t> g_launches{0};
+
 constexpr int kMaxDevices = 64;
 int* g_word_addr[kMaxDevices] = {};
 std::mutex g_word_mu;
 }  // namespace
+
+void pifa_count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+extern "C" int64_t pifa_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 int* pifa_status_word(cudaError_t* err) {
   int dev = 0;
@@ -59,5 +66,6 @@ extern "C" int pifa_selftest_wait_timeout(void* cuda_stream) {
   wait_timeout_selftest<<<1, 32, 0, reinterpret_cast<cudaStream_t>(cuda_stream)>>>(status, pifa_wait_timeout_ns());
   e = cudaGetLastError();
   if (e != cudaSuccess) return pifa_fail_cuda("wait-timeout self-test launch", e);
+  pifa_count_launch();
   return PIFA_OK;
 }

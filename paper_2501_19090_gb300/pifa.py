@@ -45,7 +45,8 @@ EXPORTS = (
     "pifa_forward", "pifa_forward_variant", "pifa_workspace_size", "pifa_select_variant",
     "pifa_variant_name", "pifa_compress", "pifa_validate_indices", "pifa_device_status",
     "pifa_status_string", "pifa_last_error", "pifa_version", "pifa_forward_decode_noalloc",
-    "pifa_set_wait_timeout", "pifa_selftest_wait_timeout", "pifa_set_decode_grid", "pifa_forward_grouped",
+    "pifa_set_wait_timeout", "pifa_selftest_wait_timeout", "pifa_launch_count", "pifa_set_decode_grid",
+    "pifa_forward_grouped",
     "pifa_workspace_size_grouped", "pifa_compress_device", "pifa_compress_device_workspace_size",
     "pifa_backward", "pifa_backward_workspace_size", "pifa_m_accumulate", "pifa_m_accumulate_workspace_size",
     "pifa_m_reconstruct", "pifa_m_reconstruct_workspace_size",
@@ -133,6 +134,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.pifa_set_wait_timeout.restype = ctypes.c_int
         lib.pifa_selftest_wait_timeout.argtypes = [_VP]
         lib.pifa_selftest_wait_timeout.restype = ctypes.c_int
+        lib.pifa_launch_count.argtypes = []
+        lib.pifa_launch_count.restype = ctypes.c_int64
         lib.pifa_set_decode_grid.argtypes = [ctypes.c_int]
         lib.pifa_set_decode_grid.restype = ctypes.c_int
         lib.pifa_version.argtypes = []
@@ -173,6 +176,11 @@ def pifa_set_decode_grid(mode: int) -> None:
 def pifa_selftest_wait_timeout(stream=None) -> None:
     """Enqueue the bounded-wait self-test kernel (latches PIFA_ERR_TIMEOUT; see include/pifa.h)."""
     _check(_lib().pifa_selftest_wait_timeout(_stream_ptr(stream)), "pifa_selftest_wait_timeout")
+
+
+def pifa_launch_count() -> int:
+    """Kernels the library has enqueued since it was loaded (see include/pifa.h)."""
+    return int(_lib().pifa_launch_count())
 
 
 def pifa_last_error() -> str:

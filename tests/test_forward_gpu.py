@@ -328,6 +328,36 @@ def test_decode_selector_matches_the_form_it_picks(m, n, r, T, forced):
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
+def test_launch_count_per_call():
+    """pifa_launch_count: a split-K decode call (both phases of 4096 rows, T = 8) enqueues four
+    kernels (a partial and a reduce kernel per phase), a waves decode call on 2048-row phases two;
+    replaying a captured call launches nothing through the library."""
+    big, small = layer_for(8192, 4096, 4096, 6, "synthetic"), layer_for(4096, 4096, 2048, 6, "synthetic")
+    for L, n_k in ((big, 4), (small, 2)):
+        X = acts(8, L.n, 6)
+        run(L, X, P.PIFA_VARIANT_DECODE)  # first call: per-shape setup out of the way
+        c0 = P.pifa_launch_count()
+        run(L, X, P.PIFA_VARIANT_DECODE)
+        assert P.pifa_launch_count() - c0 == n_k, L.name
+    Wp, C, piv, nonp = small.dev(None, None)
+    Xd = torch.from_numpy(acts(8, small.n, 7)).to(DEV, torch.bfloat16)
+    Y = torch.empty((8, small.m), dtype=torch.bfloat16, device=DEV)
+    ws = P.workspace(P.pifa_workspace_size(8, small.m, small.n, small.r, P.PIFA_VARIANT_DECODE), DEV)
+    stream = torch.cuda.Stream()
+    P.pifa_forward(Xd, Wp, C, piv, nonp, Y=Y, variant=P.PIFA_VARIANT_DECODE, workspace_tensor=ws, stream=stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        P.pifa_forward(Xd, Wp, C, piv, nonp, Y=Y, variant=P.PIFA_VARIANT_DECODE, workspace_tensor=ws, stream=stream)
+    c0 = P.pifa_launch_count()
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            g.replay()
+    stream.synchronize()
+    assert P.pifa_launch_count() == c0
+    assert P.pifa_device_status(stream) == P.PIFA_OK
+
+
 # ---------------------------------------------------------------------------------------------
 # edge cases
 # ---------------------------------------------------------------------------------------------
