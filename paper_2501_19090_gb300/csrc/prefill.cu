@@ -20,6 +20,8 @@
 // out as 16-byte stores after a transpose through shared memory. Every wait is bounded
 // (globaltimer); on timeout the CTA latches PIFA_ERR_TIMEOUT, drains what it has in flight and
 // returns.
+#include <utility>
+
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -33,16 +35,34 @@ using namespace pifa;
 using bf16 = __nv_bfloat16;
 
 constexpr int BM = 128;  // weight rows per tile (MMA M)
-constexpr int BN = 256;  // tokens per tile at most (MMA N); the launch picks bn <= BN, a multiple of 16
 constexpr int BK = 64;   // K per stage: one 128-byte swizzle row of bf16
-constexpr int STAGES = 4;
-constexpr int EPI_WARPS = 16;                 // epilogue warps: four per TMEM lane quarter
-constexpr int THREADS = 64 + 32 * EPI_WARPS;  // + the TMA producer and the MMA warp
 constexpr uint32_t A_BYTES = BM * BK * 2;
-constexpr uint32_t B_BYTES = BN * BK * 2;
-constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr uint32_t TMEM_COLS = BN;  // fp32 accumulator, one column per token
-constexpr size_t SMEM_BYTES = 1024 /*alignment slack*/ + STAGES * STAGE_BYTES + 256 /*barriers*/;
+
+// Two shapes of the same kernel. Config 0: one CTA per SM, up to 256 tokens per tile, a 4-stage
+// ring and 16 epilogue warps (the fastest when a GEMM fits one or two waves). Config 1: two CTAs
+// per SM, up to 160 tokens per tile, 3 stages and 8 epilogue warps: one CTA's epilogue runs while
+// the other's MMAs keep the tensor core busy, which pays on GEMMs of many waves (measured, T = 8192
+// on the 4096 x 4096, r = 2048 layer: 240.4 -> 219.3 us; 70B q/o T = 4096: 426.5 -> 378.1 us) and
+// loses on one wave (T = 2048 on the same layer: 57.8 -> 64.5 us).
+template <int CFG>
+struct PCfg;
+template <>
+struct PCfg<0> {
+  static constexpr int BN = 256, STAGES = 4, EPI_WARPS = 16, CTAS = 1;
+};
+template <>
+struct PCfg<1> {
+  static constexpr int BN = 160, STAGES = 3, EPI_WARPS = 8, CTAS = 2;
+};
+template <int CFG>
+struct PC : PCfg<CFG> {
+  using B = PCfg<CFG>;
+  static constexpr int THREADS = 64 + 32 * B::EPI_WARPS;  // + the TMA producer and the MMA warp
+  static constexpr uint32_t B_BYTES = B::BN * BK * 2;
+  static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr uint32_t TMEM_COLS = 256;  // fp32 accumulator, one column per token (a power of two)
+  static constexpr size_t SMEM_BYTES = 1024 /*alignment slack*/ + B::STAGES * STAGE_BYTES + 256 /*barriers*/;
+};
 
 // Epilogue modes: what GEMM 1 also writes besides Y (GEMM 2 writes Y only).
 enum { EPI_Y_ONLY = 0, EPI_SPLIT_BF16 = 1, EPI_SPLIT_F16 = 2 };
@@ -68,10 +88,12 @@ struct GemmArgs {
   uint64_t timeout_ns;
 };
 
-template <int kEpi>
-__global__ void __launch_bounds__(THREADS, 1)
+template <int kEpi, int CFG>
+__global__ void __launch_bounds__(PC<CFG>::THREADS, PC<CFG>::CTAS)
     pifa_umma_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, GemmArgs p) {
+  constexpr int STAGES = PC<CFG>::STAGES, EPI_WARPS = PC<CFG>::EPI_WARPS, BN = PC<CFG>::BN;
+  constexpr uint32_t STAGE_BYTES = PC<CFG>::STAGE_BYTES, TMEM_COLS = PC<CFG>::TMEM_COLS;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
@@ -181,7 +203,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     // EPI_WARPS / 4 warps of a quarter split the tile's tokens. Many warps keep the store issue
     // rate up: the scattered 2-byte stores into Y's columns are instruction-bound.
     constexpr int kSlices = EPI_WARPS / 4;
-    constexpr int kChunks = BN / 32 / kSlices;  // 32-token chunks per warp (the last ones may lie beyond bn)
+    constexpr int kChunks = (BN / 32 + kSlices - 1) / kSlices;  // 32-token chunks per warp (the last ones may lie beyond bn)
     const int tend = min(n0 + p.bn, p.N);       // this tile's tokens end here
     const int q = warp & 3;
     const int slice = (warp - 2) >> 2;
@@ -259,11 +281,13 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+template <int CFG>
 int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1, const GemmArgs& args,
              cudaStream_t stream) {
-  auto kern = epi == EPI_SPLIT_BF16 ? pifa_umma_gemm<EPI_SPLIT_BF16>
-              : epi == EPI_SPLIT_F16 ? pifa_umma_gemm<EPI_SPLIT_F16>
-                                    : pifa_umma_gemm<EPI_Y_ONLY>;
+  auto kern = epi == EPI_SPLIT_BF16 ? pifa_umma_gemm<EPI_SPLIT_BF16, CFG>
+              : epi == EPI_SPLIT_F16 ? pifa_umma_gemm<EPI_SPLIT_F16, CFG>
+                                    : pifa_umma_gemm<EPI_Y_ONLY, CFG>;
+  constexpr size_t SMEM_BYTES = PC<CFG>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(prefill gemm)", e);
   // programmatic dependent launch: each GEMM may start (weight tiles in flight) while the previous
@@ -280,7 +304,7 @@ int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtenso
   if ((g.tok_fast ? mt : nt) > 65535u) g.tok_fast ^= 1;  // gridDim.y is at most 65535
   if ((g.tok_fast ? mt : nt) > 65535u) return pifa_fail(PIFA_ERR_UNSUPPORTED, "more than 65535 tiles along both M and T");
   cfg.gridDim = g.tok_fast ? dim3(nt, mt) : dim3(mt, nt);
-  cfg.blockDim = dim3(THREADS);
+  cfg.blockDim = dim3(PC<CFG>::THREADS);
   cfg.dynamicSmemBytes = SMEM_BYTES;
   cfg.stream = stream;
   cudaLaunchAttribute attr;
@@ -301,23 +325,44 @@ inline int64_t pad8(int64_t v) { return (v + 7) / 8 * 8; }
 // t(bn) ~ t0 (432 + bn), most of a tile's time not shrinking with its width. There T = 2048 takes
 // 240 (144 tiles, one wave of 152 SMs, where 256 leaves 24 SMs idle: 58.3 -> 57.3 us) and
 // T = 8192 224 (254.4 -> 242.8 us).
-int pick_bn(int64_t M, int64_t T) {
+int sm_count_prefill() {
   int sms = 0, dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
       sms < 1)
     sms = 1;
+  return sms;
+}
+
+// The kernel shape and token-tile width of one GEMM: config 0 with pick_bn's width unless that
+// takes three or more waves, then config 1 (CTA slots = 2 per SM) with its own width.
+struct GemmShape {
+  int cfg, bn;
+};
+int pick_bn_slots(int64_t M, int64_t T, int bnmax, int64_t slots) {
   const int64_t mt = (M + BM - 1) / BM;
-  int best = BN;
+  int best = bnmax;
   int64_t best_cost = -1;
-  for (int bn = BN; bn >= 16; bn -= 16) {
+  for (int bn = bnmax; bn >= 16; bn -= 16) {
     const int64_t tiles = mt * ((T + bn - 1) / bn);
-    const int64_t cost = (tiles + sms - 1) / sms * (432 + bn);
+    const int64_t cost = (tiles + slots - 1) / slots * (432 + bn);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
       best = bn;
     }
   }
   return best;
+}
+GemmShape pick_shape(int64_t M, int64_t T) {
+  const int64_t sms = sm_count_prefill();
+  const int bn0 = pick_bn_slots(M, T, PC<0>::BN, sms);
+  const int64_t waves0 = ((M + BM - 1) / BM * ((T + bn0 - 1) / bn0) + sms - 1) / sms;
+  if (waves0 < 3) return {0, bn0};
+  return {1, pick_bn_slots(M, T, PC<1>::BN, 2 * sms)};
+}
+
+template <typename... A>
+int run_gemm_cfg(int cfg, A&&... args) {
+  return cfg == 0 ? run_gemm<0>(std::forward<A>(args)...) : run_gemm<1>(std::forward<A>(args)...);
 }
 
 }  // namespace
@@ -338,7 +383,8 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
 
   CUtensorMap tWp, tX, tC, tHi, tLo;
   int st;
-  const int bn1 = pick_bn(G * s.r, s.T);
+  const GemmShape sh1 = pick_shape(G * s.r, s.T);
+  const int bn1 = sh1.bn;
   if ((st = make_tmap_2d(&tWp, PIFA_DTYPE_BF16, p.Wp, G * s.r, s.n, s.ldwp, BK, BM)) != PIFA_OK) return st;
   if ((st = make_tmap_2d(&tX, PIFA_DTYPE_BF16, p.X, s.T, s.n, s.ldx, BK, bn1)) != PIFA_OK) return st;
 
@@ -358,10 +404,11 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
   g1.ldyp = ldyp;
   g1.status = status;
   g1.timeout_ns = timeout_ns;
-  if ((st = run_gemm(f16 ? EPI_SPLIT_F16 : EPI_SPLIT_BF16, tWp, tX, tX, g1, stream)) != PIFA_OK) return st;
+  if ((st = run_gemm_cfg(sh1.cfg, f16 ? EPI_SPLIT_F16 : EPI_SPLIT_BF16, tWp, tX, tX, g1, stream)) != PIFA_OK) return st;
   if (s.m == s.r) return PIFA_OK;
 
-  const int bn2 = pick_bn(G * (s.m - s.r), s.T);
+  const GemmShape sh2 = pick_shape(G * (s.m - s.r), s.T);
+  const int bn2 = sh2.bn;
   if ((st = make_tmap_2d(&tC, s.c_dtype, p.C, G * (s.m - s.r), s.r, s.ldc, BK, BM)) != PIFA_OK) return st;
   if ((st = make_tmap_2d(&tHi, s.c_dtype, hi, s.T, G * s.r, ldyp, BK, bn2)) != PIFA_OK) return st;
   if ((st = make_tmap_2d(&tLo, s.c_dtype, lo, s.T, G * s.r, ldyp, BK, bn2)) != PIFA_OK) return st;
@@ -378,6 +425,6 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
   g2.cols = p.nonpiv;
   g2.yp_hi = nullptr;
   g2.yp_lo = nullptr;
-  return run_gemm(EPI_Y_ONLY, tC, tHi, tLo, g2, stream);
+  return run_gemm_cfg(sh2.cfg, EPI_Y_ONLY, tC, tHi, tLo, g2, stream);
 }
 
