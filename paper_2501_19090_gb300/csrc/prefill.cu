@@ -41,9 +41,10 @@ constexpr uint32_t A_BYTES = BM * BK * 2;
 // Two shapes of the same kernel. Config 0: one CTA per SM, up to 256 tokens per tile, a 4-stage
 // ring and 16 epilogue warps (the fastest when a GEMM fits one or two waves). Config 1: two CTAs
 // per SM, up to 160 tokens per tile, 3 stages and 8 epilogue warps: one CTA's epilogue runs while
-// the other's MMAs keep the tensor core busy, which pays on GEMMs of many waves (measured, T = 8192
-// on the 4096 x 4096, r = 2048 layer: 240.4 -> 219.3 us; 70B q/o T = 4096: 426.5 -> 378.1 us) and
-// loses on one wave (T = 2048 on the same layer: 57.8 -> 64.5 us).
+// the other's MMAs keep the tensor core busy, which pays on GEMMs of many waves (measured, same
+// outputs bit for bit: T = 8192 on the 4096 x 4096, r = 2048 layer 241.1 -> 226.2 us; 70B q/o
+// T = 4096 427.3 -> 390.1 us). A GEMM of one or two waves leaves little to overlap, and there the
+// one-CTA shape's wider tiles and deeper ring are kept.
 template <int CFG>
 struct PCfg;
 template <>
