@@ -30,8 +30,17 @@ using bf16 = __nv_bfloat16;
 constexpr int BM = 128;
 constexpr int BNMAX = 256;
 constexpr int BK = 64;
-constexpr int STAGES = 4;
 constexpr int THREADS = 192;
+// Two shapes of the kernel. Config 0: one CTA per SM, tiles up to 256 wide, a 4-stage ring, the
+// values to add in (the old D, an addend) staged into shared memory while the MMAs run. Config 1:
+// two CTAs per SM, tiles up to 128 wide, 3 stages, the values to add in (if any) loaded right
+// before the stores: one CTA's epilogue runs under the other's MMAs. gemm_tc picks one per GEMM
+// (measured, 4096 x 4096 r = 2048 layer, T = 2048: the backward 425.7 -> 353.3 us, bit for bit
+// the same).
+template <int CFG>
+constexpr int kStages = CFG == 0 ? 4 : 3;
+template <int CFG>
+constexpr int kBnMax = CFG == 0 ? BNMAX : 128;
 constexpr uint32_t A_BYTES = BM * BK * 2;     // 16 KB
 constexpr uint32_t B_MAX = BNMAX * BK * 2;    // 32 KB
 constexpr uint32_t MN_BOX = 64 * BK * 2;      // one MN-major box: 64 (MN) x 64 (K), 8 KB
@@ -53,6 +62,7 @@ struct GemmTcArgs {
   const int32_t* add_idx;
   int64_t ldadd;
   int add_bound;      // columns of the addend (index bound)
+  int late_add;       // 1 (config 1): the epilogue loads the old D and the addend itself
   int* status;
   uint64_t timeout_ns;
 };
@@ -70,10 +80,12 @@ __device__ __forceinline__ uint64_t sw128_mn_desc(uint32_t saddr, uint32_t mn_st
   return d;
 }
 
-template <bool AMN, bool BMN>
-__global__ void __launch_bounds__(THREADS, 1)
+template <bool AMN, bool BMN, int CFG>
+__global__ void __launch_bounds__(THREADS, CFG == 0 ? 1 : 2)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
                    const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmB2, GemmTcArgs p) {
+  constexpr int STAGES = kStages<CFG>;
+  constexpr uint32_t TMEM_ALLOC = (uint32_t)kBnMax<CFG>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t b_bytes = (uint32_t)p.bn * BK * 2;
@@ -108,7 +120,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, BNMAX);
+    tmem_alloc(tmem_slot, TMEM_ALLOC);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -255,12 +267,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         } else {
           // D: one row of the block per step, the lanes covering consecutive columns (coalesced)
           const int col = n0 + c0 + lane;
-          for (int rr = 0; rr < nrows; ++rr) {
-            const int row = m0 + q * 32 + rr;
-            if (col >= p.N) break;
-            float f = p.alpha * tile[rr * 33 + lane];
-            if (p.prefetch) f += ext[rr * (p.bn + 1) + c0 + lane];
-            const int64_t o = (int64_t)row * p.ldd + col;
+          auto put = [&](int rr, float f) {
+            const int64_t o = (int64_t)(m0 + q * 32 + rr) * p.ldd + col;
             if (p.out_mode == 3) {
               const bf16 h = __float2bfloat16_rn(f);
               reinterpret_cast<bf16*>(p.D)[o] = h;
@@ -269,6 +277,44 @@ __global__ void __launch_bounds__(THREADS, 1)
               reinterpret_cast<bf16*>(p.D)[o] = __float2bfloat16_rn(f);
             } else {
               reinterpret_cast<float*>(p.D)[o] = f;
+            }
+          };
+          if (CFG == 0) {
+            for (int rr = 0; rr < nrows; ++rr) {
+              if (col >= p.N) break;
+              float f = p.alpha * tile[rr * 33 + lane];
+              if (p.prefetch) f += ext[rr * (p.bn + 1) + c0 + lane];
+              put(rr, f);
+            }
+          } else {
+            float addv[32];
+            if (p.late_add) {
+              // the block's values to add in, all 32 loads in flight before the first store
+              int ac = col;
+              if (p.add && p.add_idx && col < p.N) {
+                ac = __ldg(p.add_idx + col);
+                if ((unsigned)ac >= (unsigned)p.add_bound) {
+                  latch_status(p.status, PIFA_ERR_DEVICE_INDEX);
+                  ac = -1;
+                }
+              }
+#pragma unroll
+              for (int rr = 0; rr < 32; ++rr) {
+                const int row = m0 + q * 32 + rr;
+                float e = 0.0f;
+                if (rr < nrows && col < p.N) {
+                  if (p.out_mode == 2) e = __ldcg(reinterpret_cast<const float*>(p.D) + (int64_t)row * p.ldd + col);
+                  if (p.add && ac >= 0) e += __bfloat162float(p.add[(int64_t)row * p.ldadd + ac]);
+                }
+                addv[rr] = e;
+              }
+            }
+#pragma unroll
+            for (int rr = 0; rr < 32; ++rr) {
+              if (rr >= nrows || col >= p.N) continue;
+              float f = p.alpha * tile[rr * 33 + lane];
+              if (p.late_add) f += addv[rr];
+              put(rr, f);
             }
           }
         }
@@ -281,8 +327,18 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, BNMAX);
+    tmem_dealloc(tmem, TMEM_ALLOC);
   }
+}
+
+int sm_count_gemm() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      n = 1;
+  }
+  return n;
 }
 
 }  // namespace
@@ -298,12 +354,28 @@ int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stre
   a.K = (int)g.K;
   // tile width: MN-major B tiles come in 64-column boxes, K-major ones in multiples of 16
   const int64_t unit = g.b_mn ? 64 : 16;
-  // with values to add in, the tile is at most 128 wide so that their staging fits beside the ring
-  a.prefetch = (g.out_mode == 2 || g.add) ? 1 : 0;
-  const int64_t bnmax = a.prefetch ? 128 : BNMAX;
+  // with values to add in, a config-0 tile is at most 128 wide so that their staging fits beside
+  // the ring
+  const bool adds = g.out_mode == 2 || g.add;
+  if (g.d_trans && adds) return pifa_fail(PIFA_ERR_UNSUPPORTED, "gemm_tc: transposed store with an addend");
+  const int64_t bnmax0 = adds ? 128 : BNMAX;
+  const int64_t bn0 = g.N >= bnmax0 ? bnmax0 : (g.N + unit - 1) / unit * unit;
+  const int64_t tiles0 = ((g.N + bn0 - 1) / bn0) * ((g.M + BM - 1) / BM);
+  // Config per GEMM, from timing each backward and M-accumulator product under both (4096 x 4096,
+  // r = 2048 layer, T = 2048; us, config 0 -> 1):
+  //   gathered addend, hi/lo out (dY_p)          78.8 -> 55.4   config 1
+  //   bf16 or fp32 out, > 1 wave (dX, dW_p, dC)  81.5 -> 77.6, 82.9 -> 79.0, 42.3 -> 40.5   config 1
+  //   fp32 read-modify-write (X X^T, Y_t X^T)    155.8 -> 344.0, 219.7 -> 391.6   config 0
+  //   hi/lo out, no addend (Y_p, Y_t^T)          36.4 -> 41.0, 114.4 -> 128.4   config 0
+  // Config 0 stages the old D while the MMAs run; config 1's 128-wide tiles read shared memory at
+  // the MMA's limit, which only pays where the epilogue dominates.
+  const bool multi = tiles0 > sm_count_gemm();
+  const int cfg_id = g.out_mode == 2 ? 0 : g.add ? 1 : g.out_mode == 3 ? 0 : (multi ? 1 : 0);
+  const int64_t bnmax = cfg_id == 0 ? bnmax0 : kBnMax<1>;
   a.bn = (int)(g.N >= bnmax ? bnmax : (g.N + unit - 1) / unit * unit);
+  a.prefetch = (cfg_id == 0 && adds) ? 1 : 0;
+  a.late_add = (cfg_id == 1 && adds) ? 1 : 0;
   a.d_trans = g.d_trans ? 1 : 0;
-  if (a.d_trans && a.prefetch) return pifa_fail(PIFA_ERR_UNSUPPORTED, "gemm_tc: transposed store with an addend");
   a.idesc = idesc_bf16_f32(BM, (uint32_t)a.bn) | (g.a_mn ? (1u << 15) : 0u) | (g.b_mn ? (1u << 16) : 0u);
   a.passes = (g.A2 || g.B2) ? 2 : 1;
   a.D = g.D;
@@ -345,10 +417,13 @@ int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stre
       st = make_tmap_2d(map, PIFA_DTYPE_BF16, base, g.N, g.K, g.ldb, BK, (uint32_t)a.bn);
     if (st != PIFA_OK) return st;
   }
-  auto kern = g.a_mn ? (g.b_mn ? gemm_tc_kernel<true, true> : gemm_tc_kernel<true, false>)
-                     : (g.b_mn ? gemm_tc_kernel<false, true> : gemm_tc_kernel<false, false>);
+  auto kern = cfg_id == 0 ? (g.a_mn ? (g.b_mn ? gemm_tc_kernel<true, true, 0> : gemm_tc_kernel<true, false, 0>)
+                                    : (g.b_mn ? gemm_tc_kernel<false, true, 0> : gemm_tc_kernel<false, false, 0>))
+                          : (g.a_mn ? (g.b_mn ? gemm_tc_kernel<true, true, 1> : gemm_tc_kernel<true, false, 1>)
+                                    : (g.b_mn ? gemm_tc_kernel<false, true, 1> : gemm_tc_kernel<false, false, 1>));
   const size_t ext_bytes = a.prefetch ? (size_t)4 * 32 * (a.bn + 1) * 4 : 0;
-  const size_t smem = 1024 + (size_t)STAGES * (A_BYTES + (size_t)a.bn * BK * 2) + (ext_bytes + 15) / 16 * 16 + 256;
+  const int stages = cfg_id == 0 ? kStages<0> : kStages<1>;
+  const size_t smem = 1024 + (size_t)stages * (A_BYTES + (size_t)a.bn * BK * 2) + (ext_bytes + 15) / 16 * 16 + 256;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(gemm_tc)", e);
   const unsigned nt = (unsigned)((g.N + a.bn - 1) / a.bn), mt = (unsigned)((g.M + BM - 1) / BM);
