@@ -453,7 +453,8 @@ def backward_point(dev, stream, shape, T, tc_peak, peak_src):
 
 def m_accumulate_point(dev, stream, shape, T, tc_peak, peak_src):
     """pifa_m_accumulate (X X^T and Y_t X^T of one calibration batch, lambda = 0.25) beside the same
-    products through torch.matmul (bf16 in, fp32 out); tensor roofline on 2 T (n^2 + 2 m n)."""
+    products through torch.matmul (bf16 in, fp32 out, X X^T whole); tensor roofline on
+    T n (n + 1) + 4 T m n (the symmetric X X^T's upper triangle, Y_t = W X_mix^T, Y_t X^T)."""
     import torch
     from paper_2501_19090_gb300 import pifa as P
     m, n = shape.m, shape.n
@@ -479,7 +480,7 @@ def m_accumulate_point(dev, stream, shape, T, tc_peak, peak_src):
         us = _steady_us(macc, 4, stream)
         assert P.pifa_device_status(stream) == P.PIFA_OK
         t_us = _steady_us(ref, 4, stream)
-    flops = 2 * T * (n * n + 2 * m * n)
+    flops = T * n * (n + 1) + 4 * T * m * n
     tf = flops / us / 1e6
     del Xu, Xo, W, XXt, YtXt
     torch.cuda.empty_cache()

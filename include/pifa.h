@@ -291,7 +291,9 @@ int64_t pifa_backward_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r)
  *   Xo, Xu       DEVICE, bf16, T x n, common row pitch ldx >= n (Xo may be NULL when YtXt is).
  *   W            DEVICE, bf16, m x n, pitch ldw >= n (the dense weight; may be NULL when YtXt is).
  *   lambda       mix ratio in [0, 1] (Eq. 6; the paper uses 0.25).
- *   XXt          DEVICE in/out, fp32, n x n, pitch ldxx >= n.
+ *   XXt          DEVICE in/out, fp32, n x n, pitch ldxx >= n. X X^T is symmetric: its upper
+ *                triangle (column >= row) is accumulated; of the entries below it, those in tiles
+ *                that straddle the diagonal are accumulated too and the rest are left as they were.
  *   YtXt         DEVICE in/out, fp32, m x n, pitch ldyx >= n (NULL: only XXt is accumulated).
  *   workspace    DEVICE scratch of pifa_m_accumulate_workspace_size(T, m, n) bytes, 256-byte
  *                aligned (X_u^T, the mixed input and Y_t^T in bf16).
@@ -315,7 +317,7 @@ int64_t pifa_m_accumulate_workspace_size(int64_t T, int64_t m, int64_t n);
  * whose product U_r V_r^T is the low-rank weight that Algorithm 1 (pifa_compress_device) turns
  * into a PIFA layer.
  *
- *   XXt          DEVICE, fp32, n x n, pitch ldxx >= n (X X^T).
+ *   XXt          DEVICE, fp32, n x n, pitch ldxx >= n (X X^T; only its upper triangle is read).
  *   YtXt         DEVICE, fp32, m x n, pitch ldyx >= n (Y_t X^T).
  *   V            DEVICE, float64, n x r, contiguous (the pruned layer's right factor).
  *   W            DEVICE, bf16, m x n, pitch ldw >= n (the dense weight; used when alpha > 0).

@@ -288,8 +288,9 @@ extern "C" int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int6
                                              (int)n, XuT, ldT);
     if (e != cudaSuccess) return pifa_fail_cuda("m_accumulate: transpose", e);
   }
-  {  // XXt += X_u^T X_u
+  {  // XXt += X_u^T X_u, its upper triangle (the product is symmetric: half the tiles)
     GemmTc g = {n, n, T, XuT, ldT, false, XuT, ldT, false, XXt, ldxx, 2, 1.0f, nullptr, nullptr, 0, 0};
+    g.upper = true;
     if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
   }
   if (!YtXt) return PIFA_OK;

@@ -635,6 +635,14 @@ __global__ void add_scaled_bf16(const __nv_bfloat16* W, int64_t ldw, int64_t row
     dst[(e / cols) * lddst + e % cols] += alpha * (double)__bfloat162float(W[(e / cols) * ldw + e % cols]);
 }
 
+// A[i][j] = A[j][i] for i > j (n x n, pitch lda): the lower triangle from the upper.
+__global__ void mirror_upper(double* A, int64_t n, int64_t lda) {
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n * n; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t i = e / n, j = e % n;
+    if (i > j) A[i * lda + j] = A[j * lda + i];
+  }
+}
+
 __global__ void add_diag(double* A, int64_t k, int64_t lda, double alpha) {
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < k; i += (int64_t)gridDim.x * blockDim.x)
     A[i * lda + i] += alpha;
@@ -742,6 +750,8 @@ extern "C" int pifa_m_reconstruct(const float* XXt, int64_t ldxx, const float* Y
   cudaError_t e = cudaMemsetAsync(bad, 0, 8, s);
   if (e != cudaSuccess) return pifa_fail_cuda("reconstruct: memset", e);
   f32_to_f64<<<grid_for(n * n), 256, 0, s>>>(XXt, ldxx, n, n, A, n);
+  pifa_count_launch();
+  mirror_upper<<<grid_for(n * n), 256, 0, s>>>(A, n, n);  // pifa_m_accumulate keeps the upper triangle
   pifa_count_launch();
   f32_to_f64<<<grid_for(m * n), 256, 0, s>>>(YtXt, ldyx, m, n, B, n);
   pifa_count_launch();

@@ -63,6 +63,7 @@ struct GemmTcArgs {
   int64_t ldadd;
   int add_bound;      // columns of the addend (index bound)
   int late_add;       // 1 (config 1): the epilogue loads the old D and the addend itself
+  int upper;          // 1: tiles wholly below the diagonal (rows all > columns) do nothing
   int* status;
   uint64_t timeout_ns;
 };
@@ -86,6 +87,8 @@ __global__ void __launch_bounds__(THREADS, CFG == 0 ? 1 : 2)
                    const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmB2, GemmTcArgs p) {
   constexpr int STAGES = kStages<CFG>;
   constexpr uint32_t TMEM_ALLOC = (uint32_t)kBnMax<CFG>;
+  // a symmetric product's tiles wholly below the diagonal are not computed
+  if (p.upper && (int)blockIdx.y * BM >= (int)blockIdx.x * p.bn + p.bn) return;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t b_bytes = (uint32_t)p.bn * BK * 2;
@@ -376,6 +379,8 @@ int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stre
   a.prefetch = (cfg_id == 0 && adds) ? 1 : 0;
   a.late_add = (cfg_id == 1 && adds) ? 1 : 0;
   a.d_trans = g.d_trans ? 1 : 0;
+  if (g.upper && g.M != g.N) return pifa_fail(PIFA_ERR_INVALID_ARG, "gemm_tc: upper triangle of a non-square product");
+  a.upper = g.upper ? 1 : 0;
   a.idesc = idesc_bf16_f32(BM, (uint32_t)a.bn) | (g.a_mn ? (1u << 15) : 0u) | (g.b_mn ? (1u << 16) : 0u);
   a.passes = (g.A2 || g.B2) ? 2 : 1;
   a.D = g.D;

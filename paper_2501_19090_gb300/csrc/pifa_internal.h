@@ -137,6 +137,7 @@ struct GemmTc {
   const void* B2 = nullptr;
   void* D2 = nullptr;
   bool d_trans = false;  // store D^T: element (i, j) at D[j * ldd + i] (out_mode 0, 1 or 3 only)
+  bool upper = false;    // M == N: skip tiles wholly below the diagonal (a symmetric product's upper triangle)
 };
 int gemm_tc(const GemmTc& g, int* status, uint64_t timeout_ns, cudaStream_t stream);
 

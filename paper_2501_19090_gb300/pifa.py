@@ -497,8 +497,9 @@ def pifa_backward(X, Wp, C, pivot_idx, nonpivot_idx, dY, want=("dX", "dWp", "dC"
 
 
 def pifa_m_accumulate(Xo, Xu, W, lam, XXt, YtXt=None, workspace_tensor=None, stream=None):
-    """One calibration batch into the M accumulators (pifa_m_accumulate): XXt (fp32 n x n) and
-    YtXt (fp32 m x n, optional) are updated in place. Xo, Xu bf16 T x n; W bf16 m x n."""
+    """One calibration batch into the M accumulators (pifa_m_accumulate): XXt (fp32 n x n, its
+    upper triangle: X X^T is symmetric) and YtXt (fp32 m x n, optional) are updated in place.
+    Xo, Xu bf16 T x n; W bf16 m x n."""
     import torch
     for name, t in (("Xu", Xu), ("XXt", XXt)):
         if not isinstance(t, torch.Tensor) or t.device.type != "cuda":

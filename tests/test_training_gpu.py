@@ -113,7 +113,8 @@ def test_m_accumulate_two_batches_match_the_oracle():
         P.pifa_m_accumulate(dev_bf16(Xo), dev_bf16(Xu), dev_bf16(W0), lam, XXt, YtXt)
         ref = oracle.m_accumulate(Xo, Xu, W0, lam, *ref)
     assert P.pifa_device_status() == P.PIFA_OK
-    check(XXt.cpu().numpy(), ref[0], "X X^T")
+    # X X^T is accumulated in its upper triangle (it is symmetric)
+    check(np.triu(XXt.cpu().numpy()), np.triu(ref[0]), "X X^T")
     check(YtXt.cpu().numpy(), ref[1], "Y_t X^T")
 
 
@@ -122,7 +123,7 @@ def test_m_accumulate_xxt_only_and_lambda_edges():
     Xo, Xu, W = _macc_inputs(100, n, 128, 3)
     XXt = torch.zeros((n, n), dtype=torch.float32, device=DEV)
     P.pifa_m_accumulate(None, dev_bf16(Xu), None, 0.5, XXt)
-    check(XXt.cpu().numpy(), oracle.m_accumulate(Xo, Xu, W, 0.5)[0], "X X^T alone")
+    check(np.triu(XXt.cpu().numpy()), np.triu(oracle.m_accumulate(Xo, Xu, W, 0.5)[0]), "X X^T alone")
     for lam in (0.0, 1.0):
         XXt.zero_()
         Y = torch.zeros((128, n), dtype=torch.float32, device=DEV)
@@ -142,7 +143,8 @@ def test_m_accumulate_llama_shape_sampled_rows():
     assert P.pifa_device_status() == P.PIFA_OK
     rx, ry = inputs.random_rows(n, 48, 5), inputs.random_rows(m, 48, 6)
     a, b = oracle.m_accumulate(Xo, Xu, W, 0.25, rows=(rx, ry))
-    check(XXt[torch.from_numpy(rx)].cpu().numpy(), a, "X X^T rows")
+    upper = np.arange(n)[None, :] >= rx[:, None]  # the accumulated triangle of each sampled row
+    check(np.where(upper, XXt[torch.from_numpy(rx)].cpu().numpy(), 0.0), np.where(upper, a, 0.0), "X X^T rows")
     check(YtXt[torch.from_numpy(ry)].cpu().numpy(), b, "Y_t X^T rows")
 
 
@@ -167,6 +169,7 @@ def test_m_reconstruct_matches_the_oracle_on_the_same_accumulators(m, n, r, T, a
     Wd = dev_bf16(W)
     U_r, V_r = P.pifa_m_reconstruct(XXt, YtXt, torch.from_numpy(V).to(DEV), W=Wd, alpha=alpha)
     A, B = XXt.double().cpu().numpy(), YtXt.double().cpu().numpy()
+    A = np.triu(A) + np.triu(A, 1).T  # the library keeps X X^T's upper triangle; both sides see it whole
     rU, rV = oracle.m_reconstruct(A, B, V, W=W.astype(np.float64), alpha=alpha)
     for got, ref, what in ((U_r, rU, "U_r"), (V_r, rV, "V_r")):
         got = got.cpu().numpy()
