@@ -55,6 +55,8 @@ CASES = [
     ("r = m 64x128", (64, 128, 64, 4, "greedy"), 20),
     ("rank one 40x48", (40, 48, 1, 5, "greedy"), 13),
     ("7B attention 4096x4096 r2048", (4096, 4096, 2048, 0, "lapack"), 512),
+    # T = 2048: dX and dW_p span more than one wave of tiles and run gemm_tc's two-CTA shape
+    ("7B attention 4096x4096 r2048 T2048", (4096, 4096, 2048, 0, "lapack"), 2048),
 ]
 
 
