@@ -92,3 +92,24 @@ def test_headline_cut():
     p1, p2 = make_plan(4096, 8192, 304), make_plan(24576, 4096, 304)
     assert (p1["grid"], p1["ncf"], p1["ns"], p1["nclast"]) == (304, 13, 10, 11)
     assert (p2["grid"], p2["ncf"], p2["ns"], p2["nclast"]) == (304, 40, 2, 24)
+
+
+def make_plan_fixed(R, K, grid):
+    nrb, nck = -(-R // TM), -(-K // KB)
+    total = nrb * nck
+    u = max(1, min(total // grid, nck))
+    ns = -(-nck // u)
+    return dict(nrb=nrb, nck=nck, total=total, grid=grid, ncf=u, ns=ns, nclast=nck - (ns - 1) * u)
+
+
+@pytest.mark.parametrize("R,K", [(24576, 4096), (19456, 8192), (38912, 520), (24577, 4100), (152 * 128, 64)])
+def test_whole_row_plan_gives_each_cta_one_row_block(R, K):
+    """The whole-row plan (grid = the phase's 128-row blocks) cuts K into one slice, and every
+    CTA's range is exactly one unit: no unit is split, so the epilogue's sums are the outputs."""
+    nrb = -(-R // TM)
+    p = make_plan_fixed(R, K, nrb)
+    assert p["ns"] == 1 and p["ncf"] == p["nclast"] == p["nck"]
+    parts = walk(p)
+    assert len(parts) == nrb
+    for (s, rb), ps in parts.items():
+        assert ps == [(rb, 0, p["nck"])]
