@@ -59,10 +59,10 @@ T_DECODE = 16
 # measured with ncu, keyed by (layer, T), with the sha256 prefixes of the kernel sources it was
 # taken on. A source mismatch (a kernel changed since the capture) reports traffic as null.
 NCU_TRAFFIC = {
-    # profiles/decode_tc_gateup70b_T16_traffic.md: split-K partial + reduce, both phases
+    # profiles/decode_tc_gateup70b_T16_traffic.md: phase 1 split-K partial + reduce, phase 2 whole rows
     ("llama2_70b_gate_up_28672x8192_r4096", 16): {
-        "sha": {"decode_tc.cu": "df2f3ae613e49c89", "decode.cu": "0d83c7d91223b49c"},
-        "bytes": 285136896,
+        "sha": {"decode_tc.cu": "33c9277b7d351a3c", "decode.cu": "0d83c7d91223b49c"},
+        "bytes": 275081984,
     },
 }
 
