@@ -268,11 +268,11 @@ def layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src, name=None, c
     """One layer shape at T tokens: the selected PIFA variant, the two-factor low-rank layer and the
     dense layer on the same GPU, each a CUDA graph replayed in steady state over rotating weight
     copies (decode: every copy's bytes exceed 3x L2 in total; prefill: two copies), with the
-    roofline of the PIFA call (HBM for T <= 16, bf16 tensor otherwise) and the clocks seen."""
+    roofline of the PIFA call (HBM for decode, T <= DECODE_MAX_T; bf16 tensor otherwise) and the clocks seen."""
     import torch
     from paper_2501_19090_gb300 import pifa as P
     m, n, r = shape.m, shape.n, shape.r
-    decode = T <= 16
+    decode = T <= DECODE_MAX_T
     copies = _copies_for(dev, 2 * r * (m + n - r)) if decode else 2
     piv, nonp, Wps, Cs = timing_layer(shape, dev, 7, c_dtype, copies)
     gen = torch.Generator(device=dev)
@@ -323,8 +323,11 @@ def layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src, name=None, c
     return out
 
 
-DECODE_POINTS = [(inputs.ATTN7B, (1, 8, 16)), (inputs.MLP7B_GATE, (1, 8, 16)), (inputs.MLP7B_DOWN, (1, 8, 16)),
-                 (inputs.ATTN70B, (1, 8, 16)), (inputs.MLP70B_GATE, (1, 8, 16))]
+# the library's selector runs the decode variant up to this many tokens, the split prefill above
+DECODE_MAX_T = 64
+DECODE_POINTS = [(inputs.ATTN7B, (1, 8, 16, 64)), (inputs.MLP7B_GATE, (1, 8, 16, 64)),
+                 (inputs.MLP7B_DOWN, (1, 8, 16, 64)), (inputs.ATTN70B, (1, 8, 16, 64)),
+                 (inputs.MLP70B_GATE, (1, 8, 16, 32, 64))]
 PREFILL_POINTS = [(inputs.ATTN7B, 2048), (inputs.ATTN7B, 8192), (inputs.ATTN70B, 4096), (inputs.MLP70B_GATE, 4096)]
 
 
@@ -336,7 +339,7 @@ def mlp7b_point(dev, stream, T, hbm_peak, tc_peak, peak_src):
     import torch
     from paper_2501_19090_gb300 import pifa as P
     G_, D_ = inputs.MLP7B_GATE, inputs.MLP7B_DOWN
-    decode = T <= 16
+    decode = T <= DECODE_MAX_T
     copies = 4 if decode else 2
     lay = {name: timing_layer(s, dev, seed, copies=copies) for name, s, seed in
            (("gate", G_, 1), ("up", G_, 2), ("down", D_, 3))}
@@ -529,7 +532,7 @@ def run_ours(args, rank, world, local_rank):
     m, n, r = shape.m, shape.n, shape.r
     T = args.tokens
     K = max(1, args.steps)
-    decode = T <= 16
+    decode = T <= DECODE_MAX_T
     wbytes = 2 * r * (m + n - r)
     copies = _copies_for(dev, wbytes)
     piv, nonp, Wps, Cs = timing_layer(shape, dev, 0, args.c_dtype, copies)
@@ -954,7 +957,7 @@ def run_reference(args, rank):
     return {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": done, "requested_steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / done,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": f"{shape.name} {'decode' if T <= 16 else 'prefill'} T={T}",
+            "data": "synthetic", "config": {"workload": f"{shape.name} {'decode' if T <= DECODE_MAX_T else 'prefill'} T={T}",
                                             "m": shape.m, "n": shape.n, "r": shape.r, "tokens_per_step": T,
                                             "c_dtype": args.c_dtype, "parallelism": f"replicas{args.gpus}"},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",

@@ -56,7 +56,7 @@ typedef enum { PIFA_DTYPE_BF16 = 0, PIFA_DTYPE_FP16 = 1 } pifa_dtype;
  * the given shape returns PIFA_ERR_UNSUPPORTED. */
 typedef enum {
   PIFA_VARIANT_AUTO = 0,
-  PIFA_VARIANT_DECODE = 1,        /* T <= 16: two-phase HBM-streaming GEMV (mma.sync fragments)  */
+  PIFA_VARIANT_DECODE = 1,        /* T <= 64: two HBM-streaming phases (mma.sync or tcgen05)     */
   PIFA_VARIANT_PREFILL_SPLIT = 2, /* tcgen05 GEMM 1 -> Y_p in workspace -> tcgen05 GEMM 2        */
   PIFA_VARIANT_PREFILL_FUSED = 3  /* reserved: not built in this version (PIFA_ERR_UNSUPPORTED)   */
 } pifa_variant;
@@ -85,7 +85,7 @@ typedef struct {
  *   workspace    DEVICE scratch of at least pifa_workspace_size(T, m, n, r, c_dtype, variant) bytes,
  *                256-byte aligned; it needs no initialisation. Its first 256 bytes are reserved
  *                for library state (no kernel of this version reads or writes them); the rest
- *                holds Y_p between the two contractions. It must not overlap Y or an input
+ *                holds Y_p between the two contractions and the split-K decode's fp32 partial sums. It must not overlap Y or an input
  *                (PIFA_ERR_INVALID_ARG; only the first pifa_workspace_size() bytes are checked),
  *                nor be used by another call that may run concurrently.
  *   cuda_stream  a cudaStream_t (NULL = legacy default stream).
@@ -186,7 +186,7 @@ int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dt
 
 /* pifa_select_variant -- the selector (host, < 1 us): the pifa_variant pifa_forward runs for
  * (T, m, n, r, c_dtype) on this build, never PIFA_VARIANT_AUTO; negative pifa_status on bad
- * arguments. Decode for T <= 16, else the split prefill. */
+ * arguments. Decode for T <= 64, else the split prefill. */
 int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype);
 
 /* pifa_variant_name -- static string naming a pifa_variant ("decode", ...); "?" if unknown. */
@@ -357,7 +357,7 @@ int pifa_device_status(void* cuda_stream);
  * undefined. Process-wide; PIFA_ERR_INVALID_ARG for ns < 0. */
 int pifa_set_wait_timeout(int64_t ns);
 
-/* pifa_set_decode_grid -- how the decode variant (T <= 16) lays out each of its two phases for
+/* pifa_set_decode_grid -- how the decode variant with T <= 16 lays out each of its two phases for
  * calls made after this one (process-wide). Three forms compute a phase (R weight rows, K
  * columns): waves of one-tile clusters, every CTA staging its weight rows at launch; a persistent
  * grid of co-resident clusters that stream their tiles through a ring of TMA-filled stages; and
@@ -370,7 +370,9 @@ int pifa_set_wait_timeout(int64_t ns);
  * grid. PIFA_DECODE_GRID_WAVES (1), PIFA_DECODE_GRID_PERSISTENT (2) and PIFA_DECODE_GRID_SPLITK
  * (3) force one form for both phases (a tuning and test knob: all compute the same result up to
  * the summation order of fp32 partial sums; forced split-K runs the persistent grid instead when the
- * workspace is too small for its partial sums). PIFA_ERR_INVALID_ARG for other values. */
+ * workspace is too small for its partial sums). For 16 < T <= 64 only the split-K form exists
+ * (token tiles of 32 or 64 rows): both phases run it whatever the mode. PIFA_ERR_INVALID_ARG for
+ * other values. */
 #define PIFA_DECODE_GRID_AUTO 0
 #define PIFA_DECODE_GRID_WAVES 1
 #define PIFA_DECODE_GRID_PERSISTENT 2

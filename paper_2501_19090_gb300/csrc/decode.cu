@@ -1,5 +1,6 @@
-// decode.cu -- PIFA forward for small token counts (T <= 16): Algorithm 2 as two HBM-streaming
-// phases, one kernel each.
+// decode.cu -- PIFA forward for small token counts (T <= 64): Algorithm 2 as two HBM-streaming
+// phases. Up to T = 16 each phase runs one of the forms below or the split-K tensor-core form of
+// decode_tc.cu; for 16 < T <= 64 both phases run the latter.
 //
 //   phase 1: Y_p = X W_p^T  (the r rows of W_p, each read once)  -> Y[:, I[j]] = bf16(Y_p[:, j]),
 //            and y_p to the workspace as a hi + lo pair of C's dtype  (Algorithm 2, steps 2 and 4)
@@ -978,6 +979,10 @@ int launch_one_phase(DecodeArgs& a, uint32_t budget, int dtype, const SplitKScra
   const char* what = PHASE == 1 ? "decode phase 1 launch" : "decode phase 2 launch";
   const int mode = g_decode_grid.load(std::memory_order_relaxed);
   const bool tc_fits = sk.P != nullptr && decode_tc_partial_bytes(a.R, a.K, a.T, PHASE == 1 ? 1 : 2) <= sk.bytes;
+  if (a.T > 16) {  // token tiles of 32 and 64 rows exist only in the split-K tensor-core form
+    if (!tc_fits) return pifa_fail(PIFA_ERR_INVALID_ARG, "decode with T > 16 needs the split-K workspace");
+    return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
+  }
   if (mode == PIFA_DECODE_GRID_SPLITK && tc_fits) return launch_phase_tc<PHASE, kF16C>(a, dtype, sk, stream);
   // Auto, keyed on the phase's shape and T (phase 1: r rows of K = n; phase 2: m - r rows of
   // K = r): for T > 2 a phase of at least 32 blocks of 128 rows runs split-K on the tensor cores

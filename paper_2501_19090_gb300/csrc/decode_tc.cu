@@ -1,5 +1,6 @@
-// decode_tc.cu -- one decode phase (T <= 16 tokens) of Algorithm 2 on the 5th-generation tensor
-// cores, split over K across a persistent grid: the form used for layers too large for one wave.
+// decode_tc.cu -- one decode phase (T <= 64 tokens) of Algorithm 2 on the 5th-generation tensor
+// cores, split over K across a persistent grid: the form used for layers too large for one wave,
+// and the only decode form for 16 < T <= 64.
 //
 // A phase is a skinny product D = A B^T: A the weight rows (W_p for Y_p = X W_p^T, Algorithm 2
 // step 2; C for Y_np = Y_p C^T, step 3), B the T token rows (x, or y_p as its hi and lo planes).
@@ -12,13 +13,14 @@
 //
 // Partial kernel (two CTAs per SM, 192 threads each):
 //   warp 0     TMA producer: per chunk, the weight tile (128 rows x 64 columns, 128-byte swizzle)
-//              and the matching 64 columns of B (16 token rows per plane; rows >= T zero-filled)
+//              and the matching 64 columns of B (a token tile of TNT = 16, 32 or 64 rows per
+//              plane, the smallest that holds T; rows >= T zero-filled)
 //              into one stage of a ring; the first weight tiles go out before the dependency wait
 //              (the weights do not depend on the previous kernel), their B boxes after it.
 //   warp 1     owns 256 TMEM columns (two segments in flight) and issues tcgen05.mma.kind::f16
-//              M = 128, K = 16, N = 16 (one B plane) or 32 (the y_p hi and lo planes as one
+//              M = 128, K = 16, N = TNT (one B plane) or 2 TNT (the y_p hi and lo planes as one
 //              operand) from one thread, dealing a segment's MMAs round-robin over independent
-//              accumulators so that consecutive MMAs do not wait for each other.
+//              accumulators (128 / N of them) so that consecutive MMAs do not wait for each other.
 //   warps 2-5  sum a segment's accumulators (TMEM lane quarter each) while the next segment fills
 //              the other set, and store its partial sums P[s][t][row] (fp32, coalesced over rows).
 // A unit's head CTA writes zeros to P2 when it holds the whole unit, so P2 is defined everywhere.
@@ -43,19 +45,19 @@ using namespace pifa;
 using bf16 = __nv_bfloat16;
 
 constexpr int TM = 128;                         // weight rows per unit (MMA M = TMEM lanes)
-constexpr int TN = 16;                          // token rows of B, padded (MMA N)
+constexpr int TN = 16;                          // token rows of B, padded (MMA N), for T <= 16
+constexpr int kMaxTokensTc = 64;                // token tiles of 32 and 64 rows serve T <= 64
 constexpr int KB = 64;                          // K per chunk: one 128-byte swizzle row
 constexpr uint32_t A_BYTES = TM * KB * 2;       // one weight tile
-constexpr uint32_t BOX_BYTES = TN * KB * 2;     // one B box
 constexpr int MAX_STAGES = 10;
 constexpr int THREADS = 192;
 // A segment's MMAs are dealt round-robin over NACC independent accumulators (summed in the
 // epilogue), so that consecutive MMAs do not wait for each other. With two B planes (y_p hi and
-// lo) one MMA of N = 32 covers both: the lo box follows the hi box in shared memory, making one
-// 32-row operand, and accumulator columns t and 16 + t are added in the epilogue. Per segment
-// NACC * 16 * NB columns; two segments in flight: 256 TMEM columns either way.
-template <int NB>
-constexpr int kNacc = NB == 1 ? 8 : 4;
+// lo) one MMA of N = 2 TNT covers both: the lo box follows the hi box in shared memory, making one
+// 2 TNT-row operand, and accumulator columns t and TNT + t are added in the epilogue. Per segment
+// NACC * TNT * NB = 128 columns; two segments in flight: 256 TMEM columns in every case.
+template <int NB, int TNT = TN>
+constexpr int kNacc = 128 / (TNT * NB);
 constexpr uint32_t TMEM_COLS = 256;
 // Two CTAs per SM, each with its own producer and MMA-issuing thread: one issuing thread per SM
 // measured as the limit (70B gate/up, T = 16: 73 us with one CTA of ten stages, 60 us with two of
@@ -154,7 +156,7 @@ __device__ __forceinline__ Seg seg_at(const TcArgs& a, int64_t g, int64_t e) {
 // Column (within the unit's K-slice) of the c-th chunk a CTA loads for segment q.
 __device__ __forceinline__ int seg_col(const Seg& q, int c) { return (q.c0 + c) * KB; }
 
-template <int NB>
+template <int NB, int TNT>
 __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
     decode_tc_partial(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                       const __grid_constant__ CUtensorMap tmB1, TcArgs a) {
@@ -237,7 +239,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
             tma_load_2d(smem_u32(stage), &tmA, q.s * a.ncf * KB + kx, q.rb * TM, &full[st]);
           }
           tma_load_2d(smem_u32(stage + A_BYTES), &tmB0, x0 + kx, 0, &full[st]);
-          if (NB > 1) tma_load_2d(smem_u32(stage + A_BYTES + BOX_BYTES), &tmB1, x0 + kx, 0, &full[st]);
+          if (NB > 1) tma_load_2d(smem_u32(stage + A_BYTES + (uint32_t)TNT * KB * 2), &tmB1, x0 + kx, 0, &full[st]);
         }
       }
       int issued = dead ? it : total;
@@ -261,8 +263,8 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
           break;
         }
         tc_fence_after();
-        constexpr int NACC = kNacc<NB>;
-        const uint32_t dacc = tmem + (uint32_t)(acc * NACC * TN * NB);
+        constexpr int NACC = kNacc<NB, TNT>;
+        const uint32_t dacc = tmem + (uint32_t)(acc * NACC * TNT * NB);
         int e = 0;  // MMAs of this segment so far: accumulator e % NACC, first use overwrites
         for (int c = 0; c < q.nc; ++c, ++it) {
           const int st = it % a.stages;
@@ -274,7 +276,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
           const uint32_t at = smem_u32(ring + (size_t)st * a.stage_bytes);
 #pragma unroll
           for (int kk = 0; kk < KB / 16; ++kk, ++e)
-            mma_bf16_ss(dacc + (uint32_t)((e % NACC) * TN * NB), sw128_desc(at + kk * 32),
+            mma_bf16_ss(dacc + (uint32_t)((e % NACC) * TNT * NB), sw128_desc(at + kk * 32),
                         sw128_desc(at + A_BYTES + kk * 32), a.idesc, e >= NACC ? 1u : 0u);
           mma_commit(&empty[st]);  // the stage is free once these MMAs have read it
         }
@@ -304,24 +306,42 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
       tc_fence_after();
       // the accumulators this segment wrote (fewer than NACC only when it has fewer MMAs), summed
       // in a fixed order
-      constexpr int NACC = kNacc<NB>;
+      constexpr int NACC = kNacc<NB, TNT>;
       const int used = min(NACC, q.nc * (KB / 16));
-      const uint32_t base = tmem + ((uint32_t)(q4 * 32) << 16) + (uint32_t)(acc * NACC * TN * NB);
-      float sum[TN];
+      const uint32_t base = tmem + ((uint32_t)(q4 * 32) << 16) + (uint32_t)(acc * NACC * TNT * NB);
+      float sum[TNT];
 #pragma unroll
-      for (int t = 0; t < TN; ++t) sum[t] = 0.0f;
-      // column groups of 16: accumulator a, plane nb at (a NB + nb) 16
-      for (int c0 = 0; c0 < used * NB; c0 += 4) {
-        uint32_t v[4][16];
+      for (int t = 0; t < TNT; ++t) sum[t] = 0.0f;
+      if (TNT == TN) {
+        // column groups of 16: accumulator a, plane nb at (a NB + nb) 16, four loads in flight
+        for (int c0 = 0; c0 < used * NB; c0 += 4) {
+          uint32_t v[4][16];
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          if (c0 + k < used * NB) tmem_ld_32x32b_x16(base + (uint32_t)((c0 + k) * TN), v[k]);
-        tmem_ld_wait();
+          for (int k = 0; k < 4; ++k)
+            if (c0 + k < used * NB) tmem_ld_32x32b_x16(base + (uint32_t)((c0 + k) * TN), v[k]);
+          tmem_ld_wait();
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          if (c0 + k < used * NB)
+          for (int k = 0; k < 4; ++k)
+            if (c0 + k < used * NB)
 #pragma unroll
-            for (int t = 0; t < TN; ++t) sum[t] += __uint_as_float(v[k][t]);
+              for (int t = 0; t < TN; ++t) sum[t % TNT] += __uint_as_float(v[k][t]);
+        }
+      } else {
+        // wider token tiles: accumulator a, plane nb, tokens 16 g .. 16 g + 15 at column
+        // (a NB + nb) TNT + 16 g; one (a, nb) pair's TNT / 16 loads in flight at a time
+        for (int a2 = 0; a2 < used; ++a2)
+#pragma unroll
+          for (int nb = 0; nb < NB; ++nb) {
+            uint32_t v[TNT / 16][16];
+#pragma unroll
+            for (int g = 0; g < TNT / 16; ++g)
+              tmem_ld_32x32b_x16(base + (uint32_t)((a2 * NB + nb) * TNT + 16 * g), v[g]);
+            tmem_ld_wait();
+#pragma unroll
+            for (int g = 0; g < TNT / 16; ++g)
+#pragma unroll
+              for (int j = 0; j < 16; ++j) sum[16 * g + j] += __uint_as_float(v[g][j]);
+          }
       }
       tc_fence_before();
       __syncwarp();
@@ -335,7 +355,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
             latch_status(a.status, PIFA_ERR_DEVICE_INDEX);
           } else {
 #pragma unroll
-            for (int t = 0; t < TN; ++t)
+            for (int t = 0; t < TNT; ++t)
               if (t < a.T) a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(sum[t]);
           }
         }
@@ -346,7 +366,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
         const bool whole = q.c0 == 0 && q.nc == (q.s < a.ns - 1 ? a.ncf : a.nclast);
         float* dst = (q.c0 == 0 ? a.P : a.P2) + off;
 #pragma unroll
-        for (int t = 0; t < TN; ++t)
+        for (int t = 0; t < TNT; ++t)
           if (t < a.T) {
             dst[(size_t)t * a.R] = sum[t];
             if (whole) a.P2[off + (size_t)t * a.R] = 0.0f;
@@ -462,7 +482,10 @@ int64_t decode_tc_partial_bytes(int64_t R, int64_t K, int64_t T, int NB) {
 
 int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, cudaStream_t stream) {
   const int NB = ph.planes;
-  if (ph.R < 1 || ph.K < 1 || ph.T < 1 || ph.T > TN) return pifa_fail(PIFA_ERR_INVALID_ARG, "decode_tc: empty or oversized phase");
+  if (ph.R < 1 || ph.K < 1 || ph.T < 1 || ph.T > kMaxTokensTc)
+    return pifa_fail(PIFA_ERR_INVALID_ARG, "decode_tc: empty or oversized phase");
+  // token tile (MMA N per plane): 16, 32 or 64 rows of B, those beyond T zero-filled by TMA
+  const int TNT = ph.T <= 16 ? 16 : ph.T <= 32 ? 32 : 64;
   // Whole-row plan: when a phase without y_p planes to write has between one and two 128-row blocks
   // per SM, each CTA takes one row block over all of K. No partial sums and no reduce kernel: one
   // kernel and one kernel boundary fewer per phase (measured on the 70B gate/up layer, whose phase 2
@@ -482,9 +505,9 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   a.grid = p.grid;
   a.gsz = (int)ph.gsz;
   a.goff = (int)ph.goff;
-  a.stage_bytes = A_BYTES + (uint32_t)NB * BOX_BYTES;
+  a.stage_bytes = A_BYTES + (uint32_t)(NB * TNT) * KB * 2;
   const bool f16 = ph.mma_f16;
-  a.idesc = f16 ? idesc_f16_f32(TM, TN * NB) : idesc_bf16_f32(TM, TN * NB);
+  a.idesc = f16 ? idesc_f16_f32(TM, (uint32_t)(TNT * NB)) : idesc_bf16_f32(TM, (uint32_t)(TNT * NB));
   a.P = ph.P;
   a.P2 = ph.P + (size_t)p.ns * ph.T * ph.R;
   a.direct = direct ? 1 : 0;
@@ -502,11 +525,13 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   CUtensorMap tA, tB0, tB1;
   int st;
   if ((st = make_tmap_2d(&tA, ph.dtype, ph.A, ph.R, ph.K, ph.lda, KB, TM)) != PIFA_OK) return st;
-  if ((st = make_tmap_2d(&tB0, ph.dtype, ph.B0, ph.T, ph.bcols, ph.ldb, KB, TN)) != PIFA_OK) return st;
-  if (NB > 1 && (st = make_tmap_2d(&tB1, ph.dtype, ph.B1, ph.T, ph.bcols, ph.ldb, KB, TN)) != PIFA_OK) return st;
+  if ((st = make_tmap_2d(&tB0, ph.dtype, ph.B0, ph.T, ph.bcols, ph.ldb, KB, (uint32_t)TNT)) != PIFA_OK) return st;
+  if (NB > 1 && (st = make_tmap_2d(&tB1, ph.dtype, ph.B1, ph.T, ph.bcols, ph.ldb, KB, (uint32_t)TNT)) != PIFA_OK)
+    return st;
   if (NB == 1) tB1 = tB0;
 
-  auto kern = NB == 1 ? decode_tc_partial<1> : decode_tc_partial<2>;
+  auto kern = NB == 1 ? (TNT == 16 ? decode_tc_partial<1, 16> : TNT == 32 ? decode_tc_partial<1, 32> : decode_tc_partial<1, 64>)
+                      : (TNT == 16 ? decode_tc_partial<2, 16> : TNT == 32 ? decode_tc_partial<2, 32> : decode_tc_partial<2, 64>);
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(decode_tc)", e);
   cudaLaunchConfig_t cfg = {};

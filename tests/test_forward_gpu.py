@@ -269,11 +269,12 @@ def test_decode_persistent_grid_fp16_c_and_padding(T):
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
-@pytest.mark.parametrize("T", [1, 3, 8, 16])
+@pytest.mark.parametrize("T", [1, 3, 8, 16, 17, 33, 64])
 def test_decode_splitk_tensor_cores_ragged(T):
     """The split-K tensor-core decode form forced on a layer with ragged K in both phases (520 and
     264 columns: partial 64-column chunks and K-slices), a partial last 128-row block in phase 1
-    (264 rows) and many units per CTA in phase 2 (39736 rows)."""
+    (264 rows) and many units per CTA in phase 2 (39736 rows). T = 17 and 33 fill token tiles of
+    32 and 64 rows only partly; T = 64 fills its tile."""
     L = layer_for(40000, 520, 264, 3, "synthetic")
     P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_SPLITK)
     try:
@@ -282,7 +283,7 @@ def test_decode_splitk_tensor_cores_ragged(T):
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
-@pytest.mark.parametrize("T", [1, 8, 16])
+@pytest.mark.parametrize("T", [1, 8, 16, 32, 64])
 def test_decode_splitk_tensor_cores_compressed_layers(T):
     """The split-K form on compressed layers (C that cancels): 7B attention and the 70B gate/up
     layer, and C stored as fp16 (fp16 MMAs in phase 2, fp16 hi/lo planes) on padded pitches."""
@@ -304,6 +305,10 @@ def test_decode_splitk_deterministic_and_r_equals_m():
         assert np.array_equal(run(L, X, P.PIFA_VARIANT_DECODE), run(L, X, P.PIFA_VARIANT_DECODE))
         parity(layer_for(64, 128, 64, 4, "oracle_greedy"), 9, P.PIFA_VARIANT_DECODE)
         parity(layer_for(40, 48, 1, 5, "oracle_greedy"), 12, P.PIFA_VARIANT_DECODE)
+        X = acts(48, 4096, 5)
+        assert np.array_equal(run(L, X, P.PIFA_VARIANT_DECODE), run(L, X, P.PIFA_VARIANT_DECODE))
+        parity(layer_for(64, 128, 64, 4, "oracle_greedy"), 40, P.PIFA_VARIANT_DECODE)
+        parity(layer_for(40, 48, 1, 5, "oracle_greedy"), 64, P.PIFA_VARIANT_DECODE)
     finally:
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
@@ -361,10 +366,10 @@ def test_launch_count_per_call():
 # ---------------------------------------------------------------------------------------------
 # edge cases
 # ---------------------------------------------------------------------------------------------
-@pytest.mark.parametrize("T", [1, 3, 13, 16, 17, 100, 300])
+@pytest.mark.parametrize("T", [1, 3, 13, 16, 17, 40, 64, 65, 100, 300])
 def test_ragged_shapes_all_variants(T):
     L = layer_for(300, 200, 77, 3, "oracle_greedy")
-    variants = [P.PIFA_VARIANT_PREFILL_SPLIT] + ([P.PIFA_VARIANT_DECODE] if T <= 16 else [])
+    variants = [P.PIFA_VARIANT_PREFILL_SPLIT] + ([P.PIFA_VARIANT_DECODE] if T <= 64 else [])
     for v in variants:
         parity(L, T, v)
 
@@ -458,6 +463,8 @@ def test_selector_picks_split_prefill():
     assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(16, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
+    assert P.pifa_select_variant(64, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
+    assert P.pifa_select_variant(65, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT
 
 
 @pytest.mark.parametrize("T,sample", [(2048, None), (8192, 512), (300, None), (17, None)])
@@ -483,10 +490,10 @@ def test_fp16_c_llama70b(T):
     parity(layer_for(28672, 8192, 4096, 0, "gpu", "fp16"), T, sample=128)
 
 
-@pytest.mark.parametrize("T", [1, 17, 100, 300, 513])
+@pytest.mark.parametrize("T", [1, 17, 40, 64, 100, 300, 513])
 def test_fp16_c_ragged_split_and_decode(T):
     L = layer_for(300, 200, 77, 3, "oracle_greedy", "fp16")
-    for v in ([SPLIT] if T > 16 else [P.PIFA_VARIANT_DECODE, SPLIT]):
+    for v in ([SPLIT] if T > 64 else [P.PIFA_VARIANT_DECODE, SPLIT]):
         parity(L, T, v)
 
 
@@ -576,15 +583,15 @@ def grouped_parity(layers, T, sample=None, seed=0):
 
 
 @pytest.mark.parametrize("G", [2, 3])
-@pytest.mark.parametrize("T", [1, 3, 8, 16, 100, 300])
+@pytest.mark.parametrize("T", [1, 3, 8, 16, 40, 64, 100, 300])
 def test_grouped_layers_match_per_layer_oracle(G, T):
     """G synthetic layers of one shape (m - r = 7 x 128, ragged n) sharing X: each group's block of
-    Y equals the oracle's forward of that layer alone (decode for T <= 16, split prefill above)."""
+    Y equals the oracle's forward of that layer alone (decode for T <= 64, split prefill above)."""
     layers = [layer_for(1408, 1000, 512, 10 + g, "synthetic") for g in range(G)]
     grouped_parity(layers, T)
 
 
-@pytest.mark.parametrize("T", [2, 8, 16])
+@pytest.mark.parametrize("T", [2, 8, 16, 48])
 @pytest.mark.parametrize("grid", [P.PIFA_DECODE_GRID_PERSISTENT, P.PIFA_DECODE_GRID_WAVES,
                                   P.PIFA_DECODE_GRID_SPLITK])
 def test_grouped_layers_both_decode_grids(T, grid):
@@ -649,31 +656,35 @@ def test_grouped_layers_prefill_three_groups(T):
 # back-to-back calls in a CUDA graph (the chained kernels of one call overlap the next call's)
 # ---------------------------------------------------------------------------------------------
 @pytest.mark.parametrize("m,n,r,T", [(4096, 4096, 2048, 8), (8192, 8192, 4096, 1), (8192, 8192, 4096, 16),
-                                     (28672, 8192, 4096, 16), (4096, 4096, 2048, 300)])
+                                     (28672, 8192, 4096, 16), (4096, 4096, 2048, 40), (28672, 8192, 4096, 64),
+                                     (4096, 4096, 2048, 300)])
 def test_graph_replay_back_to_back_matches_single_calls(m, n, r, T):
     """64 calls captured in one CUDA graph and replayed, on four rotating (X, Y) pairs that share one
     workspace: every call's kernels launch while the previous call's still run (programmatic
     dependent launch), so a call that read the shared y_p planes or partial sums too early, or
     wrote them too late, would change some output. Each Y must equal, bit for bit, the same call
-    made alone. Covers the wave, split-K tensor-core and persistent decode forms and the prefill."""
+    made alone. Covers the wave, split-K tensor-core and persistent decode forms (the latter with
+    token tiles of 64 rows at T = 40 and 64) and the prefill."""
+    variant = P.PIFA_VARIANT_DECODE if T <= 64 else P.PIFA_VARIANT_PREFILL_SPLIT
     piv, nonp, Wp32, C32 = inputs.synthetic_layer(m, n, r, 40)
     L = Layer(piv, nonp, Wp32, C32, f"{m}x{n}r{r}/graph")
     Wp, C, pd, nd = L.dev()
     copies = 4
     Xs = [_pad_dev(acts(T, n, 50 + j)) for j in range(copies)]
     Ys = [torch.full((T, m), float("nan"), dtype=torch.bfloat16, device=DEV) for _ in range(copies)]
-    ws = torch.empty(P.pifa_workspace_size(T, m, n, r) + 512, dtype=torch.uint8, device=DEV)
+    ws = torch.empty(P.pifa_workspace_size(T, m, n, r, variant) + 512, dtype=torch.uint8, device=DEV)
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
     ref = []
     for j in range(copies):
         Yj = torch.empty((T, m), dtype=torch.bfloat16, device=DEV)
-        P.pifa_forward(Xs[j], Wp, C, pd, nd, Y=Yj, workspace_tensor=ws, stream=stream)
+        P.pifa_forward(Xs[j], Wp, C, pd, nd, Y=Yj, workspace_tensor=ws, stream=stream, variant=variant)
         stream.synchronize()
         ref.append(Yj)
 
     def step(i):
-        P.pifa_forward(Xs[i % copies], Wp, C, pd, nd, Y=Ys[i % copies], workspace_tensor=ws, stream=stream)
+        P.pifa_forward(Xs[i % copies], Wp, C, pd, nd, Y=Ys[i % copies], workspace_tensor=ws, stream=stream,
+                       variant=variant)
 
     with torch.cuda.stream(stream):
         for i in range(4):

@@ -75,7 +75,8 @@ def test_selector(lib):
     assert P.pifa_select_variant(1, 4096, 4096, 2048) == P.PIFA_VARIANT_DECODE
     assert P.pifa_select_variant(16, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE
     assert P.pifa_select_variant(2048, 4096, 4096, 2048) == P.PIFA_VARIANT_PREFILL_SPLIT
-    assert P.pifa_select_variant(17, 256, 256, 128) == P.PIFA_VARIANT_PREFILL_SPLIT
+    assert P.pifa_select_variant(64, 256, 256, 128) == P.PIFA_VARIANT_DECODE
+    assert P.pifa_select_variant(65, 256, 256, 128) == P.PIFA_VARIANT_PREFILL_SPLIT
     assert P.pifa_select_variant(4096, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == P.PIFA_VARIANT_PREFILL_SPLIT
     with pytest.raises(P.PifaError):
         P.pifa_select_variant(1, 100, 50, 60)      # r > n
@@ -138,7 +139,7 @@ def test_forward_argument_errors(lib):
     assert "overlap" in _last(lib)
     assert _fwd_raw(lib, variant=9) == E.PIFA_ERR_INVALID_ARG
     assert _fwd_raw(lib, cdt=7) == E.PIFA_ERR_INVALID_ARG
-    assert _fwd_raw(lib, variant=P.PIFA_VARIANT_DECODE, T=17) == E.PIFA_ERR_UNSUPPORTED
+    assert _fwd_raw(lib, variant=P.PIFA_VARIANT_DECODE, T=65) == E.PIFA_ERR_UNSUPPORTED
     assert _fwd_raw(lib, wsb=16) == E.PIFA_ERR_WORKSPACE
     assert _fwd_raw(lib, ws=None) == E.PIFA_ERR_WORKSPACE
     assert _fwd_raw(lib, ws=0x70010) == E.PIFA_ERR_ALIGNMENT
