@@ -361,10 +361,11 @@ int pifa_set_wait_timeout(int64_t ns);
  * calls made after this one (process-wide). Three forms compute a phase (R weight rows, K
  * columns): waves of one-tile clusters, every CTA staging its weight rows at launch; a persistent
  * grid of co-resident clusters that stream their tiles through a ring of TMA-filled stages; and
- * split-K on the tensor cores, where equal ranges of 128 x 64 weight tiles go to a persistent grid
- * and a second kernel sums the fp32 partial sums in a fixed order (a phase 2 whose 128-row blocks
- * number between one and two per SM instead gives each CTA one row block over all of K and needs
- * no second kernel).
+ * split-K on the tensor cores. The latter gives a phase of at most two 128-row blocks per SM 1, 2,
+ * 4 or 8 CTAs per row block, each one K-slice of it, as a thread-block cluster that adds up its
+ * slices in shared memory in rank order and writes the outputs itself (one kernel); a taller
+ * phase deals equal ranges of 128 x 64 weight tiles to a persistent grid and a second kernel sums
+ * the fp32 partial sums in a fixed order.
  * PIFA_DECODE_GRID_AUTO (0, the default) picks per phase from its shape and T: split-K when
  * T > 2 and R >= 4096, else waves while the phase takes at most two of them, else the persistent
  * grid. PIFA_DECODE_GRID_WAVES (1), PIFA_DECODE_GRID_PERSISTENT (2) and PIFA_DECODE_GRID_SPLITK

@@ -24,12 +24,16 @@
 //   warps 2-5  sum a segment's accumulators (TMEM lane quarter each) while the next segment fills
 //              the other set, and store its partial sums P[s][t][row] (fp32, coalesced over rows).
 // A unit's head CTA writes zeros to P2 when it holds the whole unit, so P2 is defined everywhere.
-// A phase without y_p planes to write and with between one and two 128-row blocks per SM runs the
-// whole-row plan instead: one CTA per row block over all of K, the epilogue writing Y itself, no
-// partial sums and no reduce kernel.
 // Reduce kernel: Y[t, cols[j]] = bf16(sum_s (P[s][t][j] + P2[s][t][j])) in slice order
 // (deterministic for a given grid); phase 1 also writes y_p as the hi + lo planes of C's dtype
 // that phase 2 reads.
+// Row-block plan, for every phase of at most two 128-row blocks per SM (all layers of LLaMA-2 7B
+// and 70B): each row block gets cs CTAs (1, 2, 4 or 8), CTA k taking the block's K-slice k. With
+// cs = 1 the epilogue's sums are the outputs. With cs > 1 the block's CTAs form a thread-block
+// cluster: each stores its slice's sums in its own shared memory (the stage ring, free once its
+// MMAs are done), and after a cluster barrier CTA k reads rows [k 128 / cs, (k + 1) 128 / cs) of
+// every peer's sums through distributed shared memory, adds them in rank order and writes Y and
+// y_p's planes. One kernel per phase: no partial sums in global memory and no reduce kernel.
 // Every wait is bounded (globaltimer); on timeout the CTA latches PIFA_ERR_TIMEOUT, drains what
 // it has in flight and returns.
 #include <cuda_bf16.h>
@@ -68,6 +72,7 @@ constexpr size_t SMEM_PER_CTA = 112 * 1024;
 // bytes of every smaller grid (a smaller grid gives longer ranges, wider slices, fewer of them).
 constexpr int GRID_MAX = 512;
 constexpr int MIN_CHUNKS_PER_CTA = 4;
+constexpr int MAX_CLUSTER_TC = 8;  // CTAs per row block in the row-block plan (portable cluster size)
 
 // How one phase is cut: slice width, slice count and grid.
 struct Plan {
@@ -96,6 +101,20 @@ Plan make_plan_fixed(int64_t R, int64_t K, int grid) {
   return p;
 }
 
+// The row-block plan: cs CTAs per 128-row block, CTA k of a block taking K-slice k (ncf chunks, the
+// last slice nclast; slices beyond ns are empty).
+Plan make_plan_rows(int64_t R, int64_t K, int cs) {
+  Plan p;
+  p.nrb = (int)((R + TM - 1) / TM);
+  p.nck = (int)((K + KB - 1) / KB);
+  p.total = (int64_t)p.nrb * p.nck;
+  p.grid = p.nrb * cs;
+  p.ncf = (p.nck + cs - 1) / cs;
+  p.ns = (p.nck + p.ncf - 1) / p.ncf;
+  p.nclast = p.nck - (p.ns - 1) * p.ncf;
+  return p;
+}
+
 // The grid for one phase: at most grid_cap CTAs, each with at least MIN_CHUNKS_PER_CTA chunks.
 Plan make_plan(int64_t R, int64_t K, int grid_cap) {
   const int64_t total = ((R + TM - 1) / TM) * ((K + KB - 1) / KB);
@@ -116,12 +135,18 @@ struct TcArgs {
   uint32_t idesc;
   float* P;   // partial sums of unit heads [ns][T][R]
   float* P2;  // partial sums of the tails of split units [ns][T][R]
-  // whole-row plan (ns = 1, one unit per CTA): the epilogue writes Y[t, cols[row]] itself
-  int direct;
+  // row-block plan (cs >= 1): CTA b takes slice b % cs of row block b / cs, one unit or none; the
+  // cs CTAs of a row block form a cluster and sum their slices in shared memory (cs = 1: the CTA
+  // holds the whole row block). 0: the balanced split-K plan with partial sums P, P2.
+  int cs;
   const int32_t* cols;
   int m;  // columns of Y (index bound)
   bf16* Y;
   int64_t ldy;
+  uint16_t* yph;  // row-block plan, phase 1 with m > r: y_p hi and lo planes, else null
+  uint16_t* ypl;
+  int64_t ldyp;
+  int split_f16;  // the planes in fp16 (else bf16)
   int* status;
   uint64_t timeout_ns;
 };
@@ -153,10 +178,31 @@ __device__ __forceinline__ Seg seg_at(const TcArgs& a, int64_t g, int64_t e) {
   return seg_at(a.nrb, a.ns, a.ncf, a.nclast, g, e);
 }
 
+// hi + lo split of an fp32 value in bf16 (kF16 = false) or fp16 (kF16 = true); fp16 saturates at
+// +-65504 and reports the overflow.
+template <bool kF16>
+__device__ __forceinline__ void split_hi_lo(float f, uint16_t& h, uint16_t& l, bool& range_err) {
+  if (kF16) {
+    if (fabsf(f) > 65504.0f) {
+      range_err = true;
+      f = copysignf(65504.0f, f);
+    }
+    const __half bh = __float2half_rn(f);
+    h = __half_as_ushort(bh);
+    l = __half_as_ushort(__float2half_rn(f - __half2float(bh)));
+  } else {
+    const bf16 bh = __float2bfloat16_rn(f);
+    h = __bfloat16_as_ushort(bh);
+    l = __bfloat16_as_ushort(__float2bfloat16_rn(f - __bfloat162float(bh)));
+  }
+}
+
 // Column (within the unit's K-slice) of the c-th chunk a CTA loads for segment q.
 __device__ __forceinline__ int seg_col(const Seg& q, int c) { return (q.c0 + c) * KB; }
 
-template <int NB, int TNT>
+// kCl: the row-block plan with cs > 1 (a cluster per row block); only these instantiations hold
+// cluster barriers and distributed shared-memory loads.
+template <int NB, int TNT, bool kCl>
 __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
     decode_tc_partial(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                       const __grid_constant__ CUtensorMap tmB1, TcArgs a) {
@@ -172,8 +218,16 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
 
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t g0 = ((int64_t)blockIdx.x * a.total) / a.grid;
-  const int64_t g1 = ((int64_t)(blockIdx.x + 1) * a.total) / a.grid;
+  int64_t g0, g1;
+  if (a.cs > 0) {  // slice k of row block rb: the unit that starts at chunk k nrb ncf + rb len(k)
+    const int rb = (int)blockIdx.x / a.cs, k = (int)blockIdx.x % a.cs;
+    const int len = k < a.ns - 1 ? a.ncf : a.nclast;
+    g0 = k < a.ns ? (int64_t)k * a.nrb * a.ncf + (int64_t)rb * len : 0;
+    g1 = k < a.ns ? g0 + len : 0;
+  } else {
+    g0 = ((int64_t)blockIdx.x * a.total) / a.grid;
+    g1 = ((int64_t)(blockIdx.x + 1) * a.total) / a.grid;
+  }
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < a.stages; ++s) {
@@ -348,8 +402,31 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
       if (lane == 0) mbar_arrive(&acce[acc]);  // this quarter of the accumulators may be refilled
       // the head of a unit goes to P and, when the unit was not split, zeros to P2; a tail to P2
       const int row = q.rb * TM + q4 * 32 + lane;
-      if (a.direct) {  // the unit is the row block over all of K: its sums are the outputs
+      if (kCl) {  // this slice's sums, [t][row of the block], for the cluster to add up
+        fence_proxy_async_smem();  // the ring's last operands were read by the MMAs (async proxy)
+        float* red = reinterpret_cast<float*>(ring);
+#pragma unroll
+        for (int t = 0; t < TNT; ++t)
+          if (t < a.T) red[t * TM + q4 * 32 + lane] = sum[t];
+        continue;
+      }
+      if (a.cs == 1) {  // the unit is the row block over all of K: its sums are the outputs
         if (row < a.R) {
+          bool range_err = false;
+          if (a.yph) {
+#pragma unroll
+            for (int t = 0; t < TNT; ++t)
+              if (t < a.T) {
+                uint16_t hi, lo;
+                if (a.split_f16)
+                  split_hi_lo<true>(sum[t], hi, lo, range_err);
+                else
+                  split_hi_lo<false>(sum[t], hi, lo, range_err);
+                a.yph[(int64_t)t * a.ldyp + row] = hi;
+                a.ypl[(int64_t)t * a.ldyp + row] = lo;
+              }
+          }
+          if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
           const int col = __ldg(a.cols + row);
           if ((unsigned)col >= (unsigned)a.m) {
             latch_status(a.status, PIFA_ERR_DEVICE_INDEX);
@@ -381,24 +458,41 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
   }
-}
-
-// hi + lo split of an fp32 value in bf16 (kF16 = false) or fp16 (kF16 = true); fp16 saturates at
-// +-65504 and reports the overflow.
-template <bool kF16>
-__device__ __forceinline__ void split_hi_lo(float f, uint16_t& h, uint16_t& l, bool& range_err) {
-  if (kF16) {
-    if (fabsf(f) > 65504.0f) {
-      range_err = true;
-      f = copysignf(65504.0f, f);
+  if (kCl) {
+    // Every CTA of the cluster has its slice's sums in its own shared memory once all arrive;
+    // CTA k then finishes rows [k rpr, (k + 1) rpr) of the block, adding the slices in rank
+    // order (deterministic). Every wait above is bounded, so each CTA reaches both barriers; the
+    // second keeps each CTA resident until no peer reads its shared memory any more.
+    cluster_sync_all();
+    const int k = (int)blockIdx.x % a.cs, rb = (int)blockIdx.x / a.cs;
+    const int rpr = TM / a.cs;
+    const int nsrc = a.ns < a.cs ? a.ns : a.cs;
+    const uint32_t red = smem_u32(ring);
+    bool range_err = false;
+    for (int idx = threadIdx.x; idx < rpr * a.T; idx += THREADS) {
+      const int t = idx / rpr, rr = k * rpr + idx % rpr;
+      const int row = rb * TM + rr;
+      const uint32_t off = red + (uint32_t)(t * TM + rr) * 4u;
+      float sum = 0.0f;
+      for (int p = 0; p < nsrc; ++p) sum += ld_dsmem_f32(mapa_shared(off, (uint32_t)p));
+      if (row >= a.R) continue;
+      if (a.yph) {
+        uint16_t hi, lo;
+        if (a.split_f16)
+          split_hi_lo<true>(sum, hi, lo, range_err);
+        else
+          split_hi_lo<false>(sum, hi, lo, range_err);
+        a.yph[(int64_t)t * a.ldyp + row] = hi;
+        a.ypl[(int64_t)t * a.ldyp + row] = lo;
+      }
+      const int col = __ldg(a.cols + row);
+      if ((unsigned)col >= (unsigned)a.m)
+        latch_status(a.status, PIFA_ERR_DEVICE_INDEX);
+      else
+        a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(sum);
     }
-    const __half bh = __float2half_rn(f);
-    h = __half_as_ushort(bh);
-    l = __half_as_ushort(__float2half_rn(f - __half2float(bh)));
-  } else {
-    const bf16 bh = __float2bfloat16_rn(f);
-    h = __bfloat16_as_ushort(bh);
-    l = __bfloat16_as_ushort(__float2bfloat16_rn(f - __bfloat162float(bh)));
+    if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
+    cluster_sync_all();
   }
 }
 
@@ -486,13 +580,20 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
     return pifa_fail(PIFA_ERR_INVALID_ARG, "decode_tc: empty or oversized phase");
   // token tile (MMA N per plane): 16, 32 or 64 rows of B, those beyond T zero-filled by TMA
   const int TNT = ph.T <= 16 ? 16 : ph.T <= 32 ? 32 : 64;
-  // Whole-row plan: when a phase without y_p planes to write has between one and two 128-row blocks
-  // per SM, each CTA takes one row block over all of K. No partial sums and no reduce kernel: one
-  // kernel and one kernel boundary fewer per phase (measured on the 70B gate/up layer, whose phase 2
-  // has 192 row blocks: T = 16 57.1 -> 53.0 us per call, T = 8 54.3 -> 51.5 us).
-  const int64_t nrb_all = (ph.R + TM - 1) / TM;
-  const bool direct = ph.yph == nullptr && nrb_all >= sm_count_tc() && nrb_all <= grid_cap();
-  Plan p = direct ? make_plan_fixed(ph.R, ph.K, (int)nrb_all) : make_plan(ph.R, ph.K, grid_cap());
+  // Row-block plan: a phase of at most grid_cap() 128-row blocks gives each block cs CTAs (cs the
+  // largest power of two up to 8 that keeps the grid within grid_cap() and every slice at least one
+  // chunk), CTA k taking K-slice k; the block's cs CTAs form a cluster that adds up its slices in
+  // shared memory and writes Y (and y_p's planes) itself. No partial sums in global memory and no
+  // reduce kernel: one kernel and one kernel boundary fewer per phase (measured on the 70B gate/up
+  // layer, whose phase 2 has 192 row blocks and takes cs = 1: T = 16 57.1 -> 53.0 us per call, T = 8
+  // 54.3 -> 51.5 us). Longer phases deal balanced chunk ranges and sum P + P2 in a second kernel.
+  const int64_t nrb_all = (ph.R + TM - 1) / TM, nck_all = (ph.K + KB - 1) / KB;
+  int cs = 0;
+  if (nrb_all <= grid_cap()) {
+    cs = 1;
+    while (cs < MAX_CLUSTER_TC && nrb_all * cs * 2 <= grid_cap() && cs * 2 <= nck_all) cs *= 2;
+  }
+  const Plan p = cs > 0 ? make_plan_rows(ph.R, ph.K, cs) : make_plan(ph.R, ph.K, grid_cap());
   TcArgs a = {};
   a.R = (int)ph.R;
   a.K = (int)ph.K;
@@ -510,17 +611,24 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   a.idesc = f16 ? idesc_f16_f32(TM, (uint32_t)(TNT * NB)) : idesc_bf16_f32(TM, (uint32_t)(TNT * NB));
   a.P = ph.P;
   a.P2 = ph.P + (size_t)p.ns * ph.T * ph.R;
-  a.direct = direct ? 1 : 0;
+  a.cs = cs;
   a.cols = ph.cols;
   a.m = (int)ph.m;
   a.Y = reinterpret_cast<bf16*>(ph.Y);
   a.ldy = ph.ldy;
+  a.yph = ph.yph;
+  a.ypl = ph.ypl;
+  a.ldyp = ph.ldyp;
+  a.split_f16 = ph.split_f16 ? 1 : 0;
   a.status = status;
   a.timeout_ns = timeout_ns;
   const size_t fixed = 1024 + 512;  // alignment slack; barriers and the TMEM slot
   const int stages = (int)((SMEM_PER_CTA - fixed) / a.stage_bytes);
   a.stages = stages > MAX_STAGES ? MAX_STAGES : stages;
   const size_t smem = fixed + (size_t)a.stages * a.stage_bytes;
+  // the row-block plan's cluster sums ([T][128] fp32) reuse the ring once its MMAs are done
+  if (cs > 1 && (size_t)TM * TNT * 4 > (size_t)a.stages * a.stage_bytes)
+    return pifa_fail(PIFA_ERR_UNSUPPORTED, "decode_tc: ring smaller than the cluster sums");
 
   CUtensorMap tA, tB0, tB1;
   int st;
@@ -530,8 +638,15 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
     return st;
   if (NB == 1) tB1 = tB0;
 
-  auto kern = NB == 1 ? (TNT == 16 ? decode_tc_partial<1, 16> : TNT == 32 ? decode_tc_partial<1, 32> : decode_tc_partial<1, 64>)
-                      : (TNT == 16 ? decode_tc_partial<2, 16> : TNT == 32 ? decode_tc_partial<2, 32> : decode_tc_partial<2, 64>);
+  using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, TcArgs);
+  static const Kern kerns[2][3][2] = {
+      {{decode_tc_partial<1, 16, false>, decode_tc_partial<1, 16, true>},
+       {decode_tc_partial<1, 32, false>, decode_tc_partial<1, 32, true>},
+       {decode_tc_partial<1, 64, false>, decode_tc_partial<1, 64, true>}},
+      {{decode_tc_partial<2, 16, false>, decode_tc_partial<2, 16, true>},
+       {decode_tc_partial<2, 32, false>, decode_tc_partial<2, 32, true>},
+       {decode_tc_partial<2, 64, false>, decode_tc_partial<2, 64, true>}}};
+  const Kern kern = kerns[NB - 1][TNT == 16 ? 0 : TNT == 32 ? 1 : 2][cs > 1 ? 1 : 0];
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(decode_tc)", e);
   cudaLaunchConfig_t cfg = {};
@@ -539,14 +654,18 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   cfg.blockDim = dim3(THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr;
-  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr.val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = &attr;
-  cfg.numAttrs = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)(cs > 1 ? cs : 1);
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cs > 1 ? 2 : 1;
   e = pifa_launch_ex(&cfg, kern, tA, tB0, tB1, a);
   if (e != cudaSuccess) return pifa_fail_cuda("decode_tc partial launch", e);
-  if (direct) return PIFA_OK;
+  if (cs > 0) return PIFA_OK;
 
   ReduceArgs r = {};
   r.P = a.P;
@@ -567,6 +686,7 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   rc.gridDim = dim3((unsigned)((n + 255) / 256));
   rc.blockDim = dim3(256);
   rc.dynamicSmemBytes = 0;
+  rc.numAttrs = 1;  // programmatic serialization only, no cluster
   void (*red)(ReduceArgs);
   if (a.ns <= 2)
     red = ph.split_f16 ? decode_tc_reduce<true, 2> : decode_tc_reduce<false, 2>;

@@ -138,6 +138,12 @@ __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wai
 __device__ __forceinline__ void st_dsmem_f32(uint32_t cluster_saddr, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(cluster_saddr), "f"(v) : "memory");
 }
+// 32-bit load from the shared memory of a CTA of this cluster (shared::cluster address).
+__device__ __forceinline__ float ld_dsmem_f32(uint32_t cluster_saddr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(cluster_saddr) : "memory");
+  return v;
+}
 // 128-bit load from this CTA's shared memory at a 32-bit shared-window address.
 __device__ __forceinline__ uint4 lds128(uint32_t saddr) {
   uint4 v;
@@ -168,6 +174,11 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity
     if ((++spins & 15u) == 0 && globaltimer_ns() - t0 > limit_ns) return false;
   }
   return true;
+}
+// Order shared-memory accesses of the async proxy (TMA writes, tcgen05 operand reads) that this
+// thread has observed complete before its later generic-proxy accesses of the same bytes.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 // Order this thread's generic-proxy global writes before later async-proxy (TMA) accesses.
 __device__ __forceinline__ void fence_proxy_async_global() {

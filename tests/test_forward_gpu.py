@@ -334,11 +334,14 @@ def test_decode_selector_matches_the_form_it_picks(m, n, r, T, forced):
 
 
 def test_launch_count_per_call():
-    """pifa_launch_count: a split-K decode call (both phases of 4096 rows, T = 8) enqueues four
-    kernels (a partial and a reduce kernel per phase), a waves decode call on 2048-row phases two;
-    replaying a captured call launches nothing through the library."""
+    """pifa_launch_count: a split-K decode call whose phases take the row-block plan (both phases
+    of 4096 rows, T = 8: clusters of 8 CTAs that add up their K-slices themselves) enqueues two
+    kernels, one whose phase 2 has more 128-row blocks than the grid holds (39736 rows) three (a
+    partial and a reduce kernel for it), a waves decode call on 2048-row phases two; replaying a
+    captured call launches nothing through the library."""
     big, small = layer_for(8192, 4096, 4096, 6, "synthetic"), layer_for(4096, 4096, 2048, 6, "synthetic")
-    for L, n_k in ((big, 4), (small, 2)):
+    long_ = layer_for(40000, 520, 264, 3, "synthetic")
+    for L, n_k in ((big, 2), (small, 2), (long_, 3)):
         X = acts(8, L.n, 6)
         run(L, X, P.PIFA_VARIANT_DECODE)  # first call: per-shape setup out of the way
         c0 = P.pifa_launch_count()

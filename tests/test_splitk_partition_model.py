@@ -94,22 +94,79 @@ def test_headline_cut():
     assert (p2["grid"], p2["ncf"], p2["ns"], p2["nclast"]) == (304, 40, 2, 24)
 
 
-def make_plan_fixed(R, K, grid):
+def pick_cs(nrb, nck, cap):
+    """CTAs per row block in the row-block plan (0: the balanced plan with a reduce kernel); cap is
+    the CTA slots (two per SM)."""
+    if nrb > cap:
+        return 0
+    cs = 1
+    while cs < 8 and nrb * cs * 2 <= cap and cs * 2 <= nck:
+        cs *= 2
+    return cs
+
+
+def make_plan_rows(R, K, cs):
     nrb, nck = -(-R // TM), -(-K // KB)
-    total = nrb * nck
-    u = max(1, min(total // grid, nck))
-    ns = -(-nck // u)
-    return dict(nrb=nrb, nck=nck, total=total, grid=grid, ncf=u, ns=ns, nclast=nck - (ns - 1) * u)
+    ncf = -(-nck // cs)
+    ns = -(-nck // ncf)
+    return dict(nrb=nrb, nck=nck, total=nrb * nck, grid=nrb * cs, ncf=ncf, ns=ns, nclast=nck - (ns - 1) * ncf)
 
 
-@pytest.mark.parametrize("R,K", [(24576, 4096), (19456, 8192), (38912, 520), (24577, 4100), (152 * 128, 64)])
-def test_whole_row_plan_gives_each_cta_one_row_block(R, K):
-    """The whole-row plan (grid = the phase's 128-row blocks) cuts K into one slice, and every
-    CTA's range is exactly one unit: no unit is split, so the epilogue's sums are the outputs."""
-    nrb = -(-R // TM)
-    p = make_plan_fixed(R, K, nrb)
-    assert p["ns"] == 1 and p["ncf"] == p["nclast"] == p["nck"]
-    parts = walk(p)
-    assert len(parts) == nrb
-    for (s, rb), ps in parts.items():
-        assert ps == [(rb, 0, p["nck"])]
+ROW_SHAPES = [(4096, 8192), (24576, 4096), (2048, 4096), (2048, 11008), (8960, 2048), (8192, 4096),
+              (19456, 8192), (38912, 520), (24577, 4100), (152 * 128, 64), (1, 1), (129, 65), (300, 837),
+              (264, 520), (64, 128), (40, 1), (1400, 1000)]
+
+
+@pytest.mark.parametrize("R,K", ROW_SHAPES)
+@pytest.mark.parametrize("cap", [296, 304])
+def test_row_block_plan_gives_each_cta_one_slice_of_its_cluster_block(R, K, cap):
+    """The row-block plan: cs CTAs (a cluster) per 128-row block, cs a power of two up to 8 with the
+    grid within the cap and every slice non-empty; CTA b takes slice b % cs of block b / cs (or
+    nothing when the block has fewer slices), as the segment walk finds it from its (g0, g1). Every
+    chunk of every block is computed once, inside the block's own cluster, and the cluster's
+    row shares (128 / cs rows each) cover the block's 128 rows once."""
+    nrb, nck = -(-R // TM), -(-K // KB)
+    cs = pick_cs(nrb, nck, cap)
+    if cs == 0:  # more blocks than CTA slots: the balanced plan
+        assert nrb > cap
+        return
+    assert cs in (1, 2, 4, 8) and nrb * cs <= cap and cs <= nck
+    assert cs == 8 or nrb * cs * 2 > cap or cs * 2 > nck   # the largest such cs
+    p = make_plan_rows(R, K, cs)
+    assert (p["ns"] - 1) * p["ncf"] + p["nclast"] == nck and 1 <= p["nclast"] <= p["ncf"] and p["ns"] <= cs
+    seen = {}
+    for b in range(p["grid"]):
+        rb, k = divmod(b, cs)
+        if k >= p["ns"]:
+            continue
+        n = p["ncf"] if k < p["ns"] - 1 else p["nclast"]
+        g0 = k * nrb * p["ncf"] + rb * n
+        g1 = g0 + n
+        assert seg_at(p, g0, g1) == (k, rb, 0, n)
+        assert (k, rb) not in seen
+        seen[(k, rb)] = n
+    assert len(seen) == nrb * p["ns"]
+    for rb in range(nrb):
+        assert sum(seen[(k, rb)] for k in range(p["ns"])) == nck
+    rpr = TM // cs
+    assert sorted(r for k in range(cs) for r in range(k * rpr, (k + 1) * rpr)) == list(range(TM))
+
+
+def test_row_block_plan_on_the_llama_phases():
+    """On 152 SMs (304 CTA slots): 70B gate/up phase 1 (32 blocks) and both 70B q/o phases take
+    clusters of 8 (256 CTAs of 16 chunks), its phase 2 (192 blocks) one CTA per block, the 7B
+    phases of 16 blocks clusters of 8 (128 CTAs), the 7B gate's phase 2 (70 blocks) clusters of 4;
+    longer phases (more than 304 blocks) keep the balanced plan."""
+    assert pick_cs(32, 128, 304) == 8 and pick_cs(192, 64, 304) == 1 and pick_cs(32, 64, 304) == 8
+    assert pick_cs(16, 64, 304) == 8 and pick_cs(70, 32, 304) == 4 and pick_cs(311, 5, 304) == 0
+    p = make_plan_rows(4096, 8192, 8)
+    assert (p["grid"], p["ncf"], p["ns"], p["nclast"]) == (256, 16, 8, 16)
+
+
+@pytest.mark.parametrize("tnt", [16, 32, 64])
+@pytest.mark.parametrize("nb", [1, 2])
+def test_cluster_sums_fit_the_ring(tnt, nb):
+    """The cluster's [T][128] fp32 sums reuse the stage ring (112 KB per CTA less 1.5 KB)."""
+    stage = TM * KB * 2 + nb * tnt * KB * 2
+    stages = min(10, (112 * 1024 - 1536) // stage)
+    assert stages >= 2 and TM * tnt * 4 <= stages * stage
