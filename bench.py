@@ -59,10 +59,11 @@ T_DECODE = 16
 # measured with ncu, keyed by (layer, T), with the sha256 prefixes of the kernel sources it was
 # taken on. A source mismatch (a kernel changed since the capture) reports traffic as null.
 NCU_TRAFFIC = {
-    # profiles/decode_tc_gateup70b_T16_traffic.md: phase 1 split-K partial + reduce, phase 2 whole rows
+    # profiles/decode_tc_gateup70b_T16_traffic.md: phase 1 in clusters of 8 CTAs per row block,
+    # phase 2 one CTA per row block; two kernels, no partial sums in global memory
     ("llama2_70b_gate_up_28672x8192_r4096", 16): {
-        "sha": {"decode_tc.cu": "33c9277b7d351a3c", "decode.cu": "0d83c7d91223b49c"},
-        "bytes": 275081984,
+        "sha": {"decode_tc.cu": "1019e523e9e64c73", "decode.cu": "ae2f58c787dfe866"},
+        "bytes": 269476608,
     },
 }
 
