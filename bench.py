@@ -324,11 +324,12 @@ def layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src, name=None, c
     return out
 
 
-# the library's selector runs the decode variant up to this many tokens, the split prefill above
-DECODE_MAX_T = 64
-DECODE_POINTS = [(inputs.ATTN7B, (1, 8, 16, 64)), (inputs.MLP7B_GATE, (1, 8, 16, 64)),
-                 (inputs.MLP7B_DOWN, (1, 8, 16, 64)), (inputs.ATTN70B, (1, 8, 16, 64)),
-                 (inputs.MLP70B_GATE, (1, 8, 16, 32, 64))]
+# the library's selector runs the decode variant up to this many tokens on every single layer
+# measured here (T <= 128 needs each phase within 296 row blocks of 128), the split prefill above
+DECODE_MAX_T = 128
+DECODE_POINTS = [(inputs.ATTN7B, (1, 8, 16, 64, 128)), (inputs.MLP7B_GATE, (1, 8, 16, 64, 128)),
+                 (inputs.MLP7B_DOWN, (1, 8, 16, 64, 128)), (inputs.ATTN70B, (1, 8, 16, 64, 128)),
+                 (inputs.MLP70B_GATE, (1, 8, 16, 32, 64, 128))]
 PREFILL_POINTS = [(inputs.ATTN7B, 2048), (inputs.ATTN7B, 8192), (inputs.ATTN70B, 4096), (inputs.MLP70B_GATE, 4096)]
 
 

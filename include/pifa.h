@@ -56,7 +56,7 @@ typedef enum { PIFA_DTYPE_BF16 = 0, PIFA_DTYPE_FP16 = 1 } pifa_dtype;
  * the given shape returns PIFA_ERR_UNSUPPORTED. */
 typedef enum {
   PIFA_VARIANT_AUTO = 0,
-  PIFA_VARIANT_DECODE = 1,        /* T <= 64: two HBM-streaming phases (mma.sync or tcgen05)     */
+  PIFA_VARIANT_DECODE = 1,        /* T <= 128: two HBM-streaming phases (mma.sync or tcgen05)    */
   PIFA_VARIANT_PREFILL_SPLIT = 2, /* tcgen05 GEMM 1 -> Y_p in workspace -> tcgen05 GEMM 2        */
   PIFA_VARIANT_PREFILL_FUSED = 3  /* reserved: not built in this version (PIFA_ERR_UNSUPPORTED)   */
 } pifa_variant;
@@ -186,7 +186,9 @@ int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dt
 
 /* pifa_select_variant -- the selector (host, < 1 us): the pifa_variant pifa_forward runs for
  * (T, m, n, r, c_dtype) on this build, never PIFA_VARIANT_AUTO; negative pifa_status on bad
- * arguments. Decode for T <= 64, else the split prefill. */
+ * arguments. Decode for T <= 64, and for T <= 128 when both phases (r and m - r rows) have at
+ * most 296 blocks of 128 rows; else the split prefill. The forced decode variant takes the same
+ * shapes (PIFA_ERR_UNSUPPORTED otherwise). */
 int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype);
 
 /* pifa_variant_name -- static string naming a pifa_variant ("decode", ...); "?" if unknown. */
@@ -371,8 +373,8 @@ int pifa_set_wait_timeout(int64_t ns);
  * grid. PIFA_DECODE_GRID_WAVES (1), PIFA_DECODE_GRID_PERSISTENT (2) and PIFA_DECODE_GRID_SPLITK
  * (3) force one form for both phases (a tuning and test knob: all compute the same result up to
  * the summation order of fp32 partial sums; forced split-K runs the persistent grid instead when the
- * workspace is too small for its partial sums). For 16 < T <= 64 only the split-K form exists
- * (token tiles of 32 or 64 rows): both phases run it whatever the mode. PIFA_ERR_INVALID_ARG for
+ * workspace is too small for its partial sums). For 16 < T <= 128 only the split-K form exists
+ * (token tiles of 32, 64 or 128 rows): both phases run it whatever the mode. PIFA_ERR_INVALID_ARG for
  * other values. */
 #define PIFA_DECODE_GRID_AUTO 0
 #define PIFA_DECODE_GRID_WAVES 1

@@ -144,16 +144,38 @@ const char* pifa_variant_name(int variant) {
   }
 }
 
+}  // extern "C"
+
+namespace {
+
+// Whether the decode variant runs T tokens of G layers of this shape: any T <= 64; up to 128 when
+// both phases (G r and G (m - r) rows) have at most kWideRowBlocks blocks of 128 rows, the limit of
+// the row-block plan that 128-token tiles need on every sm_103a part (two CTAs on each of 148 SMs).
+constexpr int64_t kWideRowBlocks = 296;
+bool decode_takes(int64_t T, int64_t G, int64_t m, int64_t r) {
+  if (T <= 64) return true;
+  if (T > 128) return false;
+  return (G * r + 127) / 128 <= kWideRowBlocks && (G * (m - r) + 127) / 128 <= kWideRowBlocks;
+}
+
+// The selector: decode wherever it runs. Decode streams each weight once with every token's
+// product per tile; against the split prefill it measured 2.0-2.8x faster at T = 24 / 32 / 64 and
+// 1.2-2.3x at T = 80 / 96 / 128 on the LLaMA-2 7B and 70B layers (70B gate/up T = 128: 83.6 us
+// against 145.0 us), whose prefill grids hold one token tile at such T, too few tiles to fill the
+// GPU.
+int select_for(int64_t T, int64_t G, int64_t m, int64_t r) {
+  return decode_takes(T, G, m, r) ? PIFA_VARIANT_DECODE : PIFA_VARIANT_PREFILL_SPLIT;
+}
+
+}  // namespace
+
+extern "C" {
+
 int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype) {
   int st = validate_shape(T, m, n, r);
   if (st != PIFA_OK) return st;
   if (c_dtype != PIFA_DTYPE_BF16 && c_dtype != PIFA_DTYPE_FP16) return pifa_fail(PIFA_ERR_INVALID_ARG, "unknown c_dtype");
-  // Decode streams each weight once with every token's product per tile; measured against the
-  // split prefill at T = 24 / 32 / 64 it is 2.0 - 2.8x faster on the LLaMA-2 7B and 70B layers
-  // (70B gate/up 57 / 58 / 67 us against 138 / 139 / 141 us), whose prefill grids hold too few
-  // tiles at such T to fill the GPU.
-  if (T <= 64) return PIFA_VARIANT_DECODE;
-  return PIFA_VARIANT_PREFILL_SPLIT;
+  return select_for(T, 1, m, r);
 }
 
 int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype, int variant) {
@@ -225,11 +247,13 @@ int forward_impl(int64_t groups, const void* X, int64_t T, int64_t n, int64_t ld
         (has_np && overlaps(y, span_of(C, G * (m - r), r, ldc, 2))))
       return pifa_fail(PIFA_ERR_INVALID_ARG, "Y overlaps an input");
   }
-  if (variant == PIFA_VARIANT_AUTO) variant = pifa_select_variant(T, m, n, r, c_dtype);
+  if (variant == PIFA_VARIANT_AUTO) variant = select_for(T, G, m, r);
 
   PifaShape s = {T, m, n, r, ldx, ldwp, has_np ? ldc : r, ldy, c_dtype};
   s.groups = G;
-  if (variant == PIFA_VARIANT_DECODE && T > 64) return pifa_fail(PIFA_ERR_UNSUPPORTED, "decode variant needs T <= 64");
+  if (variant == PIFA_VARIANT_DECODE && !decode_takes(T, G, m, r))
+    return pifa_fail(PIFA_ERR_UNSUPPORTED,
+                     "decode variant needs T <= 64, or T <= 128 with at most 296 row blocks of 128 per phase");
   const int64_t need = workspace_bytes_for(s, variant);
   if (need < 0) return (int)need;
   if (!workspace || workspace_bytes < need)
@@ -285,7 +309,7 @@ int64_t pifa_workspace_size_grouped(int64_t groups, int64_t T, int64_t m, int64_
   if (T == 0) return 0;
   PifaShape s = {T, m, n, r, n, n, r, groups * m, c_dtype};
   s.groups = groups;
-  return workspace_bytes_for(s, pifa_select_variant(T, m, n, r, c_dtype));
+  return workspace_bytes_for(s, select_for(T, groups, m, r));
 }
 
 int pifa_forward(const void* X, int64_t T, int64_t n, int64_t ldx, const void* Wp, int64_t r, int64_t ldwp,

@@ -1,6 +1,6 @@
-// decode.cu -- PIFA forward for small token counts (T <= 64): Algorithm 2 as two HBM-streaming
+// decode.cu -- PIFA forward for small token counts (T <= 128): Algorithm 2 as two HBM-streaming
 // phases. Up to T = 16 each phase runs one of the forms below or the split-K tensor-core form of
-// decode_tc.cu; for 16 < T <= 64 both phases run the latter.
+// decode_tc.cu; for 16 < T <= 128 both phases run the latter.
 //
 //   phase 1: Y_p = X W_p^T  (the r rows of W_p, each read once)  -> Y[:, I[j]] = bf16(Y_p[:, j]),
 //            and y_p to the workspace as a hi + lo pair of C's dtype  (Algorithm 2, steps 2 and 4)

@@ -1,6 +1,6 @@
-// decode_tc.cu -- one decode phase (T <= 64 tokens) of Algorithm 2 on the 5th-generation tensor
+// decode_tc.cu -- one decode phase (T <= 128 tokens) of Algorithm 2 on the 5th-generation tensor
 // cores, split over K across a persistent grid: the form used for layers too large for one wave,
-// and the only decode form for 16 < T <= 64.
+// and the only decode form for 16 < T <= 128.
 //
 // A phase is a skinny product D = A B^T: A the weight rows (W_p for Y_p = X W_p^T, Algorithm 2
 // step 2; C for Y_np = Y_p C^T, step 3), B the T token rows (x, or y_p as its hi and lo planes).
@@ -13,14 +13,16 @@
 //
 // Partial kernel (two CTAs per SM, 192 threads each):
 //   warp 0     TMA producer: per chunk, the weight tile (128 rows x 64 columns, 128-byte swizzle)
-//              and the matching 64 columns of B (a token tile of TNT = 16, 32 or 64 rows per
+//              and the matching 64 columns of B (a token tile of TNT = 16, 32, 64 or 128 rows per
 //              plane, the smallest that holds T; rows >= T zero-filled)
 //              into one stage of a ring; the first weight tiles go out before the dependency wait
 //              (the weights do not depend on the previous kernel), their B boxes after it.
 //   warp 1     owns 256 TMEM columns (two segments in flight) and issues tcgen05.mma.kind::f16
 //              M = 128, K = 16, N = TNT (one B plane) or 2 TNT (the y_p hi and lo planes as one
 //              operand) from one thread, dealing a segment's MMAs round-robin over independent
-//              accumulators (128 / N of them) so that consecutive MMAs do not wait for each other.
+//              accumulators (128 / N of them, at least one) so that consecutive MMAs do not wait
+//              for each other. A 128-token tile's accumulator (N = 128 or 256) fills the 256
+//              columns alone, so it is used only where a CTA has one segment (the row-block plan).
 //   warps 2-5  sum a segment's accumulators (TMEM lane quarter each) while the next segment fills
 //              the other set, and store its partial sums P[s][t][row] (fp32, coalesced over rows).
 // A unit's head CTA writes zeros to P2 when it holds the whole unit, so P2 is defined everywhere.
@@ -50,7 +52,7 @@ using bf16 = __nv_bfloat16;
 
 constexpr int TM = 128;                         // weight rows per unit (MMA M = TMEM lanes)
 constexpr int TN = 16;                          // token rows of B, padded (MMA N), for T <= 16
-constexpr int kMaxTokensTc = 64;                // token tiles of 32 and 64 rows serve T <= 64
+constexpr int kMaxTokensTc = 128;               // token tiles of 32, 64 and 128 rows serve T <= 128
 constexpr int KB = 64;                          // K per chunk: one 128-byte swizzle row
 constexpr uint32_t A_BYTES = TM * KB * 2;       // one weight tile
 constexpr int MAX_STAGES = 10;
@@ -61,7 +63,7 @@ constexpr int THREADS = 192;
 // 2 TNT-row operand, and accumulator columns t and TNT + t are added in the epilogue. Per segment
 // NACC * TNT * NB = 128 columns; two segments in flight: 256 TMEM columns in every case.
 template <int NB, int TNT = TN>
-constexpr int kNacc = 128 / (TNT * NB);
+constexpr int kNacc = TNT * NB >= 128 ? 1 : 128 / (TNT * NB);
 constexpr uint32_t TMEM_COLS = 256;
 // Two CTAs per SM, each with its own producer and MMA-issuing thread: one issuing thread per SM
 // measured as the limit (70B gate/up, T = 16: 73 us with one CTA of ten stages, 60 us with two of
@@ -358,6 +360,57 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
         break;
       }
       tc_fence_after();
+      if constexpr (TNT > 64) {
+        // 128-token tiles (row-block plan only: one segment per CTA, one accumulator of TNT NB
+        // columns): tokens in groups of 16, the hi and lo columns 16 g and TNT + 16 g loaded,
+        // added and written out at once
+        const uint32_t base = tmem + ((uint32_t)(q4 * 32) << 16);
+        const int row = q.rb * TM + q4 * 32 + lane;
+        const bool in = row < a.R;
+        int col = -1;
+        if (!kCl && in) {
+          col = __ldg(a.cols + row);
+          if ((unsigned)col >= (unsigned)a.m) {
+            latch_status(a.status, PIFA_ERR_DEVICE_INDEX);
+            col = -1;
+          }
+        }
+        if (kCl) fence_proxy_async_smem();  // the ring's last operands were read by the MMAs
+        float* red = reinterpret_cast<float*>(ring);
+        bool range_err = false;
+        for (int g16 = 0; g16 < TNT / 16 && 16 * g16 < a.T; ++g16) {
+          uint32_t vh[16], vl[16];
+          tmem_ld_32x32b_x16(base + (uint32_t)(16 * g16), vh);
+          if (NB > 1) tmem_ld_32x32b_x16(base + (uint32_t)(TNT + 16 * g16), vl);
+          tmem_ld_wait();
+#pragma unroll
+          for (int u = 0; u < 16; ++u) {
+            const int t = 16 * g16 + u;
+            const float v = __uint_as_float(vh[u]) + (NB > 1 ? __uint_as_float(vl[u]) : 0.0f);
+            if (t >= a.T) continue;
+            if (kCl) {
+              red[t * TM + q4 * 32 + lane] = v;
+            } else if (in) {
+              if (a.yph) {
+                uint16_t hi, lo;
+                if (a.split_f16)
+                  split_hi_lo<true>(v, hi, lo, range_err);
+                else
+                  split_hi_lo<false>(v, hi, lo, range_err);
+                a.yph[(int64_t)t * a.ldyp + row] = hi;
+                a.ypl[(int64_t)t * a.ldyp + row] = lo;
+              }
+              if (col >= 0) a.Y[(int64_t)t * a.ldy + col] = __float2bfloat16_rn(v);
+            }
+          }
+        }
+        if (range_err) latch_status(a.status, PIFA_ERR_RANGE);
+        if (!kCl && a.cs != 1) latch_status(a.status, PIFA_ERR_UNSUPPORTED);  // host never launches this
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acce[acc]);
+        continue;
+      } else {
       // the accumulators this segment wrote (fewer than NACC only when it has fewer MMAs), summed
       // in a fixed order
       constexpr int NACC = kNacc<NB, TNT>;
@@ -449,6 +502,7 @@ __global__ void __launch_bounds__(THREADS, CTAS_PER_SM)
             if (whole) a.P2[off + (size_t)t * a.R] = 0.0f;
           }
       }
+      }  // TNT <= 64
     }
   }
 
@@ -578,8 +632,8 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   const int NB = ph.planes;
   if (ph.R < 1 || ph.K < 1 || ph.T < 1 || ph.T > kMaxTokensTc)
     return pifa_fail(PIFA_ERR_INVALID_ARG, "decode_tc: empty or oversized phase");
-  // token tile (MMA N per plane): 16, 32 or 64 rows of B, those beyond T zero-filled by TMA
-  const int TNT = ph.T <= 16 ? 16 : ph.T <= 32 ? 32 : 64;
+  // token tile (MMA N per plane): 16, 32, 64 or 128 rows of B, those beyond T zero-filled by TMA
+  const int TNT = ph.T <= 16 ? 16 : ph.T <= 32 ? 32 : ph.T <= 64 ? 64 : 128;
   // Row-block plan: a phase of at most grid_cap() 128-row blocks gives each block cs CTAs (cs the
   // largest power of two up to 8 that keeps the grid within grid_cap() and every slice at least one
   // chunk), CTA k taking K-slice k; the block's cs CTAs form a cluster that adds up its slices in
@@ -593,6 +647,10 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
     cs = 1;
     while (cs < MAX_CLUSTER_TC && nrb_all * cs * 2 <= grid_cap() && cs * 2 <= nck_all) cs *= 2;
   }
+  // a 128-token tile fills all of a CTA's 256 TMEM columns with one accumulator (hi and lo as one
+  // N = 256 operand), so only the row-block plan's one segment per CTA can use it
+  if (TNT > 64 && cs == 0)
+    return pifa_fail(PIFA_ERR_UNSUPPORTED, "decode with T > 64 needs phases of at most two row blocks per SM");
   const Plan p = cs > 0 ? make_plan_rows(ph.R, ph.K, cs) : make_plan(ph.R, ph.K, grid_cap());
   TcArgs a = {};
   a.R = (int)ph.R;
@@ -639,14 +697,16 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   if (NB == 1) tB1 = tB0;
 
   using Kern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, TcArgs);
-  static const Kern kerns[2][3][2] = {
+  static const Kern kerns[2][4][2] = {
       {{decode_tc_partial<1, 16, false>, decode_tc_partial<1, 16, true>},
        {decode_tc_partial<1, 32, false>, decode_tc_partial<1, 32, true>},
-       {decode_tc_partial<1, 64, false>, decode_tc_partial<1, 64, true>}},
+       {decode_tc_partial<1, 64, false>, decode_tc_partial<1, 64, true>},
+       {decode_tc_partial<1, 128, false>, decode_tc_partial<1, 128, true>}},
       {{decode_tc_partial<2, 16, false>, decode_tc_partial<2, 16, true>},
        {decode_tc_partial<2, 32, false>, decode_tc_partial<2, 32, true>},
-       {decode_tc_partial<2, 64, false>, decode_tc_partial<2, 64, true>}}};
-  const Kern kern = kerns[NB - 1][TNT == 16 ? 0 : TNT == 32 ? 1 : 2][cs > 1 ? 1 : 0];
+       {decode_tc_partial<2, 64, false>, decode_tc_partial<2, 64, true>},
+       {decode_tc_partial<2, 128, false>, decode_tc_partial<2, 128, true>}}};
+  const Kern kern = kerns[NB - 1][TNT == 16 ? 0 : TNT == 32 ? 1 : TNT == 64 ? 2 : 3][cs > 1 ? 1 : 0];
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(decode_tc)", e);
   cudaLaunchConfig_t cfg = {};

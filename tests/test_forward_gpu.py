@@ -215,7 +215,7 @@ def test_mlp7b_three_layers_back_to_back(T):
         check(Y[rows], ref, f"{L.name} T={T}")
 
 
-@pytest.mark.parametrize("T", [1, 8, 16, 4096])
+@pytest.mark.parametrize("T", [1, 8, 16, 80, 128, 4096])
 def test_llama70b_qo(T):
     L = layer_for(8192, 8192, 4096, 0, "library")
     parity(L, T, sample=256)
@@ -234,7 +234,7 @@ def test_llama70b_qo_persistent_grid(T):
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
-@pytest.mark.parametrize("T", [1, 8, 16, 4096])
+@pytest.mark.parametrize("T", [1, 8, 16, 80, 128, 4096])
 def test_llama70b_gate_up(T):
     """The 28672 x 8192, r = 4096 layer as Algorithm 1 makes it from Gaussian U V^T (compressed on
     the GPU): its C cancels heavily, the case that makes the hi + lo split of y_p necessary."""
@@ -269,13 +269,15 @@ def test_decode_persistent_grid_fp16_c_and_padding(T):
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
-@pytest.mark.parametrize("T", [1, 3, 8, 16, 17, 33, 64])
+@pytest.mark.parametrize("T", [1, 3, 8, 16, 17, 33, 64, 65, 128])
 def test_decode_splitk_tensor_cores_ragged(T):
     """The split-K tensor-core decode form forced on a layer with ragged K in both phases (520 and
     264 columns: partial 64-column chunks and K-slices), a partial last 128-row block in phase 1
-    (264 rows) and many units per CTA in phase 2 (39736 rows). T = 17 and 33 fill token tiles of
-    32 and 64 rows only partly; T = 64 fills its tile."""
-    L = layer_for(40000, 520, 264, 3, "synthetic")
+    (264 rows) and many units per CTA in phase 2 (39736 rows). T = 17, 33 and 65 fill token tiles
+    of 32, 64 and 128 rows only partly; T = 64 and 128 fill theirs. 128-token tiles need the
+    row-block plan (at most 296 blocks per phase), so above T = 64 the layer has 30000 rows (233
+    blocks in phase 2)."""
+    L = layer_for(40000, 520, 264, 3, "synthetic") if T <= 64 else layer_for(30000, 520, 264, 3, "synthetic")
     P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_SPLITK)
     try:
         parity(L, T, P.PIFA_VARIANT_DECODE)
@@ -283,7 +285,7 @@ def test_decode_splitk_tensor_cores_ragged(T):
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
 
-@pytest.mark.parametrize("T", [1, 8, 16, 32, 64])
+@pytest.mark.parametrize("T", [1, 8, 16, 32, 64, 96, 128])
 def test_decode_splitk_tensor_cores_compressed_layers(T):
     """The split-K form on compressed layers (C that cancels): 7B attention and the 70B gate/up
     layer, and C stored as fp16 (fp16 MMAs in phase 2, fp16 hi/lo planes) on padded pitches."""
@@ -309,6 +311,10 @@ def test_decode_splitk_deterministic_and_r_equals_m():
         assert np.array_equal(run(L, X, P.PIFA_VARIANT_DECODE), run(L, X, P.PIFA_VARIANT_DECODE))
         parity(layer_for(64, 128, 64, 4, "oracle_greedy"), 40, P.PIFA_VARIANT_DECODE)
         parity(layer_for(40, 48, 1, 5, "oracle_greedy"), 64, P.PIFA_VARIANT_DECODE)
+        X = acts(128, 4096, 5)
+        assert np.array_equal(run(L, X, P.PIFA_VARIANT_DECODE), run(L, X, P.PIFA_VARIANT_DECODE))
+        parity(layer_for(64, 128, 64, 4, "oracle_greedy"), 100, P.PIFA_VARIANT_DECODE)
+        parity(layer_for(40, 48, 1, 5, "oracle_greedy"), 128, P.PIFA_VARIANT_DECODE)
     finally:
         P.pifa_set_decode_grid(P.PIFA_DECODE_GRID_AUTO)
 
@@ -369,10 +375,10 @@ def test_launch_count_per_call():
 # ---------------------------------------------------------------------------------------------
 # edge cases
 # ---------------------------------------------------------------------------------------------
-@pytest.mark.parametrize("T", [1, 3, 13, 16, 17, 40, 64, 65, 100, 300])
+@pytest.mark.parametrize("T", [1, 3, 13, 16, 17, 40, 64, 65, 100, 128, 129, 300])
 def test_ragged_shapes_all_variants(T):
     L = layer_for(300, 200, 77, 3, "oracle_greedy")
-    variants = [P.PIFA_VARIANT_PREFILL_SPLIT] + ([P.PIFA_VARIANT_DECODE] if T <= 64 else [])
+    variants = [P.PIFA_VARIANT_PREFILL_SPLIT] + ([P.PIFA_VARIANT_DECODE] if T <= 128 else [])
     for v in variants:
         parity(L, T, v)
 
@@ -466,8 +472,9 @@ def test_selector_picks_split_prefill():
     assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(16, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
-    assert P.pifa_select_variant(64, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
-    assert P.pifa_select_variant(65, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT
+    assert P.pifa_select_variant(128, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
+    assert P.pifa_select_variant(129, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT
+    assert P.pifa_select_variant(100, 40000, 520, 264, P.PIFA_DTYPE_BF16) == SPLIT  # 311 row blocks
 
 
 @pytest.mark.parametrize("T,sample", [(2048, None), (8192, 512), (300, None), (17, None)])
@@ -493,10 +500,10 @@ def test_fp16_c_llama70b(T):
     parity(layer_for(28672, 8192, 4096, 0, "gpu", "fp16"), T, sample=128)
 
 
-@pytest.mark.parametrize("T", [1, 17, 40, 64, 100, 300, 513])
+@pytest.mark.parametrize("T", [1, 17, 40, 64, 100, 128, 300, 513])
 def test_fp16_c_ragged_split_and_decode(T):
     L = layer_for(300, 200, 77, 3, "oracle_greedy", "fp16")
-    for v in ([SPLIT] if T > 64 else [P.PIFA_VARIANT_DECODE, SPLIT]):
+    for v in ([SPLIT] if T > 128 else [P.PIFA_VARIANT_DECODE, SPLIT]):
         parity(L, T, v)
 
 
@@ -586,7 +593,7 @@ def grouped_parity(layers, T, sample=None, seed=0):
 
 
 @pytest.mark.parametrize("G", [2, 3])
-@pytest.mark.parametrize("T", [1, 3, 8, 16, 40, 64, 100, 300])
+@pytest.mark.parametrize("T", [1, 3, 8, 16, 40, 64, 100, 128, 300])
 def test_grouped_layers_match_per_layer_oracle(G, T):
     """G synthetic layers of one shape (m - r = 7 x 128, ragged n) sharing X: each group's block of
     Y equals the oracle's forward of that layer alone (decode for T <= 64, split prefill above)."""
@@ -660,15 +667,15 @@ def test_grouped_layers_prefill_three_groups(T):
 # ---------------------------------------------------------------------------------------------
 @pytest.mark.parametrize("m,n,r,T", [(4096, 4096, 2048, 8), (8192, 8192, 4096, 1), (8192, 8192, 4096, 16),
                                      (28672, 8192, 4096, 16), (4096, 4096, 2048, 40), (28672, 8192, 4096, 64),
-                                     (4096, 4096, 2048, 300)])
+                                     (8192, 8192, 4096, 128), (4096, 4096, 2048, 300)])
 def test_graph_replay_back_to_back_matches_single_calls(m, n, r, T):
     """64 calls captured in one CUDA graph and replayed, on four rotating (X, Y) pairs that share one
     workspace: every call's kernels launch while the previous call's still run (programmatic
     dependent launch), so a call that read the shared y_p planes or partial sums too early, or
     wrote them too late, would change some output. Each Y must equal, bit for bit, the same call
     made alone. Covers the wave, split-K tensor-core and persistent decode forms (the latter with
-    token tiles of 64 rows at T = 40 and 64) and the prefill."""
-    variant = P.PIFA_VARIANT_DECODE if T <= 64 else P.PIFA_VARIANT_PREFILL_SPLIT
+    token tiles of 64 and 128 rows at T = 40, 64 and 128) and the prefill."""
+    variant = P.PIFA_VARIANT_DECODE if T <= 128 else P.PIFA_VARIANT_PREFILL_SPLIT
     piv, nonp, Wp32, C32 = inputs.synthetic_layer(m, n, r, 40)
     L = Layer(piv, nonp, Wp32, C32, f"{m}x{n}r{r}/graph")
     Wp, C, pd, nd = L.dev()

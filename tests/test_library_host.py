@@ -76,7 +76,17 @@ def test_selector(lib):
     assert P.pifa_select_variant(16, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE
     assert P.pifa_select_variant(2048, 4096, 4096, 2048) == P.PIFA_VARIANT_PREFILL_SPLIT
     assert P.pifa_select_variant(64, 256, 256, 128) == P.PIFA_VARIANT_DECODE
-    assert P.pifa_select_variant(65, 256, 256, 128) == P.PIFA_VARIANT_PREFILL_SPLIT
+    assert P.pifa_select_variant(128, 256, 256, 128) == P.PIFA_VARIANT_DECODE
+    assert P.pifa_select_variant(129, 256, 256, 128) == P.PIFA_VARIANT_PREFILL_SPLIT
+    # 64 < T <= 128 decodes only when both phases have at most 296 row blocks of 128
+    assert P.pifa_select_variant(100, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE       # 32 and 192
+    assert P.pifa_select_variant(100, 40000, 520, 264) == P.PIFA_VARIANT_PREFILL_SPLIT  # 3 and 311
+    assert P.pifa_select_variant(64, 40000, 520, 264) == P.PIFA_VARIANT_DECODE
+    # grouped layers count their stacked rows: 70B gate + up (2 x 192 non-pivot blocks) prefill
+    ws_dec = P.pifa_workspace_size(100, 28672, 8192, 4096, P.PIFA_VARIANT_DECODE)
+    ws_pre = P.pifa_workspace_size(100, 28672, 8192, 4096, P.PIFA_VARIANT_PREFILL_SPLIT)
+    assert P.pifa_workspace_size(100, 28672, 8192, 4096) == ws_dec
+    assert ws_dec != ws_pre
     assert P.pifa_select_variant(4096, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == P.PIFA_VARIANT_PREFILL_SPLIT
     with pytest.raises(P.PifaError):
         P.pifa_select_variant(1, 100, 50, 60)      # r > n
@@ -139,7 +149,13 @@ def test_forward_argument_errors(lib):
     assert "overlap" in _last(lib)
     assert _fwd_raw(lib, variant=9) == E.PIFA_ERR_INVALID_ARG
     assert _fwd_raw(lib, cdt=7) == E.PIFA_ERR_INVALID_ARG
-    assert _fwd_raw(lib, variant=P.PIFA_VARIANT_DECODE, T=65) == E.PIFA_ERR_UNSUPPORTED
+    assert _fwd_raw(lib, variant=P.PIFA_VARIANT_DECODE, T=129) == E.PIFA_ERR_UNSUPPORTED
+    # 64 < T <= 128 only with at most 296 row blocks of 128 per phase (39984 non-pivot rows: 313)
+    tall = dict(X=0x10000000, Wp=0x20000000, C=0x30000000, Y=0x40000000, ws=0x50000000, m=40000, ldy=40000,
+                variant=P.PIFA_VARIANT_DECODE)
+    assert _fwd_raw(lib, T=100, **tall) == E.PIFA_ERR_UNSUPPORTED
+    assert "row blocks" in _last(lib)
+    assert _fwd_raw(lib, T=64, wsb=0, **tall) == E.PIFA_ERR_WORKSPACE   # T <= 64 passes that rule
     assert _fwd_raw(lib, wsb=16) == E.PIFA_ERR_WORKSPACE
     assert _fwd_raw(lib, ws=None) == E.PIFA_ERR_WORKSPACE
     assert _fwd_raw(lib, ws=0x70010) == E.PIFA_ERR_ALIGNMENT
