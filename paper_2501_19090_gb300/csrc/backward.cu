@@ -205,11 +205,18 @@ extern "C" int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx, c
                     (void*)&dYnp, (void*)&ldnp, (void*)&status};
     if ((st = launch_small((const void*)gather_cols, args, T, m - r, s, "backward: gather")) != PIFA_OK) return st;
   }
+  // Independent products run concurrently: Y_p and then dC on side stream 0 (after the gather),
+  // dY_p and then dX on the caller's stream, dW_p on side stream 1 once dY_p is done. Each product
+  // alone fills one or two waves of the GPU; together they keep it busy (the side streams rejoin
+  // the caller's stream before this call returns, also on failure).
+  PifaSides sides(s);
+  cudaStream_t s_yp = s, s_dw = s;
   // Y_p = X W_p^T as hi + lo planes (only dC needs it)
   if (dC && has_np) {
+    if ((st = sides.fork(0, &s_yp)) != PIFA_OK) return st;
     GemmTc g = {T, r, n, X, ldx, false, Wp, ldwp, false, Yp, ldr, 3, 1.0f, nullptr, nullptr, 0, 0};
     g.D2 = Yp_lo;
-    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+    if ((st = gemm_tc(g, status, tmo, s_yp)) != PIFA_OK) return st;
   }
   // dY_p = dY[:, I] + dY_np C, as hi + lo planes
   if (has_np) {
@@ -222,20 +229,21 @@ extern "C" int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx, c
                     (void*)&dYp, (void*)&ldr, (void*)&status};
     if ((st = launch_small((const void*)gather_cols, args, T, r, s, "backward: gather")) != PIFA_OK) return st;
   }
+  if (dWp) {  // dW_p = (dY_p,hi + dY_p,lo)^T X
+    if ((st = sides.fork(1, &s_dw)) != PIFA_OK) return st;
+    GemmTc g = {r, n, T, dYp, ldr, true, X, ldx, true, dWp, lddwp, 1, 1.0f, nullptr, nullptr, 0, 0};
+    if (has_np) g.A2 = dYp_lo;
+    if ((st = gemm_tc(g, status, tmo, s_dw)) != PIFA_OK) return st;
+  }
   if (dX) {  // dX = (dY_p,hi + dY_p,lo) W_p  (dY_p exact in bf16 when r == m)
     GemmTc g = {T, n, r, dYp, ldr, false, Wp, ldwp, true, dX, lddx, 0, 1.0f, nullptr, nullptr, 0, 0};
     if (has_np) g.A2 = dYp_lo;
     if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
   }
-  if (dWp) {  // dW_p = (dY_p,hi + dY_p,lo)^T X
-    GemmTc g = {r, n, T, dYp, ldr, true, X, ldx, true, dWp, lddwp, 1, 1.0f, nullptr, nullptr, 0, 0};
-    if (has_np) g.A2 = dYp_lo;
-    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
-  }
-  if (dC && has_np) {  // dC = dY_np^T (Y_p,hi + Y_p,lo)
+  if (dC && has_np) {  // dC = dY_np^T (Y_p,hi + Y_p,lo), after Y_p on its side stream
     GemmTc g = {m - r, r, T, dYnp, ldnp, true, Yp, ldr, true, dC, lddc, 1, 1.0f, nullptr, nullptr, 0, 0};
     g.B2 = Yp_lo;
-    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
+    if ((st = gemm_tc(g, status, tmo, s_yp)) != PIFA_OK) return st;
   }
   return PIFA_OK;
 }
@@ -288,32 +296,38 @@ extern "C" int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int6
                                              (int)n, XuT, ldT);
     if (e != cudaSuccess) return pifa_fail_cuda("m_accumulate: transpose", e);
   }
+  // X X^T on the caller's stream and, concurrently, the mix, Y_t^T and Y_t X^T on a side stream
+  // (both read X_u^T; the side stream rejoins before this call returns, also on failure)
+  PifaSides sides(s);
+  if (YtXt) {
+    cudaStream_t s2 = s;
+    if ((st = sides.fork(0, &s2)) != PIFA_OK) return st;
+    bf16* Xmix = reinterpret_cast<bf16*>(ws + Ly.xmix);
+    bf16* Xmix_lo = reinterpret_cast<bf16*>(ws + Ly.xmix_lo);
+    bf16* YtT = reinterpret_cast<bf16*>(ws + Ly.ytt);
+    bf16* YtT_lo = reinterpret_cast<bf16*>(ws + Ly.ytt_lo);
+    {  // X_mix = lambda X_o + (1 - lambda) X_u, as hi + lo planes
+      int Ti = (int)T, ni = (int)n;
+      float a = lambda, b = 1.0f - lambda;
+      void* args[] = {(void*)&Xo, (void*)&Xu, (void*)&ldx, (void*)&Ti, (void*)&ni, (void*)&a, (void*)&b, (void*)&Xmix,
+                      (void*)&Xmix_lo, (void*)&ldn};
+      if ((st = launch_small((const void*)axpby_rows, args, T, n, s2, "m_accumulate: mix")) != PIFA_OK) return st;
+    }
+    {  // Y_t^T = W (X_mix,hi + X_mix,lo)^T, as hi + lo planes (m x T)
+      GemmTc g = {m, T, n, W, ldw, false, Xmix, ldn, false, YtT, ldT, 3, 1.0f, nullptr, nullptr, 0, 0};
+      g.B2 = Xmix_lo;
+      g.D2 = YtT_lo;
+      if ((st = gemm_tc(g, status, tmo, s2)) != PIFA_OK) return st;
+    }
+    {  // YtXt += (Y_t^T,hi + Y_t^T,lo) X_u
+      GemmTc g = {m, n, T, YtT, ldT, false, XuT, ldT, false, YtXt, ldyx, 2, 1.0f, nullptr, nullptr, 0, 0};
+      g.A2 = YtT_lo;
+      if ((st = gemm_tc(g, status, tmo, s2)) != PIFA_OK) return st;
+    }
+  }
   {  // XXt += X_u^T X_u, its upper triangle (the product is symmetric: half the tiles)
     GemmTc g = {n, n, T, XuT, ldT, false, XuT, ldT, false, XXt, ldxx, 2, 1.0f, nullptr, nullptr, 0, 0};
     g.upper = true;
-    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
-  }
-  if (!YtXt) return PIFA_OK;
-  bf16* Xmix = reinterpret_cast<bf16*>(ws + Ly.xmix);
-  bf16* Xmix_lo = reinterpret_cast<bf16*>(ws + Ly.xmix_lo);
-  bf16* YtT = reinterpret_cast<bf16*>(ws + Ly.ytt);
-  bf16* YtT_lo = reinterpret_cast<bf16*>(ws + Ly.ytt_lo);
-  {  // X_mix = lambda X_o + (1 - lambda) X_u, as hi + lo planes
-    int Ti = (int)T, ni = (int)n;
-    float a = lambda, b = 1.0f - lambda;
-    void* args[] = {(void*)&Xo, (void*)&Xu, (void*)&ldx, (void*)&Ti, (void*)&ni, (void*)&a, (void*)&b, (void*)&Xmix,
-                    (void*)&Xmix_lo, (void*)&ldn};
-    if ((st = launch_small((const void*)axpby_rows, args, T, n, s, "m_accumulate: mix")) != PIFA_OK) return st;
-  }
-  {  // Y_t^T = W (X_mix,hi + X_mix,lo)^T, as hi + lo planes (m x T)
-    GemmTc g = {m, T, n, W, ldw, false, Xmix, ldn, false, YtT, ldT, 3, 1.0f, nullptr, nullptr, 0, 0};
-    g.B2 = Xmix_lo;
-    g.D2 = YtT_lo;
-    if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
-  }
-  {  // YtXt += (Y_t^T,hi + Y_t^T,lo) X_u
-    GemmTc g = {m, n, T, YtT, ldT, false, XuT, ldT, false, YtXt, ldyx, 2, 1.0f, nullptr, nullptr, 0, 0};
-    g.A2 = YtT_lo;
     if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
   }
   return PIFA_OK;

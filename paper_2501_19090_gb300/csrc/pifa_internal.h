@@ -24,6 +24,23 @@ uint64_t pifa_wait_timeout_ns();
 // per successful launch; pifa_launch_count() reads the total.
 void pifa_count_launch();
 
+// Up to two side streams for independent work inside one call (status.cu): fork(i) makes side
+// stream i wait for the work enqueued on the caller's stream so far and returns it; the destructor
+// makes the caller's stream wait for every side stream that was forked. Per host thread and device.
+class PifaSides {
+ public:
+  explicit PifaSides(cudaStream_t main) : main_(main) {}
+  ~PifaSides();
+  PifaSides(const PifaSides&) = delete;
+  PifaSides& operator=(const PifaSides&) = delete;
+  int fork(int i, cudaStream_t* side);  // PIFA_OK or PIFA_ERR_CUDA
+
+ private:
+  cudaStream_t main_;
+  void* state_ = nullptr;
+  bool forked_[2] = {false, false};
+};
+
 #ifdef __CUDACC__
 #include <utility>
 // cudaLaunchKernelEx, counted.
@@ -82,9 +99,10 @@ int64_t decode_workspace_bytes(const PifaShape& s);
 int launch_decode(const PifaShape& s, const PifaPointers& p, int* status, cudaStream_t stream);
 
 // ---- decode on the tensor cores, split over K (decode_tc.cu) ------------------------------------
-// One decode phase D = A B^T (A: R x K weight rows, B: T <= 16 token rows of K columns, NB = planes
-// 1 or 2) as a persistent split-K tcgen05 kernel writing fp32 partial sums P, then a reduction
-// that writes Y[t, cols[j]] (and, for phase 1, the y_p hi/lo planes).
+// One decode phase D = A B^T (A: R x K weight rows, B: T <= 128 token rows of K columns, NB =
+// planes 1 or 2) as a split-K tcgen05 kernel: row blocks in clusters that add up their K-slices
+// and write Y[t, cols[j]] (and, for phase 1, the y_p hi/lo planes) themselves, or, for phases of
+// more row blocks than the grid holds, balanced ranges writing fp32 partial sums P and a reduction.
 struct DecodeTcPhase {
   const void* A;
   int64_t lda, R, K;

@@ -69,3 +69,61 @@ extern "C" int pifa_selftest_wait_timeout(void* cuda_stream) {
   pifa_count_launch();
   return PIFA_OK;
 }
+
+// ---- side streams: independent products of one call, run concurrently --------------------------
+// Per host thread and device, two non-blocking streams and three events, made on first use and
+// kept for the thread's life (CUDA releases them with the context). A side stream first waits for
+// everything enqueued on the caller's stream so far (PifaSides::fork), and the caller's stream
+// waits for it before the call returns (the destructor), so the call behaves as one stream's work:
+// under stream capture the side streams join the capture through these event waits and rejoin it.
+namespace {
+struct SideState {
+  bool ready = false;
+  cudaStream_t s[2] = {};
+  cudaEvent_t fork = nullptr;
+  cudaEvent_t join[2] = {};
+};
+thread_local SideState g_side[kMaxDevices];
+
+SideState* side_state(cudaError_t* err) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+    *err = e != cudaSuccess ? e : cudaErrorInvalidDevice;
+    return nullptr;
+  }
+  SideState& st = g_side[dev];
+  if (!st.ready) {
+    for (int i = 0; i < 2 && e == cudaSuccess; ++i) e = cudaStreamCreateWithFlags(&st.s[i], cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&st.fork, cudaEventDisableTiming);
+    for (int i = 0; i < 2 && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&st.join[i], cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+      *err = e;
+      return nullptr;
+    }
+    st.ready = true;
+  }
+  return &st;
+}
+}  // namespace
+
+PifaSides::~PifaSides() {
+  // the caller's stream waits for every side stream that was given work, even after a failure
+  for (int i = 0; i < 2; ++i)
+    if (forked_[i]) {
+      SideState* st = static_cast<SideState*>(state_);
+      if (cudaEventRecord(st->join[i], st->s[i]) == cudaSuccess) cudaStreamWaitEvent(main_, st->join[i], 0);
+    }
+}
+
+int PifaSides::fork(int i, cudaStream_t* side) {
+  cudaError_t e = cudaSuccess;
+  SideState* st = state_ ? static_cast<SideState*>(state_) : side_state(&e);
+  if (!st) return pifa_fail_cuda("side stream", e);
+  state_ = st;
+  if ((e = cudaEventRecord(st->fork, main_)) != cudaSuccess || (e = cudaStreamWaitEvent(st->s[i], st->fork, 0)) != cudaSuccess)
+    return pifa_fail_cuda("side stream fork", e);
+  forked_[i] = true;
+  *side = st->s[i];
+  return PIFA_OK;
+}

@@ -200,3 +200,53 @@ def test_m_reconstruct_reports_a_singular_system():
     with pytest.raises(P.PifaError) as e:
         P.pifa_m_reconstruct(XXt, YtXt, torch.from_numpy(V).to(DEV), alpha=0.0)
     assert e.value.status == P.PIFA_ERR_RANK_DEFICIENT
+
+
+def test_backward_and_m_accumulate_under_graph_capture():
+    """The backward's and the M accumulators' independent products run on side streams forked from
+    and joined back into the caller's stream. Captured into a CUDA graph (after a first eager call,
+    which creates the side streams), a replay gives every output bit for bit equal to the eager
+    call's."""
+    m, n, r, T = 1024, 768, 384, 512
+    piv, nonp, Wp32, C32 = inputs.synthetic_layer(m, n, r, 21)
+    rng = np.random.default_rng(22)
+    X = dev_bf16(inputs.make_activations(rng, T, n, "bf16"))
+    dY = dev_bf16(inputs.make_activations(rng, T, m, "bf16"))
+    Wp, C = dev_bf16(Wp32), dev_bf16(C32)
+    pd = torch.from_numpy(piv.astype(np.int32)).to(DEV)
+    nd = torch.from_numpy(nonp.astype(np.int32)).to(DEV)
+    ws = torch.empty(P.pifa_backward_workspace_size(T, m, n, r) + 256, dtype=torch.uint8, device=DEV)
+    st = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    ref = P.pifa_backward(X, Wp, C, pd, nd, dY, workspace_tensor=ws, stream=st)
+    st.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=st):
+        got = P.pifa_backward(X, Wp, C, pd, nd, dY, workspace_tensor=ws, stream=st)
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    assert P.pifa_device_status() == P.PIFA_OK
+    assert torch.equal(got[0].view(torch.int16), ref[0].view(torch.int16))
+    assert torch.equal(got[1], ref[1]) and torch.equal(got[2], ref[2])
+    del g
+
+    Xo, Xu, W = _macc_inputs(T, n, m, 23)
+    Xo, Xu, W = dev_bf16(Xo), dev_bf16(Xu), dev_bf16(W)
+    wsm = torch.empty(P.pifa_m_accumulate_workspace_size(T, m, n) + 256, dtype=torch.uint8, device=DEV)
+    XXt0 = torch.zeros((n, n), dtype=torch.float32, device=DEV)
+    Y0 = torch.zeros((m, n), dtype=torch.float32, device=DEV)
+    P.pifa_m_accumulate(Xo, Xu, W, 0.3, XXt0, Y0, workspace_tensor=wsm, stream=st)
+    st.synchronize()
+    XXt1 = torch.zeros_like(XXt0)
+    Y1 = torch.zeros_like(Y0)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=st):
+        P.pifa_m_accumulate(Xo, Xu, W, 0.3, XXt1, Y1, workspace_tensor=wsm, stream=st)
+    XXt1.zero_()
+    Y1.zero_()
+    torch.cuda.synchronize()
+    g.replay()
+    torch.cuda.synchronize()
+    assert P.pifa_device_status() == P.PIFA_OK
+    assert torch.equal(torch.triu(XXt1), torch.triu(XXt0)) and torch.equal(Y1, Y0)
