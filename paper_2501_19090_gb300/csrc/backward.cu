@@ -1,10 +1,10 @@
 // backward.cu -- the gradients of a PIFA layer (fine-tuning after compression, Sec. 5.1; the layer
 // is differentiable, Sec. 6) and the online accumulators of the M reconstruction (Sec. 4; the
-// accumulation steps of Algorithm 3), as tensor-core contractions (gemm_tc.cu) plus a column gather.
+// accumulation steps of Algorithm 3), as tensor-core contractions (gemm_tc.cu) plus a column split.
 //
 // Backward, tokens as rows (Y = X W'^T, Y_p = X W_p^T, Y_np = Y_p C^T), given dY = dL/dY:
-//   dY_np = dY[:, I^c]                       gather                 (Algorithm 2, step 5, reversed)
-//   dY_p  = dY[:, I] + dY_np C               T x r,  K = m - r      (steps 4 and 3, reversed)
+//   dY_I = dY[:, I], dY_np = dY[:, I^c]      one pass over dY       (Algorithm 2, steps 4-5, reversed)
+//   dY_p  = dY_I + dY_np C                   T x r,  K = m - r      (steps 4 and 3, reversed)
 //   dX    = dY_p W_p                         T x n,  K = r          (step 2, reversed)
 // dY_p and Y_p are kept as hi + lo pairs of bf16 planes: in exact arithmetic dX = dY W', and the
 // route through dY_p (amplified by C, then contracted with W_p) would otherwise lose the bits that
@@ -32,22 +32,26 @@ using bf16 = __nv_bfloat16;
 int64_t pad8(int64_t v) { return (v + 7) / 8 * 8; }
 int64_t a256(int64_t b) { return (b + 255) / 256 * 256; }
 
-// out[t][i] = in[t][idx[i]] for t < T, i < cnt (bf16); an index outside [0, bound) writes 0 and
-// latches PIFA_ERR_DEVICE_INDEX. Row t = blockIdx.y (grid-stride), columns across the x grid.
-__global__ void gather_cols(const bf16* in, int64_t ldin, const int32_t* idx, int cnt, int bound, int T, bf16* out,
-                            int64_t ldout, int* status) {
+// dY's columns split into its pivot and non-pivot parts (bf16): outp[t][j] = in[t][piv[j]] for
+// j < r and outnp[t][i] = in[t][nonpiv[i]] for i < nnp; an index outside [0, bound) writes 0 and
+// latches PIFA_ERR_DEVICE_INDEX. A thread owns one output column (its index read once, the lanes
+// of a warp on consecutive columns) and walks the rows of its y-block's share, so that the loads of
+// consecutive rows are independent and many are in flight.
+__global__ void split_cols(const bf16* in, int64_t ldin, const int32_t* piv, int r, const int32_t* nonpiv, int nnp,
+                           int bound, int T, bf16* outp, int64_t ldp, bf16* outnp, int64_t ldnp, int* status) {
   pdl_launch_dependents();
   pdl_wait_primary();
-  for (int t = blockIdx.y; t < T; t += gridDim.y)
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < cnt; i += gridDim.x * blockDim.x) {
-      const int c = __ldg(idx + i);
-      bf16 v = __float2bfloat16_rn(0.0f);
-      if ((unsigned)c < (unsigned)bound)
-        v = in[(int64_t)t * ldin + c];
-      else
-        latch_status(status, PIFA_ERR_DEVICE_INDEX);
-      out[(int64_t)t * ldout + i] = v;
-    }
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= r + nnp) return;
+  const bool pv = j < r;
+  const int c = __ldg(pv ? piv + j : nonpiv + (j - r));
+  bf16* out = pv ? outp + j : outnp + (j - r);
+  const int64_t ldo = pv ? ldp : ldnp;
+  const bool ok = (unsigned)c < (unsigned)bound;
+  if (!ok) latch_status(status, PIFA_ERR_DEVICE_INDEX);
+  const bf16 zero = __float2bfloat16_rn(0.0f);
+#pragma unroll 8
+  for (int t = blockIdx.y; t < T; t += gridDim.y) out[(int64_t)t * ldo] = ok ? in[(int64_t)t * ldin + c] : zero;
 }
 
 // out = a * x + b * y elementwise over T rows of n (bf16 in, fp32 arithmetic), written as a hi +
@@ -104,7 +108,7 @@ int launch_small(const void* fn, void** args, int64_t rows, int64_t cols, cudaSt
 bool al16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct BwdLayout {
-  int64_t dynp, yp, yp_lo, dyp, dyp_lo, total;
+  int64_t dynp, dyi, yp, yp_lo, dyp, dyp_lo, total;
 };
 
 BwdLayout bwd_layout(int64_t T, int64_t m, int64_t r) {
@@ -112,6 +116,8 @@ BwdLayout bwd_layout(int64_t T, int64_t m, int64_t r) {
   int64_t o = 0;
   L.dynp = o;
   o += a256(T * pad8(m - r > 0 ? m - r : 1) * 2);
+  L.dyi = o;
+  o += a256(T * pad8(r) * 2);
   L.yp = o;
   o += a256(T * pad8(r) * 2);
   L.yp_lo = o;
@@ -197,15 +203,23 @@ extern "C" int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx, c
   bf16* dYp_lo = reinterpret_cast<bf16*>(ws + Ly.dyp_lo);
   const int64_t ldnp = pad8(m - r > 0 ? m - r : 1), ldr = pad8(r);
   int st;
-  int Ti = (int)T, mi = (int)m;
-  // dY_np = dY[:, I^c]
-  if (has_np) {
-    int cnt = (int)(m - r);
-    void* args[] = {(void*)&dY, (void*)&lddy, (void*)&nonpivot_idx, (void*)&cnt, (void*)&mi, (void*)&Ti,
-                    (void*)&dYnp, (void*)&ldnp, (void*)&status};
-    if ((st = launch_small((const void*)gather_cols, args, T, m - r, s, "backward: gather")) != PIFA_OK) return st;
+  bf16* dYi = reinterpret_cast<bf16*>(ws + Ly.dyi);
+  {  // dY_I = dY[:, I] and dY_np = dY[:, I^c] in one pass over dY (dY_I straight into dY_p when r = m)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)((m + 255) / 256), (unsigned)(T < 64 ? T : 64));
+    cfg.blockDim = dim3(256);
+    cfg.stream = s;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = pifa_launch_ex(&cfg, split_cols, reinterpret_cast<const bf16*>(dY), lddy, pivot_idx, (int)r,
+                                         nonpivot_idx, (int)(m - r), (int)m, (int)T, has_np ? dYi : dYp, ldr, dYnp,
+                                         ldnp, status);
+    if (e != cudaSuccess) return pifa_fail_cuda("backward: split dY", e);
   }
-  // Independent products run concurrently: Y_p and then dC on side stream 0 (after the gather),
+  // Independent products run concurrently: Y_p and then dC on side stream 0 (after the split),
   // dY_p and then dX on the caller's stream, dW_p on side stream 1 once dY_p is done. Each product
   // alone fills one or two waves of the GPU; together they keep it busy (the side streams rejoin
   // the caller's stream before this call returns, also on failure).
@@ -218,16 +232,11 @@ extern "C" int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx, c
     g.D2 = Yp_lo;
     if ((st = gemm_tc(g, status, tmo, s_yp)) != PIFA_OK) return st;
   }
-  // dY_p = dY[:, I] + dY_np C, as hi + lo planes
+  // dY_p = dY_I + dY_np C, as hi + lo planes (dY_p = dY_I when r = m)
   if (has_np) {
-    GemmTc g = {T, r, m - r, dYnp, ldnp, false, C, ldc, true, dYp, ldr, 3, 1.0f, dY, pivot_idx, lddy, m};
+    GemmTc g = {T, r, m - r, dYnp, ldnp, false, C, ldc, true, dYp, ldr, 3, 1.0f, dYi, nullptr, ldr, r};
     g.D2 = dYp_lo;
     if ((st = gemm_tc(g, status, tmo, s)) != PIFA_OK) return st;
-  } else {
-    int cnt = (int)r;
-    void* args[] = {(void*)&dY, (void*)&lddy, (void*)&pivot_idx, (void*)&cnt, (void*)&mi, (void*)&Ti,
-                    (void*)&dYp, (void*)&ldr, (void*)&status};
-    if ((st = launch_small((const void*)gather_cols, args, T, r, s, "backward: gather")) != PIFA_OK) return st;
   }
   if (dWp) {  // dW_p = (dY_p,hi + dY_p,lo)^T X
     if ((st = sides.fork(1, &s_dw)) != PIFA_OK) return st;
