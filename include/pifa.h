@@ -264,11 +264,16 @@ int64_t pifa_compress_device_workspace_size(int64_t m, int64_t n, int64_t r);
  *   dWp          DEVICE out, fp32, r x n, pitch lddwp >= n (NULL: not computed).
  *   dC           DEVICE out, fp32, (m - r) x r, pitch lddc >= r (NULL: not computed).
  *   workspace    DEVICE scratch of pifa_backward_workspace_size(T, m, n, r) bytes, 256-byte
- *                aligned, no initialisation needed (dY_np, Y_p and dY_p in bf16).
- *   Numerics: bf16 operands, fp32 accumulation; dY_p and Y_p are rounded to bf16 between the
- *   contractions. Alignment as pifa_forward (fp32 pitches multiples of 4 elements). T == 0 writes
- *   zero dW_p and dC. Asynchronous on cuda_stream; out-of-range indices latch
+ *                aligned, no initialisation needed (dY[:, I], dY[:, I^c], Y_p and dY_p in bf16).
+ *   Numerics: bf16 operands, fp32 accumulation; dY_p and Y_p pass between the contractions as
+ *   hi + lo pairs of bf16. Alignment as pifa_forward (fp32 pitches multiples of 4 elements).
+ *   T == 0 writes zero dW_p and dC. Asynchronous on cuda_stream; out-of-range indices latch
  *   PIFA_ERR_DEVICE_INDEX (read with pifa_device_status()).
+ *   Concurrency: independent products run on two side streams that the library keeps per host
+ *   thread and device, forked from cuda_stream and joined back into it inside the call (also on
+ *   failure), so the call orders like one kernel sequence on cuda_stream and can be captured into a
+ *   CUDA graph. The first call on a thread and device creates those streams: make it before a
+ *   stream capture that contains the call.
  */
 int pifa_backward(const void* X, int64_t T, int64_t n, int64_t ldx,
                   const void* Wp, int64_t r, int64_t ldwp,
@@ -299,8 +304,9 @@ int64_t pifa_backward_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r)
  *   YtXt         DEVICE in/out, fp32, m x n, pitch ldyx >= n (NULL: only XXt is accumulated).
  *   workspace    DEVICE scratch of pifa_m_accumulate_workspace_size(T, m, n) bytes, 256-byte
  *                aligned (X_u^T, the mixed input and Y_t^T in bf16).
- *   Numerics: bf16 operands, fp32 accumulation; the mixed input and Y_t are rounded to bf16.
- *   T == 0 is a no-op. Asynchronous on cuda_stream.
+ *   Numerics: bf16 operands, fp32 accumulation; the mixed input and Y_t pass as hi + lo bf16 pairs.
+ *   T == 0 is a no-op. Asynchronous on cuda_stream; X X^T runs beside the Y_t chain on a side
+ *   stream, as in pifa_backward (same ordering and capture rules).
  */
 int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int64_t n, int64_t ldx,
                       const void* W, int64_t m, int64_t ldw, float lambda,
