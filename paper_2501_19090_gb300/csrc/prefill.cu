@@ -20,6 +20,11 @@
 // out as 16-byte stores after a transpose through shared memory. Every wait is bounded
 // (globaltimer); on timeout the CTA latches PIFA_ERR_TIMEOUT, drains what it has in flight and
 // returns.
+//
+// GEMMs whose full-width tiles leave most SMs idle (GEMM 1 of the 70B layers has 32 row blocks;
+// T of a few hundred gives one token tile) split K instead: a tile's 2 or 4 CTAs form a cluster,
+// each accumulates its K-slice, stores the fp32 partial tile in its own freed stage ring, and the
+// cluster adds the slices through distributed shared memory in rank order before the epilogue.
 #include <utility>
 
 #include <cuda_bf16.h>
@@ -87,9 +92,16 @@ struct GemmArgs {
   int64_t ldyp;
   int* status;
   uint64_t timeout_ns;
+  int ks;                // K-slices per tile (kCl): the CTAs blockIdx.z = 0 .. ks - 1 of a tile form a cluster
 };
 
-template <int kEpi, int CFG>
+// kCl: split-K over a cluster of ks CTAs per tile (grids with too few tiles to fill the GPU). CTA z
+// accumulates the K-steps [z total / ks, (z + 1) total / ks) of both passes, stores its fp32
+// partial tile in its own shared memory (the stage ring, free once its MMAs are done) and, after a
+// cluster barrier, adds rows [z 128 / ks, (z + 1) 128 / ks) of every peer's partial tile in rank
+// order (distributed shared memory) and writes them out as the epilogue would. Only these
+// instantiations hold cluster barriers and distributed shared-memory loads.
+template <int kEpi, int CFG, bool kCl>
 __global__ void __launch_bounds__(PC<CFG>::THREADS, PC<CFG>::CTAS)
     pifa_umma_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, GemmArgs p) {
@@ -111,7 +123,10 @@ __global__ void __launch_bounds__(PC<CFG>::THREADS, PC<CFG>::CTAS)
   const int n0 = (p.tok_fast ? blockIdx.x : blockIdx.y) * p.bn;
   const uint32_t b_bytes = (uint32_t)p.bn * BK * 2;  // one B box
   const int bx0 = p.gsz > 0 ? (m0 / p.gsz) * p.goff : 0;  // the tile's group's first B column
-  const int total = p.kchunks * p.passes;
+  const int ksteps = p.kchunks * p.passes;
+  const int z = kCl ? (int)blockIdx.z : 0;
+  const int i0 = kCl ? (int)(((int64_t)z * ksteps) / p.ks) : 0;  // this CTA's K-steps [i0, i0 + total)
+  const int total = kCl ? (int)(((int64_t)(z + 1) * ksteps) / p.ks) - i0 : ksteps;
 
   if (warp == 0 && lane == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -143,11 +158,11 @@ __global__ void __launch_bounds__(PC<CFG>::THREADS, PC<CFG>::CTAS)
       const int pre = total < STAGES ? total : STAGES;
       for (int i = 0; i < pre; ++i) {
         mbar_expect_tx(&full[i], A_BYTES);
-        tma_load_2d(smem_u32(smem + i * STAGE_BYTES), &tmA, (i % p.kchunks) * BK, m0, &full[i]);
+        tma_load_2d(smem_u32(smem + i * STAGE_BYTES), &tmA, ((i0 + i) % p.kchunks) * BK, m0, &full[i]);
       }
       pdl_wait_primary();
       for (int i = 0; i < pre; ++i) {
-        const int pass = i / p.kchunks, kc = i % p.kchunks;
+        const int pass = (i0 + i) / p.kchunks, kc = (i0 + i) % p.kchunks;
         mbar_arrive_expect_tx(&full[i], b_bytes);
         tma_load_2d(smem_u32(smem + i * STAGE_BYTES + A_BYTES), pass ? &tmB1 : &tmB0, bx0 + kc * BK, n0, &full[i]);
       }
@@ -161,7 +176,7 @@ __global__ void __launch_bounds__(PC<CFG>::THREADS, PC<CFG>::CTAS)
           break;
         }
         if (*abort_flag) break;
-        const int pass = i / p.kchunks, kc = i % p.kchunks;
+        const int pass = (i0 + i) / p.kchunks, kc = (i0 + i) % p.kchunks;
         uint8_t* sa = smem + s * STAGE_BYTES;
         mbar_arrive_expect_tx(&full[s], A_BYTES + b_bytes);
         tma_load_2d(smem_u32(sa), &tmA, kc * BK, m0, &full[s]);
@@ -216,7 +231,25 @@ __global__ void __launch_bounds__(PC<CFG>::THREADS, PC<CFG>::CTAS)
     const bool ok = mbar_wait(acc_full, 0, p.timeout_ns);
     if (!ok) latch_status(p.status, PIFA_ERR_TIMEOUT);
     tc_fence_after();
-    if (ok && !*abort_flag) {
+    if (kCl) {
+      // this K-slice's partial tile into the ring as [token][128 rows] fp32 (the lanes of a
+      // warp on consecutive rows): the cluster adds the slices below
+      if (ok && !*abort_flag) {
+        fence_proxy_async_smem();  // the ring's last operands were read by the MMAs (async proxy)
+        float* red = reinterpret_cast<float*>(smem);
+        const int tend = min(n0 + p.bn, p.N);
+#pragma unroll 1
+        for (int ci = 0; ci < kChunks; ++ci) {
+          const int tb = n0 + (slice * kChunks + ci) * 32;
+          if (tb >= tend) break;  // warp-uniform
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(tb - n0), v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 32; ++j) red[(tb - n0 + j) * BM + q * 32 + lane] = __uint_as_float(v[j]);
+        }
+      }
+    } else if (ok && !*abort_flag) {
       int col = -1;
       if (row < p.M) {
         col = p.cols[row];
@@ -280,14 +313,64 @@ __global__ void __launch_bounds__(PC<CFG>::THREADS, PC<CFG>::CTAS)
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
   }
+  if (kCl) {
+    // Every CTA of the cluster has its partial tile in its own shared memory once all arrive (every
+    // wait above is bounded, so each CTA gets here); CTA z then finishes rows [z rpc, (z + 1) rpc)
+    // of the tile for all its tokens, adding the slices in rank order (deterministic), and a
+    // second barrier keeps each CTA resident until no peer reads its shared memory any more.
+    cluster_sync_all();
+    const int rpc = BM / p.ks;
+    const int ntok = min(p.bn, p.N - n0);
+    const uint32_t red = smem_u32(smem);
+    bool range_err = false;
+    for (int idx = threadIdx.x; idx < rpc * ntok; idx += PC<CFG>::THREADS) {
+      const int t = idx / rpc, rr = z * rpc + idx % rpc;
+      const int row = m0 + rr;
+      const uint32_t off = red + (uint32_t)(t * BM + rr) * 4u;
+      float f = 0.0f;
+      for (int k = 0; k < p.ks; ++k) f += ld_dsmem_f32(mapa_shared(off, (uint32_t)k));
+      if (row >= p.M) continue;
+      const int tok = n0 + t;
+      const int col = __ldg(p.cols + row);
+      if ((unsigned)col >= (unsigned)p.m)
+        latch_status(p.status, PIFA_ERR_DEVICE_INDEX);
+      else
+        p.Y[(int64_t)tok * p.ldy + col] = __float2bfloat16_rn(f);
+      if (kEpi == EPI_SPLIT_BF16) {
+        const bf16 h = __float2bfloat16_rn(f);
+        reinterpret_cast<uint16_t*>(p.yp_hi)[(int64_t)tok * p.ldyp + row] = __bfloat16_as_ushort(h);
+        reinterpret_cast<uint16_t*>(p.yp_lo)[(int64_t)tok * p.ldyp + row] =
+            __bfloat16_as_ushort(__float2bfloat16_rn(f - __bfloat162float(h)));
+      } else if (kEpi == EPI_SPLIT_F16) {
+        float fs = f;
+        if (fabsf(fs) > 65504.0f) {
+          range_err = true;
+          fs = copysignf(65504.0f, fs);
+        }
+        const __half hh = __float2half_rn(fs);
+        reinterpret_cast<uint16_t*>(p.yp_hi)[(int64_t)tok * p.ldyp + row] = __half_as_ushort(hh);
+        reinterpret_cast<uint16_t*>(p.yp_lo)[(int64_t)tok * p.ldyp + row] =
+            __half_as_ushort(__float2half_rn(fs - __half2float(hh)));
+      }
+    }
+    if (range_err) latch_status(p.status, PIFA_ERR_RANGE);
+    cluster_sync_all();
+  }
 }
 
 template <int CFG>
 int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1, const GemmArgs& args,
              cudaStream_t stream) {
-  auto kern = epi == EPI_SPLIT_BF16 ? pifa_umma_gemm<EPI_SPLIT_BF16, CFG>
-              : epi == EPI_SPLIT_F16 ? pifa_umma_gemm<EPI_SPLIT_F16, CFG>
-                                    : pifa_umma_gemm<EPI_Y_ONLY, CFG>;
+  const bool cl = CFG == 0 && args.ks > 1;  // split-K clusters: config 0 only (one CTA per SM)
+  auto kern = cl ? (epi == EPI_SPLIT_BF16 ? pifa_umma_gemm<EPI_SPLIT_BF16, CFG, CFG == 0>
+                    : epi == EPI_SPLIT_F16 ? pifa_umma_gemm<EPI_SPLIT_F16, CFG, CFG == 0>
+                                          : pifa_umma_gemm<EPI_Y_ONLY, CFG, CFG == 0>)
+                 : (epi == EPI_SPLIT_BF16 ? pifa_umma_gemm<EPI_SPLIT_BF16, CFG, false>
+                    : epi == EPI_SPLIT_F16 ? pifa_umma_gemm<EPI_SPLIT_F16, CFG, false>
+                                          : pifa_umma_gemm<EPI_Y_ONLY, CFG, false>);
+  if (args.ks > 1 && !cl) return pifa_fail(PIFA_ERR_UNSUPPORTED, "prefill: split-K needs the one-CTA shape");
+  if (cl && (size_t)args.bn * BM * 4 > (size_t)PC<CFG>::B::STAGES * PC<CFG>::STAGE_BYTES)
+    return pifa_fail(PIFA_ERR_UNSUPPORTED, "prefill: partial tile larger than the stage ring");
   constexpr size_t SMEM_BYTES = PC<CFG>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SMEM_BYTES);
   if (e != cudaSuccess) return pifa_fail_cuda("cudaFuncSetAttribute(prefill gemm)", e);
@@ -304,15 +387,20 @@ int run_gemm(int epi, const CUtensorMap& a, const CUtensorMap& b0, const CUtenso
   g.tok_fast = args.M > args.N ? 1 : 0;
   if ((g.tok_fast ? mt : nt) > 65535u) g.tok_fast ^= 1;  // gridDim.y is at most 65535
   if ((g.tok_fast ? mt : nt) > 65535u) return pifa_fail(PIFA_ERR_UNSUPPORTED, "more than 65535 tiles along both M and T");
-  cfg.gridDim = g.tok_fast ? dim3(nt, mt) : dim3(mt, nt);
+  g.ks = cl ? args.ks : 1;
+  cfg.gridDim = g.tok_fast ? dim3(nt, mt, (unsigned)g.ks) : dim3(mt, nt, (unsigned)g.ks);
   cfg.blockDim = dim3(PC<CFG>::THREADS);
   cfg.dynamicSmemBytes = SMEM_BYTES;
   cfg.stream = stream;
-  cudaLaunchAttribute attr;
-  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr.val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = &attr;
-  cfg.numAttrs = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;  // a tile's K-slices: consecutive along z
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = (unsigned)g.ks;
+  cfg.attrs = attr;
+  cfg.numAttrs = cl ? 2 : 1;
   e = pifa_launch_ex(&cfg, kern, a, b0, b1, g);
   if (e != cudaSuccess) return pifa_fail_cuda("prefill gemm launch", e);
   return PIFA_OK;
@@ -337,7 +425,7 @@ int sm_count_prefill() {
 // The kernel shape and token-tile width of one GEMM: config 0 with pick_bn's width unless that
 // takes three or more waves, then config 1 (CTA slots = 2 per SM) with its own width.
 struct GemmShape {
-  int cfg, bn;
+  int cfg, bn, ks;  // kernel shape, tokens per tile, K-slices per tile (a cluster when > 1)
 };
 int pick_bn_slots(int64_t M, int64_t T, int bnmax, int64_t slots) {
   const int64_t mt = (M + BM - 1) / BM;
@@ -353,12 +441,29 @@ int pick_bn_slots(int64_t M, int64_t T, int bnmax, int64_t slots) {
   }
   return best;
 }
-GemmShape pick_shape(int64_t M, int64_t T) {
+// Split-K: when the GEMM's full-width tiles (256 tokens, or all of T) fill at most half the SMs and
+// the one-wave plan would otherwise fall back to tiles of 64 tokens or fewer, each full-width tile
+// gets ks CTAs (2 or 4, keeping one CTA per SM, every K-slice at least 16 steps of 64) as a
+// cluster that adds its partial tiles in shared memory. Measured against the narrow-tile plan (us,
+// one process, interleaved): 7B attention T = 256 44.5 -> 34.8, T = 512 47.3 -> 37.0; 7B MLP down
+// T = 256 76.7 -> 43.5, T = 512 80.4 -> 46.7; 7B MLP gate T = 256 46.6 -> 42.7; 70B q/o T = 256
+// 88.9 -> 53.0; 70B gate/up T = 256 159.4 -> 142.8; 4096 x 4096, r = 1024, T = 512 36.4 -> 32.3.
+// Splitting also where the plan keeps tiles of 96-128 tokens lost (r = 1024, T = 2048: 55.4 ->
+// 59.0), as did clusters of 8 (8 K-steps per slice: 7B attention T = 256 44.5 -> 49.2).
+GemmShape pick_shape(int64_t M, int64_t T, int64_t ksteps) {
   const int64_t sms = sm_count_prefill();
+  const int64_t mt = (M + BM - 1) / BM;
+  const int bnw = (int)(T >= PC<0>::BN ? PC<0>::BN : (T + 15) / 16 * 16);
+  const int64_t tiles_w = mt * ((T + bnw - 1) / bnw);
   const int bn0 = pick_bn_slots(M, T, PC<0>::BN, sms);
-  const int64_t waves0 = ((M + BM - 1) / BM * ((T + bn0 - 1) / bn0) + sms - 1) / sms;
-  if (waves0 < 3) return {0, bn0};
-  return {1, pick_bn_slots(M, T, PC<1>::BN, 2 * sms)};
+  if (tiles_w * 2 <= sms && bn0 <= 64) {
+    int ks = 1;
+    while (ks < 4 && tiles_w * ks * 2 <= sms && ksteps / (ks * 2) >= 16) ks *= 2;
+    if (ks > 1) return {0, bnw, ks};
+  }
+  const int64_t waves0 = (mt * ((T + bn0 - 1) / bn0) + sms - 1) / sms;
+  if (waves0 < 3) return {0, bn0, 1};
+  return {1, pick_bn_slots(M, T, PC<1>::BN, 2 * sms), 1};
 }
 
 template <typename... A>
@@ -384,7 +489,7 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
 
   CUtensorMap tWp, tX, tC, tHi, tLo;
   int st;
-  const GemmShape sh1 = pick_shape(G * s.r, s.T);
+  const GemmShape sh1 = pick_shape(G * s.r, s.T, (s.n + BK - 1) / BK);
   const int bn1 = sh1.bn;
   if ((st = make_tmap_2d(&tWp, PIFA_DTYPE_BF16, p.Wp, G * s.r, s.n, s.ldwp, BK, BM)) != PIFA_OK) return st;
   if ((st = make_tmap_2d(&tX, PIFA_DTYPE_BF16, p.X, s.T, s.n, s.ldx, BK, bn1)) != PIFA_OK) return st;
@@ -405,10 +510,11 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
   g1.ldyp = ldyp;
   g1.status = status;
   g1.timeout_ns = timeout_ns;
+  g1.ks = sh1.ks;
   if ((st = run_gemm_cfg(sh1.cfg, f16 ? EPI_SPLIT_F16 : EPI_SPLIT_BF16, tWp, tX, tX, g1, stream)) != PIFA_OK) return st;
   if (s.m == s.r) return PIFA_OK;
 
-  const GemmShape sh2 = pick_shape(G * (s.m - s.r), s.T);
+  const GemmShape sh2 = pick_shape(G * (s.m - s.r), s.T, 2 * ((s.r + BK - 1) / BK));
   const int bn2 = sh2.bn;
   if ((st = make_tmap_2d(&tC, s.c_dtype, p.C, G * (s.m - s.r), s.r, s.ldc, BK, BM)) != PIFA_OK) return st;
   if ((st = make_tmap_2d(&tHi, s.c_dtype, hi, s.T, G * s.r, ldyp, BK, bn2)) != PIFA_OK) return st;
@@ -423,6 +529,7 @@ int launch_prefill_split(const PifaShape& s, const PifaPointers& p, int* status,
   }
   g2.kchunks = (int)((s.r + BK - 1) / BK);
   g2.passes = 2;
+  g2.ks = sh2.ks;
   g2.cols = p.nonpiv;
   g2.yp_hi = nullptr;
   g2.yp_lo = nullptr;

@@ -715,3 +715,27 @@ def test_graph_replay_back_to_back_matches_single_calls(m, n, r, T):
         for j in range(copies):
             assert torch.equal(Ys[j].view(torch.int16), ref[j].view(torch.int16)), f"copy {j} differs"
     del g
+
+
+# ---------------------------------------------------------------------------------------------
+# split prefill with split-K clusters: GEMMs of too few 256-token tiles to fill the GPU
+# ---------------------------------------------------------------------------------------------
+@pytest.mark.parametrize("T", [256, 200])
+def test_prefill_split_k_clusters_llama70b(T):
+    """70B gate/up at T = 256 (GEMM 1: 32 tiles of 256 tokens, four CTAs each over K = 8192, the
+    partial tiles added in a cluster) and 70B q/o with C in fp16 at T = 200 (both GEMMs split in
+    four, one 208-token tile holding 200 tokens; fp16 hi/lo planes written by the cluster sum)."""
+    if T == 256:
+        parity(layer_for(28672, 8192, 4096, 0, "gpu"), T, P.PIFA_VARIANT_PREFILL_SPLIT, sample=96)
+    else:
+        parity(layer_for(8192, 8192, 4096, 0, "library", "fp16"), T, P.PIFA_VARIANT_PREFILL_SPLIT, sample=96)
+
+
+def test_prefill_split_k_clusters_ragged_and_deterministic():
+    """A layer with a partial last row tile in both GEMMs (1100 and 1900 rows) and ragged K (2000 and
+    1100 columns) at T = 200: each GEMM split over two CTAs (GEMM 2's slices are its hi and its lo
+    pass); the same call twice gives the same bits (the slices are added in rank order)."""
+    L = layer_for(3000, 2000, 1100, 4, "synthetic")
+    parity(L, 200, P.PIFA_VARIANT_PREFILL_SPLIT)
+    X = acts(200, 2000, 9)
+    assert np.array_equal(run(L, X, P.PIFA_VARIANT_PREFILL_SPLIT), run(L, X, P.PIFA_VARIANT_PREFILL_SPLIT))

@@ -170,3 +170,55 @@ def test_cluster_sums_fit_the_ring(tnt, nb):
     stage = TM * KB * 2 + nb * tnt * KB * 2
     stages = min(10, (112 * 1024 - 1536) // stage)
     assert stages >= 2 and TM * tnt * 4 <= stages * stage
+
+
+# ---- the split prefill's choice of tile width and K-slices (csrc/prefill.cu pick_shape) ----------
+def pick_bn_slots(M, T, bnmax, slots):
+    mt = -(-M // 128)
+    best, best_cost = bnmax, None
+    for bn in range(bnmax, 15, -16):
+        tiles = mt * -(-T // bn)
+        cost = -(-tiles // slots) * (432 + bn)
+        if best_cost is None or cost < best_cost:
+            best, best_cost = bn, cost
+    return best
+
+
+def pick_shape(M, T, ksteps, sms=152):
+    """(config, tokens per tile, K-slices per tile)."""
+    mt = -(-M // 128)
+    bnw = 256 if T >= 256 else -(-T // 16) * 16
+    tiles_w = mt * -(-T // bnw)
+    bn0 = pick_bn_slots(M, T, 256, sms)
+    if tiles_w * 2 <= sms and bn0 <= 64:
+        ks = 1
+        while ks < 4 and tiles_w * ks * 2 <= sms and ksteps // (ks * 2) >= 16:
+            ks *= 2
+        if ks > 1:
+            return 0, bnw, ks
+    waves0 = -(-(mt * -(-T // bn0)) // sms)
+    if waves0 < 3:
+        return 0, bn0, 1
+    return 1, pick_bn_slots(M, T, 160, 2 * sms), 1
+
+
+def test_prefill_split_k_choice_on_the_llama_gemms():
+    """GEMM 1 (M = r, K = n) and GEMM 2 (M = m - r, two passes over K = r): split into clusters of 4
+    where the plain plan would run tiles of 64 tokens or fewer (7B attention and 70B layers at
+    T = 256), kept whole where it fills the SMs with wider tiles (7B attention T = 2048, the
+    r = 1024 layer at T = 2048, 70B q/o at T = 512)."""
+    assert pick_shape(2048, 256, 64) == (0, 256, 4) and pick_shape(2048, 256, 64) == pick_shape(2048, 256, 2 * 32)
+    assert pick_shape(4096, 256, 128) == (0, 256, 4)                  # 70B GEMM 1
+    assert pick_shape(24576, 256, 128)[2] == 1                       # 70B gate/up GEMM 2: 192 tiles
+    assert pick_shape(2048, 2048, 64) == (0, 240, 1)                 # 7B attention prefill
+    assert pick_shape(1024, 2048, 64)[2] == 1                        # r = 1024 GEMM 1: 152 tiles of 112
+    assert pick_shape(4096, 512, 128)[2] == 1                        # 70B q/o T = 512
+    assert pick_shape(4096, 200, 128) == (0, 208, 4)                 # one ragged 208-token tile
+    assert pick_shape(1100, 200, 32) == (0, 208, 2) and pick_shape(1900, 200, 36) == (0, 208, 2)
+
+
+@pytest.mark.parametrize("ksteps,ks", [(64, 4), (36, 2), (128, 4), (33, 2), (16, 2)])
+def test_prefill_k_slices_cover_every_step_once(ksteps, ks):
+    """CTA z of a tile's cluster accumulates K-steps [z ksteps / ks, (z + 1) ksteps / ks)."""
+    steps = [i for z in range(ks) for i in range(z * ksteps // ks, (z + 1) * ksteps // ks)]
+    assert steps == list(range(ksteps))
