@@ -269,11 +269,11 @@ def layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src, name=None, c
     """One layer shape at T tokens: the selected PIFA variant, the two-factor low-rank layer and the
     dense layer on the same GPU, each a CUDA graph replayed in steady state over rotating weight
     copies (decode: every copy's bytes exceed 3x L2 in total; prefill: two copies), with the
-    roofline of the PIFA call (HBM for decode, T <= DECODE_MAX_T; bf16 tensor otherwise) and the clocks seen."""
+    roofline of the PIFA call (HBM for the decode variant, bf16 tensor otherwise) and the clocks seen."""
     import torch
     from paper_2501_19090_gb300 import pifa as P
     m, n, r = shape.m, shape.n, shape.r
-    decode = T <= DECODE_MAX_T
+    decode = is_decode(T, m, r)
     copies = _copies_for(dev, 2 * r * (m + n - r)) if decode else 2
     piv, nonp, Wps, Cs = timing_layer(shape, dev, 7, c_dtype, copies)
     gen = torch.Generator(device=dev)
@@ -324,11 +324,19 @@ def layer_point(dev, stream, shape, T, hbm_peak, tc_peak, peak_src, name=None, c
     return out
 
 
-# the library's selector runs the decode variant up to this many tokens on every single layer
-# measured here (T <= 128 needs each phase within 296 row blocks of 128), the split prefill above
+# The library's selector (pifa_select_variant) runs the decode variant for T <= 64, and up to
+# DECODE_MAX_T tokens where the non-pivot rows make 148 to 296 blocks of 128 and the pivot rows at
+# most 296; the split prefill otherwise. is_decode restates it for the bench's workload names.
 DECODE_MAX_T = 128
-DECODE_POINTS = [(inputs.ATTN7B, (1, 8, 16, 64, 128)), (inputs.MLP7B_GATE, (1, 8, 16, 64, 128)),
-                 (inputs.MLP7B_DOWN, (1, 8, 16, 64, 128)), (inputs.ATTN70B, (1, 8, 16, 64, 128)),
+
+
+def is_decode(T, m, r, groups=1):
+    if T <= 64:
+        return True
+    blocks_p, blocks_np = -(-groups * r // 128), -(-groups * (m - r) // 128)
+    return T <= DECODE_MAX_T and blocks_p <= 296 and 148 <= blocks_np <= 296
+DECODE_POINTS = [(inputs.ATTN7B, (1, 8, 16, 64)), (inputs.MLP7B_GATE, (1, 8, 16, 64)),
+                 (inputs.MLP7B_DOWN, (1, 8, 16, 64)), (inputs.ATTN70B, (1, 8, 16, 64)),
                  (inputs.MLP70B_GATE, (1, 8, 16, 32, 64, 128))]
 PREFILL_POINTS = [(inputs.ATTN7B, 2048), (inputs.ATTN7B, 8192), (inputs.ATTN70B, 4096), (inputs.MLP70B_GATE, 4096)]
 
@@ -341,7 +349,7 @@ def mlp7b_point(dev, stream, T, hbm_peak, tc_peak, peak_src):
     import torch
     from paper_2501_19090_gb300 import pifa as P
     G_, D_ = inputs.MLP7B_GATE, inputs.MLP7B_DOWN
-    decode = T <= DECODE_MAX_T
+    decode = is_decode(T, G_.m, G_.r)
     copies = 4 if decode else 2
     lay = {name: timing_layer(s, dev, seed, copies=copies) for name, s, seed in
            (("gate", G_, 1), ("up", G_, 2), ("down", D_, 3))}
@@ -534,7 +542,7 @@ def run_ours(args, rank, world, local_rank):
     m, n, r = shape.m, shape.n, shape.r
     T = args.tokens
     K = max(1, args.steps)
-    decode = T <= DECODE_MAX_T
+    decode = is_decode(T, m, r)
     wbytes = 2 * r * (m + n - r)
     copies = _copies_for(dev, wbytes)
     piv, nonp, Wps, Cs = timing_layer(shape, dev, 0, args.c_dtype, copies)
@@ -959,7 +967,7 @@ def run_reference(args, rank):
     return {"impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": done, "requested_steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / done,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": f"{shape.name} {'decode' if T <= DECODE_MAX_T else 'prefill'} T={T}",
+            "data": "synthetic", "config": {"workload": f"{shape.name} {'decode' if is_decode(T, shape.m, shape.r) else 'prefill'} T={T}",
                                             "m": shape.m, "n": shape.n, "r": shape.r, "tokens_per_step": T,
                                             "c_dtype": args.c_dtype, "parallelism": f"replicas{args.gpus}"},
             "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle",

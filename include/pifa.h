@@ -186,9 +186,10 @@ int64_t pifa_workspace_size(int64_t T, int64_t m, int64_t n, int64_t r, int c_dt
 
 /* pifa_select_variant -- the selector (host, < 1 us): the pifa_variant pifa_forward runs for
  * (T, m, n, r, c_dtype) on this build, never PIFA_VARIANT_AUTO; negative pifa_status on bad
- * arguments. Decode for T <= 64, and for T <= 128 when both phases (r and m - r rows) have at
- * most 296 blocks of 128 rows; else the split prefill. The forced decode variant takes the same
- * shapes (PIFA_ERR_UNSUPPORTED otherwise). */
+ * arguments. Decode for T <= 64, and for T <= 128 when the m - r non-pivot rows make between 148
+ * and 296 blocks of 128 rows and the r pivot rows at most 296; else the split prefill. The forced
+ * decode variant takes T <= 64, and T <= 128 when both phases have at most 296 blocks
+ * (PIFA_ERR_UNSUPPORTED otherwise). */
 int pifa_select_variant(int64_t T, int64_t m, int64_t n, int64_t r, int c_dtype);
 
 /* pifa_variant_name -- static string naming a pifa_variant ("decode", ...); "?" if unknown. */

@@ -158,15 +158,19 @@ bool decode_takes(int64_t T, int64_t G, int64_t m, int64_t r) {
   return (G * r + 127) / 128 <= kWideRowBlocks && (G * (m - r) + 127) / 128 <= kWideRowBlocks;
 }
 
-// The selector: decode wherever it runs. Decode streams each weight once with every token's
-// product per tile; against the split prefill it measured 2.0-2.8x faster at T = 24 / 32 / 64 and
-// 1.2-2.3x at T = 80 / 96 / 128 on the LLaMA-2 7B and 70B layers (70B gate/up T = 128: 83.6 us
-// against 145.0 us), whose prefill grids hold one token tile at such T, too few tiles to fill the
-// GPU.
+// The selector. Decode streams each weight once with every token's product per tile; against the
+// split prefill (one process, interleaved, us) it measured 2.0-2.8x faster at T = 24 / 32 / 64 on
+// the LLaMA-2 7B and 70B layers, whose prefill GEMMs hold one token tile at such T. From T = 65 the
+// prefill's split-K clusters catch up on layers of few non-pivot rows (T = 128: 7B attention 26.9
+// against 30.2, 7B MLP gate 36.2 against 39.3, 70B q/o 41.4 against 41.8; at T = 96 within 2-7%
+// either way), while on a non-pivot phase of at least one 128-row block per SM decode keeps its
+// lead (70B gate/up, 192 blocks: T = 128 83.7 against 124.4). So: decode for T <= 64, and up to 128
+// where the non-pivot rows make at least kWideRowBlocks / 2 blocks.
 int select_for(int64_t T, int64_t G, int64_t m, int64_t r) {
-  return decode_takes(T, G, m, r) ? PIFA_VARIANT_DECODE : PIFA_VARIANT_PREFILL_SPLIT;
+  if (T <= 64) return PIFA_VARIANT_DECODE;
+  if (decode_takes(T, G, m, r) && (G * (m - r) + 127) / 128 >= kWideRowBlocks / 2) return PIFA_VARIANT_DECODE;
+  return PIFA_VARIANT_PREFILL_SPLIT;
 }
-
 }  // namespace
 
 extern "C" {

@@ -56,10 +56,10 @@ def test_clock_summary_empty():
     assert _sampler([]) == {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
 
 
-@pytest.mark.parametrize("m,n,r", SHAPES)
+@pytest.mark.parametrize("m,n,r", SHAPES + [(40000, 520, 264), (30000, 520, 264), (19456 + 4096, 8192, 4096)])
 def test_bench_decode_rule_is_the_library_selector(m, n, r):
     """bench.py names a workload decode (HBM roofline, L2-defeating weight copies) exactly when the
     library's selector runs the decode variant."""
     from paper_2501_19090_gb300 import pifa as P
-    for T in (1, 16, bench.DECODE_MAX_T, bench.DECODE_MAX_T + 1, 2048):
-        assert (P.pifa_select_variant(T, m, n, r) == P.PIFA_VARIANT_DECODE) == (T <= bench.DECODE_MAX_T)
+    for T in (1, 16, 64, 65, 96, 128, 129, 2048):
+        assert (P.pifa_select_variant(T, m, n, r) == P.PIFA_VARIANT_DECODE) == bench.is_decode(T, m, r), T

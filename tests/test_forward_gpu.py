@@ -472,8 +472,10 @@ def test_selector_picks_split_prefill():
     assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_FP16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(2048, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT, P.pifa_last_error()
     assert P.pifa_select_variant(16, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
-    assert P.pifa_select_variant(128, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
-    assert P.pifa_select_variant(129, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT
+    assert P.pifa_select_variant(64, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE
+    assert P.pifa_select_variant(96, 4096, 4096, 2048, P.PIFA_DTYPE_BF16) == SPLIT      # 16 non-pivot blocks
+    assert P.pifa_select_variant(128, 28672, 8192, 4096, P.PIFA_DTYPE_BF16) == P.PIFA_VARIANT_DECODE  # 192
+    assert P.pifa_select_variant(129, 28672, 8192, 4096, P.PIFA_DTYPE_BF16) == SPLIT
     assert P.pifa_select_variant(100, 40000, 520, 264, P.PIFA_DTYPE_BF16) == SPLIT  # 311 row blocks
 
 

@@ -76,10 +76,12 @@ def test_selector(lib):
     assert P.pifa_select_variant(16, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE
     assert P.pifa_select_variant(2048, 4096, 4096, 2048) == P.PIFA_VARIANT_PREFILL_SPLIT
     assert P.pifa_select_variant(64, 256, 256, 128) == P.PIFA_VARIANT_DECODE
-    assert P.pifa_select_variant(128, 256, 256, 128) == P.PIFA_VARIANT_DECODE
+    assert P.pifa_select_variant(128, 256, 256, 128) == P.PIFA_VARIANT_PREFILL_SPLIT  # 1 non-pivot block
     assert P.pifa_select_variant(129, 256, 256, 128) == P.PIFA_VARIANT_PREFILL_SPLIT
-    # 64 < T <= 128 decodes only when both phases have at most 296 row blocks of 128
+    # 64 < T <= 128 decodes where the non-pivot rows make 148 to 296 blocks of 128 (and the pivot
+    # rows at most 296)
     assert P.pifa_select_variant(100, 28672, 8192, 4096) == P.PIFA_VARIANT_DECODE       # 32 and 192
+    assert P.pifa_select_variant(128, 8192, 8192, 4096) == P.PIFA_VARIANT_PREFILL_SPLIT  # 32 and 32
     assert P.pifa_select_variant(100, 40000, 520, 264) == P.PIFA_VARIANT_PREFILL_SPLIT  # 3 and 311
     assert P.pifa_select_variant(64, 40000, 520, 264) == P.PIFA_VARIANT_DECODE
     # grouped layers count their stacked rows: 70B gate + up (2 x 192 non-pivot blocks) prefill
