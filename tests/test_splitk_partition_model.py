@@ -163,13 +163,20 @@ def test_row_block_plan_on_the_llama_phases():
     assert (p["grid"], p["ncf"], p["ns"], p["nclast"]) == (256, 16, 8, 16)
 
 
-@pytest.mark.parametrize("tnt", [16, 32, 64])
+@pytest.mark.parametrize("tnt", [16, 32, 64, 128])
 @pytest.mark.parametrize("nb", [1, 2])
-def test_cluster_sums_fit_the_ring(tnt, nb):
-    """The cluster's [T][128] fp32 sums reuse the stage ring (112 KB per CTA less 1.5 KB)."""
+def test_cluster_sums_fit_the_ring_and_tensor_memory(tnt, nb):
+    """Per CTA (two per SM): the stage ring (112 KB less 1.5 KB) holds at least two stages and the
+    cluster's [T][128] fp32 sums; tensor memory holds the accumulators in its 256 columns: two
+    segments of 128 / (tnt nb) accumulators each up to 64 tokens, one accumulator of tnt nb columns
+    at 128 tokens (the row-block plan's single segment)."""
     stage = TM * KB * 2 + nb * tnt * KB * 2
     stages = min(10, (112 * 1024 - 1536) // stage)
     assert stages >= 2 and TM * tnt * 4 <= stages * stage
+    nacc = 1 if tnt * nb >= 128 else 128 // (tnt * nb)
+    segments = 2 if tnt <= 64 else 1
+    assert segments * nacc * tnt * nb <= 256
+    assert 16 <= tnt * nb <= 256 and (tnt * nb) % 16 == 0          # an MMA's N for M = 128
 
 
 # ---- the split prefill's choice of tile width and K-slices (csrc/prefill.cu pick_shape) ----------
