@@ -55,35 +55,85 @@ __global__ void split_cols(const bf16* in, int64_t ldin, const int32_t* piv, int
 }
 
 // out = a * x + b * y elementwise over T rows of n (bf16 in, fp32 arithmetic), written as a hi +
-// lo pair of bf16 planes. Rows across the y grid, columns across x.
+// lo pair of bf16 planes. A thread owns 8 consecutive columns of a row (16-byte loads and stores:
+// every pitch is a multiple of 8 elements and every base 16-byte aligned), scalar at a ragged end.
+// Rows across the y grid, column groups across x.
 __global__ void axpby_rows(const bf16* x, const bf16* y, int64_t ld, int T, int n, float a, float b, bf16* out,
                            bf16* out_lo, int64_t ldout) {
   pdl_launch_dependents();
   pdl_wait_primary();
+  const int ng = (n + 7) / 8;
   for (int t = blockIdx.y; t < T; t += gridDim.y)
-    for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < n; c += gridDim.x * blockDim.x) {
-      const float v = a * __bfloat162float(x[(int64_t)t * ld + c]) + b * __bfloat162float(y[(int64_t)t * ld + c]);
-      const bf16 h = __float2bfloat16_rn(v);
-      out[(int64_t)t * ldout + c] = h;
-      out_lo[(int64_t)t * ldout + c] = __float2bfloat16_rn(v - __bfloat162float(h));
+    for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < ng; g += gridDim.x * blockDim.x) {
+      const int c = 8 * g;
+      const bf16* xr = x + (int64_t)t * ld + c;
+      const bf16* yr = y + (int64_t)t * ld + c;
+      bf16* hr = out + (int64_t)t * ldout + c;
+      bf16* lr = out_lo + (int64_t)t * ldout + c;
+      if (c + 8 <= n) {
+        uint4 xv = *reinterpret_cast<const uint4*>(xr), yv = *reinterpret_cast<const uint4*>(yr), hv, lv;
+        const bf16* xe = reinterpret_cast<const bf16*>(&xv);
+        const bf16* ye = reinterpret_cast<const bf16*>(&yv);
+        bf16* he = reinterpret_cast<bf16*>(&hv);
+        bf16* le = reinterpret_cast<bf16*>(&lv);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float v = a * __bfloat162float(xe[e]) + b * __bfloat162float(ye[e]);
+          he[e] = __float2bfloat16_rn(v);
+          le[e] = __float2bfloat16_rn(v - __bfloat162float(he[e]));
+        }
+        *reinterpret_cast<uint4*>(hr) = hv;
+        *reinterpret_cast<uint4*>(lr) = lv;
+      } else {
+        for (int e = 0; c + e < n; ++e) {
+          const float v = a * __bfloat162float(xr[e]) + b * __bfloat162float(yr[e]);
+          const bf16 h = __float2bfloat16_rn(v);
+          hr[e] = h;
+          lr[e] = __float2bfloat16_rn(v - __bfloat162float(h));
+        }
+      }
     }
 }
 
-// out (cols x rows) = in (rows x cols)^T, bf16, through 32 x 32 shared-memory tiles (coalesced
-// reads and writes). Block (32, 8); grid (ceil(cols / 32), ceil(rows / 32)).
+// out (cols x rows) = in (rows x cols)^T, bf16, through 64 x 64 shared-memory tiles: each thread
+// loads 8 consecutive elements of an input row and stores 8 consecutive elements of an output row
+// (16-byte accesses: both pitches are multiples of 8 elements and both bases 16-byte aligned;
+// scalar at ragged edges). The tile's 8-element groups are stored XOR-swizzled by the row's group
+// (group g of row k at g ^ (k / 8 % 8)), so that the column reads of 8 rows 8 apart hit 8 different
+// banks. Block (8, 32); grid (ceil(cols / 64), ceil(rows / 64)).
 __global__ void transpose_bf16(const bf16* in, int64_t ldin, int rows, int cols, bf16* out, int64_t ldout) {
-  __shared__ bf16 t[32][34];
+  __shared__ __align__(16) bf16 t[64][64];
   pdl_launch_dependents();
   pdl_wait_primary();
-  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
-  for (int k = threadIdx.y; k < 32; k += 8) {
-    const int r = r0 + k, c = c0 + threadIdx.x;
-    t[k][threadIdx.x] = (r < rows && c < cols) ? in[(int64_t)r * ldin + c] : __float2bfloat16_rn(0.0f);
+  const int c0 = blockIdx.x * 64, r0 = blockIdx.y * 64;
+  const int tx = threadIdx.x, ty = threadIdx.y;  // 8 x 32
+  for (int k = ty; k < 64; k += 32) {  // input row r0 + k, columns c0 + 8 tx .. + 7
+    const int r = r0 + k, c = c0 + 8 * tx;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (r < rows && c + 8 <= cols) {
+      v = *reinterpret_cast<const uint4*>(in + (int64_t)r * ldin + c);
+    } else if (r < rows) {
+      bf16* ve = reinterpret_cast<bf16*>(&v);
+      for (int e = 0; e < 8 && c + e < cols; ++e) ve[e] = in[(int64_t)r * ldin + c + e];
+    }
+    *reinterpret_cast<uint4*>(&t[k][8 * (tx ^ ((k >> 3) & 7))]) = v;
   }
   __syncthreads();
-  for (int k = threadIdx.y; k < 32; k += 8) {
-    const int c = c0 + k, r = r0 + threadIdx.x;
-    if (c < cols && r < rows) out[(int64_t)c * ldout + r] = t[threadIdx.x][k];
+  for (int k = ty; k < 64; k += 32) {  // output row c0 + k (input column), rows r0 + 8 tx .. + 7
+    const int c = c0 + k, r = r0 + 8 * tx;
+    if (c >= cols) continue;
+    uint4 v;
+    bf16* ve = reinterpret_cast<bf16*>(&v);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const int kr = 8 * tx + e;  // tile row; its group (k >> 3) sits at (k >> 3) ^ tx
+      ve[e] = t[kr][8 * ((k >> 3) ^ ((kr >> 3) & 7)) + (k & 7)];
+    }
+    if (r + 8 <= rows) {
+      *reinterpret_cast<uint4*>(out + (int64_t)c * ldout + r) = v;
+    } else {
+      for (int e = 0; r + e < rows; ++e) out[(int64_t)c * ldout + r + e] = ve[e];
+    }
   }
 }
 
@@ -293,8 +343,8 @@ extern "C" int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int6
   const int64_t ldT = pad8(T), ldn = pad8(n);
   {  // X_u^T
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)((n + 31) / 32), (unsigned)((T + 31) / 32));
-    cfg.blockDim = dim3(32, 8);
+    cfg.gridDim = dim3((unsigned)((n + 63) / 64), (unsigned)((T + 63) / 64));
+    cfg.blockDim = dim3(8, 32);
     cfg.stream = s;
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -320,7 +370,8 @@ extern "C" int pifa_m_accumulate(const void* Xo, const void* Xu, int64_t T, int6
       float a = lambda, b = 1.0f - lambda;
       void* args[] = {(void*)&Xo, (void*)&Xu, (void*)&ldx, (void*)&Ti, (void*)&ni, (void*)&a, (void*)&b, (void*)&Xmix,
                       (void*)&Xmix_lo, (void*)&ldn};
-      if ((st = launch_small((const void*)axpby_rows, args, T, n, s2, "m_accumulate: mix")) != PIFA_OK) return st;
+      if ((st = launch_small((const void*)axpby_rows, args, T, (n + 7) / 8, s2, "m_accumulate: mix")) != PIFA_OK)
+        return st;
     }
     {  // Y_t^T = W (X_mix,hi + X_mix,lo)^T, as hi + lo planes (m x T)
       GemmTc g = {m, T, n, W, ldw, false, Xmix, ldn, false, YtT, ldT, 3, 1.0f, nullptr, nullptr, 0, 0};
