@@ -229,3 +229,24 @@ def test_prefill_k_slices_cover_every_step_once(ksteps, ks):
     """CTA z of a tile's cluster accumulates K-steps [z ksteps / ks, (z + 1) ksteps / ks)."""
     steps = [i for z in range(ks) for i in range(z * ksteps // ks, (z + 1) * ksteps // ks)]
     assert steps == list(range(ksteps))
+
+
+@pytest.mark.parametrize("ks,bn,ntok", [(2, 256, 256), (4, 256, 200), (4, 208, 200), (2, 208, 17)])
+def test_prefill_cluster_sums_cover_the_tile_once(ks, bn, ntok):
+    """The split prefill's cluster epilogue: every CTA stores its partial tile as [token][128 rows]
+    (bn tokens, within the ring); CTA z of ks then finishes rows [z 128 / ks, (z + 1) 128 / ks) for
+    the tile's ntok tokens, thread idx taking token idx / rpc and row z rpc + idx % rpc. Every
+    (token, row) of the tile is finished exactly once, and every read stays inside the stored
+    partial tile."""
+    rpc = 128 // ks
+    seen = set()
+    for z in range(ks):
+        for idx in range(rpc * ntok):
+            t, rr = idx // rpc, z * rpc + idx % rpc
+            assert 0 <= t < ntok <= bn and 0 <= rr < 128
+            off = t * 128 + rr
+            assert 0 <= off < bn * 128
+            assert (t, rr) not in seen
+            seen.add((t, rr))
+    assert len(seen) == ntok * 128
+    assert bn * 128 * 4 <= 4 * (16 * 1024 + 256 * 128)          # the one-CTA shape's 4-stage ring
