@@ -62,7 +62,7 @@ NCU_TRAFFIC = {
     # profiles/decode_tc_gateup70b_T16_traffic.md: phase 1 in clusters of 8 CTAs per row block,
     # phase 2 one CTA per row block; two kernels, no partial sums in global memory
     ("llama2_70b_gate_up_28672x8192_r4096", 16): {
-        "sha": {"decode_tc.cu": "ee3fc341cbb54146", "decode.cu": "d641f7870ae488ab"},
+        "sha": {"decode_tc.cu": "35b8964778d8fafd", "decode.cu": "d641f7870ae488ab"},
         "bytes": 269409536,
     },
 }

@@ -1,6 +1,7 @@
 // decode_tc.cu -- one decode phase (T <= 128 tokens) of Algorithm 2 on the 5th-generation tensor
-// cores, split over K across a persistent grid: the form used for layers too large for one wave,
-// and the only decode form for 16 < T <= 128.
+// cores, split over K: the decode form for large phases when T > 2, and the only one for
+// 16 < T <= 128. Two cuts of a phase: the row-block plan (below) for phases of at most two 128-row
+// blocks per SM, and balanced ranges with a reduce kernel for taller ones (described first).
 //
 // A phase is a skinny product D = A B^T: A the weight rows (W_p for Y_p = X W_p^T, Algorithm 2
 // step 2; C for Y_np = Y_p C^T, step 3), B the T token rows (x, or y_p as its hi and lo planes).
@@ -24,7 +25,8 @@
 //              for each other. A 128-token tile's accumulator (N = 128 or 256) fills the 256
 //              columns alone, so it is used only where a CTA has one segment (the row-block plan).
 //   warps 2-5  sum a segment's accumulators (TMEM lane quarter each) while the next segment fills
-//              the other set, and store its partial sums P[s][t][row] (fp32, coalesced over rows).
+//              the other set, and store its partial sums P[s][t][row] (fp32, coalesced over rows),
+//              or, in the row-block plan, the outputs or the cluster's shared-memory sums.
 // A unit's head CTA writes zeros to P2 when it holds the whole unit, so P2 is defined everywhere.
 // Reduce kernel: Y[t, cols[j]] = bf16(sum_s (P[s][t][j] + P2[s][t][j])) in slice order
 // (deterministic for a given grid); phase 1 also writes y_p as the hi + lo planes of C's dtype
@@ -60,8 +62,9 @@ constexpr int THREADS = 192;
 // A segment's MMAs are dealt round-robin over NACC independent accumulators (summed in the
 // epilogue), so that consecutive MMAs do not wait for each other. With two B planes (y_p hi and
 // lo) one MMA of N = 2 TNT covers both: the lo box follows the hi box in shared memory, making one
-// 2 TNT-row operand, and accumulator columns t and TNT + t are added in the epilogue. Per segment
-// NACC * TNT * NB = 128 columns; two segments in flight: 256 TMEM columns in every case.
+// 2 TNT-row operand, and accumulator columns t and TNT + t are added in the epilogue. Up to 64
+// tokens, NACC * TNT * NB = 128 columns per segment and two segments in flight: 256 TMEM columns.
+// A 128-token tile's one accumulator takes 128 or 256 columns: one segment (the row-block plan).
 template <int NB, int TNT = TN>
 constexpr int kNacc = TNT * NB >= 128 ? 1 : 128 / (TNT * NB);
 constexpr uint32_t TMEM_COLS = 256;
@@ -640,7 +643,9 @@ int launch_decode_tc(const DecodeTcPhase& ph, int* status, uint64_t timeout_ns, 
   // shared memory and writes Y (and y_p's planes) itself. No partial sums in global memory and no
   // reduce kernel: one kernel and one kernel boundary fewer per phase (measured on the 70B gate/up
   // layer, whose phase 2 has 192 row blocks and takes cs = 1: T = 16 57.1 -> 53.0 us per call, T = 8
-  // 54.3 -> 51.5 us). Longer phases deal balanced chunk ranges and sum P + P2 in a second kernel.
+  // 54.3 -> 51.5 us; clusters where a phase has fewer blocks, against balanced ranges and a reduce
+  // kernel: 70B q/o T = 16 28.9 -> 26.4 us, 70B gate/up T = 64 67.3 -> 60.8, 7B MLP down T = 64
+  // 41.4 -> 27.0). Longer phases deal balanced chunk ranges and sum P + P2 in a second kernel.
   const int64_t nrb_all = (ph.R + TM - 1) / TM, nck_all = (ph.K + KB - 1) / KB;
   int cs = 0;
   if (nrb_all <= grid_cap()) {
