@@ -289,3 +289,42 @@ def test_binding_argtypes_match_the_header(lib):
         ret, params = protos[name]
         assert [cat(t) for t in fn.argtypes] == params, name
         assert cat(fn.restype) == ret, name
+
+
+def _documented_choice(T, G, m, r):
+    """pifa.h's rule: decode for T <= 64; for 64 < T <= 128 when the G (m - r) non-pivot rows make
+    148 to 296 blocks of 128 and the G r pivot rows at most 296; the split prefill otherwise."""
+    if T <= 64:
+        return P.PIFA_VARIANT_DECODE
+    bp, bnp = -(-G * r // 128), -(-G * (m - r) // 128)
+    if T <= 128 and bp <= 296 and 148 <= bnp <= 296:
+        return P.PIFA_VARIANT_DECODE
+    return P.PIFA_VARIANT_PREFILL_SPLIT
+
+
+def test_selector_and_forced_decode_follow_the_documented_rule(lib):
+    """Random shapes and token counts: the selector's variant (single layers) and the workspace the
+    grouped entry point sizes (its own choice) follow the documented rule; a forced decode call is
+    refused exactly where 64 < T <= 128 and a phase has more than 296 blocks, or T > 128."""
+    rng = np.random.default_rng(5)
+    for _ in range(400):
+        r = int(rng.integers(1, 9000))
+        m = r + int(rng.integers(0, 45000))
+        n = int(rng.integers(r, r + 9000))
+        T = int(rng.choice([1, 16, 64, 65, 96, 128, 129, 500]))
+        assert P.pifa_select_variant(T, m, n, r) == _documented_choice(T, 1, m, r), (T, m, n, r)
+        fits = T <= 64 or (T <= 128 and -(-r // 128) <= 296 and -(-(m - r) // 128) <= 296)
+        X, Wp, C, Y = 1 << 36, 2 << 36, 3 << 36, 4 << 36
+        p8 = lambda v: (v + 7) // 8 * 8
+        st = lib.pifa_forward_variant(X, T, n, p8(n), Wp, r, p8(n), C, m, p8(r), P.PIFA_DTYPE_BF16, 0x50000, 0x60000,
+                                      Y, p8(m), None, 0, P.PIFA_VARIANT_DECODE, None)
+        # buffers 64 GB apart never overlap at these sizes; a fitting shape fails on the missing workspace
+        assert st == (P.PIFA_ERR_WORKSPACE if fits else P.PIFA_ERR_UNSUPPORTED), (T, m, n, r, st)
+    # grouped layers whose stacked non-pivot rows make fewer than 148 or more than 296 blocks take
+    # the split prefill above T = 64: the workspace the grouped entry point sizes is the prefill's,
+    # 256 reserved bytes and the hi and lo planes (T x pad8(G r) bf16 each, 256-byte rounded)
+    for G, m, r in ((2, 11008, 2048), (2, 28672, 4096), (3, 1408, 512)):
+        for T in (100, 128):
+            assert _documented_choice(T, G, m, r) == P.PIFA_VARIANT_PREFILL_SPLIT
+            plane = -(-(T * -(-G * r // 8) * 8 * 2) // 256) * 256
+            assert lib.pifa_workspace_size_grouped(G, T, m, 4096, r, P.PIFA_DTYPE_BF16) == 256 + 2 * plane
